@@ -358,7 +358,7 @@ int orc_lm_window_logits(const orc_cfg* c, const uint16_t* win_tok, int64_t n_po
 /* the LM probabilities were made integer). T = 2^P, row z[0..V) of fp32 logits:               */
 /*  (i)   m = max z                                                                            */
 /*  (ii)  y_j = fp32(fp32(z_j - m) * C), C = fp32(2^16 * log2 e)   (round to nearest, no FMA) */
-/*  (iii) a_j = -rint(y_j) >= 0, clamped to 40 * 2^16                                          */
+/*  (iii) a_j = -rint(y_j) >= 0, clamped to 40 * 2^16 (y_j < -40 * 2^16 gives the cap directly) */
 /*  (iv)  e_j = ((H[(a>>8)&255] * L[a&255] + 2^30) >> 31) >> (a >> 16)   ~ 2^31 * exp(z_j - m) */
 /*  (v)   S = sum e_j                                                                          */
 /*  (vi)  g_j = floor(e_j * (T - V) / S); freq_j = 1 + g_j; the residual (T - V) - sum g_j     */
@@ -397,7 +397,8 @@ int orc_quantize_cdf(const float* z, int V, int P, uint32_t* cdf) {
   for (int j = 0; j < V; j++) {
     float dz = z[j] - m;
     float y = dz * C;
-    int64_t a = -(int64_t)rintf(y);
+    /* (iii) with the clamp applied before the conversion: y below -40*2^16 gives the cap */
+    int64_t a = (y < -(float)ORC_A_MAX) ? ORC_A_MAX : -(int64_t)rintf(y);
     e[j] = orc_exp2_fixed(a);
     S += e[j];
     if (e[j] > e[amax]) amax = j;

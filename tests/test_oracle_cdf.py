@@ -101,3 +101,12 @@ def test_cdf_pair_matches_cdf():
     cdf = O.quantize_cdf(z, 16)
     assert np.array_equal(st, cdf[np.arange(40), sym])
     assert np.array_equal(fr, cdf[np.arange(40), sym + 1] - st)
+
+
+def test_huge_logit_gaps_clamp():
+    """Gaps far beyond the 40 * 2^16 cap (e.g. -1e30) clamp to e = 0, i.e. freq 1."""
+    for gap in [-1e30, -3.0e38, -1e6, -27.8]:
+        z = np.full(10, np.float32(gap), np.float32)
+        z[3] = 0.0
+        f = np.diff(O.quantize_cdf(z, 16)[0].astype(np.int64))
+        assert f[3] == 2 ** 16 - 9 and np.all(np.delete(f, 3) == 1), gap
