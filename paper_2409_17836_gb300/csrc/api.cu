@@ -1,0 +1,747 @@
+// api.cu -- the C ABI of liblmgc.so (include/lmgc.h): context, model forward orchestration,
+// the encode pipeline (Sec. 3: serialise -> windows from BOS -> LM -> integer CDF -> one
+// arithmetic code per window -> container) and the KV-cached decode (Sec. 3 "Compression").
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+
+static thread_local std::string g_thread_err;
+
+void set_thread_error(const std::string& s) { g_thread_err = s; }
+
+lmgc_status fail(lmgc_ctx* ctx, lmgc_status st, const std::string& msg) {
+  if (ctx) ctx->err = msg;
+  g_thread_err = msg;
+  return st;
+}
+
+lmgc_status cuda_fail(lmgc_ctx* ctx, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  return fail(ctx, e == cudaErrorMemoryAllocation ? LMGC_ERR_NOMEM : LMGC_ERR_CUDA, m);
+}
+
+// CRC-32 (IEEE 802.3, reflected 0xEDB88320), for the container header.
+static uint32_t crc32(const uint8_t* p, size_t n) {
+  static uint32_t table[256];
+  static bool init = false;
+  if (!init) {
+    for (uint32_t i = 0; i < 256; i++) {
+      uint32_t c = i;
+      for (int k = 0; k < 8; k++) c = (c & 1u) ? (0xEDB88320u ^ (c >> 1)) : (c >> 1);
+      table[i] = c;
+    }
+    init = true;
+  }
+  uint32_t c = 0xFFFFFFFFu;
+  for (size_t i = 0; i < n; i++) c = table[(c ^ p[i]) & 0xFFu] ^ (c >> 8);
+  return c ^ 0xFFFFFFFFu;
+}
+
+static uint32_t model_crc(const lmgc_config& c) {
+  uint8_t b[40];
+  int32_t iv[7] = {c.n_layers, c.d_model, c.n_heads, c.n_kv_heads, c.d_ffn, c.vocab, c.dtype == LMGC_BF16 ? 1 : 0};
+  float fv[3] = {c.init_std, c.rms_eps, c.rope_theta};
+  memcpy(b, iv, 28);
+  memcpy(b + 28, fv, 12);
+  return crc32(b, 40);
+}
+
+// ---- profiling of kernel classes (CUDA events around launches, only when enabled) ----
+enum KClass { kGemm = 0, kAttn = 1, kCdf = 2, kCoder = 3, kSer = 4, kNorm = 5, kOther = 6, kNumClasses = 7 };
+static const char* kClassNames[kNumClasses] = {"gemm", "attention", "cdf_pairs", "range_encode", "serialize",
+                                                "norm_rope_act", "other"};
+
+static cudaEvent_t prof_event(lmgc_ctx* ctx) {
+  if (!ctx->prof.pool.empty()) {
+    cudaEvent_t e = ctx->prof.pool.back();
+    ctx->prof.pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e;
+  cudaEventCreate(&e);
+  return e;
+}
+
+struct ProfScope {
+  lmgc_ctx* ctx;
+  cudaStream_t s;
+  bool on;
+  ProfScope(lmgc_ctx* c, int cls, double work, cudaStream_t st) : ctx(c), s(st), on(c->prof.enabled) {
+    if (!on) return;
+    Profiler::Rec r;
+    r.cls = cls;
+    r.work = work;
+    r.a = prof_event(ctx);
+    r.b = prof_event(ctx);
+    cudaEventRecord(r.a, s);
+    ctx->prof.pending.push_back(r);
+  }
+  ~ProfScope() {
+    if (on) cudaEventRecord(ctx->prof.pending.back().b, s);
+  }
+};
+
+static void prof_collect(lmgc_ctx* ctx) {
+  for (auto& r : ctx->prof.pending) {
+    float ms = 0.f;
+    cudaEventSynchronize(r.b);
+    cudaEventElapsedTime(&ms, r.a, r.b);
+    KernelStat& st = ctx->prof.stats[r.cls];
+    st.launches++;
+    st.ms += ms;
+    st.work += r.work;
+    ctx->prof.pool.push_back(r.a);
+    ctx->prof.pool.push_back(r.b);
+  }
+  ctx->prof.pending.clear();
+}
+
+// ---- GEMM dispatch: tcgen05 for bf16 when the shape fits, CUDA cores otherwise ----
+static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi,
+                 cudaStream_t s) {
+  ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
+  if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K))
+    launch_gemm_tc(A, B, C, M, N, K, epi, s);
+  else
+    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);
+}
+
+static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, int64_t n_win, int64_t pos_first,
+                      int n_pos, int64_t q_win_stride, cudaStream_t s) {
+  const lmgc_config& c = ctx->cfg;
+  // algorithmic flops: QK^T and PV over the causal triangle, 4*hd per (query, key) pair per head
+  double pairs = 0;
+  for (int64_t p = pos_first; p < pos_first + n_pos; p++) pairs += (double)(p + 1);
+  ProfScope ps(ctx, kAttn, 4.0 * ctx->hd * c.n_heads * pairs * (double)n_win, s);
+  const int qd = c.n_heads * ctx->hd, kd = c.n_kv_heads * ctx->hd;
+  launch_attention(q, ctx->qkv_dim, kv, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads, c.n_kv_heads, ctx->hd,
+                   c.window, n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
+}
+
+// One forward of the model over `rows` input rows already embedded into ws.x.
+//   prefill: rows = n_win * W, row r at position r mod W, keys/values from ws.qkv itself
+//   decode:  rows = n_win, every row at position pos; keys/values from the cache
+static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool decode, int64_t pos, cudaStream_t s) {
+  const lmgc_config& c = ctx->cfg;
+  const int d = c.d_model, F = c.d_ffn, hd = ctx->hd, qd = c.n_heads * hd;
+  Workspace& ws = ctx->ws;
+  const int64_t W = c.window;
+  for (int l = 0; l < c.n_layers; l++) {
+    const Layer& L = ctx->layers[l];
+    {
+      ProfScope ps(ctx, kNorm, 0, s);
+      launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
+    }
+    gemm(ctx, ws.n, L.wqkv, ws.qkv, rows, ctx->qkv_dim, d, kStore, s);
+    {
+      ProfScope ps(ctx, kNorm, 0, s);
+      launch_rope(ws.qkv, rows, ctx->qkv_dim, c.n_heads + c.n_kv_heads, hd, ctx->rope_cs, c.window,
+                  decode ? pos : 0, decode ? 1 : W, decode ? 1 : c.window, c.dtype, s);
+    }
+    if (!decode) {
+      attention(ctx, ws.qkv, ws.qkv, ws.att, n_win, 0, c.window, W, s);
+    } else {
+      char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->qkv_dim * ctx->elt;
+      launch_copy_rows(ws.qkv, ctx->qkv_dim, cache_l, W, pos, n_win, ctx->qkv_dim, c.dtype, s);
+      attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s);
+    }
+    gemm(ctx, ws.att, L.wo, ws.x, rows, d, qd, kAddResidual, s);
+    {
+      ProfScope ps(ctx, kNorm, 0, s);
+      launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
+    }
+    gemm(ctx, ws.n, L.wgu, ws.gu, rows, 2 * (int64_t)F, d, kStore, s);
+    {
+      ProfScope ps(ctx, kNorm, 0, s);
+      launch_swiglu(ws.gu, rows, F, ws.act, c.dtype, s);
+    }
+    gemm(ctx, ws.act, L.wdown, ws.x, rows, d, F, kAddResidual, s);
+  }
+  {
+    ProfScope ps(ctx, kNorm, 0, s);
+    launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
+  }
+  gemm(ctx, ws.n, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s);
+}
+
+// Model logits for windows [first_win, first_win + nb) of a token stream, into ctx->logits.
+static void forward_windows(lmgc_ctx* ctx, const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t nb,
+                            cudaStream_t s) {
+  const lmgc_config& c = ctx->cfg;
+  const int64_t rows = nb * c.window;
+  {
+    ProfScope ps(ctx, kOther, 0, s);
+    launch_window_inputs(tok, n_tok, first_win, nb, c.window, ctx->ws.tok_in, s);
+    launch_embed(ctx->ws.tok_in, rows, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
+  }
+  forward_layers(ctx, rows, nb, false, 0, s);
+}
+
+template <typename T>
+static cudaError_t dmalloc(T** p, size_t bytes) {
+  return cudaMalloc((void**)p, bytes ? bytes : 16);
+}
+
+template <typename T>
+static cudaError_t ensure(T** p, size_t* cap, size_t need) {
+  if (*cap >= need && *p) return cudaSuccess;
+  if (*p) cudaFree(*p);
+  *p = nullptr;
+  *cap = 0;
+  cudaError_t e = cudaMalloc((void**)p, need ? need : 16);
+  if (e == cudaSuccess) *cap = need;
+  return e;
+}
+
+static lmgc_status check_err_word(lmgc_ctx* ctx, cudaStream_t s, const char* what) {
+  uint32_t h = 0;
+  LMGC_CUDA(ctx, cudaMemcpyAsync(&h, ctx->d_err, 4, cudaMemcpyDeviceToHost, s));
+  LMGC_CUDA(ctx, cudaStreamSynchronize(s));
+  if (h == 0) return LMGC_OK;
+  cudaMemsetAsync(ctx->d_err, 0, 4, s);
+  cudaStreamSynchronize(s);
+  if (h & kErrLimit) return fail(ctx, LMGC_ERR_LIMIT, std::string(what) + ": device loop limit");
+  return fail(ctx, LMGC_ERR_CORRUPT, std::string(what) + ": corrupt input (device error word " +
+                                         std::to_string(h) + ")");
+}
+
+__global__ void k_fill_win_len(uint32_t* wl, int64_t n_win, int64_t W, int64_t n_tok) {
+  int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (w < n_win) wl[w] = (uint32_t)(n_tok - w * W < W ? n_tok - w * W : W);
+}
+
+__global__ void k_dec_inputs(const uint16_t* __restrict__ dec_tok, int64_t n, int64_t W, int64_t pos,
+                             uint16_t* __restrict__ tok_in) {
+  int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (w < n) tok_in[w] = pos == 0 ? (uint16_t)kTokBos : dec_tok[w * W + pos - 1];
+}
+
+}  // namespace lmgc
+
+using namespace lmgc;
+
+// ------------------------------------------------------------------------------------------
+extern "C" {
+
+lmgc_status lmgc_last_error(const lmgc_ctx* ctx, char* buf, size_t len) {
+  if (!buf || !len) return LMGC_ERR_INVALID;
+  const std::string& m = ctx ? ctx->err : g_thread_err;
+  size_t n = std::min(len - 1, m.size());
+  memcpy(buf, m.data(), n);
+  buf[n] = 0;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_tokens_per_value(const lmgc_ctx* ctx, size_t* tpv) {
+  if (!ctx || !tpv) return LMGC_ERR_INVALID;
+  *tpv = (size_t)ctx->tpv;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_destroy(lmgc_ctx* ctx) {
+  if (!ctx) return LMGC_OK;
+  cudaDeviceSynchronize();
+  void* ptrs[] = {ctx->weights_blob, ctx->rope_cs, ctx->exp2_tab, ctx->ws.x, ctx->ws.n, ctx->ws.qkv, ctx->ws.att,
+                  ctx->ws.act, ctx->ws.gu, ctx->ws.tok_in, ctx->logits, ctx->d_err, ctx->tok, ctx->pair_start,
+                  ctx->win_len, ctx->host_in, ctx->host_out, ctx->kv_cache};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  for (auto& e : ctx->ev)
+    if (e) cudaEventDestroy(e);
+  for (auto e : ctx->batch_ev) cudaEventDestroy(e);
+  for (auto& r : ctx->prof.pending) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : ctx->prof.pool) cudaEventDestroy(e);
+  delete ctx;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
+  if (!cfg || !out) return fail(nullptr, LMGC_ERR_INVALID, "null argument");
+  *out = nullptr;
+  const lmgc_config& c = *cfg;
+  if (c.n_layers < 0 || c.d_model <= 0 || c.n_heads <= 0 || c.n_kv_heads <= 0 || c.d_ffn <= 0 ||
+      c.d_model % c.n_heads || c.n_heads % c.n_kv_heads || c.vocab < 20 || c.window < 1 || c.batch_windows < 1)
+    return fail(nullptr, LMGC_ERR_INVALID, "bad model shape");
+  const int hd = c.d_model / c.n_heads;
+  if (hd != 32 && hd != 64 && hd != 128) return fail(nullptr, LMGC_ERR_INVALID, "head dim must be 32, 64 or 128");
+  if (c.d_model % 8 || c.d_ffn % 8) return fail(nullptr, LMGC_ERR_INVALID, "d_model and d_ffn must be multiples of 8");
+  if (c.cdf_bits < 1 || c.cdf_bits > 30 || (int64_t)c.vocab >= (1ll << c.cdf_bits))
+    return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must satisfy vocab < 2^cdf_bits <= 2^30");
+  if (c.dtype != LMGC_F32 && c.dtype != LMGC_BF16) return fail(nullptr, LMGC_ERR_INVALID, "bad dtype");
+  int tpv = tokens_per_value(c.input_kind, c.sep_mode);
+  if (tpv < 0) return fail(nullptr, LMGC_ERR_INVALID, "bad input kind or separator mode");
+
+  lmgc_ctx* ctx = new lmgc_ctx();
+  ctx->cfg = c;
+  cudaGetDevice(&ctx->device);
+  ctx->hd = hd;
+  ctx->qkv_dim = (c.n_heads + 2 * c.n_kv_heads) * hd;
+  ctx->tpv = tpv;
+  ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
+  const char* tc_env = getenv("LMGC_DISABLE_TC");
+  ctx->use_tc = !(tc_env && tc_env[0] == '1');
+  const int64_t d = c.d_model, F = c.d_ffn, V = c.vocab, qd = (int64_t)c.n_heads * hd;
+  const size_t e = ctx->elt;
+  // weights: one blob, every tensor 256-byte aligned
+  auto al = [](size_t x) { return (x + 255) / 256 * 256; };
+  size_t off = 0;
+  std::vector<size_t> offs;
+  offs.push_back(off); off += al(V * d * e);                        // embed
+  for (int l = 0; l < c.n_layers; l++) {
+    offs.push_back(off); off += al((size_t)ctx->qkv_dim * d * e);   // wqkv
+    offs.push_back(off); off += al((size_t)d * qd * e);             // wo
+    offs.push_back(off); off += al((size_t)2 * F * d * e);          // wgu
+    offs.push_back(off); off += al((size_t)d * F * e);              // wdown
+  }
+  offs.push_back(off); off += al(V * d * e);                        // head
+  cudaStream_t s = 0;
+  cudaError_t err = cudaMalloc(&ctx->weights_blob, off);
+  if (err != cudaSuccess) {
+    lmgc_destroy(ctx);
+    return cuda_fail(nullptr, err, "weights");
+  }
+  char* base = (char*)ctx->weights_blob;
+  int k = 0;
+  ctx->w_embed = base + offs[k++];
+  ctx->layers.resize(c.n_layers);
+  for (int l = 0; l < c.n_layers; l++) {
+    ctx->layers[l].wqkv = base + offs[k++];
+    ctx->layers[l].wo = base + offs[k++];
+    ctx->layers[l].wgu = base + offs[k++];
+    ctx->layers[l].wdown = base + offs[k++];
+  }
+  ctx->w_head = base + offs[k++];
+  // tensor ids: 0 embed, 1+7l+{q,k,v,o,gate,up,down}, 1+7L head; index = row-major canonical
+  const uint64_t seed = c.weight_seed;
+  const int dt = c.dtype;
+  launch_init_weights(ctx->w_embed, dt, seed, 0, V, d, d, 0, c.init_std, s);
+  for (int l = 0; l < c.n_layers; l++) {
+    const uint32_t t = 1 + 7 * l;
+    const Layer& L = ctx->layers[l];
+    launch_init_weights(L.wqkv, dt, seed, t + 0, qd, d, d, 0, c.init_std, s);
+    launch_init_weights(L.wqkv, dt, seed, t + 1, (int64_t)c.n_kv_heads * hd, d, d, qd, c.init_std, s);
+    launch_init_weights(L.wqkv, dt, seed, t + 2, (int64_t)c.n_kv_heads * hd, d, d,
+                        qd + (int64_t)c.n_kv_heads * hd, c.init_std, s);
+    launch_init_weights(L.wo, dt, seed, t + 3, d, qd, qd, 0, c.init_std, s);
+    launch_init_weights(L.wgu, dt, seed, t + 4, F, d, d, 0, c.init_std, s);
+    launch_init_weights(L.wgu, dt, seed, t + 5, F, d, d, F, c.init_std, s);
+    launch_init_weights(L.wdown, dt, seed, t + 6, d, F, F, 0, c.init_std, s);
+  }
+  launch_init_weights(ctx->w_head, dt, seed, 1 + 7 * c.n_layers, V, d, d, 0, c.init_std, s);
+  // RoPE table: angle pos * theta^(-2i/hd) in binary64, stored as fp32 (cos, sin)
+  {
+    std::vector<float2> cs((size_t)c.window * (hd / 2));
+    for (int64_t p = 0; p < c.window; p++)
+      for (int i = 0; i < hd / 2; i++) {
+        double ang = (double)p * pow((double)c.rope_theta, -2.0 * i / hd);
+        cs[p * (hd / 2) + i] = make_float2((float)cos(ang), (float)sin(ang));
+      }
+    err = cudaMalloc(&ctx->rope_cs, cs.size() * sizeof(float2));
+    if (err == cudaSuccess) err = cudaMemcpy(ctx->rope_cs, cs.data(), cs.size() * sizeof(float2), cudaMemcpyHostToDevice);
+  }
+  if (err == cudaSuccess) err = cudaMalloc(&ctx->exp2_tab, 512 * sizeof(uint32_t));
+  if (err == cudaSuccess) upload_exp2_tables(ctx->exp2_tab, s);
+  if (err == cudaSuccess) err = cudaMalloc(&ctx->d_err, 16);
+  if (err == cudaSuccess) err = cudaMemset(ctx->d_err, 0, 16);
+  // workspace for batch_windows windows
+  Workspace& ws = ctx->ws;
+  ws.rows = (int64_t)c.batch_windows * c.window;
+  const size_t R = (size_t)ws.rows;
+  if (err == cudaSuccess) err = dmalloc(&ws.x, R * d * 4);
+  if (err == cudaSuccess) err = dmalloc(&ws.n, R * d * e);
+  if (err == cudaSuccess) err = dmalloc(&ws.qkv, R * ctx->qkv_dim * e);
+  if (err == cudaSuccess) err = dmalloc(&ws.att, R * qd * e);
+  if (err == cudaSuccess) err = dmalloc(&ws.act, R * F * e);
+  if (err == cudaSuccess) err = dmalloc(&ws.gu, R * 2 * F * e);
+  if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
+  if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
+  for (int i = 0; i < 6 && err == cudaSuccess; i++) err = cudaEventCreate(&ctx->ev[i]);
+  if (err == cudaSuccess) err = cudaDeviceSynchronize();
+  if (err == cudaSuccess) err = cudaGetLastError();
+  if (err != cudaSuccess) {
+    lmgc_destroy(ctx);
+    return cuda_fail(nullptr, err, "lmgc_create");
+  }
+  for (int i = 0; i < kNumClasses; i++) ctx->prof.stats[i] = KernelStat{kClassNames[i], 0, 0.f, 0.0};
+  *out = ctx;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_serialize(lmgc_ctx* ctx, const void* d_in, size_t n, uint16_t* d_tok, size_t cap_tok,
+                           size_t* n_tok, lmgc_stream stream) {
+  if (!ctx || !n_tok || (n && (!d_in || !d_tok))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  size_t need = n * (size_t)ctx->tpv;
+  *n_tok = need;
+  if (cap_tok < need) return fail(ctx, LMGC_ERR_NO_SPACE, "token buffer too small");
+  cudaStream_t s = (cudaStream_t)stream;
+  launch_serialize(ctx->cfg.input_kind, ctx->cfg.sep_mode, d_in, (int64_t)n, d_tok, s);
+  LMGC_CUDA(ctx, cudaGetLastError());
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_deserialize(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, void* d_out, size_t cap_values,
+                             size_t* n_values, lmgc_stream stream) {
+  if (!ctx || !n_values || (n_tok && (!d_tok || !d_out))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  if (n_tok % (size_t)ctx->tpv) return fail(ctx, LMGC_ERR_CORRUPT, "token count not a multiple of tokens/value");
+  size_t nv = n_tok / (size_t)ctx->tpv;
+  *n_values = nv;
+  if (cap_values < nv) return fail(ctx, LMGC_ERR_NO_SPACE, "value buffer too small");
+  cudaStream_t s = (cudaStream_t)stream;
+  launch_deserialize(ctx->cfg.input_kind, ctx->cfg.sep_mode, d_tok, (int64_t)nv, d_out, ctx->d_err, s);
+  LMGC_CUDA(ctx, cudaGetLastError());
+  return check_err_word(ctx, s, "deserialize");
+}
+
+lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, size_t first_win, size_t n_win,
+                          float* d_logits, lmgc_stream stream) {
+  if (!ctx || !d_tok || !d_logits) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  const int64_t W = ctx->cfg.window, V = ctx->cfg.vocab;
+  const int64_t total_win = ((int64_t)n_tok + W - 1) / W;
+  if ((int64_t)(first_win + n_win) > total_win) return fail(ctx, LMGC_ERR_INVALID, "window range beyond the stream");
+  cudaStream_t s = (cudaStream_t)stream;
+  for (int64_t w0 = 0; w0 < (int64_t)n_win; w0 += ctx->cfg.batch_windows) {
+    int64_t nb = std::min<int64_t>(ctx->cfg.batch_windows, (int64_t)n_win - w0);
+    forward_windows(ctx, d_tok, (int64_t)n_tok, (int64_t)first_win + w0, nb, s);
+    LMGC_CUDA(ctx, cudaMemcpyAsync(d_logits + w0 * W * V, ctx->logits, (size_t)(nb * W * V) * 4,
+                                   cudaMemcpyDeviceToDevice, s));
+  }
+  LMGC_CUDA(ctx, cudaGetLastError());
+  if (ctx->prof.enabled) {
+    cudaStreamSynchronize(s);
+    prof_collect(ctx);
+  }
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_quantize_cdf(lmgc_ctx* ctx, const float* d_logits, size_t rows, uint32_t* d_cdf,
+                              lmgc_stream stream) {
+  if (!ctx || (rows && (!d_logits || !d_cdf))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  launch_quantize_cdf(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_cdf,
+                      (cudaStream_t)stream);
+  LMGC_CUDA(ctx, cudaGetLastError());
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, const uint16_t* d_sym,
+                           uint32_t* d_start, uint32_t* d_freq, lmgc_stream stream) {
+  if (!ctx || (rows && (!d_logits || !d_sym || !d_start || !d_freq)))
+    return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  launch_cdf_pairs(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0, 0,
+                   d_start, d_freq, 0, (cudaStream_t)stream);
+  LMGC_CUDA(ctx, cudaGetLastError());
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                              size_t win_tokens, const uint32_t* d_win_len, size_t stride_win, size_t stride_pos,
+                              uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
+                              lmgc_stream stream) {
+  if (!out_bytes || (n_win && (!d_start || !d_freq || !d_bitlen)))
+    return fail(nullptr, LMGC_ERR_INVALID, "null argument");
+  if (cdf_bits < 1 || cdf_bits > 30) return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must be in 1..30");
+  *out_bytes = 0;
+  if (n_win == 0) return LMGC_OK;
+  cudaStream_t s = (cudaStream_t)stream;
+  const size_t slot = slot_bytes(win_tokens, cdf_bits);
+  uint8_t* slots = nullptr;
+  uint64_t* offs = nullptr;
+  uint32_t* derr = nullptr;
+  cudaError_t e = cudaMallocAsync((void**)&slots, slot * n_win, s);
+  if (e == cudaSuccess) e = cudaMallocAsync((void**)&offs, (n_win + 1) * 8 + 16, s);
+  if (e == cudaSuccess) e = cudaMallocAsync((void**)&derr, 16, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(derr, 0, 4, s);
+  lmgc_status st = LMGC_OK;
+  if (e != cudaSuccess) {
+    st = cuda_fail(nullptr, e, "range_encode scratch");
+  } else {
+    launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
+                        (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
+    launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
+    uint64_t total = 0;
+    uint32_t herr = 0;
+    cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
+    cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) st = cuda_fail(nullptr, e, "range_encode");
+    else if (herr) st = fail(nullptr, LMGC_ERR_INVALID, "range_encode: invalid (start, freq) or window length");
+    else {
+      *out_bytes = total;
+      if (cap < total) st = fail(nullptr, LMGC_ERR_NO_SPACE, "range_encode: output too small");
+      else {
+        launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) st = cuda_fail(nullptr, e, "range_encode pack");
+      }
+    }
+  }
+  if (slots) cudaFreeAsync(slots, s);
+  if (offs) cudaFreeAsync(offs, s);
+  if (derr) cudaFreeAsync(derr, s);
+  cudaStreamSynchronize(s);
+  return st;
+}
+
+lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes) {
+  if (!ctx || !bytes) return LMGC_ERR_INVALID;
+  const size_t n_tok = n * (size_t)ctx->tpv, W = (size_t)ctx->cfg.window;
+  const size_t n_win = (n_tok + W - 1) / W;
+  *bytes = 64 + 4 * n_win + (n_tok * (size_t)ctx->cfg.cdf_bits + 2 * n_win + 7) / 8 + n_win;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_out, size_t cap, size_t* out_bytes,
+                        lmgc_stream stream) {
+  if (!ctx || !d_in || !out_bytes) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  if (n == 0) return fail(ctx, LMGC_ERR_INVALID, "empty input");
+  const lmgc_config& c = ctx->cfg;
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t W = c.window, P = c.cdf_bits;
+  const int64_t n_tok = (int64_t)n * ctx->tpv;
+  const int64_t n_win = (n_tok + W - 1) / W;
+  const size_t slot = slot_bytes((size_t)W, (int)P);
+  // staging (grown on demand; reused across calls)
+  LMGC_CUDA(ctx, ensure(&ctx->tok, &ctx->tok_cap, (size_t)n_tok * 2 + 16));
+  const size_t pair_need = (size_t)(W * n_win) * 4;
+  LMGC_CUDA(ctx, ensure(&ctx->pair_start, &ctx->pair_cap, 2 * pair_need));
+  ctx->pair_freq = ctx->pair_start + (size_t)(W * n_win);
+  // win_len [n_win] u32 | bitlen [n_win] u32 | offsets [n_win+1] u64 | slots
+  const size_t wl_off = 0, bl_off = ((size_t)n_win * 4 + 255) / 256 * 256,
+               of_off = bl_off + ((size_t)n_win * 4 + 255) / 256 * 256,
+               sl_off = of_off + (((size_t)n_win + 1) * 8 + 255) / 256 * 256;
+  LMGC_CUDA(ctx, ensure(&ctx->win_len, &ctx->win_cap, sl_off + slot * (size_t)n_win));
+  uint32_t* d_wl = (uint32_t*)((char*)ctx->win_len + wl_off);
+  uint32_t* d_bl = (uint32_t*)((char*)ctx->win_len + bl_off);
+  uint64_t* d_off = (uint64_t*)((char*)ctx->win_len + of_off);
+  uint8_t* d_slots = (uint8_t*)ctx->win_len + sl_off;
+
+  LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[0], s));
+  {
+    ProfScope ps(ctx, kSer, (double)n * (ctx->cfg.input_kind == LMGC_IN_F32 ? 4 : 1) + (double)n_tok * 2, s);
+    launch_serialize(c.input_kind, c.sep_mode, d_in, (int64_t)n, ctx->tok, s);
+  }
+  LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[1], s));
+  const int64_t n_batches = (n_win + c.batch_windows - 1) / c.batch_windows;
+  while ((int64_t)ctx->batch_ev.size() < 2 * n_batches + 1) {
+    cudaEvent_t e;
+    LMGC_CUDA(ctx, cudaEventCreate(&e));
+    ctx->batch_ev.push_back(e);
+  }
+  cudaEventRecord(ctx->batch_ev[0], s);
+  for (int64_t b = 0; b < n_batches; b++) {
+    const int64_t w0 = b * c.batch_windows;
+    const int64_t nb = std::min<int64_t>(c.batch_windows, n_win - w0);
+    forward_windows(ctx, ctx->tok, n_tok, w0, nb, s);
+    cudaEventRecord(ctx->batch_ev[2 * b + 1], s);
+    {
+      const int64_t rows = nb * W;
+      ProfScope ps(ctx, kCdf, (double)rows * ((double)c.vocab * 4 + 2 + 8), s);
+      launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
+                       ctx->pair_start, ctx->pair_freq, 1, s);
+    }
+    cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
+  }
+  LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[2], s));
+  k_fill_win_len<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(d_wl, n_win, W, n_tok);
+  {
+    ProfScope ps(ctx, kCoder, (double)n_tok * 8, s);
+    launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 1, n_win, d_slots, slot, d_bl,
+                        ctx->d_err, s);
+  }
+  LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[3], s));
+  launch_pack_codes(d_slots, slot, d_bl, n_win, d_off, nullptr, s);
+  uint64_t payload = 0;
+  LMGC_CUDA(ctx, cudaMemcpyAsync(&payload, d_off + n_win, 8, cudaMemcpyDeviceToHost, s));
+  lmgc_status st = check_err_word(ctx, s, "encode");
+  if (st != LMGC_OK) return st;
+  const size_t total = 64 + 4 * (size_t)n_win + payload;
+  *out_bytes = total;
+  if (cap < total || !d_out) return fail(ctx, LMGC_ERR_NO_SPACE, "container buffer too small");
+  // header
+  uint8_t h[64];
+  memset(h, 0, 64);
+  uint32_t u32;
+  uint64_t u64;
+  memcpy(h, "LMGC", 4);
+  u32 = 1; memcpy(h + 4, &u32, 4);
+  u64 = n; memcpy(h + 8, &u64, 8);
+  u64 = (uint64_t)n_tok; memcpy(h + 16, &u64, 8);
+  u32 = (uint32_t)W; memcpy(h + 24, &u32, 4);
+  u32 = (uint32_t)P; memcpy(h + 28, &u32, 4);
+  u32 = (uint32_t)c.input_kind; memcpy(h + 32, &u32, 4);
+  u32 = (uint32_t)c.sep_mode; memcpy(h + 36, &u32, 4);
+  u32 = (uint32_t)c.vocab; memcpy(h + 40, &u32, 4);
+  u32 = (uint32_t)n_win; memcpy(h + 44, &u32, 4);
+  u64 = c.weight_seed; memcpy(h + 48, &u64, 8);
+  u32 = model_crc(c); memcpy(h + 56, &u32, 4);
+  u32 = crc32(h, 60); memcpy(h + 60, &u32, 4);
+  LMGC_CUDA(ctx, cudaMemcpyAsync(d_out, h, 64, cudaMemcpyHostToDevice, s));
+  LMGC_CUDA(ctx, cudaMemcpyAsync(d_out + 64, d_bl, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
+  launch_pack_codes(d_slots, slot, d_bl, n_win, d_off, d_out + 64 + 4 * (size_t)n_win, s);
+  LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[5], s));
+  LMGC_CUDA(ctx, cudaStreamSynchronize(s));
+  LMGC_CUDA(ctx, cudaGetLastError());
+  float x = 0.f, ms_lm = 0.f, ms_cdf = 0.f;
+  for (int64_t b = 0; b < n_batches; b++) {
+    cudaEventElapsedTime(&x, ctx->batch_ev[2 * b], ctx->batch_ev[2 * b + 1]);
+    ms_lm += x;
+    cudaEventElapsedTime(&x, ctx->batch_ev[2 * b + 1], ctx->batch_ev[2 * b + 2]);
+    ms_cdf += x;
+  }
+  cudaEventElapsedTime(&x, ctx->ev[0], ctx->ev[1]);
+  ctx->stage_ms[0] = x;
+  ctx->stage_ms[1] = ms_lm;
+  ctx->stage_ms[2] = ms_cdf;
+  cudaEventElapsedTime(&x, ctx->ev[2], ctx->ev[3]);
+  ctx->stage_ms[3] = x;
+  cudaEventElapsedTime(&x, ctx->ev[3], ctx->ev[5]);
+  ctx->stage_ms[4] = x;
+  if (ctx->prof.enabled) prof_collect(ctx);
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t* h_out, size_t cap,
+                             size_t* out_bytes, lmgc_stream stream) {
+  if (!ctx || !h_in || !out_bytes) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  cudaStream_t s = (cudaStream_t)stream;
+  const size_t in_bytes = n * (ctx->cfg.input_kind == LMGC_IN_F32 ? 4 : 1);
+  size_t bound = 0;
+  lmgc_encode_bound(ctx, n, &bound);
+  LMGC_CUDA(ctx, ensure(&ctx->host_in, &ctx->host_in_cap, in_bytes));
+  LMGC_CUDA(ctx, ensure(&ctx->host_out, &ctx->host_out_cap, bound));
+  LMGC_CUDA(ctx, cudaMemcpyAsync(ctx->host_in, h_in, in_bytes, cudaMemcpyHostToDevice, s));
+  lmgc_status st = lmgc_encode(ctx, ctx->host_in, n, ctx->host_out, ctx->host_out_cap, out_bytes, stream);
+  if (st != LMGC_OK) return st;
+  if (cap < *out_bytes || !h_out) return fail(ctx, LMGC_ERR_NO_SPACE, "host container buffer too small");
+  LMGC_CUDA(ctx, cudaMemcpyAsync(h_out, ctx->host_out, *out_bytes, cudaMemcpyDeviceToHost, s));
+  LMGC_CUDA(ctx, cudaStreamSynchronize(s));
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, const uint32_t* h_win_ids,
+                        size_t n_ids, uint16_t* d_tok, size_t cap_tok, lmgc_stream stream) {
+  if (!ctx || !d_in || (n_ids && (!h_win_ids || !d_tok))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  const lmgc_config& c = ctx->cfg;
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t W = c.window;
+  if (in_bytes < 64) return fail(ctx, LMGC_ERR_CORRUPT, "container shorter than its header");
+  uint8_t h[64];
+  LMGC_CUDA(ctx, cudaMemcpyAsync(h, d_in, 64, cudaMemcpyDeviceToHost, s));
+  LMGC_CUDA(ctx, cudaStreamSynchronize(s));
+  uint32_t hcrc, mcrc, ver, hW, hP, kind, sep, vocab, n_win;
+  uint64_t n_tok;
+  memcpy(&hcrc, h + 60, 4);
+  if (memcmp(h, "LMGC", 4) || hcrc != crc32(h, 60)) return fail(ctx, LMGC_ERR_CORRUPT, "bad container header");
+  memcpy(&ver, h + 4, 4);
+  memcpy(&n_tok, h + 16, 8);
+  memcpy(&hW, h + 24, 4);
+  memcpy(&hP, h + 28, 4);
+  memcpy(&kind, h + 32, 4);
+  memcpy(&sep, h + 36, 4);
+  memcpy(&vocab, h + 40, 4);
+  memcpy(&n_win, h + 44, 4);
+  memcpy(&mcrc, h + 56, 4);
+  uint64_t seed;
+  memcpy(&seed, h + 48, 8);
+  if (ver != 1 || hW != (uint32_t)W || hP != (uint32_t)c.cdf_bits || kind != (uint32_t)c.input_kind ||
+      sep != (uint32_t)c.sep_mode || vocab != (uint32_t)c.vocab || mcrc != model_crc(c) || seed != c.weight_seed)
+    return fail(ctx, LMGC_ERR_CORRUPT, "container does not match this context's model or coder");
+  if ((uint64_t)n_win != (n_tok + W - 1) / W || 64 + 4 * (size_t)n_win > in_bytes)
+    return fail(ctx, LMGC_ERR_CORRUPT, "container window table truncated");
+  if (cap_tok < n_ids * (size_t)W) return fail(ctx, LMGC_ERR_NO_SPACE, "token buffer too small");
+  std::vector<uint32_t> bl(n_win);
+  if (n_win) LMGC_CUDA(ctx, cudaMemcpy(bl.data(), d_in + 64, 4 * (size_t)n_win, cudaMemcpyDeviceToHost));
+  std::vector<uint64_t> off(n_win + 1);
+  off[0] = 64 + 4 * (uint64_t)n_win;
+  for (uint32_t w = 0; w < n_win; w++) off[w + 1] = off[w] + (bl[w] + 7) / 8;
+  if (off[n_win] > in_bytes) return fail(ctx, LMGC_ERR_CORRUPT, "container payload truncated");
+  for (size_t i = 0; i < n_ids; i++)
+    if (h_win_ids[i] >= n_win) return fail(ctx, LMGC_ERR_INVALID, "window id out of range");
+  // decode batch: as many windows as the workspace holds, with the KV cache kept under 16 GiB
+  const size_t kv_per_win = (size_t)std::max(1, c.n_layers) * W * ctx->qkv_dim * ctx->elt;
+  const int64_t nd_max = std::max<int64_t>(1, std::min<int64_t>(c.batch_windows, (int64_t)((16ull << 30) / kv_per_win)));
+  const size_t kv_need = kv_per_win * (size_t)nd_max;
+  LMGC_CUDA(ctx, ensure(&ctx->kv_cache, &ctx->kv_cap, kv_need));
+  // per-chunk device arrays: code offsets, bit lengths, lengths, decoder states
+  void* dev = nullptr;
+  const size_t st_bytes = dec_state_bytes();
+  const size_t arr = (size_t)nd_max * (8 + 4 + 4) + (size_t)nd_max * st_bytes + 256;
+  LMGC_CUDA(ctx, cudaMallocAsync(&dev, arr, s));
+  uint64_t* d_coff = (uint64_t*)dev;
+  uint32_t* d_bl = (uint32_t*)(d_coff + nd_max);
+  uint32_t* d_len = d_bl + nd_max;
+  void* d_state = (void*)(((uintptr_t)(d_len + nd_max) + 63) / 64 * 64);
+  lmgc_status st = LMGC_OK;
+  for (size_t i0 = 0; i0 < n_ids && st == LMGC_OK; i0 += nd_max) {
+    const int64_t nd = std::min<int64_t>(nd_max, (int64_t)(n_ids - i0));
+    std::vector<uint64_t> hoff(nd);
+    std::vector<uint32_t> hbl(nd), hlen(nd);
+    int64_t max_len = 0;
+    for (int64_t j = 0; j < nd; j++) {
+      uint32_t w = h_win_ids[i0 + j];
+      hoff[j] = off[w];
+      hbl[j] = bl[w];
+      hlen[j] = (uint32_t)std::min<uint64_t>((uint64_t)W, n_tok - (uint64_t)w * W);
+      max_len = std::max<int64_t>(max_len, hlen[j]);
+    }
+    cudaMemcpyAsync(d_coff, hoff.data(), 8 * nd, cudaMemcpyHostToDevice, s);
+    cudaMemcpyAsync(d_bl, hbl.data(), 4 * nd, cudaMemcpyHostToDevice, s);
+    cudaMemcpyAsync(d_len, hlen.data(), 4 * nd, cudaMemcpyHostToDevice, s);
+    launch_dec_init(d_in, d_coff, d_bl, nd, d_state, s);
+    uint16_t* out = d_tok + i0 * W;
+    for (int64_t pos = 0; pos < max_len; pos++) {
+      k_dec_inputs<<<(unsigned)((nd + 127) / 128), 128, 0, s>>>(out, nd, W, pos, ctx->ws.tok_in);
+      launch_embed(ctx->ws.tok_in, nd, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
+      forward_layers(ctx, nd, nd, true, pos, s);
+      launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
+                        ctx->d_err, s);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) st = cuda_fail(ctx, e, "decode");
+    else st = check_err_word(ctx, s, "decode");
+  }
+  cudaFreeAsync(dev, s);
+  cudaStreamSynchronize(s);
+  if (ctx->prof.enabled) prof_collect(ctx);
+  return st;
+}
+
+lmgc_status lmgc_stage_times(const lmgc_ctx* ctx, float* ms, size_t n_ms) {
+  if (!ctx || !ms) return LMGC_ERR_INVALID;
+  for (size_t i = 0; i < n_ms && i < 5; i++) ms[i] = ctx->stage_ms[i];
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_profile(lmgc_ctx* ctx, int enable) {
+  if (!ctx) return LMGC_ERR_INVALID;
+  ctx->prof.enabled = enable != 0;
+  for (int i = 0; i < kNumClasses; i++) ctx->prof.stats[i] = KernelStat{kClassNames[i], 0, 0.f, 0.0};
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_kernel_stats(const lmgc_ctx* ctx, int cls, char* name, size_t name_len, int* launches, float* ms,
+                              double* work) {
+  if (!ctx || cls < 0 || cls >= kNumClasses) return LMGC_ERR_INVALID;
+  const KernelStat& st = ctx->prof.stats[cls];
+  if (name && name_len) {
+    size_t n = std::min(name_len - 1, strlen(kClassNames[cls]));
+    memcpy(name, kClassNames[cls], n);
+    name[n] = 0;
+  }
+  if (launches) *launches = st.launches;
+  if (ms) *ms = st.ms;
+  if (work) *work = st.work;
+  return LMGC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,408 @@
+// cdf.cu -- logits -> integer CDF -> (start, freq) of the coded token, plus the decoder's
+// symbol search.
+//
+// The coder of Sec. 2 needs the model's distribution p(t | BOS, t_<) (Eq. 2) as an integer CDF
+// (the paper adapts Torchac, whose CDFs are integers; Sec. 4.1). For a row z[0..V), T = 2^P:
+//   m = max z; y_j = fp32(fp32(z_j - m) * C), C = fp32(2^16 log2 e); a_j = -rint(y_j) (<= 40*2^16)
+//   e_j = ((H[(a>>8)&255] * L[a&255] + 2^30) >> 31) >> (a >> 16),   H[h] = round(2^31 2^(-h/256)),
+//         L[l] = round(2^31 2^(-l/65536))  -- a fixed-point 2^31 * exp(z_j - m)
+//   S = sum e_j; g_j = floor(e_j (T - V) / S); freq_j = 1 + g_j; the remainder (T - V) - sum g_j
+//   goes to the lowest index of the largest e_j; cdf[j] = sum_{i<j} freq_i.
+// Only the fp32 subtract/multiply and rint touch floating point; the rest is integer, so the
+// result is bit-exact on any machine that rounds fp32 to nearest.
+//
+// The encode path never materialises a CDF (V = 32000 would be 128 KB per token): one block per
+// row reduces max, sum e and argmax, then sum_{j<s} g_j and g_s for the row's symbol s.
+// floor(X / S) with X < 2^55 and S < 2^47 uses a reciprocal floor(2^64-1 / S) and one correction.
+#include <math.h>
+
+#include <algorithm>
+
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+
+// Tables H and L, computed in binary64 (each entry is >= 1e-4 away from a rounding tie, which
+// is checked, so binary64 rounding cannot change them).
+void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s) {
+  static uint32_t tab[512];
+  static bool built = false;
+  if (!built) {
+    for (int i = 0; i < 256; i++) {
+      double h = ldexp(exp2(-(double)i / 256.0), 31);
+      double l = ldexp(exp2(-(double)i / 65536.0), 31);
+      double fh = h - floor(h), fl = l - floor(l);
+      if (fabs(fh - 0.5) < 1e-4 || fabs(fl - 0.5) < 1e-4) {
+        // cannot happen for these tables; refuse to guess
+        tab[0] = 0;
+        return;
+      }
+      tab[i] = (uint32_t)llround(h);
+      tab[256 + i] = (uint32_t)llround(l);
+    }
+    built = true;
+  }
+  cudaMemcpyAsync(d_tab, tab, sizeof(tab), cudaMemcpyHostToDevice, s);
+  cudaStreamSynchronize(s);
+}
+
+constexpr int kCdfThreads = 512;
+constexpr int kAMax = 40 * 65536;
+
+__device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t* __restrict__ H,
+                                               const uint32_t* __restrict__ L) {
+  const float C = (float)(65536.0 * 1.4426950408889634073599246810019);
+  float y = __fmul_rn(__fsub_rn(z, m), C);
+  // a = -rint(y) (ties to even), capped at 40 * 2^16; y below the cap is clamped before the
+  // conversion so that huge logit gaps cannot overflow it
+  int a = (y < -(float)kAMax) ? kAMax : -__float2int_rn(y);
+  a = min(max(a, 0), kAMax);
+  uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
+  uint64_t e = (hl + (1ull << 30)) >> 31;
+  return (uint32_t)(e >> (a >> 16));
+}
+
+// floor(X / S) given minv = floor((2^64 - 1) / S), X < 2^56, S > 0
+__device__ __forceinline__ uint64_t div_floor(uint64_t X, uint64_t S, uint64_t minv) {
+  uint64_t q = __umul64hi(X, minv);
+  uint64_t r = X - q * S;
+  if (r >= S) q++;
+  return q;
+}
+
+template <typename V>
+__device__ __forceinline__ V warp_sum(V v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Block-wide reductions (kCdfThreads threads). `red` is shared scratch of >= 32 entries.
+__device__ __forceinline__ float block_max(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  v = lane < (kCdfThreads / 32) ? red[lane] : -INFINITY;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ uint64_t block_sum_u64(uint64_t v, uint64_t* red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  v = lane < (kCdfThreads / 32) ? red[lane] : 0ull;
+  return warp_sum(v);
+}
+
+// (value, index) max with the lowest index among equal values; packed as value << 32 | ~index
+__device__ __forceinline__ uint64_t block_argmax(uint64_t key, uint64_t* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    uint64_t k2 = __shfl_xor_sync(0xffffffffu, key, o);
+    key = k2 > key ? k2 : key;
+  }
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[w] = key;
+  __syncthreads();
+  key = lane < (kCdfThreads / 32) ? red[lane] : 0ull;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    uint64_t k2 = __shfl_xor_sync(0xffffffffu, key, o);
+    key = k2 > key ? k2 : key;
+  }
+  return key;
+}
+
+struct RowStats {
+  float m;
+  uint64_t S, minv, Mq;
+  int amax;
+};
+
+// Passes 1 and 2 over a row: max, sum of e, lowest-index argmax of e.
+__device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V, int P, const uint32_t* H,
+                                              const uint32_t* L, float* redf, uint64_t* redu) {
+  RowStats st;
+  float m = -INFINITY;
+  for (int j = threadIdx.x; j < V; j += kCdfThreads) m = fmaxf(m, __ldg(z + j));
+  m = block_max(m, redf);
+  uint64_t S = 0, best = 0;
+  for (int j = threadIdx.x; j < V; j += kCdfThreads) {
+    uint32_t e = exp2_fixed(__ldg(z + j), m, H, L);
+    S += e;
+    uint64_t key = ((uint64_t)e << 32) | (uint32_t)(~(uint32_t)j);
+    best = key > best ? key : best;
+  }
+  S = block_sum_u64(S, redu);
+  best = block_argmax(best, redu);
+  st.m = m;
+  st.S = S;
+  st.minv = ~0ull / S;
+  st.Mq = (1ull << P) - (uint64_t)V;
+  st.amax = (int)(~(uint32_t)(best & 0xFFFFFFFFu));
+  return st;
+}
+
+// mode 0: row r codes d_sym[r]; pair index r.
+// mode 1: rows are positions of windows first_win + r / W; the coded token is tok[w*W + i];
+//         rows past the stream end are skipped; pair index i * stride_pos + w.
+__global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restrict__ logits, int64_t rows, int V,
+                                                           int P, const uint32_t* __restrict__ tab,
+                                                           const uint16_t* __restrict__ tok, int64_t n_tok, int W,
+                                                           int64_t first_win, int64_t stride_pos,
+                                                           uint32_t* __restrict__ start, uint32_t* __restrict__ freq,
+                                                           int mode) {
+  __shared__ uint32_t H[256], L[256];
+  __shared__ float redf[32];
+  __shared__ uint64_t redu[32];
+  for (int i = threadIdx.x; i < 256; i += kCdfThreads) {
+    H[i] = tab[i];
+    L[i] = tab[256 + i];
+  }
+  __syncthreads();
+  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
+    int sym;
+    int64_t out_idx;
+    if (mode == 0) {
+      sym = tok[r];
+      out_idx = r;
+    } else {
+      int64_t wl = r / W;
+      int i = (int)(r - wl * W);
+      int64_t g = (first_win + wl) * W + i;
+      if (g >= n_tok) continue;  // block-uniform
+      sym = tok[g];
+      out_idx = (int64_t)i * stride_pos + (first_win + wl);
+    }
+    const float* z = logits + r * (int64_t)V;
+    RowStats st = row_stats(z, V, P, H, L, redf, redu);
+    uint64_t gall = 0, gbelow = 0, gsym = 0;
+    for (int j = threadIdx.x; j < V; j += kCdfThreads) {
+      uint64_t e = exp2_fixed(__ldg(z + j), st.m, H, L);
+      uint64_t g = div_floor(e * st.Mq, st.S, st.minv);
+      gall += g;
+      gbelow += j < sym ? g : 0ull;
+      gsym += j == sym ? g : 0ull;
+    }
+    gall = block_sum_u64(gall, redu);
+    gbelow = block_sum_u64(gbelow, redu);
+    gsym = block_sum_u64(gsym, redu);
+    if (threadIdx.x == 0) {
+      uint64_t resid = st.Mq - gall;
+      start[out_idx] = (uint32_t)(sym + gbelow + (st.amax < sym ? resid : 0ull));
+      freq[out_idx] = (uint32_t)(1ull + gsym + (st.amax == sym ? resid : 0ull));
+    }
+  }
+}
+
+void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
+                      int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
+                      uint32_t* freq, int mode, cudaStream_t s) {
+  if (rows <= 0) return;
+  unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
+  k_cdf_pairs<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win, pair_stride_pos,
+                                             start, freq, mode);
+}
+
+// Block inclusive scan of one u64 per thread; returns the inclusive prefix; *total the tile sum.
+__device__ __forceinline__ uint64_t block_scan_u64(uint64_t v, uint64_t* red, uint64_t* total) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint64_t x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    uint64_t y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  __syncthreads();
+  if (lane == 31) red[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    uint64_t y = lane < (kCdfThreads / 32) ? red[lane] : 0ull;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint64_t t = __shfl_up_sync(0xffffffffu, y, o);
+      if (lane >= o) y += t;
+    }
+    if (lane < (kCdfThreads / 32)) red[lane] = y;
+  }
+  __syncthreads();
+  uint64_t before = w > 0 ? red[w - 1] : 0ull;
+  *total = red[kCdfThreads / 32 - 1];
+  return x + before;
+}
+
+// Full CDF rows [rows][V+1] (parity and inspection).
+__global__ void __launch_bounds__(kCdfThreads) k_quantize_cdf(const float* __restrict__ logits, int64_t rows, int V,
+                                                              int P, const uint32_t* __restrict__ tab,
+                                                              uint32_t* __restrict__ cdf) {
+  __shared__ uint32_t H[256], L[256];
+  __shared__ float redf[32];
+  __shared__ uint64_t redu[32];
+  __shared__ uint64_t scan_red[32];
+  for (int i = threadIdx.x; i < 256; i += kCdfThreads) {
+    H[i] = tab[i];
+    L[i] = tab[256 + i];
+  }
+  __syncthreads();
+  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
+    const float* z = logits + r * (int64_t)V;
+    uint32_t* c = cdf + r * (int64_t)(V + 1);
+    RowStats st = row_stats(z, V, P, H, L, redf, redu);
+    uint64_t gall = 0;
+    for (int j = threadIdx.x; j < V; j += kCdfThreads)
+      gall += div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+    gall = block_sum_u64(gall, redu);
+    const uint64_t resid = st.Mq - gall;
+    uint64_t run = 0;
+    if (threadIdx.x == 0) c[0] = 0;
+    for (int j0 = 0; j0 < V; j0 += kCdfThreads) {
+      int j = j0 + threadIdx.x;
+      uint64_t f = 0;
+      if (j < V) {
+        f = 1 + div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+        if (j == st.amax) f += resid;
+      }
+      uint64_t tot;
+      uint64_t inc = block_scan_u64(f, scan_red, &tot);
+      if (j < V) c[j + 1] = (uint32_t)(run + inc);
+      run += tot;
+    }
+  }
+}
+
+void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
+                         cudaStream_t s) {
+  if (rows <= 0) return;
+  unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
+  k_quantize_cdf<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, cdf);
+}
+
+// ------------------------------------------------------------------------------------------
+// Decoder step (Sec. 2: the decoder repeatedly looks up the interval holding the code value).
+// State per window: R, D (62-bit window of the code value minus L), the code's bit position.
+// t = D / (R >> P); the symbol s has cdf[s] <= t < cdf[s+1]; then D -= r cdf[s], R = r freq_s,
+// k = 62 - bitlen(R), R <<= k, D = (D << k) | next k code bits.
+// ------------------------------------------------------------------------------------------
+struct DecState {
+  uint64_t R, D;
+  uint64_t bitpos;
+  uint64_t code_off;
+  uint64_t nbits;
+};
+
+size_t dec_state_bytes() { return sizeof(DecState); }
+
+__device__ __forceinline__ uint32_t code_bit(const uint8_t* code, uint64_t nbits, uint64_t pos) {
+  return pos < nbits ? (code[pos >> 3] >> (7 - (pos & 7))) & 1u : 0u;
+}
+
+__global__ void k_dec_init(const uint8_t* __restrict__ codes, const uint64_t* __restrict__ code_off,
+                           const uint32_t* __restrict__ bitlen, int64_t n, DecState* __restrict__ st) {
+  int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (w >= n) return;
+  DecState s;
+  s.R = 1ull << 62;
+  s.code_off = code_off[w];
+  s.nbits = bitlen[w];
+  s.D = 0;
+  const uint8_t* code = codes + s.code_off;
+  for (int i = 0; i < 62; i++) s.D = (s.D << 1) | code_bit(code, s.nbits, i);
+  s.bitpos = 62;
+  st[w] = s;
+}
+
+void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n, void* state,
+                     cudaStream_t s) {
+  if (n <= 0) return;
+  k_dec_init<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(codes, code_off, bitlen, n, (DecState*)state);
+}
+
+// One block per decoding window: quantise its logits row, find the symbol for the current code
+// target, update the state. Windows whose length is <= pos are left unchanged.
+__global__ void __launch_bounds__(kCdfThreads) k_dec_search(const float* __restrict__ logits, int64_t n, int V, int P,
+                                                            const uint32_t* __restrict__ tab,
+                                                            DecState* __restrict__ states,
+                                                            const uint8_t* __restrict__ codes,
+                                                            uint16_t* __restrict__ sym_out, int64_t sym_stride,
+                                                            int64_t pos, const uint32_t* __restrict__ win_len,
+                                                            uint32_t* err) {
+  __shared__ uint32_t H[256], L[256];
+  __shared__ float redf[32];
+  __shared__ uint64_t redu[32];
+  __shared__ uint64_t scan_red[32];
+  __shared__ int found_s;
+  __shared__ uint64_t found_lo, found_f;
+  for (int i = threadIdx.x; i < 256; i += kCdfThreads) {
+    H[i] = tab[i];
+    L[i] = tab[256 + i];
+  }
+  __syncthreads();
+  const int64_t w = blockIdx.x;
+  if (w >= n || (int64_t)win_len[w] <= pos) return;
+  DecState s = states[w];
+  const uint64_t r = s.R >> P;
+  const uint64_t t = s.D / r;
+  const float* z = logits + w * (int64_t)V;
+  RowStats st = row_stats(z, V, P, H, L, redf, redu);
+  uint64_t gall = 0;
+  for (int j = threadIdx.x; j < V; j += kCdfThreads)
+    gall += div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+  gall = block_sum_u64(gall, redu);
+  const uint64_t resid = st.Mq - gall;
+  if (threadIdx.x == 0) found_s = -1;
+  uint64_t run = 0;
+  for (int j0 = 0; j0 < V; j0 += kCdfThreads) {
+    int j = j0 + threadIdx.x;
+    uint64_t f = 0;
+    if (j < V) {
+      f = 1 + div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+      if (j == st.amax) f += resid;
+    }
+    uint64_t tot;
+    uint64_t inc = block_scan_u64(f, scan_red, &tot);
+    uint64_t lo = run + inc - f;
+    if (j < V && lo <= t && t < run + inc) {
+      found_s = j;
+      found_lo = lo;
+      found_f = f;
+    }
+    run += tot;
+  }
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+  int sym = found_s;
+  if (t >= (1ull << P) || sym < 0) {
+    atomicOr(err, kErrCorrupt);
+    sym = 0;
+    found_lo = 0;
+    found_f = 1;
+  }
+  s.D -= r * found_lo;
+  s.R = r * found_f;
+  int k = __clzll((long long)s.R) - 2;
+  if (k < 0) k = 0;
+  const uint8_t* code = codes + s.code_off;
+  for (int i = 0; i < k; i++) s.D = (s.D << 1) | code_bit(code, s.nbits, s.bitpos + i);
+  s.bitpos += k;
+  s.R <<= k;
+  states[w] = s;
+  sym_out[w * sym_stride + pos] = (uint16_t)sym;
+}
+
+void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
+                        const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
+                        const uint32_t* win_len, uint32_t* err, cudaStream_t s) {
+  if (n <= 0) return;
+  k_dec_search<<<(unsigned)n, kCdfThreads, 0, s>>>(logits, n, V, P, tab, (DecState*)dec_state, codes, sym_out,
+                                                   sym_stride, pos, win_len, err);
+}
+
+}  // namespace lmgc

@@ -1,0 +1,196 @@
+// coder.cu -- the arithmetic coder (Sec. 2 "Arithmetic coding") in exact integer form, one
+// independent stream per window (Sec. 3 "Compression": each window is coded from its own BOS).
+//
+// Per stream: R = 2^62, L = 0, B = 0; per token (s = start, f = freq, T = 2^P):
+//   r = R >> P;  L += r*s;  R = r*f;  k = max(0, 62 - bitlen(R));  R <<= k;  L <<= k;  B += k
+// and the code is the top B + 2 bits of v = ceil(L / 2^60) * 2^60 (v lies in [L, L + R) because
+// R >= 2^61), most significant bit first.
+//
+// The range R depends only on the freq sequence; L is the only unbounded quantity. A thread keeps
+// the low 62 bits of L in a register; the bits shifted above them are emitted into a 64-bit
+// accumulator and leave in 32-bit words to the stream's own scratch slot. A carry out of the
+// low 62 bits increments the emitted bits: in the accumulator, or -- when the accumulator was all
+// ones -- in the already written words of this stream's slot (never beyond word 0: L + R stays
+// below 2^(B+62)). The carry walk is bounded by the slot length.
+//
+// Layout: one stream per thread, 32 windows per warp. Pairs are read at
+// start[w*stride_win + i*stride_pos]; with the encode path's position-major layout
+// (stride_win = 1) a warp's 32 loads of token i are one 128-byte transaction.
+#include <algorithm>
+
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+
+size_t slot_bytes(size_t win_tokens, int P) {
+  size_t bits = win_tokens * (size_t)P + 2;
+  size_t words = (bits + 31) / 32 + 1;
+  return ((words * 4 + 15) / 16) * 16;
+}
+
+__device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
+
+struct Emitter {
+  uint32_t* slot;   // stream words (stored big-endian so the bytes are in stream order)
+  uint32_t wpos;    // words written
+  uint32_t max_words;
+  uint64_t acc;     // pending emitted bits, right-aligned
+  int nacc;         // number of pending bits (< 32 after each flush)
+  bool overflow;
+
+  __device__ __forceinline__ void carry() {
+    acc += 1;
+    if ((acc >> nacc) != 0) {  // pending bits were all ones: carry into written words
+      acc = 0;
+      int64_t i = (int64_t)wpos - 1;
+      for (; i >= 0; --i) {
+        uint32_t v = bswap32(slot[i]) + 1u;
+        slot[i] = bswap32(v);
+        if (v != 0u) break;
+      }
+      if (i < 0) overflow = true;  // impossible for valid input; reported, not propagated
+    }
+  }
+  __device__ __forceinline__ void put(uint64_t bits, int k) {  // append k (<= 32) bits
+    acc = (acc << k) | bits;
+    nacc += k;
+    if (nacc >= 32) {
+      uint32_t w = (uint32_t)(acc >> (nacc - 32));
+      if (wpos < max_words) slot[wpos] = bswap32(w);
+      else overflow = true;
+      wpos++;
+      nacc -= 32;
+      acc &= (nacc > 0) ? ((1ull << nacc) - 1ull) : 0ull;
+    }
+  }
+};
+
+__global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict__ start,
+                                                      const uint32_t* __restrict__ freq, int P, int64_t n_win,
+                                                      int64_t win_tokens, const uint32_t* __restrict__ win_len,
+                                                      int64_t stride_win, int64_t stride_pos, uint8_t* __restrict__ slots,
+                                                      size_t slot_sz, uint32_t* __restrict__ bitlen, uint32_t* err) {
+  const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (w >= n_win) return;
+  const int64_t n = win_len ? (int64_t)win_len[w] : win_tokens;
+  const uint64_t mask62 = (1ull << 62) - 1ull;
+  const uint64_t T = 1ull << P;
+  Emitter em;
+  em.slot = reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz);
+  em.wpos = 0;
+  em.max_words = (uint32_t)(slot_sz / 4);
+  em.acc = 0;
+  em.nacc = 0;
+  em.overflow = false;
+  uint64_t R = 1ull << 62, L = 0, B = 0;
+  bool bad = n > win_tokens;
+  const uint32_t* ps = start + w * stride_win;
+  const uint32_t* pf = freq + w * stride_win;
+  for (int64_t i = 0; i < n && !bad; i++) {
+    const uint64_t s = __ldcs(ps + i * stride_pos);
+    const uint64_t f = __ldcs(pf + i * stride_pos);
+    if (f == 0 || s + f > T) {
+      bad = true;
+      break;
+    }
+    const uint64_t r = R >> P;
+    L += r * s;  // < 2^63
+    if (L >> 62) {
+      L &= mask62;
+      em.carry();
+    }
+    R = r * f;
+    const int k = __clzll((long long)R) - 2;  // 62 - bitlen(R) >= 0 since R < 2^62
+    if (k > 0) {
+      em.put(L >> (62 - k), k);
+      L = (L << k) & mask62;
+      R <<= k;
+      B += (uint64_t)k;
+    }
+  }
+  // termination: v = ceil(L / 2^60) * 2^60; emit its top 2 bits of the low 62
+  L += (1ull << 60) - 1ull;
+  if (L >> 62) {
+    L &= mask62;
+    em.carry();
+  }
+  em.put(L >> 60, 2);
+  if (em.nacc > 0) {
+    uint32_t wv = (uint32_t)(em.acc << (32 - em.nacc));
+    if (em.wpos < em.max_words) em.slot[em.wpos] = bswap32(wv);
+    else em.overflow = true;
+  }
+  bitlen[w] = (uint32_t)(B + 2);
+  if (bad || em.overflow) atomicOr(err, kErrCorrupt);
+}
+
+void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
+                         const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
+                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
+  if (n_win <= 0) return;
+  k_range_encode<<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
+                                                                  stride_win, stride_pos, slots, slot_sz, bitlen, err);
+}
+
+// ------------------------------------------------------------------------------------------
+// Container payload: exclusive scan of the code byte lengths (one block), then each window's
+// ceil(bitlen/8) bytes copied from its slot to its offset.
+// ------------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(1024) k_scan_lengths(const uint32_t* __restrict__ bitlen, int64_t n,
+                                                       uint64_t* __restrict__ off) {
+  __shared__ uint64_t wsum[32];
+  __shared__ uint64_t carry;
+  const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
+  if (t == 0) carry = 0;
+  __syncthreads();
+  for (int64_t base = 0; base < n; base += 1024) {
+    int64_t i = base + t;
+    uint64_t v = i < n ? (uint64_t)((bitlen[i] + 7u) / 8u) : 0ull;
+    uint64_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      uint64_t y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    if (lane == 31) wsum[wid] = x;
+    __syncthreads();
+    if (wid == 0) {
+      uint64_t y = wsum[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        uint64_t z = __shfl_up_sync(0xffffffffu, y, o);
+        if (lane >= o) y += z;
+      }
+      wsum[lane] = y;
+    }
+    __syncthreads();
+    uint64_t excl = carry + (wid > 0 ? wsum[wid - 1] : 0ull) + x - v;
+    if (i < n) off[i] = excl;
+    __syncthreads();
+    if (t == 1023) carry = excl + v;
+    __syncthreads();
+  }
+  if (t == 0) off[n] = carry;
+}
+
+__global__ void k_copy_codes(const uint8_t* __restrict__ slots, size_t slot_sz, const uint32_t* __restrict__ bitlen,
+                             const uint64_t* __restrict__ off, int64_t n, uint8_t* __restrict__ out) {
+  for (int64_t w = blockIdx.x; w < n; w += gridDim.x) {
+    const uint32_t nb = (bitlen[w] + 7u) / 8u;
+    const uint8_t* src = slots + (size_t)w * slot_sz;
+    uint8_t* dst = out + off[w];
+    for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x) dst[b] = src[b];
+  }
+}
+
+void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win, uint64_t* offsets,
+                       uint8_t* out, cudaStream_t s) {
+  if (n_win <= 0) return;
+  k_scan_lengths<<<1, 1024, 0, s>>>(bitlen, n_win, offsets);
+  if (out) {
+    unsigned blocks = (unsigned)std::min<int64_t>(n_win, 152 * 16);
+    k_copy_codes<<<blocks, 128, 0, s>>>(slots, slot_sz, bitlen, offsets, n_win, out);
+  }
+}
+
+}  // namespace lmgc

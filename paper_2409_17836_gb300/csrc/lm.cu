@@ -1,0 +1,497 @@
+// lm.cu -- the LM prior of Eq. 2 (a Llama-family decoder, Sec. 4.1): weight generation,
+// embedding, RMSNorm, RoPE, causal GQA attention, SwiGLU, and a CUDA-core GEMM.
+//
+// Every kernel here is row-invariant: a row's result depends only on that row's inputs (and, for
+// attention, on the keys/values of its window), never on M, the batch or the row's place in a
+// tile. That is what lets the decoder (one row per window per step) reproduce the encoder's
+// logits bit for bit.
+#include <math.h>
+
+#include <algorithm>
+
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+
+template <typename T>
+__device__ __forceinline__ float to_f(T v);
+template <>
+__device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T>
+__device__ __forceinline__ T from_f(float v);
+template <>
+__device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// ------------------------------------------------------------------------------------------
+// Random-init weights: splitmix64 (Steele, Lea, Flood 2014) of seed ^ (tensor_id << 40) ^ index;
+// top 24 bits u; w = fp32((u - 2^23) * 2^-23) * a, a = fp32(init_std * sqrt(3)).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t splitmix64(uint64_t x) {
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+template <typename T>
+__global__ void k_init_weights(T* __restrict__ dst, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols,
+                               int64_t ld, int64_t row_off, float a) {
+  const int64_t total = rows * cols;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+       idx += (int64_t)gridDim.x * blockDim.x) {
+    uint64_t u = splitmix64(seed ^ ((uint64_t)tid << 40) ^ (uint64_t)idx) >> 40;
+    float unit = (float)((int32_t)u - (1 << 23)) * (1.0f / 8388608.0f);
+    float w = __fmul_rn(unit, a);
+    int64_t r = idx / cols, c = idx - r * cols;
+    dst[(row_off + r) * ld + c] = from_f<T>(w);
+  }
+}
+
+void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols, int64_t ld,
+                         int64_t row_off, float init_std, cudaStream_t s) {
+  float a = (float)((double)init_std * sqrt(3.0));
+  int64_t total = rows * cols;
+  unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 64);
+  if (dtype == LMGC_BF16)
+    k_init_weights<<<blocks, 256, 0, s>>>((__nv_bfloat16*)dst, seed, tid, rows, cols, ld, row_off, a);
+  else
+    k_init_weights<<<blocks, 256, 0, s>>>((float*)dst, seed, tid, rows, cols, ld, row_off, a);
+}
+
+// ------------------------------------------------------------------------------------------
+// Window inputs (Eq. 2): window w's model input is [BOS, t_{wW}, ..., t_{wW+W-2}]; positions past
+// the end of the token stream read padding id 0.
+// ------------------------------------------------------------------------------------------
+__global__ void k_window_inputs(const uint16_t* __restrict__ tok, int64_t n_tok, int64_t first_win, int64_t n_win,
+                                int W, uint16_t* __restrict__ tok_in) {
+  int64_t total = n_win * W;
+  for (int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; r < total; r += (int64_t)gridDim.x * blockDim.x) {
+    int64_t wl = r / W;
+    int i = (int)(r - wl * W);
+    int64_t g = (first_win + wl) * W + i - 1;
+    tok_in[r] = i == 0 ? (uint16_t)kTokBos : (g < n_tok ? tok[g] : (uint16_t)0);
+  }
+}
+
+void launch_window_inputs(const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t n_win, int W,
+                          uint16_t* tok_in, cudaStream_t s) {
+  int64_t total = n_win * W;
+  unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
+  k_window_inputs<<<blocks, 256, 0, s>>>(tok, n_tok, first_win, n_win, W, tok_in);
+}
+
+// x[r][:] = E[tok_in[r]][:] (fp32 residual stream)
+template <typename T>
+__global__ void k_embed(const uint16_t* __restrict__ tok_in, int64_t rows, const T* __restrict__ E, int d,
+                        float* __restrict__ x) {
+  int64_t r = blockIdx.x;
+  if (r >= rows) return;
+  const T* e = E + (int64_t)tok_in[r] * d;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) x[r * d + j] = to_f<T>(e[j]);
+}
+
+void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, int dtype, float* x, cudaStream_t s) {
+  if (rows <= 0) return;
+  if (dtype == LMGC_BF16) k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const __nv_bfloat16*)E, d, x);
+  else k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const float*)E, d, x);
+}
+
+// ------------------------------------------------------------------------------------------
+// RMSNorm with unit gain: y = x * rsqrt(mean(x^2) + eps). One warp per row; a fixed reduction
+// order (per-lane sequential, then a butterfly) keeps it row-invariant.
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_rmsnorm(const float* __restrict__ x, int64_t rows, int d, float eps,
+                                                 T* __restrict__ y) {
+  int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + r * d);
+  float ss = 0.f;
+  for (int j = lane; j < d / 4; j += 32) {
+    float4 v = xr[j];
+    ss += v.x * v.x;
+    ss += v.y * v.y;
+    ss += v.z * v.z;
+    ss += v.w * v.w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  float inv = rsqrtf(ss / (float)d + eps);
+  T* yr = y + r * d;
+  for (int j = lane; j < d / 4; j += 32) {
+    float4 v = xr[j];
+    yr[4 * j + 0] = from_f<T>(v.x * inv);
+    yr[4 * j + 1] = from_f<T>(v.y * inv);
+    yr[4 * j + 2] = from_f<T>(v.z * inv);
+    yr[4 * j + 3] = from_f<T>(v.w * inv);
+  }
+}
+
+void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, int dtype, cudaStream_t s) {
+  if (rows <= 0) return;
+  unsigned blocks = (unsigned)((rows + 7) / 8);
+  if (dtype == LMGC_BF16) k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (__nv_bfloat16*)out);
+  else k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (float*)out);
+}
+
+// ------------------------------------------------------------------------------------------
+// CUDA-core GEMM: C[M][N] (op)= A[M][K] . B[N][K]^T, fp32 accumulation in k order.
+// 128x128 tile, 256 threads, 8x8 outputs per thread. Used for the fp32 model and as the bf16
+// path where the tensor-core GEMM does not apply.
+// Epilogues: kStore (C has A's type), kAddResidual (C fp32 += acc), kStoreF32 (C fp32 = acc).
+// ------------------------------------------------------------------------------------------
+constexpr int GBM = 128, GBN = 128, GBK = 16;
+
+template <typename T>
+__device__ __forceinline__ void load8(const T* p, float* v, bool ok);
+template <>
+__device__ __forceinline__ void load8<float>(const float* p, float* v, bool ok) {
+  if (ok) {
+    float4 a = *reinterpret_cast<const float4*>(p);
+    float4 b = *reinterpret_cast<const float4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; i++) v[i] = 0.f;
+  }
+}
+template <>
+__device__ __forceinline__ void load8<__nv_bfloat16>(const __nv_bfloat16* p, float* v, bool ok) {
+  if (ok) {
+    uint4 q = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+    for (int i = 0; i < 4; i++) {
+      float2 f = __bfloat1622float2(h[i]);
+      v[2 * i] = f.x;
+      v[2 * i + 1] = f.y;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; i++) v[i] = 0.f;
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ A, const T* __restrict__ B, void* C,
+                                                   int64_t M, int64_t N, int64_t K, int epi) {
+  __shared__ __align__(16) float As[GBK][GBM + 4];
+  __shared__ __align__(16) float Bs[GBK][GBN + 4];
+  const int t = threadIdx.x;
+  const int tx = t & 15, ty = t >> 4;
+  const int64_t m0 = (int64_t)blockIdx.y * GBM, n0 = (int64_t)blockIdx.x * GBN;
+  // loader: each thread loads 8 consecutive k of one row of A and of B per k-tile
+  const int lr = t >> 1, lk = (t & 1) * 8;
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; i++)
+#pragma unroll
+    for (int j = 0; j < 8; j++) acc[i][j] = 0.f;
+  for (int64_t k0 = 0; k0 < K; k0 += GBK) {
+    float va[8], vb[8];
+    int64_t ar = m0 + lr, br = n0 + lr;
+    bool kok = k0 + lk < K;  // K % 8 == 0
+    load8<T>(A + ar * K + k0 + lk, va, ar < M && kok);
+    load8<T>(B + br * K + k0 + lk, vb, br < N && kok);
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+      As[lk + i][lr] = va[i];
+      Bs[lk + i][lr] = vb[i];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GBK; kk++) {
+      float a[8], b[8];
+      float4 a0 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+      float4 a1 = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
+      float4 b0 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+      float4 b1 = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
+      a[0] = a0.x; a[1] = a0.y; a[2] = a0.z; a[3] = a0.w; a[4] = a1.x; a[5] = a1.y; a[6] = a1.z; a[7] = a1.w;
+      b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w; b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
+#pragma unroll
+      for (int i = 0; i < 8; i++)
+#pragma unroll
+        for (int j = 0; j < 8; j++) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 8; i++) {
+    int64_t m = m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4);
+    if (m >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 8; j++) {
+      int64_t n = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + j - 4);
+      if (n >= N) continue;
+      if (epi == kStore) reinterpret_cast<T*>(C)[m * N + n] = from_f<T>(acc[i][j]);
+      else if (epi == kAddResidual) reinterpret_cast<float*>(C)[m * N + n] += acc[i][j];
+      else reinterpret_cast<float*>(C)[m * N + n] = acc[i][j];
+    }
+  }
+}
+
+void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
+                      cudaStream_t s) {
+  if (M <= 0 || N <= 0) return;
+  dim3 grid((unsigned)((N + GBN - 1) / GBN), (unsigned)((M + GBM - 1) / GBM));
+  if (dtype == LMGC_BF16)
+    k_gemm_simt<<<grid, 256, 0, s>>>((const __nv_bfloat16*)A, (const __nv_bfloat16*)B, C, M, N, K, epi);
+  else
+    k_gemm_simt<<<grid, 256, 0, s>>>((const float*)A, (const float*)B, C, M, N, K, epi);
+}
+
+// ------------------------------------------------------------------------------------------
+// RoPE, rotate-half pairing: in each head, dims i and i + hd/2 rotate by pos * theta^(-2i/hd).
+// Applied in place to the first n_rot_heads heads of each qkv row (the q heads then the k heads).
+// Row r sits at position pos_first + (r mod q_win_stride).
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__global__ void k_rope(T* __restrict__ qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd,
+                       const float2* __restrict__ cs, int64_t pos_first, int64_t q_win_stride) {
+  const int half = hd / 2;
+  const int64_t per_row = (int64_t)n_rot_heads * half;
+  const int64_t total = rows * per_row;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    int64_t r = e / per_row;
+    int rem = (int)(e - r * per_row);
+    int h = rem / half, i = rem - h * half;
+    int64_t pos = pos_first + (r % q_win_stride);
+    float2 c = cs[pos * half + i];
+    T* v = qkv + r * qkv_dim + (int64_t)h * hd;
+    float a = to_f<T>(v[i]), b = to_f<T>(v[i + half]);
+    v[i] = from_f<T>(a * c.x - b * c.y);
+    v[i + half] = from_f<T>(a * c.y + b * c.x);
+  }
+}
+
+void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
+                 int64_t pos_first, int64_t q_win_stride, int n_pos, int dtype, cudaStream_t s) {
+  (void)W;
+  (void)n_pos;
+  int64_t total = rows * n_rot_heads * (hd / 2);
+  if (total <= 0) return;
+  unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
+  if (dtype == LMGC_BF16)
+    k_rope<<<blocks, 256, 0, s>>>((__nv_bfloat16*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
+  else k_rope<<<blocks, 256, 0, s>>>((float*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
+}
+
+// ------------------------------------------------------------------------------------------
+// Causal softmax attention with grouped-query heads, CUDA cores, fp32 online softmax.
+// Block (qb, h, w): query positions pos_first + qb*64 + [0, 64) of window w (at most n_pos of
+// them); query row for position p: w*q_win_stride + (p - pos_first). Keys/values of window w at
+// position j: kv row w*W + j (k at column k_off + kvh*hd, v at v_off + kvh*hd). Key blocks are
+// 64-aligned and visited in order 0, 1, ..., so a row's arithmetic is the same whether it is
+// computed in a full prefill block or alone in a decode step.
+// ------------------------------------------------------------------------------------------
+constexpr int ABQ = 64, ABK = 64;
+
+template <typename T, int HD>
+__global__ void __launch_bounds__(256) k_attention(const T* __restrict__ q, int64_t q_stride,
+                                                   const T* __restrict__ kv, int64_t kv_stride, int k_off, int v_off,
+                                                   T* __restrict__ out, int64_t out_stride, int nq, int nkv, int W,
+                                                   int64_t pos_first, int n_pos, int64_t q_win_stride, float scale) {
+  extern __shared__ __align__(16) float sm[];
+  float* Qs = sm;                       // [ABQ][HD]
+  float* Kt = Qs + ABQ * HD;            // [HD][ABK] (transposed)
+  float* Vs = Kt + HD * ABK;            // [ABK][HD]
+  float* Ps = Vs + ABK * HD;            // [ABQ][ABK + 1]
+  const int t = threadIdx.x, tx = t & 15, ty = t >> 4;
+  const int qb = blockIdx.x, h = blockIdx.y;
+  const int64_t w = blockIdx.z;
+  const int kvh = h / (nq / nkv);
+  const int64_t p_lo = pos_first + (int64_t)qb * ABQ;
+  const int64_t rem_pos = pos_first + n_pos - p_lo;
+  const int nrows = rem_pos < ABQ ? (int)rem_pos : ABQ;
+  if (nrows <= 0) return;
+  const int64_t p_hi = p_lo + nrows - 1;
+  for (int e = t; e < ABQ * HD; e += 256) {
+    int r = e / HD, c = e - r * HD;
+    float v = 0.f;
+    if (r < nrows) v = to_f<T>(q[(w * q_win_stride + (p_lo + r - pos_first)) * q_stride + (int64_t)h * HD + c]);
+    Qs[e] = v;
+  }
+  constexpr int OC = HD / 16;
+  float m[4], l[4], o[4][OC];
+#pragma unroll
+  for (int r = 0; r < 4; r++) {
+    m[r] = -INFINITY;
+    l[r] = 0.f;
+#pragma unroll
+    for (int c = 0; c < OC; c++) o[r][c] = 0.f;
+  }
+  const int nkb = (int)(p_hi / ABK) + 1;
+  for (int kb = 0; kb < nkb; kb++) {
+    __syncthreads();
+    for (int e = t; e < ABK * HD; e += 256) {
+      int j = e / HD, c = e - j * HD;
+      int64_t pj = (int64_t)kb * ABK + j;
+      float kvv = 0.f, vvv = 0.f;
+      if (pj <= p_hi) {
+        const T* row = kv + (w * W + pj) * kv_stride;
+        kvv = to_f<T>(row[k_off + kvh * HD + c]);
+        vvv = to_f<T>(row[v_off + kvh * HD + c]);
+      }
+      Kt[c * ABK + j] = kvv;
+      Vs[j * HD + c] = vvv;
+    }
+    __syncthreads();
+    float s[4][4];
+#pragma unroll
+    for (int r = 0; r < 4; r++)
+#pragma unroll
+      for (int c = 0; c < 4; c++) s[r][c] = 0.f;
+#pragma unroll 4
+    for (int d = 0; d < HD; d++) {
+      float4 kk = *reinterpret_cast<const float4*>(&Kt[d * ABK + tx * 4]);
+#pragma unroll
+      for (int r = 0; r < 4; r++) {
+        float qv = Qs[(ty * 4 + r) * HD + d];
+        s[r][0] = fmaf(qv, kk.x, s[r][0]);
+        s[r][1] = fmaf(qv, kk.y, s[r][1]);
+        s[r][2] = fmaf(qv, kk.z, s[r][2]);
+        s[r][3] = fmaf(qv, kk.w, s[r][3]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 4; r++) {
+      const int64_t p = p_lo + ty * 4 + r;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        int64_t j = (int64_t)kb * ABK + tx * 4 + c;
+        s[r][c] = (j <= p) ? s[r][c] * scale : -INFINITY;
+        mx = fmaxf(mx, s[r][c]);
+      }
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      const float mn = fmaxf(m[r], mx);
+      const float corr = (mn == -INFINITY) ? 1.f : expf(m[r] - mn);
+      float rs = 0.f;
+#pragma unroll
+      for (int c = 0; c < 4; c++) {
+        float pv = (s[r][c] == -INFINITY) ? 0.f : expf(s[r][c] - mn);
+        s[r][c] = pv;
+        rs += pv;
+      }
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) rs += __shfl_xor_sync(0xffffffffu, rs, off);
+      l[r] = l[r] * corr + rs;
+      m[r] = mn;
+#pragma unroll
+      for (int c = 0; c < OC; c++) o[r][c] *= corr;
+#pragma unroll
+      for (int c = 0; c < 4; c++) Ps[(ty * 4 + r) * (ABK + 1) + tx * 4 + c] = s[r][c];
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int j = 0; j < ABK; j++) {
+      float vv[OC];
+#pragma unroll
+      for (int c = 0; c < OC; c++) vv[c] = Vs[j * HD + tx + 16 * c];
+#pragma unroll
+      for (int r = 0; r < 4; r++) {
+        float pv = Ps[(ty * 4 + r) * (ABK + 1) + j];
+#pragma unroll
+        for (int c = 0; c < OC; c++) o[r][c] = fmaf(pv, vv[c], o[r][c]);
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 4; r++) {
+    int rr = ty * 4 + r;
+    if (rr >= nrows) continue;
+    float inv = 1.f / l[r];
+    T* orow = out + (w * q_win_stride + (p_lo + rr - pos_first)) * out_stride + (int64_t)h * HD;
+#pragma unroll
+    for (int c = 0; c < OC; c++) orow[tx + 16 * c] = from_f<T>(o[r][c] * inv);
+  }
+}
+
+template <typename T, int HD>
+static void attn_launch(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
+                        void* out, int64_t out_stride, int nq, int nkv, int W, int64_t n_win, int64_t pos_first,
+                        int n_pos, int64_t q_win_stride, cudaStream_t s) {
+  size_t smem = sizeof(float) * (ABQ * HD + HD * ABK + ABK * HD + ABQ * (ABK + 1));
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaFuncSetAttribute(k_attention<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    attr_done = true;
+  }
+  dim3 grid((unsigned)((n_pos + ABQ - 1) / ABQ), (unsigned)nq, (unsigned)n_win);
+  float scale = 1.0f / sqrtf((float)HD);
+  k_attention<T, HD><<<grid, 256, smem, s>>>((const T*)q, q_stride, (const T*)kv, kv_stride, k_off, v_off, (T*)out,
+                                             out_stride, nq, nkv, W, pos_first, n_pos, q_win_stride, scale);
+}
+
+void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
+                      void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
+                      int64_t pos_first, int n_pos, int64_t q_win_stride, int dtype, cudaStream_t s) {
+  if (n_win <= 0 || n_pos <= 0) return;
+#define LMGC_ATT(T, HDV)                                                                                        \
+  attn_launch<T, HDV>(q, q_stride, kv, kv_stride, k_off, v_off, out, out_stride, nq, nkv, W, n_win, pos_first, \
+                      n_pos, q_win_stride, s)
+  if (dtype == LMGC_BF16) {
+    if (hd == 32) LMGC_ATT(__nv_bfloat16, 32);
+    else if (hd == 64) LMGC_ATT(__nv_bfloat16, 64);
+    else LMGC_ATT(__nv_bfloat16, 128);
+  } else {
+    if (hd == 32) LMGC_ATT(float, 32);
+    else if (hd == 64) LMGC_ATT(float, 64);
+    else LMGC_ATT(float, 128);
+  }
+#undef LMGC_ATT
+}
+
+// act[r][j] = silu(g) * u, g = gu[r][j], u = gu[r][ffn + j]
+template <typename T>
+__global__ void k_swiglu(const T* __restrict__ gu, int64_t rows, int ffn, T* __restrict__ act) {
+  int64_t total = rows * ffn;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    int64_t r = e / ffn;
+    int j = (int)(e - r * ffn);
+    float g = to_f<T>(gu[r * 2 * ffn + j]);
+    float u = to_f<T>(gu[r * 2 * ffn + ffn + j]);
+    act[e] = from_f<T>(g / (1.f + expf(-g)) * u);
+  }
+}
+
+void launch_swiglu(const void* gu, int64_t rows, int ffn, void* act, int dtype, cudaStream_t s) {
+  int64_t total = rows * ffn;
+  if (total <= 0) return;
+  unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
+  if (dtype == LMGC_BF16) k_swiglu<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)gu, rows, ffn, (__nv_bfloat16*)act);
+  else k_swiglu<<<blocks, 256, 0, s>>>((const float*)gu, rows, ffn, (float*)act);
+}
+
+// dst[(w * dst_win_stride + dst_pos) * row_elems + c] = src[w * src_stride + c]
+template <typename T>
+__global__ void k_copy_rows(const T* __restrict__ src, int64_t src_stride, T* __restrict__ dst, int64_t dst_win_stride,
+                            int64_t dst_pos, int64_t n_rows, int64_t row_elems) {
+  int64_t total = n_rows * row_elems;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    int64_t w = e / row_elems, c = e - w * row_elems;
+    dst[(w * dst_win_stride + dst_pos) * row_elems + c] = src[w * src_stride + c];
+  }
+}
+
+void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t dst_win_stride, int64_t dst_pos,
+                      int64_t n_rows, int64_t row_elems, int dtype, cudaStream_t s) {
+  int64_t total = n_rows * row_elems;
+  if (total <= 0) return;
+  unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
+  if (dtype == LMGC_BF16)
+    k_copy_rows<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)src, src_stride, (__nv_bfloat16*)dst, dst_win_stride,
+                                       dst_pos, n_rows, row_elems);
+  else
+    k_copy_rows<<<blocks, 256, 0, s>>>((const float*)src, src_stride, (float*)dst, dst_win_stride, dst_pos, n_rows,
+                                       row_elems);
+}
+
+}  // namespace lmgc

@@ -1,0 +1,164 @@
+// lmgc_internal.cuh -- declarations shared by the .cu files of liblmgc.so (the CUDA path only).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/lmgc.h"
+
+namespace lmgc {
+
+// Token ids (character-level reading of Sec. 3 / Fig. 1).
+constexpr int kTokSpace = 16, kTokComma = 17, kTokSemi = 18, kTokBos = 19;
+
+// Device error word bits (set by bounded device loops instead of spinning or trapping).
+enum : uint32_t { kErrCorrupt = 1u, kErrLimit = 2u, kErrDeser = 4u };
+
+struct KernelStat {
+  const char* name;
+  int launches;
+  float ms;
+  double work;  // algorithmic flops or bytes summed over launches
+};
+
+// Timing of one kernel class inside a call (only when profiling is enabled).
+struct Profiler {
+  bool enabled = false;
+  struct Rec {
+    int cls;
+    cudaEvent_t a, b;
+    double work;
+  };
+  std::vector<Rec> pending;
+  std::vector<cudaEvent_t> pool;
+  KernelStat stats[16];
+};
+
+struct Layer {
+  void* wqkv;   // [qkv_dim][d]: Wq rows, then Wk rows, then Wv rows
+  void* wo;     // [d][nq*hd]
+  void* wgu;    // [2*ffn][d]: gate/up rows, layout per GemmEpi::kSwiGLU
+  void* wdown;  // [d][ffn]
+};
+
+struct Workspace {
+  int64_t rows = 0;  // capacity in model rows (windows * W)
+  float* x = nullptr;      // residual fp32 [rows][d]
+  void* n = nullptr;       // normalised activations [rows][d] (T)
+  void* qkv = nullptr;     // [rows][qkv_dim] (T)
+  void* att = nullptr;     // [rows][nq*hd] (T)
+  void* act = nullptr;     // SwiGLU output [rows][ffn] (T)
+  void* gu = nullptr;      // gate/up GEMM output [rows][2*ffn] (T), unfused path only
+  uint16_t* tok_in = nullptr;  // model input ids [rows]
+};
+
+}  // namespace lmgc
+
+struct lmgc_ctx {
+  lmgc_config cfg;
+  int device = 0;
+  int hd = 0, qkv_dim = 0, tpv = 0;
+  size_t elt = 4;  // bytes per weight / activation element
+  void* w_embed = nullptr;
+  void* w_head = nullptr;
+  std::vector<lmgc::Layer> layers;
+  void* weights_blob = nullptr;
+  float2* rope_cs = nullptr;   // [W][hd/2] (cos, sin)
+  uint32_t* exp2_tab = nullptr;  // [512]: H then L
+  lmgc::Workspace ws;
+  float* logits = nullptr;     // [rows][V]
+  uint32_t* d_err = nullptr;   // device error word
+  // encode staging
+  uint16_t* tok = nullptr;
+  size_t tok_cap = 0;
+  uint32_t* pair_start = nullptr;
+  uint32_t* pair_freq = nullptr;
+  size_t pair_cap = 0;
+  uint32_t* win_len = nullptr;
+  size_t win_cap = 0;
+  void* host_in = nullptr;  // device staging for lmgc_encode_host
+  size_t host_in_cap = 0;
+  uint8_t* host_out = nullptr;
+  size_t host_out_cap = 0;
+  // decode state
+  void* kv_cache = nullptr;
+  size_t kv_cap = 0;
+  float stage_ms[5] = {0, 0, 0, 0, 0};
+  cudaEvent_t ev[6] = {};
+  std::vector<cudaEvent_t> batch_ev;
+  lmgc::Profiler prof;
+  bool use_tc = true;  // tcgen05 GEMM for bf16 models when available
+  std::string err;
+};
+
+namespace lmgc {
+
+// ---- error helpers (host) ----
+void set_thread_error(const std::string& s);
+lmgc_status fail(lmgc_ctx* ctx, lmgc_status st, const std::string& msg);
+lmgc_status cuda_fail(lmgc_ctx* ctx, cudaError_t e, const char* what);
+
+#define LMGC_CUDA(ctx, call)                                   \
+  do {                                                         \
+    cudaError_t e_ = (call);                                   \
+    if (e_ != cudaSuccess) return lmgc::cuda_fail(ctx, e_, #call); \
+  } while (0)
+
+// ---- kernels' launchers (stream-ordered, no sync) ----
+// serialize.cu
+int tokens_per_value(int input_kind, int sep_mode);
+void launch_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* tok, cudaStream_t s);
+void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64_t n_values, void* out,
+                        uint32_t* err, cudaStream_t s);
+
+// lm.cu
+void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols, int64_t ld,
+                         int64_t row_off, float init_std, cudaStream_t s);
+void launch_window_inputs(const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t n_win, int W,
+                          uint16_t* tok_in, cudaStream_t s);
+void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, int dtype, float* x, cudaStream_t s);
+void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, int dtype, cudaStream_t s);
+// C[M][N] = A[M][K] . B[N][K]^T with the given epilogue
+enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2 };
+void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
+                      cudaStream_t s);
+void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
+                 int64_t pos_first, int64_t q_win_stride, int n_pos, int dtype, cudaStream_t s);
+void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
+                      void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
+                      int64_t pos_first, int n_pos, int64_t q_win_stride, int dtype, cudaStream_t s);
+void launch_swiglu(const void* gu, int64_t rows, int ffn, void* act, int dtype, cudaStream_t s);
+void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t dst_win_stride, int64_t dst_pos,
+                      int64_t n_rows, int64_t row_elems, int dtype, cudaStream_t s);
+
+// cdf.cu
+void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s);  // builds H and L on the host
+void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
+                      int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
+                      uint32_t* freq, int mode, cudaStream_t s);
+void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
+                         cudaStream_t s);
+void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
+                       const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
+                       const uint32_t* win_len, uint32_t* err, cudaStream_t s);
+
+// coder.cu
+size_t slot_bytes(size_t win_tokens, int P);
+void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
+                         const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
+                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s);
+void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win,
+                       uint64_t* offsets /* [n_win+1] scratch */, uint8_t* out, cudaStream_t s);
+size_t dec_state_bytes();
+void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n,
+                     void* state, cudaStream_t s);
+
+// gemm_tc.cu (tcgen05)
+bool tc_gemm_supported(int64_t M, int64_t N, int64_t K);
+void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, cudaStream_t s);
+
+}  // namespace lmgc

@@ -1,0 +1,142 @@
+// serialize.cu -- fp32 / uint8 values -> hex-digit token ids with separators, and back.
+//
+// Sec. 3 "Serialization" and Fig. 1: each value's bits are cut into 4-bit groups, most
+// significant first (for fp32: the sign and exponent nibbles lead), each group becomes one hex
+// digit (token id = digit value 0..15), and a separator follows every value (' ' = 16,
+// ',' = 17, ', ' = 17 16, ';' = 18, or none).
+//
+// HBM-bound: 4 B read + tpv * 2 B written per fp32 value. A block stages the tokens of 1024
+// values in shared memory so that the writes leave as coalesced 16-byte vectors.
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+
+int tokens_per_value(int input_kind, int sep_mode) {
+  int nd = input_kind == LMGC_IN_F32 ? 8 : (input_kind == LMGC_IN_U8 ? 2 : -1);
+  int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
+  if (nd < 0 || sep_mode < 0 || sep_mode > 4) return -1;
+  return nd + ns;
+}
+
+static void sep_ids(int sep_mode, uint16_t* s0, uint16_t* s1) {
+  switch (sep_mode) {
+    case LMGC_SEP_SPACE: *s0 = kTokSpace; *s1 = 0; break;
+    case LMGC_SEP_COMMA: *s0 = kTokComma; *s1 = 0; break;
+    case LMGC_SEP_COMMA_SPACE: *s0 = kTokComma; *s1 = kTokSpace; break;
+    case LMGC_SEP_SEMI: *s0 = kTokSemi; *s1 = 0; break;
+    default: *s0 = 0; *s1 = 0; break;
+  }
+}
+
+constexpr int kSerThreads = 256;
+constexpr int kSerVals = 4 * kSerThreads;  // values per block
+
+template <int ND, int NS, bool VEC>
+__global__ void __launch_bounds__(kSerThreads) k_serialize(const void* __restrict__ in, int64_t n,
+                                                           uint16_t* __restrict__ tok, uint16_t sep0,
+                                                           uint16_t sep1) {
+  constexpr int TPV = ND + NS;
+  __shared__ __align__(16) uint16_t buf[kSerVals * TPV];
+  const int t = threadIdx.x;
+  const int64_t v0 = (int64_t)blockIdx.x * kSerVals;
+  const int nv = (n - v0) < kSerVals ? (int)(n - v0) : kSerVals;
+  uint32_t b[4];
+  if (ND == 8) {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(in) + v0;
+    if (VEC && nv == kSerVals) {
+      uint4 q = __ldcs(reinterpret_cast<const uint4*>(src) + t);
+      b[0] = q.x; b[1] = q.y; b[2] = q.z; b[3] = q.w;
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; i++) b[i] = (4 * t + i < nv) ? src[4 * t + i] : 0u;
+    }
+  } else {
+    const uint8_t* src = reinterpret_cast<const uint8_t*>(in) + v0;
+    if (VEC && nv == kSerVals) {
+      uint32_t q = __ldcs(reinterpret_cast<const unsigned int*>(src) + t);
+#pragma unroll
+      for (int i = 0; i < 4; i++) b[i] = (q >> (8 * i)) & 0xFFu;
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; i++) b[i] = (4 * t + i < nv) ? src[4 * t + i] : 0u;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; i++) {
+    uint16_t* o = buf + (4 * t + i) * TPV;
+#pragma unroll
+    for (int j = 0; j < ND; j++) o[j] = (uint16_t)((b[i] >> (4 * (ND - 1 - j))) & 0xFu);
+    if (NS >= 1) o[ND] = sep0;
+    if (NS >= 2) o[ND + 1] = sep1;
+  }
+  __syncthreads();
+  const int64_t tok0 = v0 * TPV;
+  const int ntok = nv * TPV;
+  uint16_t* dst = tok + tok0;
+  if (VEC && nv == kSerVals) {
+    // kSerVals * TPV * 2 bytes is a multiple of 16, and tok is 16-byte aligned (checked)
+    const uint4* s4 = reinterpret_cast<const uint4*>(buf);
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    for (int k = t; k < ntok / 8; k += kSerThreads) __stcs(d4 + k, s4[k]);
+  } else {
+    for (int k = t; k < ntok; k += kSerThreads) dst[k] = buf[k];
+  }
+}
+
+template <int ND, int NS>
+static void ser_dispatch(bool vec, const void* in, int64_t n, uint16_t* tok, uint16_t s0, uint16_t s1,
+                         cudaStream_t s) {
+  int64_t blocks = (n + kSerVals - 1) / kSerVals;
+  if (vec) k_serialize<ND, NS, true><<<(unsigned)blocks, kSerThreads, 0, s>>>(in, n, tok, s0, s1);
+  else k_serialize<ND, NS, false><<<(unsigned)blocks, kSerThreads, 0, s>>>(in, n, tok, s0, s1);
+}
+
+void launch_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* tok, cudaStream_t s) {
+  if (n <= 0) return;
+  uint16_t s0, s1;
+  sep_ids(sep_mode, &s0, &s1);
+  int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
+  bool vec = (((uintptr_t)in) % 16 == 0) && (((uintptr_t)tok) % 16 == 0);
+  if (input_kind == LMGC_IN_F32) {
+    if (ns == 0) ser_dispatch<8, 0>(vec, in, n, tok, s0, s1, s);
+    else if (ns == 1) ser_dispatch<8, 1>(vec, in, n, tok, s0, s1, s);
+    else ser_dispatch<8, 2>(vec, in, n, tok, s0, s1, s);
+  } else {
+    if (ns == 0) ser_dispatch<2, 0>(vec, in, n, tok, s0, s1, s);
+    else if (ns == 1) ser_dispatch<2, 1>(vec, in, n, tok, s0, s1, s);
+    else ser_dispatch<2, 2>(vec, in, n, tok, s0, s1, s);
+  }
+}
+
+// Inverse: one thread per value; a malformed group sets kErrDeser in *err.
+__global__ void k_deserialize(const uint16_t* __restrict__ tok, int64_t n, int nd, int ns, uint16_t sep0,
+                              uint16_t sep1, void* __restrict__ out, uint32_t* err) {
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const int tpv = nd + ns;
+  const uint16_t* g = tok + i * tpv;
+  uint32_t b = 0;
+  bool bad = false;
+  for (int j = 0; j < nd; j++) {
+    uint16_t d = g[j];
+    bad |= d > 15;
+    b = (b << 4) | (d & 0xFu);
+  }
+  if (ns >= 1) bad |= g[nd] != sep0;
+  if (ns >= 2) bad |= g[nd + 1] != sep1;
+  if (bad) atomicOr(err, kErrDeser);
+  if (nd == 8) reinterpret_cast<uint32_t*>(out)[i] = b;
+  else reinterpret_cast<uint8_t*>(out)[i] = (uint8_t)b;
+}
+
+void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64_t n_values, void* out,
+                        uint32_t* err, cudaStream_t s) {
+  if (n_values <= 0) return;
+  uint16_t s0, s1;
+  sep_ids(sep_mode, &s0, &s1);
+  int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
+  int nd = input_kind == LMGC_IN_F32 ? 8 : 2;
+  k_deserialize<<<(unsigned)((n_values + 255) / 256), 256, 0, s>>>(tok, n_values, nd, ns, s0, s1, out, err);
+}
+
+}  // namespace lmgc

@@ -1,0 +1,156 @@
+"""GPU parity of the integer stages against the oracle, through the C ABI:
+serialisation (Sec. 3), integer CDF given identical logits, and the arithmetic coder (Sec. 2)
+given identical (start, freq) pairs -- all bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2409_17836_gb300 import configs, lmgc as L
+from tests._util import random_pairs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx_tiny():
+    c = L.Context(configs.with_(configs.TINY, batch_windows=4))
+    yield c
+    c.close()
+
+
+def ctx_for(**kw):
+    return L.Context(configs.with_(configs.TINY, batch_windows=1, **kw))
+
+
+SPECIAL = np.array([0, 0x80000000, 0x7F800000, 0xFF800000, 0x7FC00000, 0x7FA00001, 0xFFFFFFFF, 1, 0x007FFFFF,
+                    0x3F800000], dtype=np.uint32)
+
+
+@pytest.mark.parametrize("sep_mode", [0, 1, 2, 3, 4])
+@pytest.mark.parametrize("n", [1, 7, 1023, 1024, 1025, 4096, 100003])
+def test_serialize_bit_exact(sep_mode, n):
+    ctx = ctx_for(sep_mode=sep_mode)
+    rng = np.random.default_rng(n + sep_mode)
+    bits = rng.integers(0, 2 ** 32, n, dtype=np.uint64).astype(np.uint32)
+    bits[: min(n, SPECIAL.size)] = SPECIAL[: min(n, SPECIAL.size)]
+    vals = bits.view(np.float32)
+    d = torch.from_numpy(bits.view(np.int32).copy()).cuda()
+    tok = L.lmgc_serialize(ctx, d)
+    ref = O.serialize(vals, sep_mode)
+    assert np.array_equal(tok.cpu().numpy().view(np.uint16), ref)
+    back = torch.empty(n, dtype=torch.int32, device="cuda")
+    assert L.lmgc_deserialize(ctx, tok, back) == n
+    assert np.array_equal(back.cpu().numpy().view(np.uint32), bits)
+    ctx.close()
+
+
+def test_serialize_unaligned_input_and_u8():
+    ctx = ctx_for()
+    rng = np.random.default_rng(3)
+    bits = rng.integers(0, 2 ** 32, 5001, dtype=np.uint64).astype(np.uint32)
+    d = torch.from_numpy(bits.view(np.int32).copy()).cuda()
+    tok = L.lmgc_serialize(ctx, d[1:])  # 4-byte aligned, not 16
+    assert np.array_equal(tok.cpu().numpy().view(np.uint16), O.serialize(bits[1:].view(np.float32), 0))
+    ctx.close()
+    ctx = ctx_for(input_kind=L.IN_U8)
+    codes = rng.integers(0, 256, 3001).astype(np.uint8)
+    tok = L.lmgc_serialize(ctx, torch.from_numpy(codes).cuda())
+    assert np.array_equal(tok.cpu().numpy().view(np.uint16), O.serialize(codes, 0))
+    out = torch.empty(3001, dtype=torch.uint8, device="cuda")
+    L.lmgc_deserialize(ctx, tok, out)
+    assert np.array_equal(out.cpu().numpy(), codes)
+    ctx.close()
+
+
+def test_deserialize_rejects_malformed(ctx_tiny):
+    tok = L.lmgc_serialize(ctx_tiny, torch.ones(10, dtype=torch.float32, device="cuda"))
+    bad = tok.clone()
+    bad[8] = 17
+    with pytest.raises(L.LmgcError) as e:
+        L.lmgc_deserialize(ctx_tiny, bad, torch.empty(10, device="cuda"))
+    assert e.value.status == L.ERR_CORRUPT
+    with pytest.raises(L.LmgcError):
+        L.lmgc_deserialize(ctx_tiny, tok[:-1], torch.empty(10, device="cuda"))
+
+
+def logit_rows(rng, rows, V):
+    z = rng.normal(size=(rows, V)) * rng.uniform(0.05, 12, size=(rows, 1))
+    z = z.astype(np.float32)
+    z[0] = 0.0                      # uniform
+    z[1] = -7.5
+    z[1, V // 3] = 100.0            # one-hot dominant (others clamp to e = 0)
+    z[2] = np.round(z[2])           # many ties
+    z[3, :] = -1e30                 # huge negative values
+    z[3, 5] = 3.0
+    z[4] = z[4] * 1e-6              # nearly uniform, ties in a
+    return z
+
+
+@pytest.mark.parametrize("V,P,rows", [(32, 16, 3000), (1000, 20, 300), (32000, 24, 64)])
+def test_cdf_bit_exact(V, P, rows):
+    ctx = L.Context(configs.with_(configs.TINY, vocab=V, cdf_bits=P, batch_windows=1))
+    rng = np.random.default_rng(V)
+    z = logit_rows(rng, rows, V)
+    dz = torch.from_numpy(z).cuda()
+    cdf = L.lmgc_quantize_cdf(ctx, dz).cpu().numpy().view(np.uint32)
+    ref = O.quantize_cdf(z, P)
+    assert np.array_equal(cdf, ref)
+    sym = rng.integers(0, V, rows).astype(np.uint16)
+    sym[1] = V // 3
+    st, fr = L.lmgc_cdf_pairs(ctx, dz, torch.from_numpy(sym.view(np.int16)).cuda())
+    rs, rf = O.cdf_pairs(z, sym, P)
+    assert np.array_equal(st.cpu().numpy().view(np.uint32), rs)
+    assert np.array_equal(fr.cpu().numpy().view(np.uint32), rf)
+    ctx.close()
+
+
+@pytest.mark.parametrize("P,layout", [(16, "row"), (24, "pos"), (24, "row"), (30, "pos")])
+def test_range_encode_bit_exact(P, layout):
+    rng = np.random.default_rng(P)
+    n_win, W = 70, 300
+    V = 32 if P == 16 else 1000
+    start, freq, lens = random_pairs(rng, n_win, W, P, V=V)
+    lens = rng.integers(1, W + 1, n_win).astype(np.uint32)
+    lens[0], lens[1], lens[-1] = W, 1, 17
+    if layout == "row":
+        s_dev, f_dev, sw, sp = start, freq, W, 1
+    else:
+        s_dev, f_dev, sw, sp = start.T.copy(), freq.T.copy(), 1, n_win
+    out, bitlen = L.lmgc_range_encode(torch.from_numpy(s_dev.view(np.int32)).cuda(),
+                                      torch.from_numpy(f_dev.view(np.int32)).cuda(), P, n_win, W,
+                                      torch.from_numpy(lens.view(np.int32)).cuda(), sw, sp)
+    payload = out.cpu().numpy().tobytes()
+    bl = bitlen.cpu().numpy()
+    off = 0
+    for w in range(n_win):
+        code, nbits = O.range_encode(start[w, :lens[w]], freq[w, :lens[w]], P)
+        assert bl[w] == nbits, w
+        assert payload[off: off + len(code)] == code, w
+        off += len(code)
+    assert off == len(payload)
+
+
+def test_range_encode_many_windows_sampled():
+    """A coder-only batch in the position-major layout: 8192 windows x 2048 tokens over
+    vocab 32000 at P = 24; sampled windows are compared with the oracle."""
+    rng = np.random.default_rng(11)
+    n_win, W, P = 8192, 2048, 24
+    start, freq, _ = random_pairs(rng, n_win, W, P)
+    out, bitlen = L.lmgc_range_encode(torch.from_numpy(start.T.copy().view(np.int32)).cuda(),
+                                      torch.from_numpy(freq.T.copy().view(np.int32)).cuda(), P, n_win, W, None, 1,
+                                      n_win)
+    bl = bitlen.cpu().numpy().astype(np.int64)
+    offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)])
+    payload = out.cpu().numpy()
+    assert offs[-1] == payload.size
+    for w in [0, 1, 31, 32, 4095, 8191] + rng.integers(0, n_win, 10).tolist():
+        code, nbits = O.range_encode(start[w], freq[w], P)
+        assert bl[w] == nbits and payload[offs[w]:offs[w + 1]].tobytes() == code, w
+
+
+def test_range_encode_rejects_bad_pairs():
+    s = torch.zeros(4, dtype=torch.int32, device="cuda")
+    f = torch.zeros(4, dtype=torch.int32, device="cuda")  # freq 0 is invalid
+    with pytest.raises(L.LmgcError):
+        L.lmgc_range_encode(s, f, 16, 1, 4, None, 4, 1)

