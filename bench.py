@@ -1,0 +1,314 @@
+"""Throughput of the LM-GC encode path on GB300 (one JSON line on rank 0).
+
+Workload (default): gradients of a seeded random-init 4-layer ConvNet (298,954 values, 3x32x32
+Gaussian inputs, batch 64), serialised as 8 hex digits + a space per value, coded with a
+TinyLlama-1.1B-shaped model (22 layers, d 2048, 32/4 heads, FFN 5632, vocab 32000, random-init
+bf16 weights) over 2048-token windows, 64 windows per model batch, 24-bit integer CDFs.
+One step = lmgc_encode of one batch: 14,563 values (131,067 tokens, 64 windows) through
+serialise -> model -> CDF pairs -> range coder -> container. Step k encodes slice k mod 20 of the
+gradient; all slices are resident in HBM before timing.
+
+value     raw-gradient MB/s (4 bytes per value) over all ranks, device buffers, CUDA events
+e2e       the same through lmgc_encode_host (pinned host buffers; H2D + D2H inside the region)
+roofline  the GEMM class (the dominant kernel): algorithmic flops / summed CUDA-event time of its
+          launches in the timed region, against the measured sustained bf16 peak
+stages    the same per kernel class (HBM-bound classes against the measured HBM copy bandwidth)
+cpu_baseline / --impl reference: the CPU oracle (test infrastructure) on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "raw gradient MB/s encoded (1 GB300); LM tensor-pipe % of bf16 peak; coder HBM GB/s"
+WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama")
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+class Clocks:
+    """nvidia-smi samples every 200 ms during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def workload(name: str):
+    from paper_2409_17836_gb300 import configs, inputs
+
+    if name == "convnet-tinyllama":
+        return configs.TINYLLAMA, inputs.convnet_gradient(0)
+    if name == "convnet-llama2-7b":
+        return configs.LLAMA2_7B, inputs.convnet_gradient(0)
+    if name == "lossy-tinyllama":
+        return configs.TINYLLAMA_LOSSY, inputs.lossy_codes(inputs.convnet_gradient(0))
+    if name == "tiny":
+        return configs.TINY, inputs.tiny_gradient(0)
+    raise ValueError(name)
+
+
+def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
+    """Oracle encode of the first `positions` tokens of window `win` (model + CDF + coder)."""
+    import numpy as np
+
+    import oracle as O
+
+    oc = O.OracleConfig(n_layers=cfg.n_layers, d_model=cfg.d_model, n_heads=cfg.n_heads, n_kv_heads=cfg.n_kv_heads,
+                        d_ffn=cfg.d_ffn, vocab=cfg.vocab, bf16=cfg.dtype == 1, window=cfg.window,
+                        cdf_bits=cfg.cdf_bits, weight_seed=cfg.weight_seed, init_std=cfg.init_std,
+                        sep_mode=cfg.sep_mode, input_kind=cfg.input_kind, n_threads=threads)
+    tok = O.serialize(vals, cfg.sep_mode)
+    W = cfg.window
+    seg = tok[win * W: win * W + W]
+    t0 = time.perf_counter()
+    st, fr, _ = O.window_pairs(oc, seg, min(positions, seg.size))
+    O.range_encode(st, fr, cfg.cdf_bits)
+    dt = time.perf_counter() - t0
+    return dt, min(positions, seg.size)
+
+
+def bytes_per_value(cfg) -> int:
+    return 4 if cfg.input_kind == 0 else 1
+
+
+def run_reference(args):
+    """The CPU oracle as the reference arm: each step encodes a bounded prefix of one window."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle as O
+
+    O.lib()
+    cfg, vals = workload(args.workload)
+    threads = max(1, len(os.sched_getaffinity(0)))
+    tpv = O.tokens_per_value(cfg.input_kind, cfg.sep_mode)
+    positions = args.ref_positions
+    n_win = -(-vals.size * tpv // cfg.window)
+    for i in range(args.warmup):
+        oracle_sample(cfg, vals, 2, i % n_win, threads)
+    total_t, total_tok = 0.0, 0
+    for k in range(args.steps):
+        dt, n = oracle_sample(cfg, vals, positions, k % n_win, threads)
+        total_t += dt
+        total_tok += n
+    mbs = total_tok / tpv * bytes_per_value(cfg) / total_t / 1e6
+    sample = (f"oracle encode of the first {positions} tokens of one window per step (model forward over those "
+              f"positions in fp64, integer CDF, range coder), {args.steps} steps")
+    out = {"impl": "reference", "metric": METRIC, "value": mbs, "unit": "MB/s", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total_t / args.steps,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": args.workload, "window": cfg.window, "batch_windows": cfg.batch_windows},
+           "cpu_baseline": {"value": mbs, "unit": "MB/s", "cores": threads, "kind": "oracle", "sample": sample},
+           "e2e": {"value": mbs, "unit": "MB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="convnet-tinyllama", choices=WORKLOADS)
+    ap.add_argument("--batch-windows", type=int, default=0)
+    ap.add_argument("--ref-positions", type=int, default=12)
+    ap.add_argument("--cpu-target-s", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2409_17836_gb300 import configs, lmgc as L
+
+    cfg, vals = workload(args.workload)
+    if args.batch_windows:
+        cfg = configs.with_(cfg, batch_windows=args.batch_windows)
+    ctx = L.Context(cfg)
+    tpv = ctx.tpv
+    per_step = (cfg.batch_windows * cfg.window) // tpv  # values filling one model batch
+    n_slices = max(1, vals.size // per_step)
+    dev = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()
+    slices = [dev[i * per_step:(i + 1) * per_step] for i in range(n_slices)]
+    out = torch.empty(L.lmgc_encode_bound(ctx, per_step), dtype=torch.uint8, device="cuda")
+
+    def step(k):
+        return L.lmgc_encode(ctx, slices[(k + rank) % n_slices], out).numel()
+
+    for k in range(args.warmup):
+        step(k)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    L.lmgc_profile(ctx, True)
+    l0 = L.lmgc_launch_count()
+    sizes = []
+    with Clocks(local) as clk:
+        torch.cuda.synchronize()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record()
+        for k in range(args.steps):
+            sizes.append(step(k))
+        ev1.record()
+        torch.cuda.synchronize()
+    launches = L.lmgc_launch_count() - l0
+    stats = L.lmgc_kernel_stats(ctx)
+    L.lmgc_profile(ctx, False)
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    bpv = bytes_per_value(cfg)
+    raw_bytes = per_step * bpv * args.steps * world
+    value = raw_bytes / (ms / 1e3) / 1e6
+
+    # end to end through host buffers
+    hin = [torch.from_numpy((vals.view(np.int32) if vals.dtype == np.float32 else vals)[i * per_step:(i + 1) *
+                                                                                          per_step].copy()).pin_memory()
+           for i in range(min(n_slices, 4))]
+    hout = torch.empty(L.lmgc_encode_bound(ctx, per_step), dtype=torch.uint8).pin_memory()
+    L.lmgc_encode_host(ctx, hin[0], hout)
+    torch.cuda.synchronize()
+    d2h = 0
+    t0 = time.perf_counter()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for k in range(args.steps):
+        d2h += L.lmgc_encode_host(ctx, hin[k % len(hin)], hout)
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    e2e = {"value": per_step * bpv * args.steps * world / (e2e_ms / 1e3) / 1e6, "unit": "MB/s",
+           "h2d_bytes_per_step": per_step * bpv, "d2h_bytes_per_step": int(d2h / args.steps),
+           "wall_s": time.perf_counter() - t0}
+
+    pk = peaks()
+    g = stats["gemm"]
+    gemm_tflops = g["work"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else 0.0
+    roofline = {"bound": "tensor", "kernel": "gemm (all linear layers and the vocabulary projection)",
+                "achieved": gemm_tflops, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+                "frac": gemm_tflops / pk["bf16_sus"], "peak_kind": f"bf16 sustained ({pk['src']})",
+                "launches": g["launches"], "avg_launch_ms": g["ms"] / max(1, g["launches"]), "traffic": None}
+    stages = {}
+    for name, st in stats.items():
+        if st["launches"] == 0:
+            continue
+        e = {"launches": st["launches"], "ms": st["ms"], "share": st["ms"] / ms if ms else None}
+        if name in ("gemm", "attention") and st["ms"] > 0:
+            e.update(achieved=st["work"] / (st["ms"] / 1e3) / 1e12, unit="TFLOP/s")
+            e["frac"] = e["achieved"] / pk["bf16_sus"]
+        elif name in ("cdf_pairs", "range_encode", "serialize") and st["ms"] > 0:
+            e.update(achieved=st["work"] / (st["ms"] / 1e3) / 1e9, unit="GB/s")
+            e["frac"] = e["achieved"] / pk["hbm"]
+        stages[name] = e
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        threads = max(1, len(os.sched_getaffinity(0)))
+        dt, n = oracle_sample(cfg, vals, 4, 0, threads)
+        per_tok = dt / n
+        positions = int(max(4, min(cfg.window, args.cpu_target_s / max(per_tok, 1e-6))))
+        dt, n = oracle_sample(cfg, vals, positions, 0, threads)
+        cpu = {"value": n / tpv * bpv / dt / 1e6, "unit": "MB/s", "cores": threads, "kind": "oracle",
+               "sample": f"oracle encode (fp64 model forward, integer CDF, range coder) of the first {n} tokens "
+                         f"of window 0, {dt:.1f} s"}
+    if rank == 0:
+        res = {"metric": METRIC, "value": value, "unit": "MB/s", "n_gpus": world, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+               "vs_baseline": None, "dtype": "bf16" if cfg.dtype == L.BF16 else "f32",
+               "data": "synthetic (seeded random-init ConvNet gradients on Gaussian inputs; random-init model)",
+               "config": {"workload": args.workload, "values_per_step": per_step, "window": cfg.window,
+                          "batch_windows": cfg.batch_windows, "cdf_bits": cfg.cdf_bits,
+                          "model": f"{cfg.n_layers}L d{cfg.d_model} {cfg.n_heads}/{cfg.n_kv_heads}h "
+                                   f"ffn{cfg.d_ffn} V{cfg.vocab}",
+                          "l2": "no flush: each step reads > L2 (model weights and per-batch logits)",
+                          "parallelism": f"windows sharded over {world} GPU(s), no collective on the data path"},
+               "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
+               "stages": stages, "stage_ms_last_step": L.lmgc_stage_times(ctx),
+               "compression_rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv), "cpu_baseline": cpu}
+        print(json.dumps(res), flush=True)
+    ctx.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -180,6 +180,9 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
  * ms[2] CDF pairs, ms[3] coder, ms[4] container assembly. n_ms: capacity of ms. */
 lmgc_status lmgc_stage_times(const lmgc_ctx* ctx, float* ms, size_t n_ms);
 
+/* Number of kernels this library has launched in the process so far (all contexts). */
+lmgc_status lmgc_launch_count(uint64_t* n);
+
 /* Kernel-class timing for roofline reports. lmgc_profile(ctx, 1) clears the counters and starts
  * recording a CUDA event pair around every launch of the classes below on the launching stream;
  * lmgc_profile(ctx, 0) stops. lmgc_kernel_stats returns, for class cls, its name, the launches

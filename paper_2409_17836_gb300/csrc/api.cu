@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <atomic>
 #include <string>
 #include <vector>
 
@@ -14,6 +15,9 @@
 namespace lmgc {
 
 static thread_local std::string g_thread_err;
+static std::atomic<unsigned long long> g_launches{0};
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 void set_thread_error(const std::string& s) { g_thread_err = s; }
 
@@ -552,6 +556,7 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[2], s));
+  note_launch();
   k_fill_win_len<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(d_wl, n_win, W, n_tok);
   {
     ProfScope ps(ctx, kCoder, (double)n_tok * 8, s);
@@ -700,6 +705,7 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
     launch_dec_init(d_in, d_coff, d_bl, nd, d_state, s);
     uint16_t* out = d_tok + i0 * W;
     for (int64_t pos = 0; pos < max_len; pos++) {
+      note_launch();
       k_dec_inputs<<<(unsigned)((nd + 127) / 128), 128, 0, s>>>(out, nd, W, pos, ctx->ws.tok_in);
       launch_embed(ctx->ws.tok_in, nd, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
       forward_layers(ctx, nd, nd, true, pos, s);
@@ -714,6 +720,12 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   cudaStreamSynchronize(s);
   if (ctx->prof.enabled) prof_collect(ctx);
   return st;
+}
+
+lmgc_status lmgc_launch_count(uint64_t* n) {
+  if (!n) return LMGC_ERR_INVALID;
+  *n = g_launches.load(std::memory_order_relaxed);
+  return LMGC_OK;
 }
 
 lmgc_status lmgc_stage_times(const lmgc_ctx* ctx, float* ms, size_t n_ms) {

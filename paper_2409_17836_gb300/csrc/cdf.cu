@@ -208,6 +208,7 @@ void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uin
                       uint32_t* freq, int mode, cudaStream_t s) {
   if (rows <= 0) return;
   unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
+  note_launch();
   k_cdf_pairs<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win, pair_stride_pos,
                                              start, freq, mode);
 }
@@ -282,6 +283,7 @@ void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const 
                          cudaStream_t s) {
   if (rows <= 0) return;
   unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
+  note_launch();
   k_quantize_cdf<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, cdf);
 }
 
@@ -322,6 +324,7 @@ __global__ void k_dec_init(const uint8_t* __restrict__ codes, const uint64_t* __
 void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n, void* state,
                      cudaStream_t s) {
   if (n <= 0) return;
+  note_launch();
   k_dec_init<<<(unsigned)((n + 127) / 128), 128, 0, s>>>(codes, code_off, bitlen, n, (DecState*)state);
 }
 
@@ -401,6 +404,7 @@ void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint3
                         const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
                         const uint32_t* win_len, uint32_t* err, cudaStream_t s) {
   if (n <= 0) return;
+  note_launch();
   k_dec_search<<<(unsigned)n, kCdfThreads, 0, s>>>(logits, n, V, P, tab, (DecState*)dec_state, codes, sym_out,
                                                    sym_stride, pos, win_len, err);
 }

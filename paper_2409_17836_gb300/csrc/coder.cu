@@ -128,6 +128,7 @@ void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int
                          const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
                          size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
   if (n_win <= 0) return;
+  note_launch();
   k_range_encode<<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
                                                                   stride_win, stride_pos, slots, slot_sz, bitlen, err);
 }
@@ -186,9 +187,11 @@ __global__ void k_copy_codes(const uint8_t* __restrict__ slots, size_t slot_sz, 
 void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win, uint64_t* offsets,
                        uint8_t* out, cudaStream_t s) {
   if (n_win <= 0) return;
+  note_launch();
   k_scan_lengths<<<1, 1024, 0, s>>>(bitlen, n_win, offsets);
   if (out) {
     unsigned blocks = (unsigned)std::min<int64_t>(n_win, 152 * 16);
+    note_launch();
     k_copy_codes<<<blocks, 128, 0, s>>>(slots, slot_sz, bitlen, offsets, n_win, out);
   }
 }

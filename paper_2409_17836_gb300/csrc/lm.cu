@@ -57,6 +57,7 @@ void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int6
   float a = (float)((double)init_std * sqrt(3.0));
   int64_t total = rows * cols;
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 64);
+  note_launch();
   if (dtype == LMGC_BF16)
     k_init_weights<<<blocks, 256, 0, s>>>((__nv_bfloat16*)dst, seed, tid, rows, cols, ld, row_off, a);
   else
@@ -82,6 +83,7 @@ void launch_window_inputs(const uint16_t* tok, int64_t n_tok, int64_t first_win,
                           uint16_t* tok_in, cudaStream_t s) {
   int64_t total = n_win * W;
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
+  note_launch();
   k_window_inputs<<<blocks, 256, 0, s>>>(tok, n_tok, first_win, n_win, W, tok_in);
 }
 
@@ -97,6 +99,7 @@ __global__ void k_embed(const uint16_t* __restrict__ tok_in, int64_t rows, const
 
 void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, int dtype, float* x, cudaStream_t s) {
   if (rows <= 0) return;
+  note_launch();
   if (dtype == LMGC_BF16) k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const __nv_bfloat16*)E, d, x);
   else k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const float*)E, d, x);
 }
@@ -135,6 +138,7 @@ __global__ void __launch_bounds__(256) k_rmsnorm(const float* __restrict__ x, in
 
 void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, int dtype, cudaStream_t s) {
   if (rows <= 0) return;
+  note_launch();
   unsigned blocks = (unsigned)((rows + 7) / 8);
   if (dtype == LMGC_BF16) k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (__nv_bfloat16*)out);
   else k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (float*)out);
@@ -239,6 +243,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ A, cons
 void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
                       cudaStream_t s) {
   if (M <= 0 || N <= 0) return;
+  note_launch();
   dim3 grid((unsigned)((N + GBN - 1) / GBN), (unsigned)((M + GBM - 1) / GBM));
   if (dtype == LMGC_BF16)
     k_gemm_simt<<<grid, 256, 0, s>>>((const __nv_bfloat16*)A, (const __nv_bfloat16*)B, C, M, N, K, epi);
@@ -276,6 +281,7 @@ void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, 
   (void)n_pos;
   int64_t total = rows * n_rot_heads * (hd / 2);
   if (total <= 0) return;
+  note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
   if (dtype == LMGC_BF16)
     k_rope<<<blocks, 256, 0, s>>>((__nv_bfloat16*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
@@ -426,6 +432,7 @@ static void attn_launch(const void* q, int64_t q_stride, const void* kv, int64_t
   }
   dim3 grid((unsigned)((n_pos + ABQ - 1) / ABQ), (unsigned)nq, (unsigned)n_win);
   float scale = 1.0f / sqrtf((float)HD);
+  note_launch();
   k_attention<T, HD><<<grid, 256, smem, s>>>((const T*)q, q_stride, (const T*)kv, kv_stride, k_off, v_off, (T*)out,
                                              out_stride, nq, nkv, W, pos_first, n_pos, q_win_stride, scale);
 }
@@ -465,6 +472,7 @@ __global__ void k_swiglu(const T* __restrict__ gu, int64_t rows, int ffn, T* __r
 void launch_swiglu(const void* gu, int64_t rows, int ffn, void* act, int dtype, cudaStream_t s) {
   int64_t total = rows * ffn;
   if (total <= 0) return;
+  note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
   if (dtype == LMGC_BF16) k_swiglu<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)gu, rows, ffn, (__nv_bfloat16*)act);
   else k_swiglu<<<blocks, 256, 0, s>>>((const float*)gu, rows, ffn, (float*)act);
@@ -485,6 +493,7 @@ void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t ds
                       int64_t n_rows, int64_t row_elems, int dtype, cudaStream_t s) {
   int64_t total = n_rows * row_elems;
   if (total <= 0) return;
+  note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
   if (dtype == LMGC_BF16)
     k_copy_rows<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)src, src_stride, (__nv_bfloat16*)dst, dst_win_stride,

@@ -108,6 +108,9 @@ lmgc_status cuda_fail(lmgc_ctx* ctx, cudaError_t e, const char* what);
     if (e_ != cudaSuccess) return lmgc::cuda_fail(ctx, e_, #call); \
   } while (0)
 
+// Counts kernel launches of this library (every launcher calls it once per launch).
+void note_launch();
+
 // ---- kernels' launchers (stream-ordered, no sync) ----
 // serialize.cu
 int tokens_per_value(int input_kind, int sep_mode);

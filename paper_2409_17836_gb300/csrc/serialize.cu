@@ -93,6 +93,7 @@ static void ser_dispatch(bool vec, const void* in, int64_t n, uint16_t* tok, uin
 
 void launch_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* tok, cudaStream_t s) {
   if (n <= 0) return;
+  note_launch();
   uint16_t s0, s1;
   sep_ids(sep_mode, &s0, &s1);
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
@@ -136,6 +137,7 @@ void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64
   sep_ids(sep_mode, &s0, &s1);
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
   int nd = input_kind == LMGC_IN_F32 ? 8 : 2;
+  note_launch();
   k_deserialize<<<(unsigned)((n_values + 255) / 256), 256, 0, s>>>(tok, n_values, nd, ns, s0, s1, out, err);
 }
 

@@ -83,6 +83,7 @@ SYMBOLS = {
     "lmgc_decode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t,
                               C.c_void_p]),
     "lmgc_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t]),
+    "lmgc_launch_count": (C.c_int, [C.c_void_p]),
     "lmgc_profile": (C.c_int, [C.c_void_p, C.c_int]),
     "lmgc_kernel_stats": (C.c_int, [C.c_void_p, C.c_int, C.c_char_p, C.c_size_t, C.c_void_p, C.c_void_p,
                                     C.c_void_p]),
@@ -266,6 +267,12 @@ def lmgc_stage_times(ctx: Context) -> list[float]:
     ms = (C.c_float * 5)()
     _check(ctx, load().lmgc_stage_times(ctx.handle, ms, 5))
     return list(ms)
+
+
+def lmgc_launch_count() -> int:
+    n = C.c_uint64()
+    _check(None, load().lmgc_launch_count(C.byref(n)))
+    return n.value
 
 
 def lmgc_profile(ctx: Context, enable: bool) -> None:
