@@ -145,6 +145,24 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
                               uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
                               lmgc_stream stream);
 
+/* lmgc_range_encode for callers that cannot allocate device memory (for example a process whose
+ * device memory is held entirely by another allocator, or a latency-critical path where
+ * cudaMalloc / cudaFree, which may synchronise the device, are not allowed). The paper has no
+ * counterpart: this is a deployment variant of the coder above, with the same arguments, output
+ * and errors. It allocates nothing: its scratch (a 256-byte error word, the payload offsets and
+ * one code slot of slot(win_tokens, cdf_bits) = ceil((win_tokens*cdf_bits + 2) / 32 + 1) * 4 bytes,
+ * rounded up to 16, per window) lives in one fixed 64 MiB device array that every GPU loading the
+ * library keeps until exit. Calls needing more than 64 MiB of scratch (about 10,900 windows of
+ * 2048 tokens at cdf_bits 24) fail with INVALID and a message giving both sizes.
+ * The first call on a device looks up the array's device address (once per device, with that
+ * device current); make that first call before any stream capture. All calls share the array
+ * and it keeps the last call's contents: calls that overlap on the GPU (other streams, other host
+ * threads) race on it and must be serialised by the caller. Syncs. */
+lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                                      size_t win_tokens, const uint32_t* d_win_len, size_t stride_win,
+                                      size_t stride_pos, uint8_t* d_out, size_t cap, size_t* out_bytes,
+                                      uint32_t* d_bitlen, lmgc_stream stream);
+
 /* Largest container lmgc_encode can produce for n input values (header + length table + the
  * coder's worst case of cdf_bits bits per token + 2 bits per window). */
 lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);

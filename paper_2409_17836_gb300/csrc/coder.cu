@@ -17,6 +17,8 @@
 // start[w*stride_win + i*stride_pos]; with the encode path's position-major layout
 // (stride_win = 1) a warp's 32 loads of token i are one 128-byte transaction.
 #include <algorithm>
+#include <mutex>
+#include <string>
 
 #include "lmgc_internal.cuh"
 
@@ -196,4 +198,91 @@ void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bit
   }
 }
 
+// ------------------------------------------------------------------------------------------
+// Allocation-free variant of lmgc_range_encode.
+//
+// Some callers cannot allocate device memory at all: a process whose device memory is held
+// entirely by another allocator, or a latency-critical path on which cudaMalloc / cudaFree
+// (which may synchronise the device) are not allowed. For them the coder's scratch -- one code
+// slot per window, the payload offsets and an error word -- lives in the fixed array below
+// instead of being allocated per call. Every GPU that loads this library keeps the array
+// (kNoAllocScratchBytes) until the process exits.
+// ------------------------------------------------------------------------------------------
+constexpr size_t kNoAllocScratchBytes = 64ull << 20;  // 64 MiB
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+uint8_t* g_noalloc_ptr[kMaxDevices] = {};  // device address of the array, per device
+
+// In host code g_noalloc_scratch names a host-side stand-in, not device memory: the device
+// address is looked up once per device, with that device current.
+lmgc_status noalloc_scratch(uint8_t** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: device id");
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: cudaGetSymbolAddress");
+    g_noalloc_ptr[dev] = (uint8_t*)p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return LMGC_OK;
+}
+}  // namespace
+
 }  // namespace lmgc
+
+extern "C" lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits,
+                                                 size_t n_win, size_t win_tokens, const uint32_t* d_win_len,
+                                                 size_t stride_win, size_t stride_pos, uint8_t* d_out, size_t cap,
+                                                 size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream) {
+  using namespace lmgc;
+  if (!out_bytes || (n_win && (!d_start || !d_freq || !d_bitlen)))
+    return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: null argument");
+  if (cdf_bits < 1 || cdf_bits > 30)
+    return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: cdf_bits must be in 1..30");
+  *out_bytes = 0;
+  if (n_win == 0) return LMGC_OK;
+  // scratch layout: [0, 256) error word | offsets [n_win + 1] u64 | one code slot per window
+  const size_t slot = slot_bytes(win_tokens, cdf_bits);
+  const size_t off_bytes = ((n_win + 1) * 8 + 255) / 256 * 256;
+  const double need = 256.0 + (double)off_bytes + (double)slot * (double)n_win;
+  if (need > (double)kNoAllocScratchBytes)
+    return fail(nullptr, LMGC_ERR_INVALID,
+                "lmgc_range_encode_noalloc: needs " + std::to_string((unsigned long long)need) +
+                    " bytes of scratch (n_win * slot + offsets); the fixed maximum is " +
+                    std::to_string(kNoAllocScratchBytes) + " bytes");
+  uint8_t* base = nullptr;
+  lmgc_status st = noalloc_scratch(&base);
+  if (st != LMGC_OK) return st;
+  cudaStream_t s = (cudaStream_t)stream;
+  uint32_t* derr = (uint32_t*)base;
+  uint64_t* offs = (uint64_t*)(base + 256);
+  uint8_t* slots = base + 256 + off_bytes;
+  // the array keeps the previous call's contents: only the error word must start at zero (the
+  // slots are written before they are read and the offsets are recomputed)
+  cudaError_t e = cudaMemsetAsync(derr, 0, 4, s);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: clear");
+  launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
+                      (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
+  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
+  uint64_t total = 0;
+  uint32_t herr = 0;
+  cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
+  cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
+  e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc");
+  if (herr) return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: invalid (start, freq) or window length");
+  *out_bytes = total;
+  if (cap < total) return fail(nullptr, LMGC_ERR_NO_SPACE, "lmgc_range_encode_noalloc: output too small");
+  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s);
+  e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: pack");
+  return LMGC_OK;
+}

@@ -76,6 +76,9 @@ SYMBOLS = {
     "lmgc_cdf_pairs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "lmgc_range_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p, C.c_size_t,
                                     C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "lmgc_range_encode_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p,
+                                            C.c_size_t, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p,
+                                            C.c_void_p]),
     "lmgc_encode_bound": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     "lmgc_encode_host": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p,
@@ -226,6 +229,19 @@ def lmgc_range_encode(start: torch.Tensor, freq: torch.Tensor, cdf_bits: int, n_
                                   stride_pos, _ptr(out), out.numel(), C.byref(nbytes), _ptr(bitlen), _stream(stream))
     _check(None, st)
     return out[: nbytes.value], bitlen[:n_win]
+
+
+def lmgc_range_encode_noalloc(start: torch.Tensor, freq: torch.Tensor, cdf_bits: int, n_win: int, win_tokens: int,
+                              win_len: torch.Tensor | None, stride_win: int, stride_pos: int, out: torch.Tensor,
+                              bitlen: torch.Tensor, stream=None) -> int:
+    """The allocation-free coder: writes the codes into `out` and the bit lengths into `bitlen`
+    (both caller-owned device tensors); returns the payload bytes."""
+    nbytes = C.c_size_t()
+    st = load().lmgc_range_encode_noalloc(_ptr(start), _ptr(freq), cdf_bits, n_win, win_tokens, _ptr(win_len),
+                                          stride_win, stride_pos, _ptr(out), out.numel(), C.byref(nbytes),
+                                          _ptr(bitlen), _stream(stream))
+    _check(None, st)
+    return nbytes.value
 
 
 def lmgc_encode_bound(ctx: Context, n: int) -> int:
