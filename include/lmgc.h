@@ -114,6 +114,14 @@ lmgc_status lmgc_deserialize(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok,
 lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, size_t first_win, size_t n_win,
                           float* d_logits, lmgc_stream stream);
 
+/* The model's dense contraction (every linear layer of the Eq. 2 model and its vocabulary
+ * projection), exposed for parity tests of the GEMM kernels: C[M][N] (op)= A[M][K] . B[N][K]^T,
+ * A and B row-major in the context's dtype (bf16: the tcgen05 kernel; fp32: CUDA cores), fp32
+ * accumulation in k order. epi 0: C = result in the context's dtype; 1: fp32 C += result;
+ * 2: fp32 C = result. Errors: INVALID (K % 8 != 0, epi outside 0..2), LIMIT, CUDA. Syncs. */
+lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
+                      int epi, lmgc_stream stream);
+
 /* Integer CDF of each logit row (the coder input; the paper adapts Torchac, whose CDFs are
  * integers, Sec. 4.1). For a row z[0..V) with T = 2^P: m = max z; y_j = fp32(fp32(z_j - m) *
  * fp32(2^16 log2 e)); a_j = -rint(y_j) clamped to 40*2^16; e_j = 2^31 * 2^(-a_j/65536) in fixed

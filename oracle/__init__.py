@@ -375,3 +375,9 @@ def encode(cfg: OracleConfig, values: np.ndarray, n_par: int = 1) -> bytes:
 def compression_rate(container_bytes: int, n_values: int, bytes_per_value: int = 4) -> float:
     """Eq. 3: 100 * compressed size / original size."""
     return 100.0 * container_bytes / (bytes_per_value * n_values)
+
+
+def gemm_nt(a: np.ndarray, b: np.ndarray) -> np.ndarray:
+    """C = A . B^T in fp64 (the plain definition of the model's linear layers; a library matmul
+    serves as the step)."""
+    return np.asarray(a, dtype=np.float64) @ np.asarray(b, dtype=np.float64).T

@@ -113,7 +113,7 @@ static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M
                  cudaStream_t s) {
   ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
   if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K))
-    launch_gemm_tc(A, B, C, M, N, K, epi, s);
+    launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s);
   else
     launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);
 }
@@ -726,6 +726,20 @@ lmgc_status lmgc_launch_count(uint64_t* n) {
   if (!n) return LMGC_ERR_INVALID;
   *n = g_launches.load(std::memory_order_relaxed);
   return LMGC_OK;
+}
+
+lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
+                      int epi, lmgc_stream stream) {
+  if (!ctx || (M && N && (!d_a || !d_b || !d_c))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  if (K % 8 || epi < 0 || epi > 2) return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..2");
+  cudaStream_t s = (cudaStream_t)stream;
+  gemm(ctx, d_a, d_b, d_c, (int64_t)M, (int64_t)N, (int64_t)K, epi, s);
+  LMGC_CUDA(ctx, cudaGetLastError());
+  if (ctx->prof.enabled) {
+    cudaStreamSynchronize(s);
+    prof_collect(ctx);
+  }
+  return check_err_word(ctx, s, "gemm");
 }
 
 lmgc_status lmgc_stage_times(const lmgc_ctx* ctx, float* ms, size_t n_ms) {

@@ -1,10 +1,378 @@
-// gemm_tc.cu -- tensor-core (tcgen05) GEMM for the bf16 model.
+// gemm_tc.cu -- the model's dense contractions (the linear layers and the vocabulary projection of
+// the LM prior, Eq. 2) on the 5th-generation tensor cores: C[M][N] (op)= A[M][K] . B[N][K]^T,
+// bf16 operands, fp32 accumulation in tensor memory.
+//
+// Persistent, warp-specialised kernel, one CTA per SM (192 threads):
+//   warp 0      TMA producer: 128x64 A and 256x64 B tiles (128-byte swizzle) into a 4-stage ring
+//   warp 1      allocates 512 TMEM columns; one lane issues tcgen05.mma (M 128, N 256, K 16) and
+//               tcgen05.commit to the ring's empty barriers and to the accumulator-full barriers
+//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns, convert / add, store to global
+// Two 128x256 fp32 accumulators (2 x 256 TMEM columns) let the epilogue of one tile run under the
+// main loop of the next. Tiles are visited in groups of 16 M-blocks so the A and B tiles in
+// flight stay in L2.
+//
+// Row invariance (needed by the KV-cached decoder): every output element is accumulated over k
+// in the same order by the same MMA shape whatever M is; rows past M are zero-filled by TMA and
+// never stored.
+//
+// Every mbarrier wait is bounded (about 2 s of %globaltimer); on expiry the kernel records
+// kErrLimit, leaves its loops and still frees its tensor memory.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
 #include "lmgc_internal.cuh"
 
 namespace lmgc {
+namespace tc {
 
-bool tc_gemm_supported(int64_t, int64_t, int64_t) { return false; }
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int kThreads = 192;
+constexpr uint32_t A_BYTES = BM * BK * 2;  // 16 KiB
+constexpr uint32_t B_BYTES = BN * BK * 2;  // 32 KiB
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
+constexpr int GROUP_M = 16;
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
 
-void launch_gemm_tc(const void*, const void*, void*, int64_t, int64_t, int64_t, int, cudaStream_t) {}
+// instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1), B bf16 (10-12 = 1),
+// both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait for the phase with the given parity; false (and kErrLimit) after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
+  if (mbar_try(a, parity)) return true;
+  const uint64_t t0 = gtimer();
+  for (uint32_t i = 1; i < (1u << 28); ++i) {
+    if (mbar_try(a, parity)) return true;
+    if ((i & 127) == 0 && gtimer() - t0 > 2000000000ull) break;
+  }
+  atomicOr(err, kErrLimit);
+  return false;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          dst),
+      "l"((uint64_t)map), "r"(mbar), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar) : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
+          d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(IDESC), "r"(accumulate)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile written by TMA with the 128-byte
+// swizzle: rows of 64 bf16 (128 B), 8-row groups 1024 B apart (stride byte offset), leading
+// byte offset unused for swizzled K-major layouts, version 1, layout SWIZZLE_128B (2).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// 32 TMEM lanes x 32 columns of 32-bit: thread i of the warp gets lane (base + i), 32 columns.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+struct Params {
+  void* C;
+  int64_t M, N, K;
+  int tiles_m, tiles_n, num_kb;
+  uint32_t* err;
+};
+
+__device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int& nb) {
+  const int per_group = GROUP_M * p.tiles_n;
+  const int g = t / per_group;
+  const int first_m = g * GROUP_M;
+  const int gm = min(p.tiles_m - first_m, GROUP_M);
+  const int r = t - g * per_group;
+  mb = first_m + r % gm;
+  nb = r / gm;
+}
+
+template <int EPI>
+__device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t n0, const uint32_t (&r)[32]) {
+  if (EPI == kStore) {
+    __nv_bfloat16* c = reinterpret_cast<__nv_bfloat16*>(p.C) + m * p.N + n0;
+    if (n0 + 32 <= p.N && (p.N & 7) == 0) {
+      uint32_t w[16];
+#pragma unroll
+      for (int j = 0; j < 16; j++) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+        w[j] = *reinterpret_cast<uint32_t*>(&h);
+      }
+      uint4* d = reinterpret_cast<uint4*>(c);
+#pragma unroll
+      for (int j = 0; j < 4; j++) d[j] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; j++)
+        if (n0 + j < p.N) c[j] = __float2bfloat16_rn(__uint_as_float(r[j]));
+    }
+  } else {
+    float* c = reinterpret_cast<float*>(p.C) + m * p.N + n0;
+    if (n0 + 32 <= p.N && (p.N & 3) == 0) {
+      float4* d = reinterpret_cast<float4*>(c);
+#pragma unroll
+      for (int j = 0; j < 8; j++) {
+        float4 v = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
+                               __uint_as_float(r[4 * j + 3]));
+        if (EPI == kAddResidual) {
+          float4 o = d[j];
+          v.x += o.x;
+          v.y += o.y;
+          v.z += o.z;
+          v.w += o.w;
+        }
+        d[j] = v;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; j++)
+        if (n0 + j < p.N) c[j] = (EPI == kAddResidual ? c[j] : 0.f) + __uint_as_float(r[j]);
+    }
+  }
+}
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  const uint32_t smem_base = smem_u32(smem);
+  auto sA = [&](int s) { return smem_base + (uint32_t)s * STAGE_BYTES; };
+  auto sB = [&](int s) { return smem_base + (uint32_t)s * STAGE_BYTES + A_BYTES; };
+  auto full = [&](int s) { return smem_u32(bars + s); };
+  auto empty = [&](int s) { return smem_u32(bars + STAGES + s); };
+  auto tfull = [&](int a) { return smem_u32(bars + 2 * STAGES + a); };
+  auto tempty = [&](int a) { return smem_u32(bars + 2 * STAGES + 2 + a); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; s++) {
+      mbar_init(full(s), 1);
+      mbar_init(empty(s), 1);
+    }
+    for (int a = 0; a < 2; a++) {
+      mbar_init(tfull(a), 1);
+      mbar_init(tempty(a), 128);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int n_tiles = p.tiles_m * p.tiles_n;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    uint32_t g = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      int mb, nb;
+      tile_coords(t, p, mb, nb);
+      for (int kb = 0; kb < p.num_kb; ++kb, ++g) {
+        const int s = (int)(g % STAGES);
+        const uint32_t ph = (g / STAGES) & 1u;
+        ok = __all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u, p.err));
+        if (!ok) break;
+        if (lane == 0) {
+          mbar_expect_tx(full(s), STAGE_BYTES);
+          tma_load_2d(sA(s), &tma_a, full(s), kb * BK, mb * BM);
+          tma_load_2d(sB(s), &tma_b, full(s), kb * BK, nb * BN);
+        }
+        __syncwarp();
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    uint32_t g = 0;
+    int i = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+      const int a = i & 1;
+      const uint32_t aph = (uint32_t)(i >> 1) & 1u;
+      ok = __all_sync(0xffffffffu, mbar_wait(tempty(a), aph ^ 1u, p.err));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t d = tmem + (uint32_t)(a * BN);
+      for (int kb = 0; kb < p.num_kb; ++kb, ++g) {
+        const int s = (int)(g % STAGES);
+        const uint32_t ph = (g / STAGES) & 1u;
+        ok = __all_sync(0xffffffffu, mbar_wait(full(s), ph, p.err));
+        if (!ok) break;
+        tc_fence_after();
+        if (lane == 0) {
+          const uint64_t da = sw128_desc(sA(s)), db = sw128_desc(sB(s));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), (kb > 0 || k > 0) ? 1u : 0u);
+          tc_commit(empty(s));
+        }
+        __syncwarp();
+      }
+      if (lane == 0) tc_commit(tfull(a));
+      __syncwarp();
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int q = warp & 3;  // TMEM lanes 32q .. 32q+31
+    int i = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+      int mb, nb;
+      tile_coords(t, p, mb, nb);
+      const int a = i & 1;
+      const uint32_t aph = (uint32_t)(i >> 1) & 1u;
+      if (!__all_sync(0xffffffffu, mbar_wait(tfull(a), aph, p.err))) break;
+      tc_fence_after();
+      const int64_t m = (int64_t)mb * BM + q * 32 + lane;
+      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tbase + (uint32_t)(c * 32), r);
+        const int64_t n0 = (int64_t)nb * BN + c * 32;
+        if (m < p.M && n0 < p.N) store_chunk<EPI>(p, m, n0, r);
+      }
+      tc_fence_before();
+      mbar_arrive(tempty(a));
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+  }
+}
+
+// ---------------- host side ----------------
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static std::once_flag g_once;
+static int g_num_sms = 0;
+
+static void init_once() {
+  cudaDriverEntryPointQueryResult q;
+  void* fn = nullptr;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (major != 10) g_encode = nullptr;  // tcgen05 path only on Blackwell-class devices
+  cudaFuncSetAttribute(k_gemm_tc<kStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+}
+
+static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t rows, uint32_t box_rows) {
+  cuuint64_t dims[2] = {k, rows};
+  cuuint64_t strides[1] = {k * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace tc
+
+bool tc_gemm_supported(int64_t M, int64_t N, int64_t K) {
+  std::call_once(tc::g_once, tc::init_once);
+  return tc::g_encode != nullptr && M > 0 && N > 0 && K > 0 && K % 8 == 0 && M < (1ll << 31) && N < (1ll << 31);
+}
+
+void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
+                    cudaStream_t s) {
+  using namespace tc;
+  std::call_once(g_once, init_once);
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) {
+    set_thread_error("cuTensorMapEncodeTiled failed");
+    return;
+  }
+  Params p;
+  p.C = C;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.tiles_m = (int)((M + BM - 1) / BM);
+  p.tiles_n = (int)((N + BN - 1) / BN);
+  p.num_kb = (int)((K + BK - 1) / BK);
+  p.err = err;
+  const int tiles = p.tiles_m * p.tiles_n;
+  const int grid = std::max(1, std::min(tiles, g_num_sms));
+  note_launch();
+  if (epi == kStore) k_gemm_tc<kStore><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else if (epi == kAddResidual) k_gemm_tc<kAddResidual><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else k_gemm_tc<kStoreF32><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+}
 
 }  // namespace lmgc

@@ -162,6 +162,7 @@ void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint3
 
 // gemm_tc.cu (tcgen05)
 bool tc_gemm_supported(int64_t M, int64_t N, int64_t K);
-void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, cudaStream_t s);
+void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
+                    cudaStream_t s);
 
 }  // namespace lmgc

@@ -73,6 +73,8 @@ SYMBOLS = {
                                    C.c_void_p]),
     "lmgc_lm_probs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_size_t, C.c_size_t, C.c_void_p, C.c_void_p]),
     "lmgc_quantize_cdf": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
+    "lmgc_gemm": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_size_t, C.c_size_t, C.c_int,
+                            C.c_void_p]),
     "lmgc_cdf_pairs": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "lmgc_range_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p, C.c_size_t,
                                     C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -193,6 +195,14 @@ def lmgc_lm_probs(ctx: Context, tokens: torch.Tensor, first_win: int, n_win: int
     _check(ctx, load().lmgc_lm_probs(ctx.handle, _ptr(tokens), tokens.numel(), first_win, n_win, _ptr(logits),
                                      _stream(stream)))
     return logits
+
+
+def lmgc_gemm(ctx: Context, a: torch.Tensor, b: torch.Tensor, c: torch.Tensor, epi: int, stream=None) -> torch.Tensor:
+    """c (op)= a @ b.T; a [M][K], b [N][K] in the context's dtype; c per epi (0: dtype, 1/2: fp32)."""
+    M, K = a.shape
+    N = b.shape[0]
+    _check(ctx, load().lmgc_gemm(ctx.handle, _ptr(a), _ptr(b), _ptr(c), M, N, K, epi, _stream(stream)))
+    return c
 
 
 def lmgc_quantize_cdf(ctx: Context, logits: torch.Tensor, stream=None) -> torch.Tensor:

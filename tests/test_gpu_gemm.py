@@ -1,0 +1,89 @@
+"""The model's dense contraction (lmgc_gemm): C = A . B^T for the linear layers and the
+vocabulary projection of the Eq. 2 model. bf16 operands on the tcgen05 kernel, fp32 on CUDA
+cores; compared with the fp64 definition. Bound per element: fp32 accumulation error
+<= 2^-22 * sum_k |a_k b_k| (plus one bf16 rounding of the output for epilogue 0)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2409_17836_gb300 import configs, lmgc as L
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx_bf16():
+    c = L.Context(L.ModelConfig(n_layers=1, d_model=64, n_heads=1, n_kv_heads=1, d_ffn=64, vocab=32, dtype=L.BF16,
+                                window=64, cdf_bits=16))
+    yield c
+    c.close()
+
+
+def run(ctx, M, N, K, epi, seed=0, scale=1.0):
+    g = torch.Generator().manual_seed(seed)
+    a = (torch.randn(M, K, generator=g) * scale).to(torch.bfloat16)
+    b = (torch.randn(N, K, generator=g) * scale).to(torch.bfloat16)
+    c0 = torch.randn(M, N, generator=g)
+    if epi == 0:
+        c = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    else:
+        c = c0.clone().cuda()
+    L.lmgc_gemm(ctx, a.cuda(), b.cuda(), c, epi)
+    af, bf = a.float().numpy(), b.float().numpy()
+    ref = O.gemm_nt(af, bf)
+    bound = 2.0 ** -22 * O.gemm_nt(np.abs(af), np.abs(bf)) + 1e-30
+    if epi == 1:
+        ref = ref + c0.numpy().astype(np.float64)
+        bound += 2.0 ** -23 * np.abs(ref)
+    got = c.float().cpu().numpy().astype(np.float64)
+    if epi == 0:
+        bound += 2.0 ** -8 * np.abs(ref)
+    err = np.abs(got - ref)
+    assert np.all(err <= bound), float((err / bound).max())
+    return c
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 136), (1, 256, 2048), (7, 2560, 2048),
+                                   (1000, 2048, 5632), (2048, 32000, 2048)])
+@pytest.mark.parametrize("epi", [0, 1, 2])
+def test_gemm_tc_shapes(ctx_bf16, M, N, K, epi):
+    if M * N > 2048 * 32000 // 2 and epi != 2:
+        pytest.skip("the vocabulary shape is checked with the fp32 epilogue only")
+    run(ctx_bf16, M, N, K, epi, seed=M + N + K)
+
+
+def test_gemm_tc_row_invariance(ctx_bf16):
+    """A row's result does not depend on M or on the row's place in a tile (the decoder relies on
+    this): rows computed alone equal the same rows inside a 1000-row product, bit for bit."""
+    g = torch.Generator().manual_seed(5)
+    a = torch.randn(1000, 2048, generator=g).to(torch.bfloat16).cuda()
+    b = torch.randn(2560, 2048, generator=g).to(torch.bfloat16).cuda()
+    full = torch.empty(1000, 2560, device="cuda")
+    L.lmgc_gemm(ctx_bf16, a, b, full, 2)
+    for r in [0, 1, 127, 128, 517, 999]:
+        one = torch.empty(1, 2560, device="cuda")
+        L.lmgc_gemm(ctx_bf16, a[r:r + 1].contiguous(), b, one, 2)
+        assert torch.equal(one[0], full[r]), r
+    part = torch.empty(3, 2560, device="cuda")
+    L.lmgc_gemm(ctx_bf16, a[517:520].contiguous(), b, part, 2)
+    assert torch.equal(part, full[517:520])
+
+
+def test_gemm_fp32_simt():
+    ctx = L.Context(configs.with_(configs.TINY, batch_windows=1))
+    g = torch.Generator().manual_seed(1)
+    a = torch.randn(300, 136, generator=g)
+    b = torch.randn(520, 136, generator=g)
+    c = torch.empty(300, 520, device="cuda")
+    L.lmgc_gemm(ctx, a.cuda(), b.cuda(), c, 2)
+    ref = O.gemm_nt(a.numpy(), b.numpy())
+    bound = 2.0 ** -22 * O.gemm_nt(np.abs(a.numpy()), np.abs(b.numpy()))
+    assert np.all(np.abs(c.cpu().numpy() - ref) <= bound)
+    ctx.close()
+
+
+def test_gemm_rejects_bad_k(ctx_bf16):
+    a = torch.zeros(4, 12, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(L.LmgcError):
+        L.lmgc_gemm(ctx_bf16, a, a, torch.zeros(4, 4, device="cuda"), 2)
