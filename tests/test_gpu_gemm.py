@@ -2,8 +2,8 @@
 vocabulary projection of the Eq. 2 model. bf16 operands on the tcgen05 kernel, fp32 on CUDA
 cores; compared with the fp64 definition. Bound per element: accumulation error
 <= 2^-19 * sum_k |a_k b_k| on the tensor cores (their fp32 accumulation aligns products
-with truncation, measured at up to 1.4 x 2^-22 * sum |a b|), 2^-22 * sum |a b| on CUDA
-cores; plus one bf16 rounding of the output for epilogue 0."""
+with truncation, measured at up to 1.4 x 2^-22 * sum |a b|), and the standard bound of sequential fp32 summation,
+K * 2^-24 * sum |a b|, on CUDA cores; plus one bf16 rounding of the output for epilogue 0."""
 import numpy as np
 import pytest
 import torch
@@ -80,7 +80,7 @@ def test_gemm_fp32_simt():
     c = torch.empty(300, 520, device="cuda")
     L.lmgc_gemm(ctx, a.cuda(), b.cuda(), c, 2)
     ref = O.gemm_nt(a.numpy(), b.numpy())
-    bound = 2.0 ** -22 * O.gemm_nt(np.abs(a.numpy()), np.abs(b.numpy()))
+    bound = 136 * 2.0 ** -24 * O.gemm_nt(np.abs(a.numpy()), np.abs(b.numpy()))
     assert np.all(np.abs(c.cpu().numpy() - ref) <= bound)
     ctx.close()
 
