@@ -118,7 +118,10 @@ lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, si
  * projection), exposed for parity tests of the GEMM kernels: C[M][N] (op)= A[M][K] . B[N][K]^T,
  * A and B row-major in the context's dtype (bf16: the tcgen05 kernel; fp32: CUDA cores), fp32
  * accumulation in k order. epi 0: C = result in the context's dtype; 1: fp32 C += result;
- * 2: fp32 C = result. Errors: INVALID (K % 8 != 0, epi outside 0..2), LIMIT, CUDA. Syncs. */
+ * 2: fp32 C = result; 3 (bf16, N % 256 == 0): the SwiGLU MLP input -- B's rows hold gate and up
+ * rows interleaved in 128-row blocks (rows 256t..256t+127 gate, 256t+128..256t+255 up) and
+ * C[M][N/2] (bf16) = silu(gate) * up, i.e. C[m][128t+j] = silu(R[m][256t+j]) * R[m][256t+128+j].
+ * Errors: INVALID (K % 8 != 0, epi outside 0..3, epi 3 unsupported), LIMIT, CUDA. Syncs. */
 lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
                       int epi, lmgc_stream stream);
 

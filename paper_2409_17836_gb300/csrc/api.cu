@@ -112,10 +112,10 @@ static void prof_collect(lmgc_ctx* ctx) {
 static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi,
                  cudaStream_t s) {
   ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
-  if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K))
+  if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi))
     launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s);
   else
-    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);
+    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);  // kSwiGLU never reaches here
 }
 
 static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, int64_t n_win, int64_t pos_first,
@@ -162,8 +162,10 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
       ProfScope ps(ctx, kNorm, 0, s);
       launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
     }
-    gemm(ctx, ws.n, L.wgu, ws.gu, rows, 2 * (int64_t)F, d, kStore, s);
-    {
+    if (ctx->fused_swiglu) {
+      gemm(ctx, ws.n, L.wgu, ws.act, rows, 2 * (int64_t)F, d, kSwiGLU, s);
+    } else {
+      gemm(ctx, ws.n, L.wgu, ws.gu, rows, 2 * (int64_t)F, d, kStore, s);
       ProfScope ps(ctx, kNorm, 0, s);
       launch_swiglu(ws.gu, rows, F, ws.act, c.dtype, s);
     }
@@ -295,6 +297,7 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
   const char* tc_env = getenv("LMGC_DISABLE_TC");
   ctx->use_tc = !(tc_env && tc_env[0] == '1');
+  ctx->fused_swiglu = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_ffn % 128 == 0 && tc_gemm_supported(1, 2 * c.d_ffn, c.d_model, kSwiGLU);
   const int64_t d = c.d_model, F = c.d_ffn, V = c.vocab, qd = (int64_t)c.n_heads * hd;
   const size_t e = ctx->elt;
   // weights: one blob, every tensor 256-byte aligned
@@ -338,8 +341,13 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
     launch_init_weights(L.wqkv, dt, seed, t + 2, (int64_t)c.n_kv_heads * hd, d, d,
                         qd + (int64_t)c.n_kv_heads * hd, c.init_std, s);
     launch_init_weights(L.wo, dt, seed, t + 3, d, qd, qd, 0, c.init_std, s);
-    launch_init_weights(L.wgu, dt, seed, t + 4, F, d, d, 0, c.init_std, s);
-    launch_init_weights(L.wgu, dt, seed, t + 5, F, d, d, F, c.init_std, s);
+    if (ctx->fused_swiglu) {  // gate/up interleaved in 128-row blocks
+      launch_init_weights(L.wgu, dt, seed, t + 4, F, d, d, 0, c.init_std, s, 128, 256);
+      launch_init_weights(L.wgu, dt, seed, t + 5, F, d, d, 128, c.init_std, s, 128, 256);
+    } else {
+      launch_init_weights(L.wgu, dt, seed, t + 4, F, d, d, 0, c.init_std, s);
+      launch_init_weights(L.wgu, dt, seed, t + 5, F, d, d, F, c.init_std, s);
+    }
     launch_init_weights(L.wdown, dt, seed, t + 6, d, F, F, 0, c.init_std, s);
   }
   launch_init_weights(ctx->w_head, dt, seed, 1 + 7 * c.n_layers, V, d, d, 0, c.init_std, s);
@@ -367,7 +375,7 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (err == cudaSuccess) err = dmalloc(&ws.qkv, R * ctx->qkv_dim * e);
   if (err == cudaSuccess) err = dmalloc(&ws.att, R * qd * e);
   if (err == cudaSuccess) err = dmalloc(&ws.act, R * F * e);
-  if (err == cudaSuccess) err = dmalloc(&ws.gu, R * 2 * F * e);
+  if (err == cudaSuccess && !ctx->fused_swiglu) err = dmalloc(&ws.gu, R * 2 * F * e);
   if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
   if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
   for (int i = 0; i < 6 && err == cudaSuccess; i++) err = cudaEventCreate(&ctx->ev[i]);
@@ -731,7 +739,9 @@ lmgc_status lmgc_launch_count(uint64_t* n) {
 lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
                       int epi, lmgc_stream stream) {
   if (!ctx || (M && N && (!d_a || !d_b || !d_c))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
-  if (K % 8 || epi < 0 || epi > 2) return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..2");
+  if (K % 8 || epi < 0 || epi > 3) return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..3");
+  if (epi == kSwiGLU && !(ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi)))
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epi 3 needs the bf16 tensor-core path and N % 256 == 0");
   cudaStream_t s = (cudaStream_t)stream;
   gemm(ctx, d_a, d_b, d_c, (int64_t)M, (int64_t)N, (int64_t)K, epi, s);
   LMGC_CUDA(ctx, cudaGetLastError());

@@ -289,12 +289,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const int64_t m = (int64_t)mb * BM + q * 32 + lane;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);
+      if (EPI == kSwiGLU) {
+        // columns [0, 128) of the tile are gate, [128, 256) the matching up columns
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tbase + (uint32_t)(c * 32), r);
-        const int64_t n0 = (int64_t)nb * BN + c * 32;
-        if (m < p.M && n0 < p.N) store_chunk<EPI>(p, m, n0, r);
+        for (int c = 0; c < BN / 64; ++c) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tbase + (uint32_t)(c * 32), g);
+          tmem_ld32(tbase + (uint32_t)(BN / 2 + c * 32), u);
+          if (m < p.M) {
+            const int64_t half_n = p.N / 2;
+            __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.C) + m * half_n + (int64_t)nb * (BN / 2) + c * 32;
+            uint32_t w[16];
+#pragma unroll
+            for (int j = 0; j < 16; j++) {
+              const float g0 = __uint_as_float(g[2 * j]), g1 = __uint_as_float(g[2 * j + 1]);
+              const float a0 = g0 / (1.f + expf(-g0)) * __uint_as_float(u[2 * j]);
+              const float a1 = g1 / (1.f + expf(-g1)) * __uint_as_float(u[2 * j + 1]);
+              __nv_bfloat162 h = __floats2bfloat162_rn(a0, a1);
+              w[j] = *reinterpret_cast<uint32_t*>(&h);
+            }
+            uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+            for (int j = 0; j < 4; j++) d4[j] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tbase + (uint32_t)(c * 32), r);
+          const int64_t n0 = (int64_t)nb * BN + c * 32;
+          if (m < p.M && n0 < p.N) store_chunk<EPI>(p, m, n0, r);
+        }
       }
       tc_fence_before();
       mbar_arrive(tempty(a));
@@ -329,6 +355,7 @@ static void init_once() {
   cudaFuncSetAttribute(k_gemm_tc<kStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaFuncSetAttribute(k_gemm_tc<kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
 }
 
 static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t rows, uint32_t box_rows) {
@@ -344,8 +371,9 @@ static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t row
 
 }  // namespace tc
 
-bool tc_gemm_supported(int64_t M, int64_t N, int64_t K) {
+bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi) {
   std::call_once(tc::g_once, tc::init_once);
+  if (epi == kSwiGLU && N % tc::BN != 0) return false;
   return tc::g_encode != nullptr && M > 0 && N > 0 && K > 0 && K % 8 == 0 && M < (1ll << 31) && N < (1ll << 31);
 }
 
@@ -372,7 +400,8 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   note_launch();
   if (epi == kStore) k_gemm_tc<kStore><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
   else if (epi == kAddResidual) k_gemm_tc<kAddResidual><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else k_gemm_tc<kStoreF32><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else if (epi == kStoreF32) k_gemm_tc<kStoreF32><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else k_gemm_tc<kSwiGLU><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
 }
 
 }  // namespace lmgc

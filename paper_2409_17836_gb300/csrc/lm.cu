@@ -40,7 +40,7 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t x) {
 
 template <typename T>
 __global__ void k_init_weights(T* __restrict__ dst, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols,
-                               int64_t ld, int64_t row_off, float a) {
+                               int64_t ld, int64_t row_off, int64_t rblk, int64_t rstride, float a) {
   const int64_t total = rows * cols;
   for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
@@ -48,20 +48,25 @@ __global__ void k_init_weights(T* __restrict__ dst, uint64_t seed, uint32_t tid,
     float unit = (float)((int32_t)u - (1 << 23)) * (1.0f / 8388608.0f);
     float w = __fmul_rn(unit, a);
     int64_t r = idx / cols, c = idx - r * cols;
-    dst[(row_off + r) * ld + c] = from_f<T>(w);
+    const int64_t dr = row_off + (r / rblk) * rstride + r % rblk;
+    dst[dr * ld + c] = from_f<T>(w);
   }
 }
 
 void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols, int64_t ld,
-                         int64_t row_off, float init_std, cudaStream_t s) {
+                         int64_t row_off, float init_std, cudaStream_t s, int64_t rblk, int64_t rstride) {
+  if (rblk <= 0) {
+    rblk = rows;
+    rstride = 0;
+  }
   float a = (float)((double)init_std * sqrt(3.0));
   int64_t total = rows * cols;
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 64);
   note_launch();
   if (dtype == LMGC_BF16)
-    k_init_weights<<<blocks, 256, 0, s>>>((__nv_bfloat16*)dst, seed, tid, rows, cols, ld, row_off, a);
+    k_init_weights<<<blocks, 256, 0, s>>>((__nv_bfloat16*)dst, seed, tid, rows, cols, ld, row_off, rblk, rstride, a);
   else
-    k_init_weights<<<blocks, 256, 0, s>>>((float*)dst, seed, tid, rows, cols, ld, row_off, a);
+    k_init_weights<<<blocks, 256, 0, s>>>((float*)dst, seed, tid, rows, cols, ld, row_off, rblk, rstride, a);
 }
 
 // ------------------------------------------------------------------------------------------

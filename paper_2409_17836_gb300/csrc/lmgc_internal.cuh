@@ -91,7 +91,8 @@ struct lmgc_ctx {
   cudaEvent_t ev[6] = {};
   std::vector<cudaEvent_t> batch_ev;
   lmgc::Profiler prof;
-  bool use_tc = true;  // tcgen05 GEMM for bf16 models when available
+  bool use_tc = true;        // tcgen05 GEMM for bf16 models when available
+  bool fused_swiglu = false;  // gate/up interleaved, SwiGLU in the tcgen05 epilogue
   std::string err;
 };
 
@@ -119,14 +120,18 @@ void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64
                         uint32_t* err, cudaStream_t s);
 
 // lm.cu
+// Canonical row r of tensor tid goes to dst row row_off + (r / rblk) * rstride + r % rblk
+// (rblk <= 0: dst row row_off + r).
 void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols, int64_t ld,
-                         int64_t row_off, float init_std, cudaStream_t s);
+                         int64_t row_off, float init_std, cudaStream_t s, int64_t rblk = 0, int64_t rstride = 0);
 void launch_window_inputs(const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t n_win, int W,
                           uint16_t* tok_in, cudaStream_t s);
 void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, int dtype, float* x, cudaStream_t s);
 void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, int dtype, cudaStream_t s);
 // C[M][N] = A[M][K] . B[N][K]^T with the given epilogue
-enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2 };
+// kSwiGLU: B's rows are gate/up blocks interleaved 128 by 128 (rows 256t..256t+127 = gate rows
+// 128t.., rows 256t+128.. = up rows 128t..); C[m][128t + j] = silu(gate) * up, N/2 columns.
+enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3 };
 void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
                       cudaStream_t s);
 void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
@@ -161,7 +166,7 @@ void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint3
                      void* state, cudaStream_t s);
 
 // gemm_tc.cu (tcgen05)
-bool tc_gemm_supported(int64_t M, int64_t N, int64_t K);
+bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi = 0);
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
                     cudaStream_t s);
 

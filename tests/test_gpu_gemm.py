@@ -89,3 +89,28 @@ def test_gemm_rejects_bad_k(ctx_bf16):
     a = torch.zeros(4, 12, dtype=torch.bfloat16, device="cuda")
     with pytest.raises(L.LmgcError):
         L.lmgc_gemm(ctx_bf16, a, a, torch.zeros(4, 4, device="cuda"), 2)
+
+
+@pytest.mark.parametrize("M,F,K", [(300, 512, 136), (1, 5632, 2048), (1000, 1408, 2048)])
+def test_gemm_tc_swiglu_epilogue(ctx_bf16, M, F, K):
+    """Epilogue 3: gate/up rows interleaved in 128-row blocks, C = silu(gate) * up in bf16."""
+    g = torch.Generator().manual_seed(F + M)
+    a = torch.randn(M, K, generator=g).to(torch.bfloat16)
+    wg = (torch.randn(F, K, generator=g) * 0.05).to(torch.bfloat16)
+    wu = (torch.randn(F, K, generator=g) * 0.05).to(torch.bfloat16)
+    inter = torch.empty(2 * F, K, dtype=torch.bfloat16)
+    for t in range(F // 128):
+        inter[256 * t: 256 * t + 128] = wg[128 * t: 128 * t + 128]
+        inter[256 * t + 128: 256 * t + 256] = wu[128 * t: 128 * t + 128]
+    c = torch.empty(M, F, dtype=torch.bfloat16, device="cuda")
+    L.lmgc_gemm(ctx_bf16, a.cuda(), inter.cuda(), c, 3)
+    af = a.float().numpy()
+    gr = O.gemm_nt(af, wg.float().numpy())
+    ur = O.gemm_nt(af, wu.float().numpy())
+    ref = O.swiglu(gr, ur)
+    eg = 2.0 ** -19 * O.gemm_nt(np.abs(af), np.abs(wg.float().numpy()))
+    eu = 2.0 ** -19 * O.gemm_nt(np.abs(af), np.abs(wu.float().numpy()))
+    silu = gr / (1 + np.exp(-gr))
+    bound = 1.1 * np.abs(ur) * eg + np.abs(silu) * eu + 2.0 ** -8 * np.abs(ref) + 1e-30
+    err = np.abs(c.float().cpu().numpy() - ref)
+    assert np.all(err <= bound), float((err / bound).max())
