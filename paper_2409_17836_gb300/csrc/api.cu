@@ -126,8 +126,14 @@ static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, i
   for (int64_t p = pos_first; p < pos_first + n_pos; p++) pairs += (double)(p + 1);
   ProfScope ps(ctx, kAttn, 4.0 * ctx->hd * c.n_heads * pairs * (double)n_win, s);
   const int qd = c.n_heads * ctx->hd, kd = c.n_kv_heads * ctx->hd;
-  launch_attention(q, ctx->qkv_dim, kv, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads, c.n_kv_heads, ctx->hd,
-                   c.window, n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
+  if (c.dtype == LMGC_BF16 && ctx->use_tc && tc_attention_supported(ctx->hd, ctx->qkv_dim)) {
+    const int64_t q_rows = q_win_stride == 1 ? n_win : n_win * c.window;
+    launch_attention_tc(q, q_rows, kv, n_win * c.window, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads,
+                        c.n_kv_heads, ctx->hd, c.window, n_win, pos_first, n_pos, q_win_stride, ctx->d_err, s);
+  } else {
+    launch_attention(q, ctx->qkv_dim, kv, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads, c.n_kv_heads, ctx->hd,
+                     c.window, n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
+  }
 }
 
 // One forward of the model over `rows` input rows already embedded into ws.x.
@@ -684,7 +690,11 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   const size_t kv_per_win = (size_t)std::max(1, c.n_layers) * W * ctx->qkv_dim * ctx->elt;
   const int64_t nd_max = std::max<int64_t>(1, std::min<int64_t>(c.batch_windows, (int64_t)((16ull << 30) / kv_per_win)));
   const size_t kv_need = kv_per_win * (size_t)nd_max;
-  LMGC_CUDA(ctx, ensure(&ctx->kv_cache, &ctx->kv_cap, kv_need));
+  if (ctx->kv_cap < kv_need || !ctx->kv_cache) {
+    LMGC_CUDA(ctx, ensure(&ctx->kv_cache, &ctx->kv_cap, kv_need));
+    // keys/values past a decoded position are read (and multiplied by probability 0): keep them finite
+    LMGC_CUDA(ctx, cudaMemsetAsync(ctx->kv_cache, 0, ctx->kv_cap, s));
+  }
   // per-chunk device arrays: code offsets, bit lengths, lengths, decoder states
   void* dev = nullptr;
   const size_t st_bytes = dec_state_bytes();

@@ -1,0 +1,408 @@
+// attn_tc.cu -- causal softmax attention of the LM prior (Eq. 2's Llama decoder) on the
+// 5th-generation tensor cores, bf16 inputs, fp32 softmax and accumulation.
+//
+// One CTA per (128 query rows, query head, window); 192 threads:
+//   warp 0      TMA: the Q tile once, then 64-key K and V blocks into a 2-stage ring
+//   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64) and O_blk = P V
+//               (M 128, N hd, V as an MN-major operand) and commits to mbarriers
+//   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
+//               per-thread loops; P is written as bf16 into shared memory in the 128-byte
+//               swizzled K-major layout the MMA reads; the running output O stays in registers
+//               and is rescaled by the online-softmax correction before each block's P V is added.
+// Key blocks are 64-aligned and visited in order 0, 1, ...; a block whose keys all lie past a
+// row's position leaves that row's state exactly unchanged (correction 1, P = 0). A decode step
+// (one query row per window, keys from the cache) therefore reproduces the prefill row bit for
+// bit: the tensor cores' row results do not depend on the other rows of the tile.
+// Every mbarrier wait is bounded (~2 s), after which kErrLimit is recorded and the loops end.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "lmgc_internal.cuh"
+
+namespace lmgc {
+namespace attn {
+
+constexpr int BQ = 128, BKV = 64;
+constexpr int kThreads = 192;
+
+template <int HD>
+struct Shape {
+  static constexpr int KCH = HD / 64;                   // 64-column (128-byte) chunks of a row
+  static constexpr uint32_t Q_BYTES = BQ * HD * 2;
+  static constexpr uint32_t KV_CHUNK = BKV * 128;       // one 64x64 bf16 chunk (8 KiB)
+  static constexpr uint32_t K_BYTES = BKV * HD * 2;
+  static constexpr uint32_t V_BYTES = BKV * HD * 2;
+  static constexpr uint32_t STAGE_BYTES = K_BYTES + V_BYTES;
+  static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB
+  static constexpr int STAGES = 2;
+  static constexpr uint32_t TMEM_S = 0;                 // 64 columns
+  static constexpr uint32_t TMEM_O = 64;                // HD columns
+  static constexpr uint32_t TMEM_COLS = (64 + HD <= 128) ? 128 : 256;
+  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + P_BYTES + 1024 + 256;
+  // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
+  static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BKV >> 3) << 17) |
+                                      ((uint32_t)(BQ >> 4) << 24);
+  static constexpr uint32_t IDESC_PV = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+                                       ((uint32_t)(HD >> 3) << 17) | ((uint32_t)(BQ >> 4) << 24);
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
+  if (mbar_try(a, parity)) return true;
+  const uint64_t t0 = gtimer();
+  for (uint32_t i = 1; i < (1u << 28); ++i) {
+    if (mbar_try(a, parity)) return true;
+    if ((i & 127) == 0 && gtimer() - t0 > 2000000000ull) break;
+  }
+  atomicOr(err, kErrLimit);
+  return false;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
+          dst),
+      "l"((uint64_t)map), "r"(mbar), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar) : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
+          d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// K-major operand, 128-byte swizzle: 8-row groups 1024 B apart (SBO), LBO unused.
+__device__ __forceinline__ uint64_t desc_kmajor(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// MN-major operand, 128-byte swizzle: 64-element MN chunks `lbo` bytes apart (LBO), 8-row K
+// groups 1024 B apart (SBO).
+__device__ __forceinline__ uint64_t desc_mnmajor(uint32_t saddr, uint32_t lbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; i++) v[i] = __uint_as_float(r[i]);
+}
+
+struct Params {
+  __nv_bfloat16* out;
+  int64_t out_stride;    // elements per output row
+  int64_t q_win_stride;  // query rows per window in the q buffer (W prefill, 1 decode)
+  int64_t pos_first;     // position of the first query row of a window
+  int n_pos;             // query positions per window
+  int W;                 // keys rows per window in the kv buffer
+  int nq, nkv;
+  int q_col0, k_col0, v_col0;  // column offsets of q head 0, k head 0, v head 0
+  float scale_log2;            // log2(e) / sqrt(hd)
+  uint32_t* err;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(kThreads)
+    k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv, Params p) {
+  using S = Shape<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+  const uint32_t sq = smem_u32(smem);
+  const uint32_t skv = sq + S::Q_BYTES;
+  const uint32_t sp = skv + S::STAGES * S::STAGE_BYTES;
+  uint8_t* p_gen = smem + S::Q_BYTES + S::STAGES * S::STAGE_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + S::P_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+  const uint32_t b_q = smem_u32(bars + 0), b_s = smem_u32(bars + 1), b_p = smem_u32(bars + 2),
+                 b_pv = smem_u32(bars + 3);
+  auto b_kvfull = [&](int s) { return smem_u32(bars + 4 + s); };
+  auto b_kvempty = [&](int s) { return smem_u32(bars + 6 + s); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y;
+  const int64_t w = blockIdx.z;
+  const int kvh = h / (p.nq / p.nkv);
+  // heavy (late) query tiles first
+  const int qb = (int)gridDim.x - 1 - (int)blockIdx.x;
+  const int64_t pos0 = p.pos_first + (int64_t)qb * BQ;                     // position of tile row 0
+  const int64_t rem = p.pos_first + p.n_pos - pos0;
+  const int nrows = rem < BQ ? (int)rem : BQ;  // valid rows
+  const int64_t last_pos = pos0 + nrows - 1;
+  const int nkb = (int)(last_pos / BKV) + 1;
+  const int q_row0 = (int)(w * p.q_win_stride + (pos0 - p.pos_first));
+  const int kv_row0 = (int)(w * p.W);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 10; i++) mbar_init(smem_u32(bars + i), i == 2 ? 128 : 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(S::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      mbar_expect_tx(b_q, S::Q_BYTES);
+#pragma unroll
+      for (int c = 0; c < S::KCH; c++) tma_load_2d(sq + c * (BQ * 128), &tq, b_q, p.q_col0 + h * HD + 64 * c, q_row0);
+    }
+    __syncwarp();
+    for (int kb = 0; kb < nkb; kb++) {
+      const int st = kb & 1;
+      const uint32_t ph = (uint32_t)(kb >> 1) & 1u;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kvempty(st), ph ^ 1u, p.err))) break;
+      if (lane == 0) {
+        const uint32_t base = skv + st * S::STAGE_BYTES;
+        mbar_expect_tx(b_kvfull(st), S::STAGE_BYTES);
+#pragma unroll
+        for (int c = 0; c < S::KCH; c++) {
+          tma_load_2d(base + c * S::KV_CHUNK, &tkv, b_kvfull(st), p.k_col0 + kvh * HD + 64 * c, kv_row0 + kb * BKV);
+          tma_load_2d(base + S::K_BYTES + c * S::KV_CHUNK, &tkv, b_kvfull(st), p.v_col0 + kvh * HD + 64 * c,
+                      kv_row0 + kb * BKV);
+        }
+      }
+      __syncwarp();
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
+    for (int kb = 0; kb < nkb && ok; kb++) {
+      const int st = kb & 1;
+      const uint32_t ph = (uint32_t)(kb >> 1) & 1u;
+      ok = __all_sync(0xffffffffu, mbar_wait(b_kvfull(st), ph, p.err));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t kbase = skv + st * S::STAGE_BYTES, vbase = kbase + S::K_BYTES;
+      if (lane == 0) {
+        // S = Q K^T over hd in steps of 16 (32 bytes inside a 128-byte chunk)
+#pragma unroll
+        for (int k = 0; k < HD / 16; k++) {
+          const int c = k >> 2, o = (k & 3) * 32;
+          tc_mma(tmem + S::TMEM_S, desc_kmajor(sq + c * (BQ * 128) + o), desc_kmajor(kbase + c * S::KV_CHUNK + o),
+                 S::IDESC_S, k > 0 ? 1u : 0u);
+        }
+        tc_commit(b_s);
+      }
+      __syncwarp();
+      ok = __all_sync(0xffffffffu, mbar_wait(b_p, (uint32_t)kb & 1u, p.err));
+      if (!ok) break;
+      tc_fence_after();
+      if (lane == 0) {
+        // O_blk = P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
+#pragma unroll
+        for (int k = 0; k < BKV / 16; k++)
+          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + k * 32), desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV,
+                 k > 0 ? 1u : 0u);
+        tc_commit(b_pv);
+        tc_commit(b_kvempty(st));
+      }
+      __syncwarp();
+    }
+  } else {
+    // ---------------- softmax (warps 2..5): thread = query row ----------------
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const int64_t qpos = pos0 + r;
+    const uint32_t tl = (uint32_t)(q4 * 32) << 16;
+    float m = -INFINITY, l = 0.f;
+    float o[HD];
+#pragma unroll
+    for (int i = 0; i < HD; i++) o[i] = 0.f;
+    // this row's P row in the swizzled layout: 8-row groups of 1024 B, rows of 128 B, 16-byte
+    // chunk index XOR (row mod 8)
+    uint8_t* prow = p_gen + (r >> 3) * 1024 + (r & 7) * 128;
+    for (int kb = 0; kb < nkb; kb++) {
+      if (!__all_sync(0xffffffffu, mbar_wait(b_s, (uint32_t)kb & 1u, p.err))) break;
+      tc_fence_after();
+      float s[64];
+      {
+        float a[32], b[32];
+        tmem_ld32(tmem + tl + S::TMEM_S, a);
+        tmem_ld32(tmem + tl + S::TMEM_S + 32, b);
+#pragma unroll
+        for (int j = 0; j < 32; j++) {
+          s[j] = a[j];
+          s[32 + j] = b[j];
+        }
+      }
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 64; j++) {
+        const int64_t kpos = (int64_t)kb * BKV + j;
+        s[j] = (kpos <= qpos) ? s[j] : -INFINITY;
+        mx = fmaxf(mx, s[j]);
+      }
+      const float mn = fmaxf(m, mx);
+      const float corr = (mn == -INFINITY) ? 1.f : exp2f((m - mn) * p.scale_log2);
+      float rs = 0.f;
+#pragma unroll
+      for (int j = 0; j < 64; j++) {
+        const float e = (s[j] == -INFINITY) ? 0.f : exp2f((s[j] - mn) * p.scale_log2);
+        s[j] = e;
+        rs += e;
+      }
+      l = l * corr + rs;
+      m = mn;
+#pragma unroll
+      for (int c = 0; c < 8; c++) {
+        uint32_t wv[4];
+#pragma unroll
+        for (int t = 0; t < 4; t++) {
+          __nv_bfloat162 hb = __floats2bfloat162_rn(s[8 * c + 2 * t], s[8 * c + 2 * t + 1]);
+          wv[t] = *reinterpret_cast<uint32_t*>(&hb);
+        }
+        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(b_p);
+      if (!__all_sync(0xffffffffu, mbar_wait(b_pv, (uint32_t)kb & 1u, p.err))) break;
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < HD / 32; c++) {
+        float pv[32];
+        tmem_ld32(tmem + tl + S::TMEM_O + c * 32, pv);
+#pragma unroll
+        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + pv[j];
+      }
+      tc_fence_before();
+    }
+    if (r < nrows) {
+      const float inv = 1.f / l;
+      __nv_bfloat16* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
+#pragma unroll
+      for (int c = 0; c < HD / 8; c++) {
+        uint32_t wv[4];
+#pragma unroll
+        for (int t = 0; t < 4; t++) {
+          __nv_bfloat162 hb = __floats2bfloat162_rn(o[8 * c + 2 * t] * inv, o[8 * c + 2 * t + 1] * inv);
+          wv[t] = *reinterpret_cast<uint32_t*>(&hb);
+        }
+        reinterpret_cast<uint4*>(dst)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(S::TMEM_COLS) : "memory");
+  }
+}
+
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static std::once_flag g_once;
+
+static void init_once() {
+  cudaDriverEntryPointQueryResult q;
+  void* fn = nullptr;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  int dev = 0, major = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  if (major != 10) g_encode = nullptr;
+  cudaFuncSetAttribute(k_attn_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<64>::SMEM);
+  cudaFuncSetAttribute(k_attn_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<128>::SMEM);
+}
+
+static bool make_map(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint32_t box_rows) {
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace attn
+
+bool tc_attention_supported(int hd, int64_t qkv_dim) {
+  std::call_once(attn::g_once, attn::init_once);
+  return attn::g_encode != nullptr && (hd == 64 || hd == 128) && qkv_dim % 64 == 0;
+}
+
+void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t kv_rows, int64_t qkv_dim, int k_off,
+                         int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
+                         int64_t pos_first, int n_pos, int64_t q_win_stride, uint32_t* err, cudaStream_t s) {
+  using namespace attn;
+  std::call_once(g_once, init_once);
+  CUtensorMap tq, tkv;
+  if (!make_map(&tq, q, (uint64_t)qkv_dim, (uint64_t)q_rows, BQ) ||
+      !make_map(&tkv, kv, (uint64_t)qkv_dim, (uint64_t)kv_rows, BKV)) {
+    set_thread_error("cuTensorMapEncodeTiled failed (attention)");
+    return;
+  }
+  Params p;
+  p.out = (__nv_bfloat16*)out;
+  p.out_stride = out_stride;
+  p.q_win_stride = q_win_stride;
+  p.pos_first = pos_first;
+  p.n_pos = n_pos;
+  p.W = W;
+  p.nq = nq;
+  p.nkv = nkv;
+  p.q_col0 = 0;
+  p.k_col0 = k_off;
+  p.v_col0 = v_off;
+  p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)hd));
+  p.err = err;
+  dim3 grid((unsigned)((n_pos + BQ - 1) / BQ), (unsigned)nq, (unsigned)n_win);
+  note_launch();
+  if (hd == 64) k_attn_tc<64><<<grid, kThreads, Shape<64>::SMEM, s>>>(tq, tkv, p);
+  else k_attn_tc<128><<<grid, kThreads, Shape<128>::SMEM, s>>>(tq, tkv, p);
+}
+
+}  // namespace lmgc

@@ -165,6 +165,12 @@ size_t dec_state_bytes();
 void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n,
                      void* state, cudaStream_t s);
 
+// attn_tc.cu (tcgen05)
+bool tc_attention_supported(int hd, int64_t qkv_dim);
+void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t kv_rows, int64_t qkv_dim, int k_off,
+                         int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
+                         int64_t pos_first, int n_pos, int64_t q_win_stride, uint32_t* err, cudaStream_t s);
+
 // gemm_tc.cu (tcgen05)
 bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi = 0);
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
