@@ -36,12 +36,12 @@ struct Shape {
   static constexpr uint32_t K_BYTES = BKV * HD * 2;
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
   static constexpr uint32_t STAGE_BYTES = K_BYTES + V_BYTES;
-  static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB
+  static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB per P buffer (two)
   static constexpr int STAGES = 2;
-  static constexpr uint32_t TMEM_S = 0;                 // 64 columns
-  static constexpr uint32_t TMEM_O = 64;                // HD columns
-  static constexpr uint32_t TMEM_COLS = (64 + HD <= 128) ? 128 : 256;
-  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + P_BYTES + 1024 + 256;
+  static constexpr uint32_t TMEM_S = 0;                 // S double buffer: columns 0..127
+  static constexpr uint32_t TMEM_O = 128;               // P V double buffer: 2 x HD columns
+  static constexpr uint32_t TMEM_COLS = (128 + 2 * HD <= 256) ? 256 : 512;
+  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + 2 * P_BYTES + 1024 + 256;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
@@ -150,14 +150,18 @@ __global__ void __launch_bounds__(kThreads)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const uint32_t sq = smem_u32(smem);
   const uint32_t skv = sq + S::Q_BYTES;
-  const uint32_t sp = skv + S::STAGES * S::STAGE_BYTES;
+  const uint32_t sp = skv + S::STAGES * S::STAGE_BYTES;  // two P buffers
   uint8_t* p_gen = smem + S::Q_BYTES + S::STAGES * S::STAGE_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + S::P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
-  const uint32_t b_q = smem_u32(bars + 0), b_s = smem_u32(bars + 1), b_p = smem_u32(bars + 2),
-                 b_pv = smem_u32(bars + 3);
-  auto b_kvfull = [&](int s) { return smem_u32(bars + 4 + s); };
-  auto b_kvempty = [&](int s) { return smem_u32(bars + 6 + s); };
+  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + 2 * S::P_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (128 arrivals) | 5-6 P V ready |
+  //           7-8 K/V stage loaded | 9-10 K/V stage free
+  const uint32_t b_q = smem_u32(bars + 0);
+  auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
+  auto b_p = [&](int i) { return smem_u32(bars + 3 + i); };
+  auto b_pv = [&](int i) { return smem_u32(bars + 5 + i); };
+  auto b_kvfull = [&](int i) { return smem_u32(bars + 7 + i); };
+  auto b_kvempty = [&](int i) { return smem_u32(bars + 9 + i); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -165,7 +169,7 @@ __global__ void __launch_bounds__(kThreads)
   const int kvh = h / (p.nq / p.nkv);
   // heavy (late) query tiles first
   const int qb = (int)gridDim.x - 1 - (int)blockIdx.x;
-  const int64_t pos0 = p.pos_first + (int64_t)qb * BQ;                     // position of tile row 0
+  const int64_t pos0 = p.pos_first + (int64_t)qb * BQ;  // position of tile row 0
   const int64_t rem = p.pos_first + p.n_pos - pos0;
   const int nrows = rem < BQ ? (int)rem : BQ;  // valid rows
   const int64_t last_pos = pos0 + nrows - 1;
@@ -174,7 +178,7 @@ __global__ void __launch_bounds__(kThreads)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 10; i++) mbar_init(smem_u32(bars + i), i == 2 ? 128 : 1);
+    for (int i = 0; i < 11; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 128 : 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -214,36 +218,42 @@ __global__ void __launch_bounds__(kThreads)
       __syncwarp();
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
-    for (int kb = 0; kb < nkb && ok; kb++) {
+    // ---------------- MMA issuer: S(kb+1) is issued before P V(kb) so the softmax of block kb
+    // overlaps the tensor cores ----------------
+    auto issue_s = [&](int kb) -> bool {
       const int st = kb & 1;
-      const uint32_t ph = (uint32_t)(kb >> 1) & 1u;
-      ok = __all_sync(0xffffffffu, mbar_wait(b_kvfull(st), ph, p.err));
-      if (!ok) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kvfull(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
       tc_fence_after();
-      const uint32_t kbase = skv + st * S::STAGE_BYTES, vbase = kbase + S::K_BYTES;
       if (lane == 0) {
+        const uint32_t kbase = skv + st * S::STAGE_BYTES;
         // S = Q K^T over hd in steps of 16 (32 bytes inside a 128-byte chunk)
 #pragma unroll
         for (int k = 0; k < HD / 16; k++) {
           const int c = k >> 2, o = (k & 3) * 32;
-          tc_mma(tmem + S::TMEM_S, desc_kmajor(sq + c * (BQ * 128) + o), desc_kmajor(kbase + c * S::KV_CHUNK + o),
-                 S::IDESC_S, k > 0 ? 1u : 0u);
+          tc_mma(tmem + S::TMEM_S + st * 64, desc_kmajor(sq + c * (BQ * 128) + o),
+                 desc_kmajor(kbase + c * S::KV_CHUNK + o), S::IDESC_S, k > 0 ? 1u : 0u);
         }
-        tc_commit(b_s);
+        tc_commit(b_s(st));
       }
       __syncwarp();
-      ok = __all_sync(0xffffffffu, mbar_wait(b_p, (uint32_t)kb & 1u, p.err));
+      return true;
+    };
+    bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
+    if (ok) ok = issue_s(0);
+    for (int kb = 0; kb < nkb && ok; kb++) {
+      const int st = kb & 1;
+      if (kb + 1 < nkb && !(ok = issue_s(kb + 1))) break;
+      ok = __all_sync(0xffffffffu, mbar_wait(b_p(st), (uint32_t)(kb >> 1) & 1u, p.err));
       if (!ok) break;
       tc_fence_after();
       if (lane == 0) {
+        const uint32_t vbase = skv + st * S::STAGE_BYTES + S::K_BYTES;
         // O_blk = P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
-          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + k * 32), desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV,
-                 k > 0 ? 1u : 0u);
-        tc_commit(b_pv);
+          tc_mma(tmem + S::TMEM_O + st * HD, desc_kmajor(sp + st * S::P_BYTES + k * 32),
+                 desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, k > 0 ? 1u : 0u);
+        tc_commit(b_pv(st));
         tc_commit(b_kvempty(st));
       }
       __syncwarp();
@@ -254,21 +264,38 @@ __global__ void __launch_bounds__(kThreads)
     const int r = q4 * 32 + lane;
     const int64_t qpos = pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
-    float m = -INFINITY, l = 0.f;
+    float m = -INFINITY, l = 0.f, corr_prev = 1.f;
     float o[HD];
 #pragma unroll
     for (int i = 0; i < HD; i++) o[i] = 0.f;
+    // O = O * corr + (P V) of a block; deferred by one block so the P V MMA runs meanwhile
+    auto add_pv = [&](int kb, float corr) -> bool {
+      const int st = kb & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < HD / 32; c++) {
+        float pv[32];
+        tmem_ld32(tmem + tl + S::TMEM_O + st * HD + c * 32, pv);
+#pragma unroll
+        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + pv[j];
+      }
+      tc_fence_before();
+      return true;
+    };
     // this row's P row in the swizzled layout: 8-row groups of 1024 B, rows of 128 B, 16-byte
     // chunk index XOR (row mod 8)
-    uint8_t* prow = p_gen + (r >> 3) * 1024 + (r & 7) * 128;
+    const int prow_off = (r >> 3) * 1024 + (r & 7) * 128;
+    bool ok = true;
     for (int kb = 0; kb < nkb; kb++) {
-      if (!__all_sync(0xffffffffu, mbar_wait(b_s, (uint32_t)kb & 1u, p.err))) break;
+      const int st = kb & 1;
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(st), (uint32_t)(kb >> 1) & 1u, p.err)))) break;
       tc_fence_after();
       float s[64];
       {
         float a[32], b[32];
-        tmem_ld32(tmem + tl + S::TMEM_S, a);
-        tmem_ld32(tmem + tl + S::TMEM_S + 32, b);
+        tmem_ld32(tmem + tl + S::TMEM_S + st * 64, a);
+        tmem_ld32(tmem + tl + S::TMEM_S + st * 64 + 32, b);
 #pragma unroll
         for (int j = 0; j < 32; j++) {
           s[j] = a[j];
@@ -293,6 +320,7 @@ __global__ void __launch_bounds__(kThreads)
       }
       l = l * corr + rs;
       m = mn;
+      uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
 #pragma unroll
       for (int c = 0; c < 8; c++) {
         uint32_t wv[4];
@@ -305,19 +333,12 @@ __global__ void __launch_bounds__(kThreads)
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
-      mbar_arrive(b_p);
-      if (!__all_sync(0xffffffffu, mbar_wait(b_pv, (uint32_t)kb & 1u, p.err))) break;
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < HD / 32; c++) {
-        float pv[32];
-        tmem_ld32(tmem + tl + S::TMEM_O + c * 32, pv);
-#pragma unroll
-        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + pv[j];
-      }
-      tc_fence_before();
+      mbar_arrive(b_p(st));
+      if (kb > 0 && !(ok = add_pv(kb - 1, corr_prev))) break;
+      corr_prev = corr;
     }
-    if (r < nrows) {
+    if (ok) ok = add_pv(nkb - 1, corr_prev);
+    if (ok && r < nrows) {
       const float inv = 1.f / l;
       __nv_bfloat16* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
 #pragma unroll
