@@ -114,6 +114,12 @@ __device__ __forceinline__ uint64_t desc_mnmajor(uint32_t saddr, uint32_t lbo) {
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
+// 2^x on the special-function unit (flushes subnormal results to zero; ex2(-inf) = 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -262,7 +268,7 @@ __global__ void __launch_bounds__(kThreads)
     // ---------------- softmax (warps 2..5): thread = query row ----------------
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
-    const int64_t qpos = pos0 + r;
+    const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
     float m = -INFINITY, l = 0.f, corr_prev = 1.f;
     float o[HD];
@@ -302,22 +308,34 @@ __global__ void __launch_bounds__(kThreads)
           s[32 + j] = b[j];
         }
       }
-      float mx = -INFINITY;
+      // causal mask, only on blocks that reach past the tile's first position
+      if ((int)(kb * BKV + BKV - 1) > pos0_i) {
 #pragma unroll
-      for (int j = 0; j < 64; j++) {
-        const int64_t kpos = (int64_t)kb * BKV + j;
-        s[j] = (kpos <= qpos) ? s[j] : -INFINITY;
-        mx = fmaxf(mx, s[j]);
+        for (int j = 0; j < 64; j++)
+          if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
       }
-      const float mn = fmaxf(m, mx);
-      const float corr = (mn == -INFINITY) ? 1.f : exp2f((m - mn) * p.scale_log2);
-      float rs = 0.f;
+      // row max and row sum with 8 independent chains
+      float mx8[8];
+#pragma unroll
+      for (int i = 0; i < 8; i++) mx8[i] = s[i];
+#pragma unroll
+      for (int j = 8; j < 64; j++) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      const float mn = fmaxf(m, mx);  // finite: key 0 is never masked
+      // exactly 1 when the maximum does not change (a fully masked block is then a no-op)
+      const float corr = ex2_approx((m - mn) * p.scale_log2);
+      const float nb = -mn * p.scale_log2;
+      float sum8[8];
+#pragma unroll
+      for (int i = 0; i < 8; i++) sum8[i] = 0.f;
 #pragma unroll
       for (int j = 0; j < 64; j++) {
-        const float e = (s[j] == -INFINITY) ? 0.f : exp2f((s[j] - mn) * p.scale_log2);
+        const float e = ex2_approx(fmaf(s[j], p.scale_log2, nb));
         s[j] = e;
-        rs += e;
+        sum8[j & 7] += e;
       }
+      const float rs = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
       l = l * corr + rs;
       m = mn;
       uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
