@@ -150,8 +150,12 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
       ProfScope ps(ctx, kNorm, 0, s);
       launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
     }
-    gemm(ctx, ws.n, L.wqkv, ws.qkv, rows, ctx->qkv_dim, d, kStore, s);
-    {
+    if (ctx->fused_rope) {
+      RopeArgs ra{ctx->rope_cs, (c.n_heads + c.n_kv_heads) * hd, hd, decode ? 1 : c.window, decode ? pos : 0};
+      ProfScope ps(ctx, kGemm, 2.0 * (double)rows * (double)ctx->qkv_dim * (double)d, s);
+      launch_gemm_tc(ws.n, L.wqkv, ws.qkv, rows, ctx->qkv_dim, d, kQKVRope, ctx->d_err, s, &ra);
+    } else {
+      gemm(ctx, ws.n, L.wqkv, ws.qkv, rows, ctx->qkv_dim, d, kStore, s);
       ProfScope ps(ctx, kNorm, 0, s);
       launch_rope(ws.qkv, rows, ctx->qkv_dim, c.n_heads + c.n_kv_heads, hd, ctx->rope_cs, c.window,
                   decode ? pos : 0, decode ? 1 : W, decode ? 1 : c.window, c.dtype, s);
@@ -303,6 +307,8 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
   const char* tc_env = getenv("LMGC_DISABLE_TC");
   ctx->use_tc = !(tc_env && tc_env[0] == '1');
+  ctx->fused_rope = c.dtype == LMGC_BF16 && ctx->use_tc && (hd == 64 || hd == 128) &&
+                    tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kQKVRope);
   ctx->fused_swiglu = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_ffn % 128 == 0 && tc_gemm_supported(1, 2 * c.d_ffn, c.d_model, kSwiGLU);
   const int64_t d = c.d_model, F = c.d_ffn, V = c.vocab, qd = (int64_t)c.n_heads * hd;
   const size_t e = ctx->elt;

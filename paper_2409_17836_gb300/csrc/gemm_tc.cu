@@ -130,6 +130,11 @@ struct Params {
   int64_t M, N, K;
   int tiles_m, tiles_n, num_kb;
   uint32_t* err;
+  // kQKVRope: rotary embedding of columns [0, rope_cols) in heads of rope_hd; row m sits at
+  // position rope_pos0 + m % rope_pos_mod; rope_cs[pos * rope_hd/2 + i] = (cos, sin)
+  const float2* rope_cs;
+  int rope_cols, rope_hd, rope_pos_mod;
+  int64_t rope_pos0;
 };
 
 __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int& nb) {
@@ -289,7 +294,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const int64_t m = (int64_t)mb * BM + q * 32 + lane;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);
-      if (EPI == kSwiGLU) {
+      if (EPI == kQKVRope) {
+        // one head at a time: halves [0, hd/2) and [hd/2, hd) rotate pairwise by pos * theta_i
+        const int hd = p.rope_hd, hh = hd / 2;
+        const int64_t pos = p.rope_pos0 + m % p.rope_pos_mod;
+        const float2* cs = p.rope_cs + pos * hh;
+#pragma unroll 1
+        for (int hs = 0; hs < BN / hd; ++hs) {
+          const int64_t col0 = (int64_t)nb * BN + hs * hd;
+          const bool rot = col0 < p.rope_cols;
+#pragma unroll 1
+          for (int c = 0; c < hh / 32; ++c) {
+            uint32_t a[32], b[32];
+            tmem_ld32(tbase + (uint32_t)(hs * hd + c * 32), a);
+            tmem_ld32(tbase + (uint32_t)(hs * hd + hh + c * 32), b);
+            if (m < p.M && col0 < p.N) {
+              if (rot) {
+#pragma unroll
+                for (int j = 0; j < 32; j++) {
+                  const float2 t = cs[c * 32 + j];
+                  const float x = __uint_as_float(a[j]), y = __uint_as_float(b[j]);
+                  a[j] = __float_as_uint(x * t.x - y * t.y);
+                  b[j] = __float_as_uint(x * t.y + y * t.x);
+                }
+              }
+              store_chunk<kStore>(p, m, col0 + c * 32, a);
+              store_chunk<kStore>(p, m, col0 + hh + c * 32, b);
+            }
+          }
+        }
+      } else if (EPI == kSwiGLU) {
         // columns [0, 128) of the tile are gate, [128, 256) the matching up columns
 #pragma unroll 1
         for (int c = 0; c < BN / 64; ++c) {
@@ -356,6 +390,7 @@ static void init_once() {
   cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   cudaFuncSetAttribute(k_gemm_tc<kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaFuncSetAttribute(k_gemm_tc<kQKVRope>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
 }
 
 static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t rows, uint32_t box_rows) {
@@ -374,11 +409,12 @@ static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t row
 bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi) {
   std::call_once(tc::g_once, tc::init_once);
   if (epi == kSwiGLU && N % tc::BN != 0) return false;
+  if (epi == kQKVRope && N % 64 != 0) return false;
   return tc::g_encode != nullptr && M > 0 && N > 0 && K > 0 && K % 8 == 0 && M < (1ll << 31) && N < (1ll << 31);
 }
 
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
-                    cudaStream_t s) {
+                    cudaStream_t s, const RopeArgs* rope) {
   using namespace tc;
   std::call_once(g_once, init_once);
   CUtensorMap ma, mb;
@@ -395,13 +431,19 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.tiles_n = (int)((N + BN - 1) / BN);
   p.num_kb = (int)((K + BK - 1) / BK);
   p.err = err;
+  p.rope_cs = rope ? rope->cs : nullptr;
+  p.rope_cols = rope ? rope->cols : 0;
+  p.rope_hd = rope ? rope->hd : 64;
+  p.rope_pos_mod = rope ? rope->pos_mod : 1;
+  p.rope_pos0 = rope ? rope->pos0 : 0;
   const int tiles = p.tiles_m * p.tiles_n;
   const int grid = std::max(1, std::min(tiles, g_num_sms));
   note_launch();
   if (epi == kStore) k_gemm_tc<kStore><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
   else if (epi == kAddResidual) k_gemm_tc<kAddResidual><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
   else if (epi == kStoreF32) k_gemm_tc<kStoreF32><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else k_gemm_tc<kSwiGLU><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else if (epi == kSwiGLU) k_gemm_tc<kSwiGLU><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  else k_gemm_tc<kQKVRope><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
 }
 
 }  // namespace lmgc

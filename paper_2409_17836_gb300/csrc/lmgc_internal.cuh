@@ -93,6 +93,7 @@ struct lmgc_ctx {
   lmgc::Profiler prof;
   bool use_tc = true;        // tcgen05 GEMM for bf16 models when available
   bool fused_swiglu = false;  // gate/up interleaved, SwiGLU in the tcgen05 epilogue
+  bool fused_rope = false;    // RoPE in the QKV tcgen05 epilogue
   std::string err;
 };
 
@@ -131,7 +132,15 @@ void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, i
 // C[M][N] = A[M][K] . B[N][K]^T with the given epilogue
 // kSwiGLU: B's rows are gate/up blocks interleaved 128 by 128 (rows 256t..256t+127 = gate rows
 // 128t.., rows 256t+128.. = up rows 128t..); C[m][128t + j] = silu(gate) * up, N/2 columns.
-enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3 };
+// kQKVRope: kStore with the rotary embedding applied to the q and k heads (RopeArgs).
+enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3, kQKVRope = 4 };
+struct RopeArgs {
+  const float2* cs;  // [W][hd/2] (cos, sin)
+  int cols;          // columns [0, cols) are rotated: (n_heads + n_kv_heads) * hd
+  int hd;
+  int pos_mod;       // row m sits at position pos0 + m % pos_mod
+  int64_t pos0;
+};
 void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
                       cudaStream_t s);
 void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
@@ -174,6 +183,6 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
 // gemm_tc.cu (tcgen05)
 bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi = 0);
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
-                    cudaStream_t s);
+                    cudaStream_t s, const RopeArgs* rope = nullptr);
 
 }  // namespace lmgc
