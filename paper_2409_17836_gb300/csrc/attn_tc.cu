@@ -120,6 +120,18 @@ __device__ __forceinline__ float ex2_approx(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// tcgen05.ld without the wait (several loads may be in flight; then tmem_wait())
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -280,11 +292,16 @@ __global__ void __launch_bounds__(kThreads)
       if (!__all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
       tc_fence_after();
 #pragma unroll
-      for (int c = 0; c < HD / 32; c++) {
-        float pv[32];
-        tmem_ld32(tmem + tl + S::TMEM_O + st * HD + c * 32, pv);
+      for (int c = 0; c < HD / 64; c++) {
+        uint32_t pa[32], pb[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + c * 64, pa);
+        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + c * 64 + 32, pb);
+        tmem_wait();
 #pragma unroll
-        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + pv[j];
+        for (int j = 0; j < 32; j++) {
+          o[c * 64 + j] = o[c * 64 + j] * corr + __uint_as_float(pa[j]);
+          o[c * 64 + 32 + j] = o[c * 64 + 32 + j] * corr + __uint_as_float(pb[j]);
+        }
       }
       tc_fence_before();
       return true;
@@ -299,13 +316,14 @@ __global__ void __launch_bounds__(kThreads)
       tc_fence_after();
       float s[64];
       {
-        float a[32], b[32];
-        tmem_ld32(tmem + tl + S::TMEM_S + st * 64, a);
-        tmem_ld32(tmem + tl + S::TMEM_S + st * 64 + 32, b);
+        uint32_t a[32], b[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64, a);
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + 32, b);
+        tmem_wait();
 #pragma unroll
         for (int j = 0; j < 32; j++) {
-          s[j] = a[j];
-          s[32 + j] = b[j];
+          s[j] = __uint_as_float(a[j]);
+          s[32 + j] = __uint_as_float(b[j]);
         }
       }
       // causal mask, only on blocks that reach past the tile's first position

@@ -88,9 +88,29 @@ __global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict
   bool bad = n > win_tokens;
   const uint32_t* ps = start + w * stride_win;
   const uint32_t* pf = freq + w * stride_win;
-  for (int64_t i = 0; i < n && !bad; i++) {
-    const uint64_t s = __ldcs(ps + i * stride_pos);
-    const uint64_t f = __ldcs(pf + i * stride_pos);
+  // the pairs of the next kPre tokens are loaded ahead so their latency overlaps the serial chain
+  constexpr int kPre = 8;
+  uint32_t bs[kPre], bf[kPre];
+#pragma unroll
+  for (int j = 0; j < kPre; j++) {
+    bs[j] = j < n ? __ldcs(ps + j * stride_pos) : 0u;
+    bf[j] = j < n ? __ldcs(pf + j * stride_pos) : 1u;
+  }
+  for (int64_t i0 = 0; i0 < n && !bad; i0 += kPre) {
+    uint32_t cs[kPre], cf[kPre];
+#pragma unroll
+    for (int j = 0; j < kPre; j++) {
+      cs[j] = bs[j];
+      cf[j] = bf[j];
+      const int64_t nx = i0 + kPre + j;
+      bs[j] = nx < n ? __ldcs(ps + nx * stride_pos) : 0u;
+      bf[j] = nx < n ? __ldcs(pf + nx * stride_pos) : 1u;
+    }
+#pragma unroll
+  for (int j = 0; j < kPre; j++) {
+    if (i0 + j >= n) break;
+    const uint64_t s = cs[j];
+    const uint64_t f = cf[j];
     if (f == 0 || s + f > T) {
       bad = true;
       break;
@@ -109,6 +129,7 @@ __global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict
       R <<= k;
       B += (uint64_t)k;
     }
+  }
   }
   // termination: v = ceil(L / 2^60) * 2^60; emit its top 2 bits of the low 62
   L += (1ull << 60) - 1ull;

@@ -300,11 +300,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t pos = p.rope_pos0 + m % p.rope_pos_mod;
         const float2* cs = p.rope_cs + pos * hh;
 #pragma unroll 1
-        for (int hs = 0; hs < BN / hd; ++hs) {
-          const int64_t col0 = (int64_t)nb * BN + hs * hd;
-          const bool rot = col0 < p.rope_cols;
+        for (int c = 0; c < hh / 32; ++c) {
+          float ct[32], st[32];
+          const bool any_rot = (int64_t)nb * BN < p.rope_cols && m < p.M;
+          if (any_rot) {
+            const float4* c4 = reinterpret_cast<const float4*>(cs + c * 32);
+#pragma unroll
+            for (int j = 0; j < 16; j++) {
+              const float4 t = __ldg(c4 + j);
+              ct[2 * j] = t.x;
+              st[2 * j] = t.y;
+              ct[2 * j + 1] = t.z;
+              st[2 * j + 1] = t.w;
+            }
+          }
 #pragma unroll 1
-          for (int c = 0; c < hh / 32; ++c) {
+          for (int hs = 0; hs < BN / hd; ++hs) {
+            const int64_t col0 = (int64_t)nb * BN + hs * hd;
+            const bool rot = col0 < p.rope_cols;
             uint32_t a[32], b[32];
             tmem_ld32(tbase + (uint32_t)(hs * hd + c * 32), a);
             tmem_ld32(tbase + (uint32_t)(hs * hd + hh + c * 32), b);
@@ -312,10 +325,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (rot) {
 #pragma unroll
                 for (int j = 0; j < 32; j++) {
-                  const float2 t = cs[c * 32 + j];
                   const float x = __uint_as_float(a[j]), y = __uint_as_float(b[j]);
-                  a[j] = __float_as_uint(x * t.x - y * t.y);
-                  b[j] = __float_as_uint(x * t.y + y * t.x);
+                  a[j] = __float_as_uint(x * ct[j] - y * st[j]);
+                  b[j] = __float_as_uint(x * st[j] + y * ct[j]);
                 }
               }
               store_chunk<kStore>(p, m, col0 + c * 32, a);
