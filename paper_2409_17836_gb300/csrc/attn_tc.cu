@@ -26,7 +26,7 @@ namespace lmgc {
 namespace attn {
 
 constexpr int BQ = 128, BKV = 64;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;  // TMA warp, MMA warp, 8 softmax warps
 
 template <int HD>
 struct Shape {
@@ -41,7 +41,7 @@ struct Shape {
   static constexpr uint32_t TMEM_S = 0;                 // S double buffer: columns 0..127
   static constexpr uint32_t TMEM_O = 128;               // P V double buffer: 2 x HD columns
   static constexpr uint32_t TMEM_COLS = (128 + 2 * HD <= 256) ? 256 : 512;
-  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + 2 * P_BYTES + 1024 + 256;
+  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
@@ -161,7 +161,7 @@ struct Params {
 };
 
 template <int HD>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv, Params p) {
   using S = Shape<HD>;
   extern __shared__ uint8_t smem_raw[];
@@ -171,9 +171,11 @@ __global__ void __launch_bounds__(kThreads)
   const uint32_t sp = skv + S::STAGES * S::STAGE_BYTES;  // two P buffers
   uint8_t* p_gen = smem + S::Q_BYTES + S::STAGES * S::STAGE_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + 2 * S::P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
-  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (128 arrivals) | 5-6 P V ready |
-  //           7-8 K/V stage loaded | 9-10 K/V stage free
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  float* red_m = reinterpret_cast<float*>(bars + 32);  // [2 parities][2 halves][128 rows]
+  float* red_l = red_m + 512;                          // [2 halves][128 rows]
+  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (256 arrivals) | 5-6 P V ready |
+  //           7-8 K/V stage loaded | 9-10 K/V stage free | 11-14 softmax warp pairs (64 arrivals)
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
   auto b_p = [&](int i) { return smem_u32(bars + 3 + i); };
@@ -196,7 +198,7 @@ __global__ void __launch_bounds__(kThreads)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 11; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 128 : 1);
+    for (int i = 0; i < 15; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 256 : (i >= 11 ? 64 : 1));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -277,31 +279,32 @@ __global__ void __launch_bounds__(kThreads)
       __syncwarp();
     }
   } else {
-    // ---------------- softmax (warps 2..5): thread = query row ----------------
-    const int q4 = warp & 3;
+    // ---------------- softmax (warps 2..9): a row is shared by two warps with the same TMEM
+    // lanes (warp mod 4); half hf of them takes key columns [32 hf, 32 hf + 32) and output
+    // columns [hf hd/2, (hf + 1) hd/2). The pair exchanges its partial row maxima through shared
+    // memory behind an mbarrier of 64 arrivals; the two partial row sums are added at the end.
+    const int q4 = warp & 3, hf = (warp - 2) >> 2;
     const int r = q4 * 32 + lane;
     const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
+    constexpr int OH = HD / 2;
+    const uint32_t b_pair = smem_u32(bars + 11 + q4);
     float m = -INFINITY, l = 0.f, corr_prev = 1.f;
-    float o[HD];
+    float o[OH];
 #pragma unroll
-    for (int i = 0; i < HD; i++) o[i] = 0.f;
+    for (int i = 0; i < OH; i++) o[i] = 0.f;
     // O = O * corr + (P V) of a block; deferred by one block so the P V MMA runs meanwhile
     auto add_pv = [&](int kb, float corr) -> bool {
       const int st = kb & 1;
       if (!__all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
       tc_fence_after();
 #pragma unroll
-      for (int c = 0; c < HD / 64; c++) {
-        uint32_t pa[32], pb[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + c * 64, pa);
-        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + c * 64 + 32, pb);
+      for (int c = 0; c < OH / 32; c++) {
+        uint32_t pa[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + hf * OH + c * 32, pa);
         tmem_wait();
 #pragma unroll
-        for (int j = 0; j < 32; j++) {
-          o[c * 64 + j] = o[c * 64 + j] * corr + __uint_as_float(pa[j]);
-          o[c * 64 + 32 + j] = o[c * 64 + 32 + j] * corr + __uint_as_float(pb[j]);
-        }
+        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + __uint_as_float(pa[j]);
       }
       tc_fence_before();
       return true;
@@ -314,55 +317,51 @@ __global__ void __launch_bounds__(kThreads)
       const int st = kb & 1;
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(st), (uint32_t)(kb >> 1) & 1u, p.err)))) break;
       tc_fence_after();
-      float s[64];
+      float s[32];
       {
-        uint32_t a[32], b[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64, a);
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + 32, b);
+        uint32_t a[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + hf * 32, a);
         tmem_wait();
 #pragma unroll
-        for (int j = 0; j < 32; j++) {
-          s[j] = __uint_as_float(a[j]);
-          s[32 + j] = __uint_as_float(b[j]);
-        }
+        for (int j = 0; j < 32; j++) s[j] = __uint_as_float(a[j]);
       }
       // causal mask, only on blocks that reach past the tile's first position
       if ((int)(kb * BKV + BKV - 1) > pos0_i) {
 #pragma unroll
-        for (int j = 0; j < 64; j++)
-          if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
+        for (int j = 0; j < 32; j++)
+          if (kb * BKV + hf * 32 + j > qpos_i) s[j] = -INFINITY;
       }
-      // row max and row sum with 8 independent chains
-      float mx8[8];
+      float mx4[4];
 #pragma unroll
-      for (int i = 0; i < 8; i++) mx8[i] = s[i];
+      for (int i = 0; i < 4; i++) mx4[i] = s[i];
 #pragma unroll
-      for (int j = 8; j < 64; j++) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      for (int j = 4; j < 32; j++) mx4[j & 3] = fmaxf(mx4[j & 3], s[j]);
+      const float pm = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+      red_m[(kb & 1) * 256 + hf * 128 + r] = pm;
+      mbar_arrive(b_pair);
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pair, (uint32_t)kb & 1u, p.err)))) break;
+      const float mx = fmaxf(pm, red_m[(kb & 1) * 256 + (1 - hf) * 128 + r]);
       const float mn = fmaxf(m, mx);  // finite: key 0 is never masked
       // exactly 1 when the maximum does not change (a fully masked block is then a no-op)
       const float corr = ex2_approx((m - mn) * p.scale_log2);
       const float nb = -mn * p.scale_log2;
-      float sum8[8];
+      float sum4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int i = 0; i < 8; i++) sum8[i] = 0.f;
-#pragma unroll
-      for (int j = 0; j < 64; j++) {
+      for (int j = 0; j < 32; j++) {
         const float e = ex2_approx(fmaf(s[j], p.scale_log2, nb));
         s[j] = e;
-        sum8[j & 7] += e;
+        sum4[j & 3] += e;
       }
-      const float rs = ((sum8[0] + sum8[1]) + (sum8[2] + sum8[3])) + ((sum8[4] + sum8[5]) + (sum8[6] + sum8[7]));
-      l = l * corr + rs;
+      l = l * corr + ((sum4[0] + sum4[1]) + (sum4[2] + sum4[3]));
       m = mn;
       uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
 #pragma unroll
-      for (int c = 0; c < 8; c++) {
+      for (int cc = 0; cc < 4; cc++) {
+        const int c = hf * 4 + cc;
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-          __nv_bfloat162 hb = __floats2bfloat162_rn(s[8 * c + 2 * t], s[8 * c + 2 * t + 1]);
+          __nv_bfloat162 hb = __floats2bfloat162_rn(s[8 * cc + 2 * t], s[8 * cc + 2 * t + 1]);
           wv[t] = *reinterpret_cast<uint32_t*>(&hb);
         }
         *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
@@ -374,11 +373,18 @@ __global__ void __launch_bounds__(kThreads)
       corr_prev = corr;
     }
     if (ok) ok = add_pv(nkb - 1, corr_prev);
+    if (ok) {
+      // row sum = half 0's partial + half 1's partial (the same order in both threads)
+      red_l[hf * 128 + r] = l;
+      mbar_arrive(b_pair);
+      ok = __all_sync(0xffffffffu, mbar_wait(b_pair, (uint32_t)nkb & 1u, p.err));
+    }
     if (ok && r < nrows) {
-      const float inv = 1.f / l;
-      __nv_bfloat16* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
+      const float other = red_l[(1 - hf) * 128 + r];
+      const float inv = 1.f / (hf == 0 ? l + other : other + l);
+      __nv_bfloat16* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD + hf * OH;
 #pragma unroll
-      for (int c = 0; c < HD / 8; c++) {
+      for (int c = 0; c < OH / 8; c++) {
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
