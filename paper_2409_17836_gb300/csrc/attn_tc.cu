@@ -35,13 +35,12 @@ struct Shape {
   static constexpr uint32_t KV_CHUNK = BKV * 128;       // one 64x64 bf16 chunk (8 KiB)
   static constexpr uint32_t K_BYTES = BKV * HD * 2;
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
-  static constexpr uint32_t STAGE_BYTES = K_BYTES + V_BYTES;
+  static constexpr int KS = 3;                          // stages of the K ring and of the V ring
   static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB per P buffer (two)
-  static constexpr int STAGES = 2;
   static constexpr uint32_t TMEM_S = 0;                 // S double buffer: columns 0..127
   static constexpr uint32_t TMEM_O = 128;               // P V double buffer: 2 x HD columns
   static constexpr uint32_t TMEM_COLS = (128 + 2 * HD <= 256) ? 256 : 512;
-  static constexpr size_t SMEM = Q_BYTES + STAGES * STAGE_BYTES + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
+  static constexpr size_t SMEM = Q_BYTES + KS * (K_BYTES + V_BYTES) + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
@@ -167,21 +166,25 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const uint32_t sq = smem_u32(smem);
-  const uint32_t skv = sq + S::Q_BYTES;
-  const uint32_t sp = skv + S::STAGES * S::STAGE_BYTES;  // two P buffers
-  uint8_t* p_gen = smem + S::Q_BYTES + S::STAGES * S::STAGE_BYTES;
+  const uint32_t sk = sq + S::Q_BYTES;                // K ring
+  const uint32_t sv = sk + S::KS * S::K_BYTES;         // V ring
+  const uint32_t sp = sv + S::KS * S::V_BYTES;         // two P buffers
+  uint8_t* p_gen = smem + (sp - sq);
   uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + 2 * S::P_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   float* red_m = reinterpret_cast<float*>(bars + 32);  // [2 parities][2 halves][128 rows]
   float* red_l = red_m + 512;                          // [2 halves][128 rows]
   // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (256 arrivals) | 5-6 P V ready |
-  //           7-8 K/V stage loaded | 9-10 K/V stage free | 11-14 softmax warp pairs (64 arrivals)
+  //           7-9 K stage loaded | 10-12 K stage free | 13-15 V stage loaded | 16-18 V stage free |
+  //           19-22 softmax warp pairs (64 arrivals)
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
   auto b_p = [&](int i) { return smem_u32(bars + 3 + i); };
   auto b_pv = [&](int i) { return smem_u32(bars + 5 + i); };
-  auto b_kvfull = [&](int i) { return smem_u32(bars + 7 + i); };
-  auto b_kvempty = [&](int i) { return smem_u32(bars + 9 + i); };
+  auto b_kfull = [&](int i) { return smem_u32(bars + 7 + i); };
+  auto b_kempty = [&](int i) { return smem_u32(bars + 10 + i); };
+  auto b_vfull = [&](int i) { return smem_u32(bars + 13 + i); };
+  auto b_vempty = [&](int i) { return smem_u32(bars + 16 + i); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -198,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 15; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 256 : (i >= 11 ? 64 : 1));
+    for (int i = 0; i < 23; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 256 : (i >= 19 ? 64 : 1));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -222,38 +225,45 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     }
     __syncwarp();
     for (int kb = 0; kb < nkb; kb++) {
-      const int st = kb & 1;
-      const uint32_t ph = (uint32_t)(kb >> 1) & 1u;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kvempty(st), ph ^ 1u, p.err))) break;
+      const int ks = kb % S::KS;
+      const uint32_t ph = (uint32_t)(kb / S::KS) & 1u;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kempty(ks), ph ^ 1u, p.err))) break;
       if (lane == 0) {
-        const uint32_t base = skv + st * S::STAGE_BYTES;
-        mbar_expect_tx(b_kvfull(st), S::STAGE_BYTES);
+        mbar_expect_tx(b_kfull(ks), S::K_BYTES);
 #pragma unroll
-        for (int c = 0; c < S::KCH; c++) {
-          tma_load_2d(base + c * S::KV_CHUNK, &tkv, b_kvfull(st), p.k_col0 + kvh * HD + 64 * c, kv_row0 + kb * BKV);
-          tma_load_2d(base + S::K_BYTES + c * S::KV_CHUNK, &tkv, b_kvfull(st), p.v_col0 + kvh * HD + 64 * c,
+        for (int c = 0; c < S::KCH; c++)
+          tma_load_2d(sk + ks * S::K_BYTES + c * S::KV_CHUNK, &tkv, b_kfull(ks), p.k_col0 + kvh * HD + 64 * c,
                       kv_row0 + kb * BKV);
-        }
+      }
+      __syncwarp();
+      if (!__all_sync(0xffffffffu, mbar_wait(b_vempty(ks), ph ^ 1u, p.err))) break;
+      if (lane == 0) {
+        mbar_expect_tx(b_vfull(ks), S::V_BYTES);
+#pragma unroll
+        for (int c = 0; c < S::KCH; c++)
+          tma_load_2d(sv + ks * S::V_BYTES + c * S::KV_CHUNK, &tkv, b_vfull(ks), p.v_col0 + kvh * HD + 64 * c,
+                      kv_row0 + kb * BKV);
       }
       __syncwarp();
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer: S(kb+1) is issued before P V(kb) so the softmax of block kb
-    // overlaps the tensor cores ----------------
+    // overlaps the tensor cores; a K stage is released as soon as its S is done ----------------
     auto issue_s = [&](int kb) -> bool {
-      const int st = kb & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kvfull(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
+      const int ks = kb % S::KS;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KS) & 1u, p.err))) return false;
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t kbase = skv + st * S::STAGE_BYTES;
+        const uint32_t kbase = sk + ks * S::K_BYTES;
         // S = Q K^T over hd in steps of 16 (32 bytes inside a 128-byte chunk)
 #pragma unroll
         for (int k = 0; k < HD / 16; k++) {
           const int c = k >> 2, o = (k & 3) * 32;
-          tc_mma(tmem + S::TMEM_S + st * 64, desc_kmajor(sq + c * (BQ * 128) + o),
+          tc_mma(tmem + S::TMEM_S + (kb & 1) * 64, desc_kmajor(sq + c * (BQ * 128) + o),
                  desc_kmajor(kbase + c * S::KV_CHUNK + o), S::IDESC_S, k > 0 ? 1u : 0u);
         }
-        tc_commit(b_s(st));
+        tc_commit(b_s(kb & 1));
+        tc_commit(b_kempty(ks));
       }
       __syncwarp();
       return true;
@@ -261,20 +271,21 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
     if (ok) ok = issue_s(0);
     for (int kb = 0; kb < nkb && ok; kb++) {
-      const int st = kb & 1;
+      const int st = kb & 1, ks = kb % S::KS;
       if (kb + 1 < nkb && !(ok = issue_s(kb + 1))) break;
-      ok = __all_sync(0xffffffffu, mbar_wait(b_p(st), (uint32_t)(kb >> 1) & 1u, p.err));
+      ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(ks), (uint32_t)(kb / S::KS) & 1u, p.err));
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(st), (uint32_t)(kb >> 1) & 1u, p.err));
       if (!ok) break;
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t vbase = skv + st * S::STAGE_BYTES + S::K_BYTES;
+        const uint32_t vbase = sv + ks * S::V_BYTES;
         // O_blk = P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
           tc_mma(tmem + S::TMEM_O + st * HD, desc_kmajor(sp + st * S::P_BYTES + k * 32),
                  desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, k > 0 ? 1u : 0u);
         tc_commit(b_pv(st));
-        tc_commit(b_kvempty(st));
+        tc_commit(b_vempty(ks));
       }
       __syncwarp();
     }
@@ -288,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
     constexpr int OH = HD / 2;
-    const uint32_t b_pair = smem_u32(bars + 11 + q4);
+    const uint32_t b_pair = smem_u32(bars + 19 + q4);
     float m = -INFINITY, l = 0.f, corr_prev = 1.f;
     float o[OH];
 #pragma unroll
