@@ -131,6 +131,67 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
     return dt, min(positions, seg.size)
 
 
+def microbenchmarks(L, ctx, pk, reps: int = 3) -> dict:
+    """HBM-bound stages at sizes where bandwidth, not launch latency, decides: the serialiser on
+    the 64M-value Laplace mixture, and the coder alone on 2^18 windows x 2048 tokens of seeded
+    random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most likely)."""
+    import numpy as np
+    import torch
+
+    from paper_2409_17836_gb300 import inputs
+
+    out = {}
+    vals = inputs.laplace_gradient()
+    d = torch.from_numpy(vals.view(np.int32)).cuda()
+    tok = torch.empty(d.numel() * ctx.tpv, dtype=torch.int16, device="cuda")
+    L.lmgc_serialize(ctx, d, tok)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        L.lmgc_serialize(ctx, d, tok)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    nbytes = d.numel() * 4 + tok.numel() * 2
+    out["serialize"] = {"values": d.numel(), "ms": ms, "bytes": nbytes, "achieved": nbytes / ms / 1e6,
+                        "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
+    del d, tok
+    V, P, W, n_win = 32000, 24, 2048, 1 << 18
+    g = torch.Generator(device="cuda").manual_seed(5)
+    z = torch.randn(256, V, generator=g, device="cuda") * torch.linspace(0.3, 6.0, 256, device="cuda")[:, None]
+    cdf = L.lmgc_quantize_cdf(ctx, z).long()
+    likely = torch.argmax(cdf[:, 1:] - cdf[:, :-1], dim=1)
+    start = torch.empty((W, n_win), dtype=torch.int32, device="cuda")  # position-major
+    freq = torch.empty_like(start)
+    step = 1 << 15
+    for w0 in range(0, n_win, step):
+        row = torch.randint(0, 256, (W, step), generator=g, device="cuda")
+        sym = torch.randint(0, V, (W, step), generator=g, device="cuda")
+        sym = torch.where(torch.rand((W, step), generator=g, device="cuda") < 0.5, likely[row], sym)
+        st = cdf[row, sym]
+        start[:, w0:w0 + step] = st.int()
+        freq[:, w0:w0 + step] = (cdf[row, sym + 1] - st).int()
+        del row, sym, st
+    payload, _ = L.lmgc_range_encode(start, freq, P, n_win, W, None, 1, n_win)
+    torch.cuda.synchronize()
+    L.lmgc_profile(None, True)
+    for _ in range(reps):
+        payload, _ = L.lmgc_range_encode(start, freq, P, n_win, W, None, 1, n_win, out=payload)
+    st = L.lmgc_kernel_stats(None)["range_encode"]
+    L.lmgc_profile(None, False)
+    kms = st["ms"] / max(1, st["launches"])
+    rd = 8.0 * W * n_win
+    wr = float(payload.numel())
+    out["range_encode"] = {"windows": n_win, "tokens": W * n_win, "ms": kms, "read_bytes": rd, "write_bytes": wr,
+                           "bits_per_token": 8.0 * wr / (W * n_win), "achieved": (rd + wr) / kms / 1e6,
+                           "unit": "GB/s", "frac": (rd + wr) / kms / 1e6 / pk["hbm"],
+                           "tokens_per_s": W * n_win / (kms / 1e3)}
+    del start, freq, payload
+    torch.cuda.empty_cache()
+    return out
+
+
 def bytes_per_value(cfg) -> int:
     return 4 if cfg.input_kind == 0 else 1
 
@@ -178,6 +239,7 @@ def main():
     ap.add_argument("--ref-positions", type=int, default=12)
     ap.add_argument("--cpu-target-s", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-micro", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -280,6 +342,9 @@ def main():
             e.update(achieved=st["work"] / (st["ms"] / 1e3) / 1e9, unit="GB/s")
             e["frac"] = e["achieved"] / pk["hbm"]
         stages[name] = e
+    micro = None
+    if rank == 0 and not args.no_micro and cfg.vocab == 32000:
+        micro = microbenchmarks(L, ctx, pk)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         threads = max(1, len(os.sched_getaffinity(0)))
@@ -302,7 +367,7 @@ def main():
                           "l2": "no flush: each step reads > L2 (model weights and per-batch logits)",
                           "parallelism": f"windows sharded over {world} GPU(s), no collective on the data path"},
                "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
-               "stages": stages, "stage_ms_last_step": L.lmgc_stage_times(ctx),
+               "stages": stages, "microbench": micro, "stage_ms_last_step": L.lmgc_stage_times(ctx),
                "compression_rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv), "cpu_baseline": cpu}
         print(json.dumps(res), flush=True)
     ctx.close()

@@ -217,7 +217,9 @@ lmgc_status lmgc_launch_count(uint64_t* n);
  * lmgc_profile(ctx, 0) stops. lmgc_kernel_stats returns, for class cls, its name, the launches
  * and summed device milliseconds recorded, and the summed algorithmic work of those launches
  * (flops for 0 "gemm" and 1 "attention"; bytes for 2 "cdf_pairs", 3 "range_encode",
- * 4 "serialize"; 0 for 5 "norm_rope_act" and 6 "other"). Errors: INVALID (cls outside 0..6). */
+ * 4 "serialize"; 0 for 5 "norm_rope_act" and 6 "other"). ctx == NULL selects the process-wide
+ * counters of the context-free entry points (lmgc_range_encode: its coder kernel, class 3).
+ * Errors: INVALID (cls outside 0..6). */
 lmgc_status lmgc_profile(lmgc_ctx* ctx, int enable);
 lmgc_status lmgc_kernel_stats(const lmgc_ctx* ctx, int cls, char* name, size_t name_len, int* launches, float* ms,
                               double* work);

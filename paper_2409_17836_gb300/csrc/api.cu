@@ -74,11 +74,22 @@ static cudaEvent_t prof_event(lmgc_ctx* ctx) {
   return e;
 }
 
+// Context-free entry points (lmgc_range_encode) record into this process-wide context.
+static lmgc_ctx* free_ctx() {
+  static lmgc_ctx* c = [] {
+    lmgc_ctx* x = new lmgc_ctx();
+    for (int i = 0; i < kNumClasses; i++) x->prof.stats[i] = KernelStat{kClassNames[i], 0, 0.f, 0.0};
+    return x;
+  }();
+  return c;
+}
+
 struct ProfScope {
   lmgc_ctx* ctx;
   cudaStream_t s;
   bool on;
-  ProfScope(lmgc_ctx* c, int cls, double work, cudaStream_t st) : ctx(c), s(st), on(c->prof.enabled) {
+  ProfScope(lmgc_ctx* c, int cls, double work, cudaStream_t st) : ctx(c ? c : free_ctx()), s(st) {
+    on = ctx->prof.enabled;
     if (!on) return;
     Profiler::Rec r;
     r.cls = cls;
@@ -489,8 +500,11 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
   if (e != cudaSuccess) {
     st = cuda_fail(nullptr, e, "range_encode scratch");
   } else {
-    launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
-                        (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
+    {
+      ProfScope ps(nullptr, kCoder, 8.0 * (double)n_win * (double)win_tokens, s);
+      launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
+                          (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
+    }
     launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
     uint64_t total = 0;
     uint32_t herr = 0;
@@ -513,6 +527,7 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
   if (offs) cudaFreeAsync(offs, s);
   if (derr) cudaFreeAsync(derr, s);
   cudaStreamSynchronize(s);
+  if (free_ctx()->prof.enabled) prof_collect(free_ctx());
   return st;
 }
 
@@ -775,7 +790,7 @@ lmgc_status lmgc_stage_times(const lmgc_ctx* ctx, float* ms, size_t n_ms) {
 }
 
 lmgc_status lmgc_profile(lmgc_ctx* ctx, int enable) {
-  if (!ctx) return LMGC_ERR_INVALID;
+  if (!ctx) ctx = free_ctx();
   ctx->prof.enabled = enable != 0;
   for (int i = 0; i < kNumClasses; i++) ctx->prof.stats[i] = KernelStat{kClassNames[i], 0, 0.f, 0.0};
   return LMGC_OK;
@@ -783,7 +798,8 @@ lmgc_status lmgc_profile(lmgc_ctx* ctx, int enable) {
 
 lmgc_status lmgc_kernel_stats(const lmgc_ctx* ctx, int cls, char* name, size_t name_len, int* launches, float* ms,
                               double* work) {
-  if (!ctx || cls < 0 || cls >= kNumClasses) return LMGC_ERR_INVALID;
+  if (!ctx) ctx = free_ctx();
+  if (cls < 0 || cls >= kNumClasses) return LMGC_ERR_INVALID;
   const KernelStat& st = ctx->prof.stats[cls];
   if (name && name_len) {
     size_t n = std::min(name_len - 1, strlen(kClassNames[cls]));

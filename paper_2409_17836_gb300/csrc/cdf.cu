@@ -13,7 +13,7 @@
 //
 // The encode path never materialises a CDF (V = 32000 would be 128 KB per token): one block per
 // row reduces max, sum e and argmax, then sum_{j<s} g_j and g_s for the row's symbol s.
-// floor(X / S) with X < 2^55 and S < 2^47 uses a reciprocal floor(2^64-1 / S) and one correction.
+// floor(e (T - V) / S) uses a 32-bit fixed-point reciprocal of S and one exact remainder test.
 #include <math.h>
 
 #include <algorithm>
@@ -60,14 +60,6 @@ __device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t*
   uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
   uint64_t e = (hl + (1ull << 30)) >> 31;
   return (uint32_t)(e >> (a >> 16));
-}
-
-// floor(X / S) given minv = floor((2^64 - 1) / S), X < 2^56, S > 0
-__device__ __forceinline__ uint64_t div_floor(uint64_t X, uint64_t S, uint64_t minv) {
-  uint64_t q = __umul64hi(X, minv);
-  uint64_t r = X - q * S;
-  if (r >= S) q++;
-  return q;
 }
 
 template <typename V>
@@ -123,9 +115,19 @@ __device__ __forceinline__ uint64_t block_argmax(uint64_t key, uint64_t* red) {
 
 struct RowStats {
   float m;
-  uint64_t S, minv, Mq;
+  uint64_t S, Mq;
+  uint32_t F;  // floor(Mq * 2^32 / S): floor(e * Mq / S) is (e * F) >> 32 or one more
   int amax;
 };
+
+// g = floor(e * Mq / S) exactly: q0 = (e F) >> 32 satisfies g - 1 <= q0 <= g (e <= 2^31 and
+// S >= 2^31, the largest e being 2^31), and q0 S <= e Mq < 2^61, so one remainder test fixes it.
+__device__ __forceinline__ uint64_t gfloor(uint32_t e, const RowStats& st) {
+  const uint64_t X = (uint64_t)e * st.Mq;
+  uint64_t q = ((uint64_t)e * st.F) >> 32;
+  if (X - q * st.S >= st.S) q++;
+  return q;
+}
 
 // Passes 1 and 2 over a row: max, sum of e, lowest-index argmax of e.
 __device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V, int P, const uint32_t* H,
@@ -134,19 +136,23 @@ __device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V
   float m = -INFINITY;
   for (int j = threadIdx.x; j < V; j += kCdfThreads) m = fmaxf(m, __ldg(z + j));
   m = block_max(m, redf);
-  uint64_t S = 0, best = 0;
-  for (int j = threadIdx.x; j < V; j += kCdfThreads) {
-    uint32_t e = exp2_fixed(__ldg(z + j), m, H, L);
+  uint64_t S = 0;
+  uint32_t best_e = 0;
+  int best_j = 0x7fffffff;
+  for (int j = threadIdx.x; j < V; j += kCdfThreads) {  // j increases: strict > keeps the lowest index
+    const uint32_t e = exp2_fixed(__ldg(z + j), m, H, L);
     S += e;
-    uint64_t key = ((uint64_t)e << 32) | (uint32_t)(~(uint32_t)j);
-    best = key > best ? key : best;
+    if (e > best_e) {
+      best_e = e;
+      best_j = j;
+    }
   }
   S = block_sum_u64(S, redu);
-  best = block_argmax(best, redu);
+  const uint64_t best = block_argmax(((uint64_t)best_e << 32) | (uint32_t)(~(uint32_t)best_j), redu);
   st.m = m;
   st.S = S;
-  st.minv = ~0ull / S;
   st.Mq = (1ull << P) - (uint64_t)V;
+  st.F = (uint32_t)((st.Mq << 32) / S);
   st.amax = (int)(~(uint32_t)(best & 0xFFFFFFFFu));
   return st;
 }
@@ -184,17 +190,18 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
     }
     const float* z = logits + r * (int64_t)V;
     RowStats st = row_stats(z, V, P, H, L, redf, redu);
-    uint64_t gall = 0, gbelow = 0, gsym = 0;
-    for (int j = threadIdx.x; j < V; j += kCdfThreads) {
-      uint64_t e = exp2_fixed(__ldg(z + j), st.m, H, L);
-      uint64_t g = div_floor(e * st.Mq, st.S, st.minv);
-      gall += g;
-      gbelow += j < sym ? g : 0ull;
-      gsym += j == sym ? g : 0ull;
+    uint64_t gall = 0;
+    for (int j = threadIdx.x; j < V; j += kCdfThreads) gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
+    // g below the coded symbol and g of the symbol: only j <= sym, packed as (below << 32) + at
+    // (each part < 2^31)
+    uint64_t packed = 0;
+    for (int j = threadIdx.x; j <= sym && j < V; j += kCdfThreads) {
+      const uint64_t g = gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
+      packed += j < sym ? (g << 32) : g;
     }
     gall = block_sum_u64(gall, redu);
-    gbelow = block_sum_u64(gbelow, redu);
-    gsym = block_sum_u64(gsym, redu);
+    packed = block_sum_u64(packed, redu);
+    const uint64_t gbelow = packed >> 32, gsym = packed & 0xFFFFFFFFull;
     if (threadIdx.x == 0) {
       uint64_t resid = st.Mq - gall;
       start[out_idx] = (uint32_t)(sym + gbelow + (st.amax < sym ? resid : 0ull));
@@ -259,7 +266,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_quantize_cdf(const float* __res
     RowStats st = row_stats(z, V, P, H, L, redf, redu);
     uint64_t gall = 0;
     for (int j = threadIdx.x; j < V; j += kCdfThreads)
-      gall += div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+      gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
     gall = block_sum_u64(gall, redu);
     const uint64_t resid = st.Mq - gall;
     uint64_t run = 0;
@@ -268,7 +275,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_quantize_cdf(const float* __res
       int j = j0 + threadIdx.x;
       uint64_t f = 0;
       if (j < V) {
-        f = 1 + div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+        f = 1 + gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
         if (j == st.amax) f += resid;
       }
       uint64_t tot;
@@ -357,7 +364,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_dec_search(const float* __restr
   RowStats st = row_stats(z, V, P, H, L, redf, redu);
   uint64_t gall = 0;
   for (int j = threadIdx.x; j < V; j += kCdfThreads)
-    gall += div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+    gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
   gall = block_sum_u64(gall, redu);
   const uint64_t resid = st.Mq - gall;
   if (threadIdx.x == 0) found_s = -1;
@@ -366,7 +373,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_dec_search(const float* __restr
     int j = j0 + threadIdx.x;
     uint64_t f = 0;
     if (j < V) {
-      f = 1 + div_floor((uint64_t)exp2_fixed(__ldg(z + j), st.m, H, L) * st.Mq, st.S, st.minv);
+      f = 1 + gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
       if (j == st.amax) f += resid;
     }
     uint64_t tot;

@@ -301,17 +301,18 @@ def lmgc_launch_count() -> int:
     return n.value
 
 
-def lmgc_profile(ctx: Context, enable: bool) -> None:
-    _check(ctx, load().lmgc_profile(ctx.handle, int(enable)))
+def lmgc_profile(ctx: Context | None, enable: bool) -> None:
+    """ctx None: the process-wide counters of the context-free entry points."""
+    _check(ctx, load().lmgc_profile(ctx.handle if ctx is not None else None, int(enable)))
 
 
-def lmgc_kernel_stats(ctx: Context) -> dict:
+def lmgc_kernel_stats(ctx: Context | None) -> dict:
     out = {}
     for cls in range(len(KERNEL_CLASSES)):
         name = C.create_string_buffer(32)
         launches, ms, work = C.c_int(), C.c_float(), C.c_double()
-        _check(ctx, load().lmgc_kernel_stats(ctx.handle, cls, name, 32, C.byref(launches), C.byref(ms),
-                                             C.byref(work)))
+        _check(ctx, load().lmgc_kernel_stats(ctx.handle if ctx is not None else None, cls, name, 32,
+                                             C.byref(launches), C.byref(ms), C.byref(work)))
         out[name.value.decode()] = dict(launches=launches.value, ms=ms.value, work=work.value)
     return out
 
