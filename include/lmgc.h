@@ -189,6 +189,22 @@ lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);
 lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_out, size_t cap, size_t* out_bytes,
                         lmgc_stream stream);
 
+/* The windows [first_win, first_win + n_win) of lmgc_encode's container, for encoding a stream
+ * sharded over several GPUs (windows are independent, Sec. 3 "Compression"): all n values are
+ * serialised, only the given windows are modelled and coded. d_payload receives their codes
+ * byte-aligned in window order (the container's payload slice), d_bitlen (device, n_win) their
+ * bit lengths, *payload_bytes (host) the slice size. A container is the header of
+ * lmgc_container_header, the bit lengths of all windows in order, then all payload slices in
+ * order. Errors: INVALID (range outside the stream), NO_SPACE (*payload_bytes = required), CUDA.
+ * Syncs. */
+lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_t first_win, size_t n_win,
+                                uint8_t* d_payload, size_t cap, size_t* payload_bytes, uint32_t* d_bitlen,
+                                lmgc_stream stream);
+
+/* The 64-byte container header (layout under lmgc_encode) for n input values, written to the
+ * host buffer h_header. */
+lmgc_status lmgc_container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h_header);
+
 /* lmgc_encode with HOST buffers: copies h_in to the device, encodes, copies the container back
  * to h_out. The device staging buffers are owned by the context and reused across calls. */
 lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t* h_out, size_t cap,

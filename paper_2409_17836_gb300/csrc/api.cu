@@ -539,15 +539,19 @@ lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes) {
   return LMGC_OK;
 }
 
-lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_out, size_t cap, size_t* out_bytes,
-                        lmgc_stream stream) {
-  if (!ctx || !d_in || !out_bytes) return fail(ctx, LMGC_ERR_INVALID, "null argument");
-  if (n == 0) return fail(ctx, LMGC_ERR_INVALID, "empty input");
+}  // extern "C"
+
+namespace lmgc {
+
+// Phase 1 of an encode: serialise all n values, then model, CDF pairs and coder for the windows
+// [w_begin, w_begin + w_count) of the token stream. The codes stay in the context's slot scratch;
+// *payload receives their packed size. Phase 2 (encode_pack) writes them out.
+static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64_t w_begin, int64_t w_count,
+                                uint64_t* payload, cudaStream_t s) {
   const lmgc_config& c = ctx->cfg;
-  cudaStream_t s = (cudaStream_t)stream;
   const int64_t W = c.window, P = c.cdf_bits;
   const int64_t n_tok = (int64_t)n * ctx->tpv;
-  const int64_t n_win = (n_tok + W - 1) / W;
+  const int64_t n_win = w_count;
   const size_t slot = slot_bytes((size_t)W, (int)P);
   // staging (grown on demand; reused across calls)
   LMGC_CUDA(ctx, ensure(&ctx->tok, &ctx->tok_cap, (size_t)n_tok * 2 + 16));
@@ -560,9 +564,11 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
                sl_off = of_off + (((size_t)n_win + 1) * 8 + 255) / 256 * 256;
   LMGC_CUDA(ctx, ensure(&ctx->win_len, &ctx->win_cap, sl_off + slot * (size_t)n_win));
   uint32_t* d_wl = (uint32_t*)((char*)ctx->win_len + wl_off);
-  uint32_t* d_bl = (uint32_t*)((char*)ctx->win_len + bl_off);
-  uint64_t* d_off = (uint64_t*)((char*)ctx->win_len + of_off);
-  uint8_t* d_slots = (uint8_t*)ctx->win_len + sl_off;
+  ctx->enc_bl = (uint32_t*)((char*)ctx->win_len + bl_off);
+  ctx->enc_off = (uint64_t*)((char*)ctx->win_len + of_off);
+  ctx->enc_slots = (uint8_t*)ctx->win_len + sl_off;
+  ctx->enc_slot = slot;
+  ctx->enc_nwin = n_win;
 
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[0], s));
   {
@@ -578,61 +584,45 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
   }
   cudaEventRecord(ctx->batch_ev[0], s);
   for (int64_t b = 0; b < n_batches; b++) {
-    const int64_t w0 = b * c.batch_windows;
-    const int64_t nb = std::min<int64_t>(c.batch_windows, n_win - w0);
+    const int64_t w0 = w_begin + b * c.batch_windows;
+    const int64_t nb = std::min<int64_t>(c.batch_windows, w_begin + n_win - w0);
     forward_windows(ctx, ctx->tok, n_tok, w0, nb, s);
     cudaEventRecord(ctx->batch_ev[2 * b + 1], s);
     {
       const int64_t rows = nb * W;
       ProfScope ps(ctx, kCdf, (double)rows * ((double)c.vocab * 4 + 2 + 8), s);
       launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
-                       ctx->pair_start, ctx->pair_freq, 1, s);
+                       ctx->pair_start, ctx->pair_freq, 1, s, w_begin);
     }
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[2], s));
   note_launch();
-  k_fill_win_len<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(d_wl, n_win, W, n_tok);
+  k_fill_win_len<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(d_wl, n_win, W, n_tok - w_begin * W);
   {
-    ProfScope ps(ctx, kCoder, (double)n_tok * 8, s);
-    launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 1, n_win, d_slots, slot, d_bl,
-                        ctx->d_err, s);
+    ProfScope ps(ctx, kCoder, (double)n_win * (double)W * 8, s);
+    launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 1, n_win, ctx->enc_slots, slot,
+                        ctx->enc_bl, ctx->d_err, s);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[3], s));
-  launch_pack_codes(d_slots, slot, d_bl, n_win, d_off, nullptr, s);
-  uint64_t payload = 0;
-  LMGC_CUDA(ctx, cudaMemcpyAsync(&payload, d_off + n_win, 8, cudaMemcpyDeviceToHost, s));
+  launch_pack_codes(ctx->enc_slots, slot, ctx->enc_bl, n_win, ctx->enc_off, nullptr, s);
+  LMGC_CUDA(ctx, cudaMemcpyAsync(payload, ctx->enc_off + n_win, 8, cudaMemcpyDeviceToHost, s));
   lmgc_status st = check_err_word(ctx, s, "encode");
-  if (st != LMGC_OK) return st;
-  const size_t total = 64 + 4 * (size_t)n_win + payload;
-  *out_bytes = total;
-  if (cap < total || !d_out) return fail(ctx, LMGC_ERR_NO_SPACE, "container buffer too small");
-  // header
-  uint8_t h[64];
-  memset(h, 0, 64);
-  uint32_t u32;
-  uint64_t u64;
-  memcpy(h, "LMGC", 4);
-  u32 = 1; memcpy(h + 4, &u32, 4);
-  u64 = n; memcpy(h + 8, &u64, 8);
-  u64 = (uint64_t)n_tok; memcpy(h + 16, &u64, 8);
-  u32 = (uint32_t)W; memcpy(h + 24, &u32, 4);
-  u32 = (uint32_t)P; memcpy(h + 28, &u32, 4);
-  u32 = (uint32_t)c.input_kind; memcpy(h + 32, &u32, 4);
-  u32 = (uint32_t)c.sep_mode; memcpy(h + 36, &u32, 4);
-  u32 = (uint32_t)c.vocab; memcpy(h + 40, &u32, 4);
-  u32 = (uint32_t)n_win; memcpy(h + 44, &u32, 4);
-  u64 = c.weight_seed; memcpy(h + 48, &u64, 8);
-  u32 = model_crc(c); memcpy(h + 56, &u32, 4);
-  u32 = crc32(h, 60); memcpy(h + 60, &u32, 4);
-  LMGC_CUDA(ctx, cudaMemcpyAsync(d_out, h, 64, cudaMemcpyHostToDevice, s));
-  LMGC_CUDA(ctx, cudaMemcpyAsync(d_out + 64, d_bl, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
-  launch_pack_codes(d_slots, slot, d_bl, n_win, d_off, d_out + 64 + 4 * (size_t)n_win, s);
+  ctx->enc_batches = n_batches;
+  return st;
+}
+
+// Phase 2: the codes of the last encode_codes call, byte-aligned in window order, to d_payload;
+// their bit lengths to d_bitlen (device).
+static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bitlen, cudaStream_t s) {
+  const int64_t n_win = ctx->enc_nwin;
+  LMGC_CUDA(ctx, cudaMemcpyAsync(d_bitlen, ctx->enc_bl, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
+  launch_pack_codes(ctx->enc_slots, ctx->enc_slot, ctx->enc_bl, n_win, ctx->enc_off, d_payload, s);
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[5], s));
   LMGC_CUDA(ctx, cudaStreamSynchronize(s));
   LMGC_CUDA(ctx, cudaGetLastError());
   float x = 0.f, ms_lm = 0.f, ms_cdf = 0.f;
-  for (int64_t b = 0; b < n_batches; b++) {
+  for (int64_t b = 0; b < ctx->enc_batches; b++) {
     cudaEventElapsedTime(&x, ctx->batch_ev[2 * b], ctx->batch_ev[2 * b + 1]);
     ms_lm += x;
     cudaEventElapsedTime(&x, ctx->batch_ev[2 * b + 1], ctx->batch_ev[2 * b + 2]);
@@ -647,6 +637,74 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
   cudaEventElapsedTime(&x, ctx->ev[3], ctx->ev[5]);
   ctx->stage_ms[4] = x;
   if (ctx->prof.enabled) prof_collect(ctx);
+  return LMGC_OK;
+}
+
+static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
+  const lmgc_config& c = ctx->cfg;
+  const uint64_t n_tok = (uint64_t)n * (uint64_t)ctx->tpv;
+  const uint64_t n_win = (n_tok + (uint64_t)c.window - 1) / (uint64_t)c.window;
+  memset(h, 0, 64);
+  uint32_t u32;
+  uint64_t u64;
+  memcpy(h, "LMGC", 4);
+  u32 = 1; memcpy(h + 4, &u32, 4);
+  u64 = n; memcpy(h + 8, &u64, 8);
+  u64 = n_tok; memcpy(h + 16, &u64, 8);
+  u32 = (uint32_t)c.window; memcpy(h + 24, &u32, 4);
+  u32 = (uint32_t)c.cdf_bits; memcpy(h + 28, &u32, 4);
+  u32 = (uint32_t)c.input_kind; memcpy(h + 32, &u32, 4);
+  u32 = (uint32_t)c.sep_mode; memcpy(h + 36, &u32, 4);
+  u32 = (uint32_t)c.vocab; memcpy(h + 40, &u32, 4);
+  u32 = (uint32_t)n_win; memcpy(h + 44, &u32, 4);
+  u64 = c.weight_seed; memcpy(h + 48, &u64, 8);
+  u32 = model_crc(c); memcpy(h + 56, &u32, 4);
+  u32 = crc32(h, 60); memcpy(h + 60, &u32, 4);
+}
+
+}  // namespace lmgc
+
+extern "C" {
+
+lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_out, size_t cap, size_t* out_bytes,
+                        lmgc_stream stream) {
+  if (!ctx || !d_in || !out_bytes) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  if (n == 0) return fail(ctx, LMGC_ERR_INVALID, "empty input");
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t W = ctx->cfg.window;
+  const int64_t n_win = ((int64_t)n * ctx->tpv + W - 1) / W;
+  uint64_t payload = 0;
+  lmgc_status st = encode_codes(ctx, d_in, n, 0, n_win, &payload, s);
+  if (st != LMGC_OK) return st;
+  const size_t total = 64 + 4 * (size_t)n_win + payload;
+  *out_bytes = total;
+  if (cap < total || !d_out) return fail(ctx, LMGC_ERR_NO_SPACE, "container buffer too small");
+  uint8_t h[64];
+  container_header(ctx, n, h);
+  LMGC_CUDA(ctx, cudaMemcpyAsync(d_out, h, 64, cudaMemcpyHostToDevice, s));
+  return encode_pack(ctx, d_out + 64 + 4 * (size_t)n_win, (uint32_t*)(d_out + 64), s);
+}
+
+lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_t first_win, size_t n_win,
+                                uint8_t* d_payload, size_t cap, size_t* payload_bytes, uint32_t* d_bitlen,
+                                lmgc_stream stream) {
+  if (!ctx || !d_in || !payload_bytes || (n_win && !d_bitlen)) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  const int64_t W = ctx->cfg.window;
+  const int64_t total_win = ((int64_t)n * ctx->tpv + W - 1) / W;
+  if (n == 0 || n_win == 0 || (int64_t)(first_win + n_win) > total_win)
+    return fail(ctx, LMGC_ERR_INVALID, "window range outside the stream");
+  cudaStream_t s = (cudaStream_t)stream;
+  uint64_t payload = 0;
+  lmgc_status st = encode_codes(ctx, d_in, n, (int64_t)first_win, (int64_t)n_win, &payload, s);
+  if (st != LMGC_OK) return st;
+  *payload_bytes = payload;
+  if (cap < payload || !d_payload) return fail(ctx, LMGC_ERR_NO_SPACE, "payload buffer too small");
+  return encode_pack(ctx, d_payload, d_bitlen, s);
+}
+
+lmgc_status lmgc_container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h_header) {
+  if (!ctx || !h_header) return LMGC_ERR_INVALID;
+  container_header(ctx, n, h_header);
   return LMGC_OK;
 }
 

@@ -165,7 +165,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
                                                            const uint16_t* __restrict__ tok, int64_t n_tok, int W,
                                                            int64_t first_win, int64_t stride_pos,
                                                            uint32_t* __restrict__ start, uint32_t* __restrict__ freq,
-                                                           int mode) {
+                                                           int mode, int64_t pair_win0) {
   __shared__ uint32_t H[256], L[256];
   __shared__ float redf[32];
   __shared__ uint64_t redu[32];
@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
       int64_t g = (first_win + wl) * W + i;
       if (g >= n_tok) continue;  // block-uniform
       sym = tok[g];
-      out_idx = (int64_t)i * stride_pos + (first_win + wl);
+      out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
     }
     const float* z = logits + r * (int64_t)V;
     RowStats st = row_stats(z, V, P, H, L, redf, redu);
@@ -212,12 +212,12 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
 
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
                       int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s) {
+                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0) {
   if (rows <= 0) return;
   unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
   note_launch();
   k_cdf_pairs<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win, pair_stride_pos,
-                                             start, freq, mode);
+                                             start, freq, mode, pair_win0);
 }
 
 // Block inclusive scan of one u64 per thread; returns the inclusive prefix; *total the tile sum.

@@ -87,6 +87,12 @@ struct lmgc_ctx {
   // decode state
   void* kv_cache = nullptr;
   size_t kv_cap = 0;
+  // codes of the last encode (slot scratch inside win_len)
+  uint32_t* enc_bl = nullptr;
+  uint64_t* enc_off = nullptr;
+  uint8_t* enc_slots = nullptr;
+  size_t enc_slot = 0;
+  int64_t enc_nwin = 0, enc_batches = 0;
   float stage_ms[5] = {0, 0, 0, 0, 0};
   cudaEvent_t ev[6] = {};
   std::vector<cudaEvent_t> batch_ev;
@@ -154,9 +160,10 @@ void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t ds
 
 // cdf.cu
 void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s);  // builds H and L on the host
+// mode 1: pair index i * pair_stride_pos + (window - pair_win0)
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
                       int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s);
+                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0 = 0);
 void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
                          cudaStream_t s);
 void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,

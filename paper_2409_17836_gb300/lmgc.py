@@ -83,6 +83,9 @@ SYMBOLS = {
                                             C.c_void_p]),
     "lmgc_encode_bound": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
+    "lmgc_encode_windows": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_size_t, C.c_size_t, C.c_void_p,
+                                      C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "lmgc_container_header": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_encode_host": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p,
                                    C.c_void_p]),
     "lmgc_decode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t,
@@ -268,6 +271,26 @@ def lmgc_encode(ctx: Context, values: torch.Tensor, out: torch.Tensor | None = N
     _check(ctx, load().lmgc_encode(ctx.handle, _ptr(values), n, _ptr(out), out.numel(), C.byref(nb),
                                    _stream(stream)))
     return out[: nb.value]
+
+
+def lmgc_encode_windows(ctx: Context, values: torch.Tensor, first_win: int, n_win: int, stream=None):
+    """Codes of windows [first_win, first_win + n_win): (payload uint8 tensor, bitlen int32 tensor)."""
+    bitlen = torch.empty(max(n_win, 1), dtype=torch.int32, device=values.device)
+    nb = C.c_size_t()
+    st = load().lmgc_encode_windows(ctx.handle, _ptr(values), values.numel(), first_win, n_win, None, 0, C.byref(nb),
+                                    _ptr(bitlen), _stream(stream))
+    if st != ERR_NO_SPACE:
+        _check(ctx, st)
+    out = torch.empty(max(nb.value, 1), dtype=torch.uint8, device=values.device)
+    _check(ctx, load().lmgc_encode_windows(ctx.handle, _ptr(values), values.numel(), first_win, n_win, _ptr(out),
+                                           out.numel(), C.byref(nb), _ptr(bitlen), _stream(stream)))
+    return out[: nb.value], bitlen[:n_win]
+
+
+def lmgc_container_header(ctx: Context, n: int) -> bytes:
+    buf = (C.c_uint8 * 64)()
+    _check(ctx, load().lmgc_container_header(ctx.handle, n, buf))
+    return bytes(buf)
 
 
 def lmgc_encode_host(ctx: Context, values: torch.Tensor, out: torch.Tensor, stream=None) -> int:

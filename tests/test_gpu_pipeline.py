@@ -131,3 +131,22 @@ def test_tinyllama_shape_sampled_round_trip():
     flat = np.concatenate([toks[0], toks[1, : h["n_tok"] - 2048]])
     assert O.deserialize(flat, 0, 0).tobytes() == vals.tobytes()
     ctx.close()
+
+
+def test_window_ranges_assemble_to_the_container():
+    """lmgc_encode_windows on two window ranges (as two GPUs would) plus lmgc_container_header,
+    assembled, equal lmgc_encode's container byte for byte."""
+    from paper_2409_17836_gb300 import shard
+
+    ctx = L.Context(configs.with_(configs.TINY, batch_windows=5))
+    vals = I.tiny_gradient(4)[:1000]
+    d = torch.from_numpy(vals.view(np.int32).copy()).cuda()
+    ref = L.lmgc_encode(ctx, d).cpu().numpy().tobytes()
+    n_win = -(-vals.size * 9 // 256)
+    parts = []
+    for first, count in shard.window_ranges(n_win, 2):
+        pay, bl = L.lmgc_encode_windows(ctx, d, first, count)
+        parts.append((bl.cpu().numpy().view(np.uint32), pay.cpu().numpy().tobytes()))
+    got = shard.assemble(L.lmgc_container_header(ctx, vals.size), [p[0] for p in parts], [p[1] for p in parts])
+    assert got == ref
+    ctx.close()
