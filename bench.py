@@ -358,12 +358,14 @@ def main():
     if rank == 0:
         res = {"metric": METRIC, "value": value, "unit": "MB/s", "n_gpus": world, "steps": args.steps,
                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
-               "vs_baseline": None, "dtype": "bf16" if cfg.dtype == L.BF16 else "f32",
+               "vs_baseline": None, "dtype": "f16" if cfg.dtype == L.BF16 else "f32",
                "data": "synthetic (seeded random-init ConvNet gradients on Gaussian inputs; random-init model)",
                "config": {"workload": args.workload, "values_per_step": per_step, "window": cfg.window,
                           "batch_windows": cfg.batch_windows, "cdf_bits": cfg.cdf_bits,
                           "model": f"{cfg.n_layers}L d{cfg.d_model} {cfg.n_heads}/{cfg.n_kv_heads}h "
                                    f"ffn{cfg.d_ffn} V{cfg.vocab}",
+                          "weights": "bf16 values (random init), held in fp16; fp16 activations, fp32 accumulation"
+                          if cfg.dtype == L.BF16 else "fp32",
                           "l2": "no flush: each step reads > L2 (model weights and per-batch logits)",
                           "parallelism": f"windows sharded over {world} GPU(s), no collective on the data path"},
                "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches, "roofline": roofline,

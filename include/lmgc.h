@@ -66,7 +66,10 @@ enum { LMGC_IN_F32 = 0, LMGC_IN_U8 = 1 };
  * for dtype LMGC_BF16). */
 typedef struct {
   int32_t n_layers, d_model, n_heads, n_kv_heads, d_ffn, vocab;
-  int32_t dtype;         /* LMGC_F32 or LMGC_BF16: weights and activations */
+  int32_t dtype;         /* LMGC_F32: fp32 weights and activations; LMGC_BF16: bf16-valued weights,
+                            computed with fp16 activations and fp16 x fp16 -> fp32 MMAs (every bf16
+                            value >= 2^-17 in magnitude is exact in fp16, smaller ones round to
+                            the 2^-24 grid) */
   int32_t window;        /* W: tokens per independently coded window (Sec. 4.3 "Context window size") */
   int32_t cdf_bits;      /* P: the integer CDFs sum to 2^P; 2^P > vocab, P <= 30 */
   int32_t sep_mode;      /* LMGC_SEP_* */
@@ -116,11 +119,12 @@ lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, si
 
 /* The model's dense contraction (every linear layer of the Eq. 2 model and its vocabulary
  * projection), exposed for parity tests of the GEMM kernels: C[M][N] (op)= A[M][K] . B[N][K]^T,
- * A and B row-major in the context's dtype (bf16: the tcgen05 kernel; fp32: CUDA cores), fp32
- * accumulation in k order. epi 0: C = result in the context's dtype; 1: fp32 C += result;
+ * A and B row-major (bf16-weight contexts: fp16 on the tcgen05 kernel; fp32: CUDA cores), fp32
+ * accumulation in k order (for LMGC_BF16 contexts A and B are fp16, see lmgc_config.dtype).
+ * epi 0: C = result in the operand type; 1: fp32 C += result;
  * 2: fp32 C = result; 3 (bf16, N % 256 == 0): the SwiGLU MLP input -- B's rows hold gate and up
  * rows interleaved in 128-row blocks (rows 256t..256t+127 gate, 256t+128..256t+255 up) and
- * C[M][N/2] (bf16) = silu(gate) * up, i.e. C[m][128t+j] = silu(R[m][256t+j]) * R[m][256t+128+j].
+ * C[M][N/2] (fp16) = silu(gate) * up, i.e. C[m][128t+j] = silu(R[m][256t+j]) * R[m][256t+128+j].
  * Errors: INVALID (K % 8 != 0, epi outside 0..3, epi 3 unsupported), LIMIT, CUDA. Syncs. */
 lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
                       int epi, lmgc_stream stream);

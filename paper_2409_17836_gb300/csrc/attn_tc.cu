@@ -1,12 +1,12 @@
 // attn_tc.cu -- causal softmax attention of the LM prior (Eq. 2's Llama decoder) on the
-// 5th-generation tensor cores, bf16 inputs, fp32 softmax and accumulation.
+// 5th-generation tensor cores, fp16 inputs and probabilities, fp32 softmax and accumulation.
 //
 // One CTA per (128 query rows, query head, window); 192 threads:
 //   warp 0      TMA: the Q tile once, then 64-key K and V blocks into a 2-stage ring
 //   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64) and O_blk = P V
 //               (M 128, N hd, V as an MN-major operand) and commits to mbarriers
 //   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
-//               per-thread loops; P is written as bf16 into shared memory in the 128-byte
+//               per-thread loops; P is written as fp16 into shared memory in the 128-byte
 //               swizzled K-major layout the MMA reads; the running output O stays in registers
 //               and is rescaled by the online-softmax correction before each block's P V is added.
 // Key blocks are 64-aligned and visited in order 0, 1, ...; a block whose keys all lie past a
@@ -42,9 +42,9 @@ struct Shape {
   static constexpr uint32_t TMEM_COLS = (128 + 2 * HD <= 256) ? 256 : 512;
   static constexpr size_t SMEM = Q_BYTES + KS * (K_BYTES + V_BYTES) + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
-  static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BKV >> 3) << 17) |
+  static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
-  static constexpr uint32_t IDESC_PV = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) |
+  static constexpr uint32_t IDESC_PV = (1u << 4) | (1u << 16) |
                                        ((uint32_t)(HD >> 3) << 17) | ((uint32_t)(BQ >> 4) << 24);
 };
 
@@ -147,7 +147,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 }
 
 struct Params {
-  __nv_bfloat16* out;
+  __half* out;
   int64_t out_stride;    // elements per output row
   int64_t q_win_stride;  // query rows per window in the q buffer (W prefill, 1 decode)
   int64_t pos_first;     // position of the first query row of a window
@@ -372,7 +372,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-          __nv_bfloat162 hb = __floats2bfloat162_rn(s[8 * cc + 2 * t], s[8 * cc + 2 * t + 1]);
+          __half2 hb = __floats2half2_rn(s[8 * cc + 2 * t], s[8 * cc + 2 * t + 1]);
           wv[t] = *reinterpret_cast<uint32_t*>(&hb);
         }
         *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
@@ -393,13 +393,13 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     if (ok && r < nrows) {
       const float other = red_l[(1 - hf) * 128 + r];
       const float inv = 1.f / (hf == 0 ? l + other : other + l);
-      __nv_bfloat16* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD + hf * OH;
+      __half* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD + hf * OH;
 #pragma unroll
       for (int c = 0; c < OH / 8; c++) {
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-          __nv_bfloat162 hb = __floats2bfloat162_rn(o[8 * c + 2 * t] * inv, o[8 * c + 2 * t + 1] * inv);
+          __half2 hb = __floats2half2_rn(o[8 * c + 2 * t] * inv, o[8 * c + 2 * t + 1] * inv);
           wv[t] = *reinterpret_cast<uint32_t*>(&hb);
         }
         reinterpret_cast<uint4*>(dst)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
@@ -436,7 +436,7 @@ static bool make_map(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t 
   cuuint64_t strides[1] = {cols * 2};
   cuuint32_t box[2] = {64, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+  return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -460,7 +460,7 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
     return;
   }
   Params p;
-  p.out = (__nv_bfloat16*)out;
+  p.out = (__half*)out;
   p.out_stride = out_stride;
   p.q_win_stride = q_win_stride;
   p.pos_first = pos_first;

@@ -1,6 +1,7 @@
 // gemm_tc.cu -- the model's dense contractions (the linear layers and the vocabulary projection of
 // the LM prior, Eq. 2) on the 5th-generation tensor cores: C[M][N] (op)= A[M][K] . B[N][K]^T,
-// bf16 operands, fp32 accumulation in tensor memory.
+// fp16 operands (the model's bf16-valued weights held exactly in fp16, fp16 activations), fp32
+// accumulation in tensor memory.
 //
 // Persistent, warp-specialised kernel, one CTA per SM (192 threads):
 //   warp 0      TMA producer: 128x64 A and 256x64 B tiles (128-byte swizzle) into a 4-stage ring
@@ -37,9 +38,9 @@ constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 constexpr int GROUP_M = 16;
 constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
 
-// instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (7-9 = 1), B bf16 (10-12 = 1),
+// instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B f16 (bits 7-9, 10-12 = 0),
 // both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -150,12 +151,12 @@ __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int
 template <int EPI>
 __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t n0, const uint32_t (&r)[32]) {
   if (EPI == kStore) {
-    __nv_bfloat16* c = reinterpret_cast<__nv_bfloat16*>(p.C) + m * p.N + n0;
+    __half* c = reinterpret_cast<__half*>(p.C) + m * p.N + n0;
     if (n0 + 32 <= p.N && (p.N & 7) == 0) {
       uint32_t w[16];
 #pragma unroll
       for (int j = 0; j < 16; j++) {
-        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+        __half2 h = __floats2half2_rn(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
         w[j] = *reinterpret_cast<uint32_t*>(&h);
       }
       uint4* d = reinterpret_cast<uint4*>(c);
@@ -164,7 +165,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
     } else {
 #pragma unroll
       for (int j = 0; j < 32; j++)
-        if (n0 + j < p.N) c[j] = __float2bfloat16_rn(__uint_as_float(r[j]));
+        if (n0 + j < p.N) c[j] = __float2half_rn(__uint_as_float(r[j]));
     }
   } else {
     float* c = reinterpret_cast<float*>(p.C) + m * p.N + n0;
@@ -344,14 +345,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32(tbase + (uint32_t)(BN / 2 + c * 32), u);
           if (m < p.M) {
             const int64_t half_n = p.N / 2;
-            __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.C) + m * half_n + (int64_t)nb * (BN / 2) + c * 32;
+            __half* dst = reinterpret_cast<__half*>(p.C) + m * half_n + (int64_t)nb * (BN / 2) + c * 32;
             uint32_t w[16];
 #pragma unroll
             for (int j = 0; j < 16; j++) {
               const float g0 = __uint_as_float(g[2 * j]), g1 = __uint_as_float(g[2 * j + 1]);
               const float a0 = g0 / (1.f + expf(-g0)) * __uint_as_float(u[2 * j]);
               const float a1 = g1 / (1.f + expf(-g1)) * __uint_as_float(u[2 * j + 1]);
-              __nv_bfloat162 h = __floats2bfloat162_rn(a0, a1);
+              __half2 h = __floats2half2_rn(a0, a1);
               w[j] = *reinterpret_cast<uint32_t*>(&h);
             }
             uint4* d4 = reinterpret_cast<uint4*>(dst);
@@ -410,7 +411,7 @@ static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t row
   cuuint64_t strides[1] = {k * 2};
   cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;

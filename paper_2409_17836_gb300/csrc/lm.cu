@@ -18,14 +18,14 @@ __device__ __forceinline__ float to_f(T v);
 template <>
 __device__ __forceinline__ float to_f<float>(float v) { return v; }
 template <>
-__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ float to_f<__half>(__half v) { return __half2float(v); }
 
 template <typename T>
 __device__ __forceinline__ T from_f(float v);
 template <>
 __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <>
-__device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+__device__ __forceinline__ __half from_f<__half>(float v) { return __float2half_rn(v); }
 
 // ------------------------------------------------------------------------------------------
 // Random-init weights: splitmix64 (Steele, Lea, Flood 2014) of seed ^ (tensor_id << 40) ^ index;
@@ -38,6 +38,13 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t x) {
   return z ^ (z >> 31);
 }
 
+// A bf16 model keeps its bf16-valued weights in fp16 containers (every bf16 value with magnitude
+// >= 2^-17 is exact in fp16; smaller ones round to the 2^-24 grid of fp16 subnormals).
+template <typename T>
+constexpr bool kBf16Values = false;
+template <>
+constexpr bool kBf16Values<__half> = true;
+
 template <typename T>
 __global__ void k_init_weights(T* __restrict__ dst, uint64_t seed, uint32_t tid, int64_t rows, int64_t cols,
                                int64_t ld, int64_t row_off, int64_t rblk, int64_t rstride, float a) {
@@ -47,6 +54,7 @@ __global__ void k_init_weights(T* __restrict__ dst, uint64_t seed, uint32_t tid,
     uint64_t u = splitmix64(seed ^ ((uint64_t)tid << 40) ^ (uint64_t)idx) >> 40;
     float unit = (float)((int32_t)u - (1 << 23)) * (1.0f / 8388608.0f);
     float w = __fmul_rn(unit, a);
+    if (kBf16Values<T>) w = __bfloat162float(__float2bfloat16_rn(w));  // the bf16 model's weight value
     int64_t r = idx / cols, c = idx - r * cols;
     const int64_t dr = row_off + (r / rblk) * rstride + r % rblk;
     dst[dr * ld + c] = from_f<T>(w);
@@ -64,7 +72,7 @@ void launch_init_weights(void* dst, int dtype, uint64_t seed, uint32_t tid, int6
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 64);
   note_launch();
   if (dtype == LMGC_BF16)
-    k_init_weights<<<blocks, 256, 0, s>>>((__nv_bfloat16*)dst, seed, tid, rows, cols, ld, row_off, rblk, rstride, a);
+    k_init_weights<<<blocks, 256, 0, s>>>((__half*)dst, seed, tid, rows, cols, ld, row_off, rblk, rstride, a);
   else
     k_init_weights<<<blocks, 256, 0, s>>>((float*)dst, seed, tid, rows, cols, ld, row_off, rblk, rstride, a);
 }
@@ -105,7 +113,7 @@ __global__ void k_embed(const uint16_t* __restrict__ tok_in, int64_t rows, const
 void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, int dtype, float* x, cudaStream_t s) {
   if (rows <= 0) return;
   note_launch();
-  if (dtype == LMGC_BF16) k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const __nv_bfloat16*)E, d, x);
+  if (dtype == LMGC_BF16) k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const __half*)E, d, x);
   else k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const float*)E, d, x);
 }
 
@@ -145,7 +153,7 @@ void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, i
   if (rows <= 0) return;
   note_launch();
   unsigned blocks = (unsigned)((rows + 7) / 8);
-  if (dtype == LMGC_BF16) k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (__nv_bfloat16*)out);
+  if (dtype == LMGC_BF16) k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (__half*)out);
   else k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (float*)out);
 }
 
@@ -171,13 +179,13 @@ __device__ __forceinline__ void load8<float>(const float* p, float* v, bool ok) 
   }
 }
 template <>
-__device__ __forceinline__ void load8<__nv_bfloat16>(const __nv_bfloat16* p, float* v, bool ok) {
+__device__ __forceinline__ void load8<__half>(const __half* p, float* v, bool ok) {
   if (ok) {
     uint4 q = *reinterpret_cast<const uint4*>(p);
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+    const __half2* h = reinterpret_cast<const __half2*>(&q);
 #pragma unroll
     for (int i = 0; i < 4; i++) {
-      float2 f = __bfloat1622float2(h[i]);
+      float2 f = __half22float2(h[i]);
       v[2 * i] = f.x;
       v[2 * i + 1] = f.y;
     }
@@ -251,7 +259,7 @@ void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t 
   note_launch();
   dim3 grid((unsigned)((N + GBN - 1) / GBN), (unsigned)((M + GBM - 1) / GBM));
   if (dtype == LMGC_BF16)
-    k_gemm_simt<<<grid, 256, 0, s>>>((const __nv_bfloat16*)A, (const __nv_bfloat16*)B, C, M, N, K, epi);
+    k_gemm_simt<<<grid, 256, 0, s>>>((const __half*)A, (const __half*)B, C, M, N, K, epi);
   else
     k_gemm_simt<<<grid, 256, 0, s>>>((const float*)A, (const float*)B, C, M, N, K, epi);
 }
@@ -289,7 +297,7 @@ void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, 
   note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
   if (dtype == LMGC_BF16)
-    k_rope<<<blocks, 256, 0, s>>>((__nv_bfloat16*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
+    k_rope<<<blocks, 256, 0, s>>>((__half*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
   else k_rope<<<blocks, 256, 0, s>>>((float*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
 }
 
@@ -450,9 +458,9 @@ void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t k
   attn_launch<T, HDV>(q, q_stride, kv, kv_stride, k_off, v_off, out, out_stride, nq, nkv, W, n_win, pos_first, \
                       n_pos, q_win_stride, s)
   if (dtype == LMGC_BF16) {
-    if (hd == 32) LMGC_ATT(__nv_bfloat16, 32);
-    else if (hd == 64) LMGC_ATT(__nv_bfloat16, 64);
-    else LMGC_ATT(__nv_bfloat16, 128);
+    if (hd == 32) LMGC_ATT(__half, 32);
+    else if (hd == 64) LMGC_ATT(__half, 64);
+    else LMGC_ATT(__half, 128);
   } else {
     if (hd == 32) LMGC_ATT(float, 32);
     else if (hd == 64) LMGC_ATT(float, 64);
@@ -479,7 +487,7 @@ void launch_swiglu(const void* gu, int64_t rows, int ffn, void* act, int dtype, 
   if (total <= 0) return;
   note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
-  if (dtype == LMGC_BF16) k_swiglu<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)gu, rows, ffn, (__nv_bfloat16*)act);
+  if (dtype == LMGC_BF16) k_swiglu<<<blocks, 256, 0, s>>>((const __half*)gu, rows, ffn, (__half*)act);
   else k_swiglu<<<blocks, 256, 0, s>>>((const float*)gu, rows, ffn, (float*)act);
 }
 
@@ -501,7 +509,7 @@ void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t ds
   note_launch();
   unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 32);
   if (dtype == LMGC_BF16)
-    k_copy_rows<<<blocks, 256, 0, s>>>((const __nv_bfloat16*)src, src_stride, (__nv_bfloat16*)dst, dst_win_stride,
+    k_copy_rows<<<blocks, 256, 0, s>>>((const __half*)src, src_stride, (__half*)dst, dst_win_stride,
                                        dst_pos, n_rows, row_elems);
   else
     k_copy_rows<<<blocks, 256, 0, s>>>((const float*)src, src_stride, (float*)dst, dst_win_stride, dst_pos, n_rows,

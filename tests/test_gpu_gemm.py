@@ -1,9 +1,11 @@
 """The model's dense contraction (lmgc_gemm): C = A . B^T for the linear layers and the
-vocabulary projection of the Eq. 2 model. bf16 operands on the tcgen05 kernel, fp32 on CUDA
-cores; compared with the fp64 definition. Bound per element: accumulation error
+vocabulary projection of the Eq. 2 model. A bf16-weight model computes with fp16 operands on the
+tcgen05 kernel (its bf16 weight values are exact in fp16), an fp32 model on CUDA cores; compared
+with the fp64 definition. Bound per element: accumulation error
 <= 2^-19 * sum_k |a_k b_k| on the tensor cores (their fp32 accumulation aligns products
 with truncation, measured at up to 1.4 x 2^-22 * sum |a b|), and the standard bound of sequential fp32 summation,
-K * 2^-24 * sum |a b|, on CUDA cores; plus one bf16 rounding of the output for epilogue 0."""
+K * 2^-24 * sum |a b|, on CUDA cores; plus one fp16 rounding (2^-11 relative, 2^-10 allowed) of
+the output for epilogues 0 and 3."""
 import numpy as np
 import pytest
 import torch
@@ -15,7 +17,7 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.fixture(scope="module")
-def ctx_bf16():
+def ctx_f16():
     c = L.Context(L.ModelConfig(n_layers=1, d_model=64, n_heads=1, n_kv_heads=1, d_ffn=64, vocab=32, dtype=L.BF16,
                                 window=64, cdf_bits=16))
     yield c
@@ -24,11 +26,11 @@ def ctx_bf16():
 
 def run(ctx, M, N, K, epi, seed=0, scale=1.0):
     g = torch.Generator().manual_seed(seed)
-    a = (torch.randn(M, K, generator=g) * scale).to(torch.bfloat16)
-    b = (torch.randn(N, K, generator=g) * scale).to(torch.bfloat16)
+    a = (torch.randn(M, K, generator=g) * scale).to(torch.float16)
+    b = (torch.randn(N, K, generator=g) * scale).to(torch.float16)
     c0 = torch.randn(M, N, generator=g)
     if epi == 0:
-        c = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+        c = torch.empty(M, N, dtype=torch.float16, device="cuda")
     else:
         c = c0.clone().cuda()
     L.lmgc_gemm(ctx, a.cuda(), b.cuda(), c, epi)
@@ -40,7 +42,7 @@ def run(ctx, M, N, K, epi, seed=0, scale=1.0):
         bound += 2.0 ** -23 * np.abs(ref)
     got = c.float().cpu().numpy().astype(np.float64)
     if epi == 0:
-        bound += 2.0 ** -8 * np.abs(ref)
+        bound += 2.0 ** -10 * np.abs(ref)
     err = np.abs(got - ref)
     assert np.all(err <= bound), float((err / bound).max())
     return c
@@ -49,26 +51,26 @@ def run(ctx, M, N, K, epi, seed=0, scale=1.0):
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 136), (1, 256, 2048), (7, 2560, 2048),
                                    (1000, 2048, 5632), (2048, 32000, 2048)])
 @pytest.mark.parametrize("epi", [0, 1, 2])
-def test_gemm_tc_shapes(ctx_bf16, M, N, K, epi):
+def test_gemm_tc_shapes(ctx_f16, M, N, K, epi):
     if M * N > 2048 * 32000 // 2 and epi != 2:
         pytest.skip("the vocabulary shape is checked with the fp32 epilogue only")
-    run(ctx_bf16, M, N, K, epi, seed=M + N + K)
+    run(ctx_f16, M, N, K, epi, seed=M + N + K)
 
 
-def test_gemm_tc_row_invariance(ctx_bf16):
+def test_gemm_tc_row_invariance(ctx_f16):
     """A row's result does not depend on M or on the row's place in a tile (the decoder relies on
     this): rows computed alone equal the same rows inside a 1000-row product, bit for bit."""
     g = torch.Generator().manual_seed(5)
-    a = torch.randn(1000, 2048, generator=g).to(torch.bfloat16).cuda()
-    b = torch.randn(2560, 2048, generator=g).to(torch.bfloat16).cuda()
+    a = torch.randn(1000, 2048, generator=g).to(torch.float16).cuda()
+    b = torch.randn(2560, 2048, generator=g).to(torch.float16).cuda()
     full = torch.empty(1000, 2560, device="cuda")
-    L.lmgc_gemm(ctx_bf16, a, b, full, 2)
+    L.lmgc_gemm(ctx_f16, a, b, full, 2)
     for r in [0, 1, 127, 128, 517, 999]:
         one = torch.empty(1, 2560, device="cuda")
-        L.lmgc_gemm(ctx_bf16, a[r:r + 1].contiguous(), b, one, 2)
+        L.lmgc_gemm(ctx_f16, a[r:r + 1].contiguous(), b, one, 2)
         assert torch.equal(one[0], full[r]), r
     part = torch.empty(3, 2560, device="cuda")
-    L.lmgc_gemm(ctx_bf16, a[517:520].contiguous(), b, part, 2)
+    L.lmgc_gemm(ctx_f16, a[517:520].contiguous(), b, part, 2)
     assert torch.equal(part, full[517:520])
 
 
@@ -85,25 +87,25 @@ def test_gemm_fp32_simt():
     ctx.close()
 
 
-def test_gemm_rejects_bad_k(ctx_bf16):
-    a = torch.zeros(4, 12, dtype=torch.bfloat16, device="cuda")
+def test_gemm_rejects_bad_k(ctx_f16):
+    a = torch.zeros(4, 12, dtype=torch.float16, device="cuda")
     with pytest.raises(L.LmgcError):
-        L.lmgc_gemm(ctx_bf16, a, a, torch.zeros(4, 4, device="cuda"), 2)
+        L.lmgc_gemm(ctx_f16, a, a, torch.zeros(4, 4, device="cuda"), 2)
 
 
 @pytest.mark.parametrize("M,F,K", [(300, 512, 136), (1, 5632, 2048), (1000, 1408, 2048)])
-def test_gemm_tc_swiglu_epilogue(ctx_bf16, M, F, K):
-    """Epilogue 3: gate/up rows interleaved in 128-row blocks, C = silu(gate) * up in bf16."""
+def test_gemm_tc_swiglu_epilogue(ctx_f16, M, F, K):
+    """Epilogue 3: gate/up rows interleaved in 128-row blocks, C = silu(gate) * up in fp16."""
     g = torch.Generator().manual_seed(F + M)
-    a = torch.randn(M, K, generator=g).to(torch.bfloat16)
-    wg = (torch.randn(F, K, generator=g) * 0.05).to(torch.bfloat16)
-    wu = (torch.randn(F, K, generator=g) * 0.05).to(torch.bfloat16)
-    inter = torch.empty(2 * F, K, dtype=torch.bfloat16)
+    a = torch.randn(M, K, generator=g).to(torch.float16)
+    wg = (torch.randn(F, K, generator=g) * 0.05).to(torch.float16)
+    wu = (torch.randn(F, K, generator=g) * 0.05).to(torch.float16)
+    inter = torch.empty(2 * F, K, dtype=torch.float16)
     for t in range(F // 128):
         inter[256 * t: 256 * t + 128] = wg[128 * t: 128 * t + 128]
         inter[256 * t + 128: 256 * t + 256] = wu[128 * t: 128 * t + 128]
-    c = torch.empty(M, F, dtype=torch.bfloat16, device="cuda")
-    L.lmgc_gemm(ctx_bf16, a.cuda(), inter.cuda(), c, 3)
+    c = torch.empty(M, F, dtype=torch.float16, device="cuda")
+    L.lmgc_gemm(ctx_f16, a.cuda(), inter.cuda(), c, 3)
     af = a.float().numpy()
     gr = O.gemm_nt(af, wg.float().numpy())
     ur = O.gemm_nt(af, wu.float().numpy())
@@ -111,6 +113,6 @@ def test_gemm_tc_swiglu_epilogue(ctx_bf16, M, F, K):
     eg = 2.0 ** -19 * O.gemm_nt(np.abs(af), np.abs(wg.float().numpy()))
     eu = 2.0 ** -19 * O.gemm_nt(np.abs(af), np.abs(wu.float().numpy()))
     silu = gr / (1 + np.exp(-gr))
-    bound = 1.1 * np.abs(ur) * eg + np.abs(silu) * eu + 2.0 ** -8 * np.abs(ref) + 1e-30
+    bound = 1.1 * np.abs(ur) * eg + np.abs(silu) * eu + 2.0 ** -10 * np.abs(ref) + 1e-30
     err = np.abs(c.float().cpu().numpy() - ref)
     assert np.all(err <= bound), float((err / bound).max())
