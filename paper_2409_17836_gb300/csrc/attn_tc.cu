@@ -60,10 +60,11 @@ __device__ __forceinline__ void mbar_arrive(uint32_t a) {
 }
 __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
   uint32_t ok;
+  // the suspend-time hint lets a waiting warp sleep until the phase completes instead of spinning
   asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(a), "r"(parity)
+      : "r"(a), "r"(parity), "r"(0x989680u)
       : "memory");
   return ok != 0;
 }
@@ -112,6 +113,25 @@ __device__ __forceinline__ uint64_t desc_kmajor(uint32_t saddr) {
 __device__ __forceinline__ uint64_t desc_mnmajor(uint32_t saddr, uint32_t lbo) {
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// packed pairs of fp32 (Blackwell's two-wide FMA / ADD: each lane an IEEE round-to-nearest op)
+__device__ __forceinline__ uint64_t f2pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
 }
 // 2^x on the special-function unit (flushes subnormal results to zero; ex2(-inf) = 0)
 __device__ __forceinline__ float ex2_approx(float x) {
@@ -301,9 +321,9 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     constexpr int OH = HD / 2;
     const uint32_t b_pair = smem_u32(bars + 19 + q4);
     float m = -INFINITY, l = 0.f, corr_prev = 1.f;
-    float o[OH];
+    uint64_t o2[OH / 2];  // output columns in packed pairs
 #pragma unroll
-    for (int i = 0; i < OH; i++) o[i] = 0.f;
+    for (int i = 0; i < OH / 2; i++) o2[i] = 0ull;
     // O = O * corr + (P V) of a block; deferred by one block so the P V MMA runs meanwhile
     auto add_pv = [&](int kb, float corr) -> bool {
       const int st = kb & 1;
@@ -314,8 +334,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         uint32_t pa[32];
         tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + hf * OH + c * 32, pa);
         tmem_wait();
+        const uint64_t corr2 = f2pack(corr, corr);
 #pragma unroll
-        for (int j = 0; j < 32; j++) o[c * 32 + j] = o[c * 32 + j] * corr + __uint_as_float(pa[j]);
+        for (int j = 0; j < 16; j++)
+          o2[c * 16 + j] = ffma2(o2[c * 16 + j], corr2, f2pack(__uint_as_float(pa[2 * j]), __uint_as_float(pa[2 * j + 1])));
       }
       tc_fence_before();
       return true;
@@ -356,14 +378,21 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       // exactly 1 when the maximum does not change (a fully masked block is then a no-op)
       const float corr = ex2_approx((m - mn) * p.scale_log2);
       const float nb = -mn * p.scale_log2;
-      float sum4[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint64_t c2 = f2pack(p.scale_log2, p.scale_log2), nb2 = f2pack(nb, nb);
+      uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
 #pragma unroll
-      for (int j = 0; j < 32; j++) {
-        const float e = ex2_approx(fmaf(s[j], p.scale_log2, nb));
-        s[j] = e;
-        sum4[j & 3] += e;
+      for (int j = 0; j < 32; j += 2) {
+        float t0, t1;
+        f2unpack(ffma2(f2pack(s[j], s[j + 1]), c2, nb2), t0, t1);
+        s[j] = ex2_approx(t0);
+        s[j + 1] = ex2_approx(t1);
+        if ((j >> 1) & 1) acc1 = fadd2(acc1, f2pack(s[j], s[j + 1]));
+        else acc0 = fadd2(acc0, f2pack(s[j], s[j + 1]));
       }
-      l = l * corr + ((sum4[0] + sum4[1]) + (sum4[2] + sum4[3]));
+      float a0, a1, a2, a3;
+      f2unpack(acc0, a0, a1);
+      f2unpack(acc1, a2, a3);
+      l = l * corr + ((a0 + a1) + (a2 + a3));
       m = mn;
       uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
 #pragma unroll
@@ -399,7 +428,9 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-          __half2 hb = __floats2half2_rn(o[8 * c + 2 * t] * inv, o[8 * c + 2 * t + 1] * inv);
+          float x0, x1;
+          f2unpack(o2[4 * c + t], x0, x1);
+          __half2 hb = __floats2half2_rn(x0 * inv, x1 * inv);
           wv[t] = *reinterpret_cast<uint32_t*>(&hb);
         }
         reinterpret_cast<uint4*>(dst)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
