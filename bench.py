@@ -192,6 +192,18 @@ def microbenchmarks(L, ctx, pk, reps: int = 3) -> dict:
     return out
 
 
+def profiled_traffic(workload: str, kernel: str):
+    """DRAM bytes per launch of a kernel class from the committed ncu launch-list summary of this
+    workload (profiles/launches_<workload>.md), or None when there is none."""
+    path = os.path.join(ROOT, "profiles", f"launches_{workload}.md")
+    try:
+        text = open(path).read()
+        block = text.split("```json", 1)[1].split("```", 1)[0]
+        return json.loads(block)[kernel]["traffic_bytes_per_launch"], os.path.relpath(path, ROOT)
+    except Exception:
+        return None, None
+
+
 def bytes_per_value(cfg) -> int:
     return 4 if cfg.input_kind == 0 else 1
 
@@ -326,10 +338,15 @@ def main():
     pk = peaks()
     g = stats["gemm"]
     gemm_tflops = g["work"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else 0.0
+    traffic, traffic_src = profiled_traffic(args.workload, "gemm_tc")
     roofline = {"bound": "tensor", "kernel": "gemm (all linear layers and the vocabulary projection)",
                 "achieved": gemm_tflops, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-                "frac": gemm_tflops / pk["bf16_sus"], "peak_kind": f"bf16 sustained ({pk['src']})",
-                "launches": g["launches"], "avg_launch_ms": g["ms"] / max(1, g["launches"]), "traffic": None}
+                "frac": gemm_tflops / pk["bf16_sus"],
+                "peak_kind": f"bf16 sustained ({pk['src']}; fp16 MMAs run at the bf16 rate)",
+                "launches": g["launches"], "avg_launch_ms": g["ms"] / max(1, g["launches"]),
+                "algorithmic_flops_per_launch": g["work"] / max(1, g["launches"]),
+                "traffic": traffic, "traffic_unit": "bytes per launch (DRAM read + write)",
+                "traffic_source": traffic_src}
     stages = {}
     for name, st in stats.items():
         if st["launches"] == 0:
