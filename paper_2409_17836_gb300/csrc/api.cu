@@ -121,10 +121,10 @@ static void prof_collect(lmgc_ctx* ctx) {
 
 // ---- GEMM dispatch: tcgen05 for bf16 when the shape fits, CUDA cores otherwise ----
 static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi,
-                 cudaStream_t s) {
+                 cudaStream_t s, const RopeArgs* rope = nullptr, const NormArgs* norm = nullptr) {
   ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
   if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi))
-    launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s);
+    launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s, rope, norm);
   else
     launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);  // kSwiGLU never reaches here
 }
@@ -155,6 +155,31 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
   const int d = c.d_model, F = c.d_ffn, hd = ctx->hd, qd = c.n_heads * hd;
   Workspace& ws = ctx->ws;
   const int64_t W = c.window;
+  if (ctx->fused_norm) {
+    // RMSNorm folded into the GEMMs: the residual producers (embedding, O and down projections)
+    // leave x (fp32), fp16(x) in ws.n and per-256-column sums of squares in ws.ss; the consumers
+    // (QKV, gate/up, vocabulary) read fp16(x) and scale each row by rsqrt(mean(x^2) + eps).
+    __half* xh = (__half*)ws.n;
+    const NormArgs consume{ws.ss, d / 256, 1.0f / (float)d, c.rms_eps, nullptr, nullptr};
+    const NormArgs produce{nullptr, 0, 0.f, 0.f, xh, ws.ss};
+    for (int l = 0; l < c.n_layers; l++) {
+      const Layer& L = ctx->layers[l];
+      RopeArgs ra{ctx->rope_cs, (c.n_heads + c.n_kv_heads) * hd, hd, decode ? 1 : c.window, decode ? pos : 0};
+      gemm(ctx, xh, L.wqkv, ws.qkv, rows, ctx->qkv_dim, d, kQKVRope, s, &ra, &consume);
+      if (!decode) {
+        attention(ctx, ws.qkv, ws.qkv, ws.att, n_win, 0, c.window, W, s);
+      } else {
+        char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->qkv_dim * ctx->elt;
+        launch_copy_rows(ws.qkv, ctx->qkv_dim, cache_l, W, pos, n_win, ctx->qkv_dim, c.dtype, s);
+        attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s);
+      }
+      gemm(ctx, ws.att, L.wo, ws.x, rows, d, qd, kAddResidual, s, nullptr, &produce);
+      gemm(ctx, xh, L.wgu, ws.act, rows, 2 * (int64_t)F, d, kSwiGLU, s, nullptr, &consume);
+      gemm(ctx, ws.act, L.wdown, ws.x, rows, d, F, kAddResidual, s, nullptr, &produce);
+    }
+    gemm(ctx, xh, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s, nullptr, &consume);
+    return;
+  }
   for (int l = 0; l < c.n_layers; l++) {
     const Layer& L = ctx->layers[l];
     {
@@ -199,6 +224,15 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
   gemm(ctx, ws.n, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s);
 }
 
+// x = E[tok_in] for `rows` rows (and, on the fused-RMSNorm path, fp16(x) and its sums of squares)
+static void embed_rows(lmgc_ctx* ctx, int64_t rows, cudaStream_t s) {
+  const lmgc_config& c = ctx->cfg;
+  if (ctx->fused_norm)
+    launch_embed_fused(ctx->ws.tok_in, rows, ctx->w_embed, c.d_model, ctx->ws.x, (__half*)ctx->ws.n, ctx->ws.ss, s);
+  else
+    launch_embed(ctx->ws.tok_in, rows, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
+}
+
 // Model logits for windows [first_win, first_win + nb) of a token stream, into ctx->logits.
 static void forward_windows(lmgc_ctx* ctx, const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t nb,
                             cudaStream_t s) {
@@ -207,7 +241,7 @@ static void forward_windows(lmgc_ctx* ctx, const uint16_t* tok, int64_t n_tok, i
   {
     ProfScope ps(ctx, kOther, 0, s);
     launch_window_inputs(tok, n_tok, first_win, nb, c.window, ctx->ws.tok_in, s);
-    launch_embed(ctx->ws.tok_in, rows, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
+    embed_rows(ctx, rows, s);
   }
   forward_layers(ctx, rows, nb, false, 0, s);
 }
@@ -277,7 +311,7 @@ lmgc_status lmgc_destroy(lmgc_ctx* ctx) {
   if (!ctx) return LMGC_OK;
   cudaDeviceSynchronize();
   void* ptrs[] = {ctx->weights_blob, ctx->rope_cs, ctx->exp2_tab, ctx->ws.x, ctx->ws.n, ctx->ws.qkv, ctx->ws.att,
-                  ctx->ws.act, ctx->ws.gu, ctx->ws.tok_in, ctx->logits, ctx->d_err, ctx->tok, ctx->pair_start,
+                  ctx->ws.act, ctx->ws.gu, ctx->ws.ss, ctx->ws.tok_in, ctx->logits, ctx->d_err, ctx->tok, ctx->pair_start,
                   ctx->win_len, ctx->host_in, ctx->host_out, ctx->kv_cache};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -320,6 +354,10 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->use_tc = !(tc_env && tc_env[0] == '1');
   ctx->fused_rope = c.dtype == LMGC_BF16 && ctx->use_tc && (hd == 64 || hd == 128) &&
                     tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kQKVRope);
+  ctx->fused_norm = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_model % 256 == 0 &&
+                    tc_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd, kAddResidual) &&
+                    tc_gemm_supported(1, c.d_model, c.d_ffn, kAddResidual) &&
+                    tc_gemm_supported(1, c.vocab, c.d_model, kStoreF32);
   ctx->fused_swiglu = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_ffn % 128 == 0 && tc_gemm_supported(1, 2 * c.d_ffn, c.d_model, kSwiGLU);
   const int64_t d = c.d_model, F = c.d_ffn, V = c.vocab, qd = (int64_t)c.n_heads * hd;
   const size_t e = ctx->elt;
@@ -399,6 +437,8 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (err == cudaSuccess) err = dmalloc(&ws.att, R * qd * e);
   if (err == cudaSuccess) err = dmalloc(&ws.act, R * F * e);
   if (err == cudaSuccess && !ctx->fused_swiglu) err = dmalloc(&ws.gu, R * 2 * F * e);
+  ctx->fused_norm = ctx->fused_norm && ctx->fused_rope && ctx->fused_swiglu;
+  if (err == cudaSuccess && ctx->fused_norm) err = dmalloc(&ws.ss, R * (size_t)(d / 256) * 4);
   if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
   if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
   for (int i = 0; i < 6 && err == cudaSuccess; i++) err = cudaEventCreate(&ctx->ev[i]);
@@ -804,7 +844,7 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
     for (int64_t pos = 0; pos < max_len; pos++) {
       note_launch();
       k_dec_inputs<<<(unsigned)((nd + 127) / 128), 128, 0, s>>>(out, nd, W, pos, ctx->ws.tok_in);
-      launch_embed(ctx->ws.tok_in, nd, ctx->w_embed, c.d_model, c.dtype, ctx->ws.x, s);
+      embed_rows(ctx, nd, s);
       forward_layers(ctx, nd, nd, true, pos, s);
       launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
                         ctx->d_err, s);

@@ -36,7 +36,11 @@ constexpr uint32_t B_BYTES = BN * BK * 2;  // 32 KiB
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 constexpr int GROUP_M = 16;
-constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 1024 + 256;
+// residual epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, row pitch 36 words so
+// that both the row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B
+constexpr int STG_PITCH = 36;
+constexpr uint32_t STG_BYTES = 4 * 32 * STG_PITCH * 4;
+constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 256 + STG_BYTES + 1024;
 
 // instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B f16 (bits 7-9, 10-12 = 0),
 // both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28
@@ -137,7 +141,23 @@ struct Params {
   const float2* rope_cs;
   int rope_cols, rope_hd, rope_pos_mod;
   int64_t rope_pos0;
+  // fused RMSNorm of the A rows: when row_ss is set, the result of row m is scaled by
+  // rsqrt(sum_k row_ss[m * ss_parts + k] * ss_inv_d + ss_eps) before the epilogue's operation
+  const float* row_ss;
+  int ss_parts;
+  float ss_inv_d, ss_eps;
+  // kAddResidual: also write fp16(x) to xh and the tile's sum of squares to ss_out[m * tiles_n + nb]
+  __half* xh;
+  float* ss_out;
 };
+
+__device__ __forceinline__ float row_scale(const Params& p, int64_t m) {
+  if (!p.row_ss || m >= p.M) return 1.f;
+  const float* s = p.row_ss + m * p.ss_parts;
+  float t = 0.f;
+  for (int k = 0; k < p.ss_parts; k++) t += s[k];
+  return rsqrtf(t * p.ss_inv_d + p.ss_eps);
+}
 
 __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int& nb) {
   const int per_group = GROUP_M * p.tiles_n;
@@ -147,6 +167,14 @@ __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int
   const int r = t - g * per_group;
   mb = first_m + r % gm;
   nb = r / gm;
+}
+
+// L2 prefetch of row m's BN residual columns starting at column block nb (N % 32 == 0)
+__device__ __forceinline__ void prefetch_residual(const Params& p, int64_t m, int nb) {
+  if (m >= p.M) return;
+  const char* xr = reinterpret_cast<const char*>(reinterpret_cast<const float*>(p.C) + m * p.N + (int64_t)nb * BN);
+  const int lines = (int)(min((int64_t)BN, p.N - (int64_t)nb * BN) * 4 / 128);
+  for (int j = 0; j < lines; j++) asm volatile("prefetch.global.L2 [%0];" ::"l"(xr + j * 128));
 }
 
 template <int EPI>
@@ -172,16 +200,20 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
     float* c = reinterpret_cast<float*>(p.C) + m * p.N + n0;
     if (n0 + 32 <= p.N && (p.N & 3) == 0) {
       float4* d = reinterpret_cast<float4*>(c);
+      float4 o[8];
+      if (EPI == kAddResidual) {
+#pragma unroll
+        for (int j = 0; j < 8; j++) o[j] = d[j];  // all loads in flight before the first store
+      }
 #pragma unroll
       for (int j = 0; j < 8; j++) {
         float4 v = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
                                __uint_as_float(r[4 * j + 3]));
         if (EPI == kAddResidual) {
-          float4 o = d[j];
-          v.x += o.x;
-          v.y += o.y;
-          v.z += o.z;
-          v.w += o.w;
+          v.x += o[j].x;
+          v.y += o[j].y;
+          v.z += o[j].z;
+          v.w += o[j].w;
         }
         d[j] = v;
       }
@@ -200,6 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  float* staging = reinterpret_cast<float*>(smem + STAGES * STAGE_BYTES + 256);
   const uint32_t smem_base = smem_u32(smem);
   auto sA = [&](int s) { return smem_base + (uint32_t)s * STAGE_BYTES; };
   auto sB = [&](int s) { return smem_base + (uint32_t)s * STAGE_BYTES + A_BYTES; };
@@ -292,9 +325,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       tile_coords(t, p, mb, nb);
       const int a = i & 1;
       const uint32_t aph = (uint32_t)(i >> 1) & 1u;
+      const int64_t m = (int64_t)mb * BM + q * 32 + lane;
+      if (EPI == kAddResidual && (p.N & 31) == 0) {
+        // pull the residual rows of this tile (first visit) and of the next one into L2 ahead of use
+        if (i == 0) prefetch_residual(p, m, nb);
+        if (t + (int)gridDim.x < n_tiles) {
+          int mb2, nb2;
+          tile_coords(t + (int)gridDim.x, p, mb2, nb2);
+          prefetch_residual(p, (int64_t)mb2 * BM + q * 32 + lane, nb2);
+        }
+      }
+      const float rs = row_scale(p, m);
       if (!__all_sync(0xffffffffu, mbar_wait(tfull(a), aph, p.err))) break;
       tc_fence_after();
-      const int64_t m = (int64_t)mb * BM + q * 32 + lane;
       const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);
       if (EPI == kQKVRope) {
         // one head at a time: halves [0, hd/2) and [hd/2, hd) rotate pairwise by pos * theta_i
@@ -327,9 +370,15 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (rot) {
 #pragma unroll
                 for (int j = 0; j < 32; j++) {
-                  const float x = __uint_as_float(a[j]), y = __uint_as_float(b[j]);
+                  const float x = __uint_as_float(a[j]) * rs, y = __uint_as_float(b[j]) * rs;
                   a[j] = __float_as_uint(x * ct[j] - y * st[j]);
                   b[j] = __float_as_uint(x * st[j] + y * ct[j]);
+                }
+              } else if (p.row_ss) {
+#pragma unroll
+                for (int j = 0; j < 32; j++) {
+                  a[j] = __float_as_uint(__uint_as_float(a[j]) * rs);
+                  b[j] = __float_as_uint(__uint_as_float(b[j]) * rs);
                 }
               }
               store_chunk<kStore>(p, m, col0 + c * 32, a);
@@ -350,9 +399,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t w[16];
 #pragma unroll
             for (int j = 0; j < 16; j++) {
-              const float g0 = __uint_as_float(g[2 * j]), g1 = __uint_as_float(g[2 * j + 1]);
-              const float a0 = g0 / (1.f + expf(-g0)) * __uint_as_float(u[2 * j]);
-              const float a1 = g1 / (1.f + expf(-g1)) * __uint_as_float(u[2 * j + 1]);
+              const float g0 = __uint_as_float(g[2 * j]) * rs, g1 = __uint_as_float(g[2 * j + 1]) * rs;
+              const float a0 = g0 / (1.f + expf(-g0)) * (__uint_as_float(u[2 * j]) * rs);
+              const float a1 = g1 / (1.f + expf(-g1)) * (__uint_as_float(u[2 * j + 1]) * rs);
               __half2 h = __floats2half2_rn(a0, a1);
               w[j] = *reinterpret_cast<uint32_t*>(&h);
             }
@@ -361,12 +410,79 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < 4; j++) d4[j] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
           }
         }
+      } else if (EPI == kAddResidual && (p.N & 31) == 0) {
+        // x += acc through a shared-memory transpose: the warp's 32 rows x 32 columns go in one row
+        // per thread and come out as 8 lanes per row, so each global access covers 4 full rows of
+        // 128 B. With xh set, fp16(x) is written too and ss_out[row * tiles_n + nb] receives the
+        // row's sum of squares over this tile's columns (fixed order: per lane over chunks, then
+        // a butterfly over the row's 8 lanes).
+        float* stg = staging + q * 32 * STG_PITCH;
+        const int cr = lane >> 3, cc = (lane & 7) * 4;
+        const int64_t row0 = (int64_t)mb * BM + q * 32;
+        float ssl[8];
+#pragma unroll
+        for (int k = 0; k < 8; k++) ssl[k] = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          const int64_t n0 = (int64_t)nb * BN + c * 32;
+          if (n0 >= p.N) break;
+          uint32_t r[32];
+          tmem_ld32(tbase + (uint32_t)(c * 32), r);
+          float4* srow = reinterpret_cast<float4*>(stg + lane * STG_PITCH);
+#pragma unroll
+          for (int j = 0; j < 8; j++)
+            srow[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
+                                  __uint_as_float(r[4 * j + 3]));
+          __syncwarp();
+          float* xbase = reinterpret_cast<float*>(p.C) + n0 + cc;
+          float4 o[8];
+#pragma unroll
+          for (int k = 0; k < 8; k++) {
+            const int64_t gm = row0 + 4 * k + cr;
+            o[k] = gm < p.M ? *reinterpret_cast<const float4*>(xbase + gm * p.N) : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+#pragma unroll
+          for (int k = 0; k < 8; k++) {
+            const int64_t gm = row0 + 4 * k + cr;
+            const float4 acc = *reinterpret_cast<const float4*>(stg + (4 * k + cr) * STG_PITCH + cc);
+            float4 v;
+            v.x = o[k].x + acc.x;
+            v.y = o[k].y + acc.y;
+            v.z = o[k].z + acc.z;
+            v.w = o[k].w + acc.w;
+            if (gm < p.M) {
+              *reinterpret_cast<float4*>(xbase + gm * p.N) = v;
+              if (p.xh) {
+                __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
+                *reinterpret_cast<uint2*>(p.xh + gm * p.N + n0 + cc) =
+                    make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1));
+              }
+            }
+            ssl[k] += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+          }
+          __syncwarp();
+        }
+        if (p.xh) {
+#pragma unroll
+          for (int k = 0; k < 8; k++) {
+            float v = ssl[k];
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            const int64_t gm = row0 + 4 * k + cr;
+            if ((lane & 7) == 0 && gm < p.M) p.ss_out[gm * p.tiles_n + nb] = v;
+          }
+        }
       } else {
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(tbase + (uint32_t)(c * 32), r);
           const int64_t n0 = (int64_t)nb * BN + c * 32;
+          if (p.row_ss) {
+#pragma unroll
+            for (int j = 0; j < 32; j++) r[j] = __float_as_uint(__uint_as_float(r[j]) * rs);
+          }
           if (m < p.M && n0 < p.N) store_chunk<EPI>(p, m, n0, r);
         }
       }
@@ -428,7 +544,7 @@ bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi) {
 }
 
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
-                    cudaStream_t s, const RopeArgs* rope) {
+                    cudaStream_t s, const RopeArgs* rope, const NormArgs* norm) {
   using namespace tc;
   std::call_once(g_once, init_once);
   CUtensorMap ma, mb;
@@ -450,6 +566,12 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.rope_hd = rope ? rope->hd : 64;
   p.rope_pos_mod = rope ? rope->pos_mod : 1;
   p.rope_pos0 = rope ? rope->pos0 : 0;
+  p.row_ss = norm ? norm->row_ss : nullptr;
+  p.ss_parts = norm ? norm->parts : 0;
+  p.ss_inv_d = norm ? norm->inv_d : 0.f;
+  p.ss_eps = norm ? norm->eps : 0.f;
+  p.xh = norm ? norm->xh : nullptr;
+  p.ss_out = norm ? norm->ss_out : nullptr;
   const int tiles = p.tiles_m * p.tiles_n;
   const int grid = std::max(1, std::min(tiles, g_num_sms));
   note_launch();

@@ -117,6 +117,40 @@ void launch_embed(const uint16_t* tok_in, int64_t rows, const void* E, int d, in
   else k_embed<<<(unsigned)rows, 128, 0, s>>>(tok_in, rows, (const float*)E, d, x);
 }
 
+// Embedding for the fused-RMSNorm path: 8 warps per row; warp w handles the 256-column chunks
+// w, w + 8, ...; each chunk's sum of squares is reduced in a fixed order.
+__global__ void __launch_bounds__(256) k_embed_fused(const uint16_t* __restrict__ tok_in, int64_t rows,
+                                                     const __half* __restrict__ E, int d, float* __restrict__ x,
+                                                     __half* __restrict__ xh, float* __restrict__ ss) {
+  const int64_t r = blockIdx.x;
+  if (r >= rows) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const __half* e = E + (int64_t)tok_in[r] * d;
+  const int parts = d / 256;
+  for (int k = warp; k < parts; k += 8) {
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; i++) {
+      const int c = k * 256 + i * 32 + lane;
+      const __half hv = e[c];
+      const float v = __half2float(hv);
+      x[r * d + c] = v;
+      xh[r * d + c] = hv;
+      acc += v * v;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) ss[r * parts + k] = acc;
+  }
+}
+
+void launch_embed_fused(const uint16_t* tok_in, int64_t rows, const void* E, int d, float* x, __half* xh, float* ss,
+                        cudaStream_t s) {
+  if (rows <= 0) return;
+  note_launch();
+  k_embed_fused<<<(unsigned)rows, 256, 0, s>>>(tok_in, rows, (const __half*)E, d, x, xh, ss);
+}
+
 // ------------------------------------------------------------------------------------------
 // RMSNorm with unit gain: y = x * rsqrt(mean(x^2) + eps). One warp per row; a fixed reduction
 // order (per-lane sequential, then a butterfly) keeps it row-invariant.

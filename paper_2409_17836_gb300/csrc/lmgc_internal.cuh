@@ -54,6 +54,7 @@ struct Workspace {
   void* att = nullptr;     // [rows][nq*hd] (T)
   void* act = nullptr;     // SwiGLU output [rows][ffn] (T)
   void* gu = nullptr;      // gate/up GEMM output [rows][2*ffn] (T), unfused path only
+  float* ss = nullptr;     // fused RMSNorm: per-row partial sums of squares [rows][d/256]
   uint16_t* tok_in = nullptr;  // model input ids [rows]
 };
 
@@ -101,6 +102,7 @@ struct lmgc_ctx {
   bool use_tc = true;        // tcgen05 GEMM for bf16 models when available
   bool fused_swiglu = false;  // gate/up interleaved, SwiGLU in the tcgen05 epilogue
   bool fused_rope = false;    // RoPE in the QKV tcgen05 epilogue
+  bool fused_norm = false;    // RMSNorm folded into the GEMM epilogues (row scale + residual side outputs)
   std::string err;
 };
 
@@ -141,6 +143,15 @@ void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, i
 // 128t.., rows 256t+128.. = up rows 128t..); C[m][128t + j] = silu(gate) * up, N/2 columns.
 // kQKVRope: kStore with the rotary embedding applied to the q and k heads (RopeArgs).
 enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3, kQKVRope = 4 };
+// Fused RMSNorm (see gemm_tc.cu Params): consumers read row_ss (parts per row), residual
+// producers write xh and ss_out.
+struct NormArgs {
+  const float* row_ss;
+  int parts;
+  float inv_d, eps;
+  __half* xh;
+  float* ss_out;
+};
 struct RopeArgs {
   const float2* cs;  // [W][hd/2] (cos, sin)
   int cols;          // columns [0, cols) are rotated: (n_heads + n_kv_heads) * hd
@@ -191,6 +202,10 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
 // gemm_tc.cu (tcgen05)
 bool tc_gemm_supported(int64_t M, int64_t N, int64_t K, int epi = 0);
 void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi, uint32_t* err,
-                    cudaStream_t s, const RopeArgs* rope = nullptr);
+                    cudaStream_t s, const RopeArgs* rope = nullptr, const NormArgs* norm = nullptr);
+// x[r][:] = E[tok_in[r]][:] (fp32), xh = fp16(x), ss[r * (d/256) + k] = sum of squares of columns
+// [256k, 256k + 256) of row r (d % 256 == 0)
+void launch_embed_fused(const uint16_t* tok_in, int64_t rows, const void* E, int d, float* x, __half* xh, float* ss,
+                        cudaStream_t s);
 
 }  // namespace lmgc
