@@ -178,16 +178,18 @@ lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const uint32_t* d
                                       size_t stride_pos, uint8_t* d_out, size_t cap, size_t* out_bytes,
                                       uint32_t* d_bitlen, lmgc_stream stream);
 
-/* Largest container lmgc_encode can produce for n input values (header + length table + the
- * coder's worst case of cdf_bits bits per token + 2 bits per window). */
+/* Largest container lmgc_encode can produce for n input values (header + length and checksum
+ * tables + the coder's worst case of cdf_bits bits per token + 2 bits per window). */
 lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);
 
 /* The whole encode path (Sec. 3): serialise -> windows from BOS -> model logits -> integer CDF
  * pairs -> one code per window -> container. Container layout (little-endian):
- *   0 "LMGC" | 4 u32 version=1 | 8 u64 n_values | 16 u64 n_tok | 24 u32 window | 28 u32 cdf_bits |
+ *   0 "LMGC" | 4 u32 version=2 | 8 u64 n_values | 16 u64 n_tok | 24 u32 window | 28 u32 cdf_bits |
  *   32 u32 input_kind | 36 u32 sep_mode | 40 u32 vocab | 44 u32 n_win | 48 u64 weight_seed |
  *   56 u32 crc32 of the model shape | 60 u32 crc32 of bytes [0, 60) |
- *   64 u32 bitlen[n_win] | codes, ceil(bitlen/8) bytes each, in window order.
+ *   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | codes, ceil(bitlen/8) bytes each, in window order.
+ * crc_tok[w] is the CRC-32 (IEEE 802.3) of window w's token ids as little-endian u16 bytes (the
+ * window's own length), which lmgc_decode checks on every window it restores.
  * d_in: n values; d_out: capacity cap bytes. *out_bytes (host) = container size.
  * Errors: INVALID (n == 0), NO_SPACE (*out_bytes = required), CUDA. Syncs. */
 lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_out, size_t cap, size_t* out_bytes,
@@ -196,14 +198,14 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
 /* The windows [first_win, first_win + n_win) of lmgc_encode's container, for encoding a stream
  * sharded over several GPUs (windows are independent, Sec. 3 "Compression"): all n values are
  * serialised, only the given windows are modelled and coded. d_payload receives their codes
- * byte-aligned in window order (the container's payload slice), d_bitlen (device, n_win) their
- * bit lengths, *payload_bytes (host) the slice size. A container is the header of
- * lmgc_container_header, the bit lengths of all windows in order, then all payload slices in
- * order. Errors: INVALID (range outside the stream), NO_SPACE (*payload_bytes = required), CUDA.
- * Syncs. */
+ * byte-aligned in window order (the container's payload slice), d_bitlen and d_crc (device, n_win
+ * each) their bit lengths and token checksums, *payload_bytes (host) the slice size. A container
+ * is the header of lmgc_container_header, the bit lengths of all windows in order, their token
+ * checksums in order, then all payload slices in order. Errors: INVALID (range outside the
+ * stream, null table pointer), NO_SPACE (*payload_bytes = required), CUDA. Syncs. */
 lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_t first_win, size_t n_win,
                                 uint8_t* d_payload, size_t cap, size_t* payload_bytes, uint32_t* d_bitlen,
-                                lmgc_stream stream);
+                                uint32_t* d_crc, lmgc_stream stream);
 
 /* The 64-byte container header (layout under lmgc_encode) for n input values, written to the
  * host buffer h_header. */
@@ -219,7 +221,8 @@ lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t*
  * container d_in (device, in_bytes) into d_tok (device, [n_ids][W] uint16; a partial last window
  * fills only its length). Each decode step runs the same kernels as lmgc_encode on one row per
  * window, so its logits -- and hence its CDFs -- are bit-identical to the encoder's.
- * Errors: CORRUPT (bad header, model mismatch, or a code that leaves its interval), INVALID
+ * Errors: CORRUPT (bad header, model mismatch, a code that leaves its interval, or a restored
+ * window whose token checksum differs from the container's), INVALID
  * (window id out of range), NO_SPACE (cap_tok < n_ids * W), CUDA. Syncs. */
 lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, const uint32_t* h_win_ids,
                         size_t n_ids, uint16_t* d_tok, size_t cap_tok, lmgc_stream stream);

@@ -323,11 +323,13 @@ def crc32(b: bytes) -> int:
 
 # ------------------------------------------------------------------------------------------
 # Container (a build choice; the paper stores one code per window without a format).
-#   0  "LMGC"            4  u32 version (1)      8  u64 n_values       16 u64 n_tok
+#   0  "LMGC"            4  u32 version (2)      8  u64 n_values       16 u64 n_tok
 #   24 u32 window        28 u32 cdf_bits         32 u32 input_kind     36 u32 sep_mode
 #   40 u32 vocab         44 u32 n_win            48 u64 weight_seed    56 u32 model crc
 #   60 u32 crc32 of bytes [0, 60)
-#   64 u32 bitlen[n_win], then each window's code, ceil(bitlen/8) bytes, in window order.
+#   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | each window's code, ceil(bitlen/8) bytes, in
+#   window order. crc_tok[w] = crc32 of window w's token ids as little-endian u16 (its own
+#   length: W, or fewer for the last window), so that a decoder can check each window it restores.
 # model crc = crc32 of '<7i3f' (n_layers, d_model, n_heads, n_kv_heads, d_ffn, vocab, bf16,
 # init_std, rms_eps, rope_theta).
 # ------------------------------------------------------------------------------------------
@@ -339,12 +341,25 @@ def model_crc(cfg: OracleConfig) -> int:
                              cfg.vocab, int(cfg.bf16), cfg.init_std, cfg.rms_eps, cfg.rope_theta))
 
 
-def build_container(cfg: OracleConfig, n_values: int, n_tok: int, codes: list[tuple[bytes, int]]) -> bytes:
-    head = struct.pack("<4sIQQIIIIIIQI", b"LMGC", 1, n_values, n_tok, cfg.window, cfg.cdf_bits, cfg.input_kind,
-                       cfg.sep_mode, cfg.vocab, len(codes), cfg.weight_seed, model_crc(cfg))
+CONTAINER_VERSION = 2
+
+
+def window_crcs(tok: np.ndarray, window: int, first: int = 0, count: int | None = None) -> np.ndarray:
+    """crc_tok of windows [first, first + count): crc32 of each window's ids as little-endian u16."""
+    t = np.ascontiguousarray(tok, dtype="<u2")
+    n_win = -(-t.size // window)
+    count = n_win - first if count is None else count
+    return np.array([crc32(t[w * window: (w + 1) * window].tobytes()) for w in range(first, first + count)],
+                    dtype=np.uint32)
+
+
+def build_container(cfg: OracleConfig, n_values: int, n_tok: int, codes: list[tuple[bytes, int]],
+                    crcs: np.ndarray) -> bytes:
+    head = struct.pack("<4sIQQIIIIIIQI", b"LMGC", CONTAINER_VERSION, n_values, n_tok, cfg.window, cfg.cdf_bits,
+                       cfg.input_kind, cfg.sep_mode, cfg.vocab, len(codes), cfg.weight_seed, model_crc(cfg))
     head += struct.pack("<I", crc32(head))
-    assert len(head) == HEADER_BYTES
-    table = np.array([bl for _, bl in codes], dtype="<u4").tobytes()
+    assert len(head) == HEADER_BYTES and len(crcs) == len(codes)
+    table = np.array([bl for _, bl in codes], dtype="<u4").tobytes() + np.asarray(crcs, dtype="<u4").tobytes()
     return head + table + b"".join(c for c, _ in codes)
 
 
@@ -355,12 +370,17 @@ def parse_container(buf: bytes) -> dict:
     (crc,) = struct.unpack("<I", buf[60:64])
     if crc != crc32(buf[:60]):
         raise ValueError("header crc mismatch")
+    if f[1] != CONTAINER_VERSION:
+        raise ValueError("unknown container version")
     n_win = f[9]
+    if len(buf) < 64 + 8 * n_win:
+        raise ValueError("window table truncated")
     bl = np.frombuffer(buf[64: 64 + 4 * n_win], dtype="<u4").astype(np.int64)
-    offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)]) + 64 + 4 * n_win
+    crc_tok = np.frombuffer(buf[64 + 4 * n_win: 64 + 8 * n_win], dtype="<u4").astype(np.uint32)
+    offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)]) + 64 + 8 * n_win
     return dict(version=f[1], n_values=f[2], n_tok=f[3], window=f[4], cdf_bits=f[5], input_kind=f[6],
                 sep_mode=f[7], vocab=f[8], n_win=n_win, weight_seed=f[10], model_crc=f[11], bitlen=bl,
-                offsets=offs)
+                crc_tok=crc_tok, offsets=offs)
 
 
 def encode(cfg: OracleConfig, values: np.ndarray, n_par: int = 1) -> bytes:
@@ -369,7 +389,7 @@ def encode(cfg: OracleConfig, values: np.ndarray, n_par: int = 1) -> bytes:
     W = cfg.window
     n_win = (tok.size + W - 1) // W
     codes = encode_windows(cfg, tok, 0, n_win, n_par)
-    return build_container(cfg, values.size, tok.size, codes)
+    return build_container(cfg, values.size, tok.size, codes, window_crcs(tok, W))
 
 
 def compression_rate(container_bytes: int, n_values: int, bytes_per_value: int = 4) -> float:

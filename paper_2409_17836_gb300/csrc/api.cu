@@ -575,7 +575,7 @@ lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes) {
   if (!ctx || !bytes) return LMGC_ERR_INVALID;
   const size_t n_tok = n * (size_t)ctx->tpv, W = (size_t)ctx->cfg.window;
   const size_t n_win = (n_tok + W - 1) / W;
-  *bytes = 64 + 4 * n_win + (n_tok * (size_t)ctx->cfg.cdf_bits + 2 * n_win + 7) / 8 + n_win;
+  *bytes = 64 + 8 * n_win + (n_tok * (size_t)ctx->cfg.cdf_bits + 2 * n_win + 7) / 8 + n_win;
   return LMGC_OK;
 }
 
@@ -598,13 +598,14 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   const size_t pair_need = (size_t)(W * n_win) * 4;
   LMGC_CUDA(ctx, ensure(&ctx->pair_start, &ctx->pair_cap, 2 * pair_need));
   ctx->pair_freq = ctx->pair_start + (size_t)(W * n_win);
-  // win_len [n_win] u32 | bitlen [n_win] u32 | offsets [n_win+1] u64 | slots
-  const size_t wl_off = 0, bl_off = ((size_t)n_win * 4 + 255) / 256 * 256,
-               of_off = bl_off + ((size_t)n_win * 4 + 255) / 256 * 256,
+  // win_len [n_win] u32 | bitlen [n_win] u32 | token crc [n_win] u32 | offsets [n_win+1] u64 | slots
+  const size_t tbl = ((size_t)n_win * 4 + 255) / 256 * 256;
+  const size_t wl_off = 0, bl_off = tbl, cr_off = 2 * tbl, of_off = 3 * tbl,
                sl_off = of_off + (((size_t)n_win + 1) * 8 + 255) / 256 * 256;
   LMGC_CUDA(ctx, ensure(&ctx->win_len, &ctx->win_cap, sl_off + slot * (size_t)n_win));
   uint32_t* d_wl = (uint32_t*)((char*)ctx->win_len + wl_off);
   ctx->enc_bl = (uint32_t*)((char*)ctx->win_len + bl_off);
+  ctx->enc_crc = (uint32_t*)((char*)ctx->win_len + cr_off);
   ctx->enc_off = (uint64_t*)((char*)ctx->win_len + of_off);
   ctx->enc_slots = (uint8_t*)ctx->win_len + sl_off;
   ctx->enc_slot = slot;
@@ -639,6 +640,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[2], s));
   note_launch();
   k_fill_win_len<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(d_wl, n_win, W, n_tok - w_begin * W);
+  launch_window_crc(ctx->tok + w_begin * W, W, d_wl, n_win, ctx->enc_crc, s);
   {
     ProfScope ps(ctx, kCoder, (double)n_win * (double)W * 8, s);
     launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 1, n_win, ctx->enc_slots, slot,
@@ -653,10 +655,12 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
 }
 
 // Phase 2: the codes of the last encode_codes call, byte-aligned in window order, to d_payload;
-// their bit lengths to d_bitlen (device).
-static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bitlen, cudaStream_t s) {
+// their bit lengths to d_bitlen and their token checksums to d_crc (device).
+static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bitlen, uint32_t* d_crc,
+                               cudaStream_t s) {
   const int64_t n_win = ctx->enc_nwin;
   LMGC_CUDA(ctx, cudaMemcpyAsync(d_bitlen, ctx->enc_bl, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
+  LMGC_CUDA(ctx, cudaMemcpyAsync(d_crc, ctx->enc_crc, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
   launch_pack_codes(ctx->enc_slots, ctx->enc_slot, ctx->enc_bl, n_win, ctx->enc_off, d_payload, s);
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[5], s));
   LMGC_CUDA(ctx, cudaStreamSynchronize(s));
@@ -680,6 +684,8 @@ static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bi
   return LMGC_OK;
 }
 
+constexpr uint32_t kContainerVersion = 2;  // 2: per-window token checksums after the bit lengths
+
 static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
   const lmgc_config& c = ctx->cfg;
   const uint64_t n_tok = (uint64_t)n * (uint64_t)ctx->tpv;
@@ -688,7 +694,7 @@ static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
   uint32_t u32;
   uint64_t u64;
   memcpy(h, "LMGC", 4);
-  u32 = 1; memcpy(h + 4, &u32, 4);
+  u32 = kContainerVersion; memcpy(h + 4, &u32, 4);
   u64 = n; memcpy(h + 8, &u64, 8);
   u64 = n_tok; memcpy(h + 16, &u64, 8);
   u32 = (uint32_t)c.window; memcpy(h + 24, &u32, 4);
@@ -716,19 +722,21 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
   uint64_t payload = 0;
   lmgc_status st = encode_codes(ctx, d_in, n, 0, n_win, &payload, s);
   if (st != LMGC_OK) return st;
-  const size_t total = 64 + 4 * (size_t)n_win + payload;
+  const size_t total = 64 + 8 * (size_t)n_win + payload;
   *out_bytes = total;
   if (cap < total || !d_out) return fail(ctx, LMGC_ERR_NO_SPACE, "container buffer too small");
   uint8_t h[64];
   container_header(ctx, n, h);
   LMGC_CUDA(ctx, cudaMemcpyAsync(d_out, h, 64, cudaMemcpyHostToDevice, s));
-  return encode_pack(ctx, d_out + 64 + 4 * (size_t)n_win, (uint32_t*)(d_out + 64), s);
+  return encode_pack(ctx, d_out + 64 + 8 * (size_t)n_win, (uint32_t*)(d_out + 64),
+                     (uint32_t*)(d_out + 64 + 4 * (size_t)n_win), s);
 }
 
 lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_t first_win, size_t n_win,
                                 uint8_t* d_payload, size_t cap, size_t* payload_bytes, uint32_t* d_bitlen,
-                                lmgc_stream stream) {
-  if (!ctx || !d_in || !payload_bytes || (n_win && !d_bitlen)) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+                                uint32_t* d_crc, lmgc_stream stream) {
+  if (!ctx || !d_in || !payload_bytes || (n_win && (!d_bitlen || !d_crc)))
+    return fail(ctx, LMGC_ERR_INVALID, "null argument");
   const int64_t W = ctx->cfg.window;
   const int64_t total_win = ((int64_t)n * ctx->tpv + W - 1) / W;
   if (n == 0 || n_win == 0 || (int64_t)(first_win + n_win) > total_win)
@@ -739,7 +747,7 @@ lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_
   if (st != LMGC_OK) return st;
   *payload_bytes = payload;
   if (cap < payload || !d_payload) return fail(ctx, LMGC_ERR_NO_SPACE, "payload buffer too small");
-  return encode_pack(ctx, d_payload, d_bitlen, s);
+  return encode_pack(ctx, d_payload, d_bitlen, d_crc, s);
 }
 
 lmgc_status lmgc_container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h_header) {
@@ -791,16 +799,20 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   memcpy(&mcrc, h + 56, 4);
   uint64_t seed;
   memcpy(&seed, h + 48, 8);
-  if (ver != 1 || hW != (uint32_t)W || hP != (uint32_t)c.cdf_bits || kind != (uint32_t)c.input_kind ||
+  if (ver != kContainerVersion || hW != (uint32_t)W || hP != (uint32_t)c.cdf_bits || kind != (uint32_t)c.input_kind ||
       sep != (uint32_t)c.sep_mode || vocab != (uint32_t)c.vocab || mcrc != model_crc(c) || seed != c.weight_seed)
     return fail(ctx, LMGC_ERR_CORRUPT, "container does not match this context's model or coder");
-  if ((uint64_t)n_win != (n_tok + W - 1) / W || 64 + 4 * (size_t)n_win > in_bytes)
+  if ((uint64_t)n_win != (n_tok + W - 1) / W || 64 + 8 * (size_t)n_win > in_bytes)
     return fail(ctx, LMGC_ERR_CORRUPT, "container window table truncated");
   if (cap_tok < n_ids * (size_t)W) return fail(ctx, LMGC_ERR_NO_SPACE, "token buffer too small");
-  std::vector<uint32_t> bl(n_win);
-  if (n_win) LMGC_CUDA(ctx, cudaMemcpy(bl.data(), d_in + 64, 4 * (size_t)n_win, cudaMemcpyDeviceToHost));
+  std::vector<uint32_t> bl(n_win), crc_tab(n_win);
+  if (n_win) {
+    LMGC_CUDA(ctx, cudaMemcpy(bl.data(), d_in + 64, 4 * (size_t)n_win, cudaMemcpyDeviceToHost));
+    LMGC_CUDA(ctx, cudaMemcpy(crc_tab.data(), d_in + 64 + 4 * (size_t)n_win, 4 * (size_t)n_win,
+                              cudaMemcpyDeviceToHost));
+  }
   std::vector<uint64_t> off(n_win + 1);
-  off[0] = 64 + 4 * (uint64_t)n_win;
+  off[0] = 64 + 8 * (uint64_t)n_win;
   for (uint32_t w = 0; w < n_win; w++) off[w + 1] = off[w] + (bl[w] + 7) / 8;
   if (off[n_win] > in_bytes) return fail(ctx, LMGC_ERR_CORRUPT, "container payload truncated");
   for (size_t i = 0; i < n_ids; i++)
@@ -817,12 +829,13 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   // per-chunk device arrays: code offsets, bit lengths, lengths, decoder states
   void* dev = nullptr;
   const size_t st_bytes = dec_state_bytes();
-  const size_t arr = (size_t)nd_max * (8 + 4 + 4) + (size_t)nd_max * st_bytes + 256;
+  const size_t arr = (size_t)nd_max * (8 + 4 + 4 + 4) + (size_t)nd_max * st_bytes + 256;
   LMGC_CUDA(ctx, cudaMallocAsync(&dev, arr, s));
   uint64_t* d_coff = (uint64_t*)dev;
   uint32_t* d_bl = (uint32_t*)(d_coff + nd_max);
   uint32_t* d_len = d_bl + nd_max;
-  void* d_state = (void*)(((uintptr_t)(d_len + nd_max) + 63) / 64 * 64);
+  uint32_t* d_crc = d_len + nd_max;
+  void* d_state = (void*)(((uintptr_t)(d_crc + nd_max) + 63) / 64 * 64);
   lmgc_status st = LMGC_OK;
   for (size_t i0 = 0; i0 < n_ids && st == LMGC_OK; i0 += nd_max) {
     const int64_t nd = std::min<int64_t>(nd_max, (int64_t)(n_ids - i0));
@@ -849,9 +862,16 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
       launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
                         ctx->d_err, s);
     }
+    // every restored window must reproduce the container's token checksum
+    launch_window_crc(out, W, d_len, nd, d_crc, s);
+    std::vector<uint32_t> got(nd);
+    cudaMemcpyAsync(got.data(), d_crc, 4 * nd, cudaMemcpyDeviceToHost, s);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) st = cuda_fail(ctx, e, "decode");
     else st = check_err_word(ctx, s, "decode");
+    for (int64_t j = 0; j < nd && st == LMGC_OK; j++)
+      if (got[j] != crc_tab[h_win_ids[i0 + j]])
+        st = fail(ctx, LMGC_ERR_CORRUPT, "decoded window does not match its token checksum");
   }
   cudaFreeAsync(dev, s);
   cudaStreamSynchronize(s);

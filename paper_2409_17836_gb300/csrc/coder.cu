@@ -220,6 +220,55 @@ void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bit
 }
 
 // ------------------------------------------------------------------------------------------
+// Token checksums of the container: CRC-32 (IEEE 802.3, reflected polynomial 0xEDB88320, initial
+// value and final xor 0xFFFFFFFF) of each window's token ids as little-endian u16 bytes. One
+// thread per window, one table lookup per byte; the 256-entry table is built in shared memory
+// from the polynomial by every block.
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t crc_byte(const uint32_t* tab, uint32_t c, uint32_t b) {
+  return tab[(c ^ b) & 0xFFu] ^ (c >> 8);
+}
+
+__global__ void __launch_bounds__(256) k_window_crc(const uint16_t* __restrict__ tok, int64_t stride,
+                                                    const uint32_t* __restrict__ len, int64_t n_win,
+                                                    uint32_t* __restrict__ out) {
+  __shared__ uint32_t tab[256];
+  {
+    uint32_t c = threadIdx.x;
+    for (int k = 0; k < 8; k++) c = (c & 1u) ? 0xEDB88320u ^ (c >> 1) : c >> 1;
+    tab[threadIdx.x] = c;
+  }
+  __syncthreads();
+  const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (w >= n_win) return;
+  const uint16_t* t = tok + w * stride;
+  const uint32_t n = len[w];
+  uint32_t c = 0xFFFFFFFFu, i = 0;
+  if ((reinterpret_cast<uintptr_t>(t) & 15) == 0) {
+    for (; i + 8 <= n; i += 8) {
+      const uint4 v = *reinterpret_cast<const uint4*>(t + i);
+      const uint32_t words[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int k = 0; k < 4; k++)
+#pragma unroll
+        for (int b = 0; b < 4; b++) c = crc_byte(tab, c, (words[k] >> (8 * b)) & 0xFFu);
+    }
+  }
+  for (; i < n; i++) {
+    c = crc_byte(tab, c, t[i] & 0xFFu);
+    c = crc_byte(tab, c, t[i] >> 8);
+  }
+  out[w] = c ^ 0xFFFFFFFFu;
+}
+
+void launch_window_crc(const uint16_t* tok, int64_t stride, const uint32_t* len, int64_t n_win, uint32_t* out,
+                       cudaStream_t s) {
+  if (n_win <= 0) return;
+  note_launch();
+  k_window_crc<<<(unsigned)((n_win + 255) / 256), 256, 0, s>>>(tok, stride, len, n_win, out);
+}
+
+// ------------------------------------------------------------------------------------------
 // Allocation-free variant of lmgc_range_encode.
 //
 // Some callers cannot allocate device memory at all: a process whose device memory is held

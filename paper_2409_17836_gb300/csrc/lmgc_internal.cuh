@@ -91,6 +91,7 @@ struct lmgc_ctx {
   size_t kv_cap = 0;
   // codes of the last encode (slot scratch inside win_len)
   uint32_t* enc_bl = nullptr;
+  uint32_t* enc_crc = nullptr;
   uint64_t* enc_off = nullptr;
   uint8_t* enc_slots = nullptr;
   size_t enc_slot = 0;
@@ -189,6 +190,9 @@ void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int
                          size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s);
 void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win,
                        uint64_t* offsets /* [n_win+1] scratch */, uint8_t* out, cudaStream_t s);
+// crc32 of the little-endian bytes of tok[w * stride .. w * stride + len[w]) for each w < n_win
+void launch_window_crc(const uint16_t* tok, int64_t stride, const uint32_t* len, int64_t n_win, uint32_t* out,
+                       cudaStream_t s);
 size_t dec_state_bytes();
 void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n,
                      void* state, cudaStream_t s);

@@ -84,7 +84,7 @@ SYMBOLS = {
     "lmgc_encode_bound": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     "lmgc_encode_windows": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_size_t, C.c_size_t, C.c_void_p,
-                                      C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p]),
+                                      C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     "lmgc_container_header": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_encode_host": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p,
                                    C.c_void_p]),
@@ -274,17 +274,19 @@ def lmgc_encode(ctx: Context, values: torch.Tensor, out: torch.Tensor | None = N
 
 
 def lmgc_encode_windows(ctx: Context, values: torch.Tensor, first_win: int, n_win: int, stream=None):
-    """Codes of windows [first_win, first_win + n_win): (payload uint8 tensor, bitlen int32 tensor)."""
+    """Codes of windows [first_win, first_win + n_win): (payload uint8 tensor, bitlen int32 tensor,
+    token checksum int32 tensor)."""
     bitlen = torch.empty(max(n_win, 1), dtype=torch.int32, device=values.device)
+    crc = torch.empty(max(n_win, 1), dtype=torch.int32, device=values.device)
     nb = C.c_size_t()
     st = load().lmgc_encode_windows(ctx.handle, _ptr(values), values.numel(), first_win, n_win, None, 0, C.byref(nb),
-                                    _ptr(bitlen), _stream(stream))
+                                    _ptr(bitlen), _ptr(crc), _stream(stream))
     if st != ERR_NO_SPACE:
         _check(ctx, st)
     out = torch.empty(max(nb.value, 1), dtype=torch.uint8, device=values.device)
     _check(ctx, load().lmgc_encode_windows(ctx.handle, _ptr(values), values.numel(), first_win, n_win, _ptr(out),
-                                           out.numel(), C.byref(nb), _ptr(bitlen), _stream(stream)))
-    return out[: nb.value], bitlen[:n_win]
+                                           out.numel(), C.byref(nb), _ptr(bitlen), _ptr(crc), _stream(stream)))
+    return out[: nb.value], bitlen[:n_win], crc[:n_win]
 
 
 def lmgc_container_header(ctx: Context, n: int) -> bytes:

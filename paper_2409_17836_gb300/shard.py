@@ -1,8 +1,9 @@
 """Encoding one gradient on several GPUs: windows are independent (Sec. 3 "Compression": every
 window is coded from its own BOS), so each rank codes a contiguous range of windows with no data
 exchange. The one exchange step builds the container: the ranks all-gather their windows' bit
-lengths (4 bytes per window); an exclusive scan of the byte lengths gives each payload slice's
-offset, and the slices are concatenated in rank order after the header and the length table."""
+lengths and token checksums (8 bytes per window) and payload slices; an exclusive scan of the
+byte lengths gives each slice's offset, and the slices are concatenated in rank order after the
+header, the length table and the checksum table."""
 from __future__ import annotations
 
 import numpy as np
@@ -25,27 +26,33 @@ def payload_offsets(bitlen_all: np.ndarray) -> np.ndarray:
     return np.concatenate([[0], np.cumsum(nb)])
 
 
-def assemble(header: bytes, bitlen_parts: list[np.ndarray], payload_parts: list[bytes]) -> bytes:
-    """The container from the header, every rank's bit lengths and payload slice (rank order)."""
+def assemble(header: bytes, bitlen_parts: list[np.ndarray], crc_parts: list[np.ndarray],
+             payload_parts: list[bytes]) -> bytes:
+    """The container from the header and every rank's bit lengths, token checksums and payload
+    slice (rank order)."""
     bl = np.concatenate([np.asarray(b, dtype="<u4") for b in bitlen_parts])
+    crc = np.concatenate([np.asarray(c, dtype="<u4") for c in crc_parts])
+    if crc.size != bl.size:
+        raise ValueError("one token checksum per window expected")
     offs = payload_offsets(bl)
     body = b"".join(payload_parts)
     if len(body) != offs[-1]:
         raise ValueError("payload slices do not match their bit lengths")
-    return header + bl.tobytes() + body
+    return header + bl.tobytes() + crc.tobytes() + body
 
 
-def gather_container(header: bytes, bitlen: np.ndarray, payload: bytes, group=None) -> bytes | None:
-    """Exchange step over torch.distributed: every rank contributes its range's bit lengths and
-    payload slice; rank 0 returns the assembled container, the other ranks None."""
+def gather_container(header: bytes, bitlen: np.ndarray, crc: np.ndarray, payload: bytes, group=None) -> bytes | None:
+    """Exchange step over torch.distributed: every rank contributes its range's bit lengths, token
+    checksums and payload slice; rank 0 returns the assembled container, the other ranks None."""
     import torch.distributed as dist
 
     world = dist.get_world_size(group)
     parts: list = [None] * world
-    dist.all_gather_object(parts, (np.asarray(bitlen, dtype=np.uint32), bytes(payload)), group=group)
+    dist.all_gather_object(parts, (np.asarray(bitlen, dtype=np.uint32), np.asarray(crc, dtype=np.uint32),
+                                   bytes(payload)), group=group)
     if dist.get_rank(group) != 0:
         return None
-    return assemble(header, [p[0] for p in parts], [p[1] for p in parts])
+    return assemble(header, [p[0] for p in parts], [p[1] for p in parts], [p[2] for p in parts])
 
 
 def encode_sharded(ctx, values, rank: int, world: int, group=None) -> bytes | None:
@@ -56,8 +63,9 @@ def encode_sharded(ctx, values, rank: int, world: int, group=None) -> bytes | No
     n_win = -(-values.numel() * ctx.tpv // ctx.cfg.window)
     first, count = window_ranges(n_win, world)[rank]
     if count:
-        payload, bitlen = L.lmgc_encode_windows(ctx, values, first, count)
+        payload, bitlen, crc = L.lmgc_encode_windows(ctx, values, first, count)
         pb, bl = payload.cpu().numpy().tobytes(), bitlen.cpu().numpy().view(np.uint32)
+        cr = crc.cpu().numpy().view(np.uint32)
     else:
-        pb, bl = b"", np.zeros(0, np.uint32)
-    return gather_container(L.lmgc_container_header(ctx, values.numel()), bl, pb, group)
+        pb, bl, cr = b"", np.zeros(0, np.uint32), np.zeros(0, np.uint32)
+    return gather_container(L.lmgc_container_header(ctx, values.numel()), bl, cr, pb, group)

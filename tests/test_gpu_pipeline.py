@@ -101,6 +101,23 @@ def test_corrupt_container_rejected():
     assert e.value.status == L.ERR_CORRUPT
     with pytest.raises(L.LmgcError):
         decode_all(ctx, bytes(buf), [10 ** 6])
+    # the token checksum table: it equals the oracle's, a flipped checksum bit fails the window it
+    # covers, and a flipped payload bit (which the coder alone would decode into other tokens)
+    # fails too, while the untouched window still decodes
+    h = parse(bytes(buf))
+    assert np.array_equal(h["crc_tok"], O.window_crcs(O.serialize(I.tiny_gradient(1)[:100], 0), 256))
+    bad = bytearray(buf)
+    bad[64 + 4 * h["n_win"] + 1] ^= 0x10
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(ctx, bytes(bad), [0])
+    assert e.value.status == L.ERR_CORRUPT
+    decode_all(ctx, bytes(bad), [1])
+    bad = bytearray(buf)
+    bad[h["offsets"][1] + 5] ^= 0x04
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(ctx, bytes(bad), [1])
+    assert e.value.status == L.ERR_CORRUPT
+    decode_all(ctx, bytes(bad), [0])
     ctx.close()
     other.close()
 
@@ -145,8 +162,9 @@ def test_window_ranges_assemble_to_the_container():
     n_win = -(-vals.size * 9 // 256)
     parts = []
     for first, count in shard.window_ranges(n_win, 2):
-        pay, bl = L.lmgc_encode_windows(ctx, d, first, count)
-        parts.append((bl.cpu().numpy().view(np.uint32), pay.cpu().numpy().tobytes()))
-    got = shard.assemble(L.lmgc_container_header(ctx, vals.size), [p[0] for p in parts], [p[1] for p in parts])
+        pay, bl, crc = L.lmgc_encode_windows(ctx, d, first, count)
+        parts.append((bl.cpu().numpy().view(np.uint32), crc.cpu().numpy().view(np.uint32), pay.cpu().numpy().tobytes()))
+    got = shard.assemble(L.lmgc_container_header(ctx, vals.size), [p[0] for p in parts], [p[1] for p in parts],
+                         [p[2] for p in parts])
     assert got == ref
     ctx.close()

@@ -1,6 +1,8 @@
 """Oracle end to end (Sec. 3): serialise -> windows with BOS -> LM -> integer CDF -> one code per
 window -> container; decoding each window token by token (KV-cached, Sec. 3 "Compression")
 must return the serialised tokens, and deserialising must return the input bits (lossless)."""
+import zlib
+
 import numpy as np
 import pytest
 
@@ -32,6 +34,7 @@ def test_round_trip(sep_mode, kind):
         n = min(50, tok.size - 50 * w)
         code = buf[h["offsets"][w]: h["offsets"][w + 1]]
         out.append(O.decode_window(c, code, int(h["bitlen"][w]), n))
+        assert h["crc_tok"][w] == O.crc32(out[-1].astype("<u2").tobytes())
     out = np.concatenate(out)
     assert np.array_equal(out, tok)
     back = O.deserialize(out, kind, sep_mode)
@@ -69,3 +72,28 @@ def test_config1_sample_windows_round_trip():
         assert np.array_equal(dec, tok[w * 256:(w + 1) * 256])
         # random-init weights: the prior is weak, so a code costs more than 4 bits per token
         assert nbits > 4 * 256
+
+
+def test_crc32_check_value_and_library():
+    """The container's CRC-32 (IEEE 802.3, reflected polynomial 0xEDB88320): the published check
+    value of the nine ASCII digits, and agreement with zlib on random buffers and lengths."""
+    assert O.crc32(b"123456789") == 0xCBF43926
+    assert O.crc32(b"") == 0
+    rng = np.random.default_rng(7)
+    for n in (1, 2, 3, 17, 4096, 10001):
+        b = rng.integers(0, 256, n, dtype=np.uint8).tobytes()
+        assert O.crc32(b) == zlib.crc32(b)
+
+
+def test_window_crc_table_matches_tokens():
+    c = small_cfg()
+    vals = I.tiny_gradient(5)[:19]
+    buf = O.encode(c, vals)
+    h = O.parse_container(buf)
+    tok = O.serialize(vals, 0).astype("<u2")
+    for w in range(h["n_win"]):
+        assert h["crc_tok"][w] == zlib.crc32(tok[50 * w: 50 * (w + 1)].tobytes())
+    # a flipped bit in the table is caught by comparing against the decoded tokens
+    bad = bytearray(buf)
+    bad[64 + 4 * h["n_win"]] ^= 1
+    assert O.parse_container(bytes(bad))["crc_tok"][0] != h["crc_tok"][0]

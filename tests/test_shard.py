@@ -40,9 +40,10 @@ def _worker(rank, world, port, out_path):
     first, count = shard.window_ranges(n_win, world)[rank]
     codes = O.encode_windows(c, tok, first, count)
     bl = np.array([b for _, b in codes], np.uint32)
+    crc = O.window_crcs(tok, c.window, first, count)
     pb = b"".join(cd for cd, _ in codes)
     header = O.encode(c, vals)[:64]  # the single-process container's header
-    res = shard.gather_container(header, bl, pb)
+    res = shard.gather_container(header, bl, crc, pb)
     if rank == 0:
         with open(out_path, "wb") as f:
             f.write(res)
