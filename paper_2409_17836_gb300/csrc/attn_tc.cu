@@ -2,15 +2,20 @@
 // 5th-generation tensor cores, fp16 inputs and probabilities, fp32 softmax and accumulation.
 //
 // One CTA per (128 query rows, query head, window); 192 threads:
-//   warp 0      TMA: the Q tile once, then 64-key K and V blocks into a 2-stage ring
-//   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64) and O_blk = P V
-//               (M 128, N hd, V as an MN-major operand) and commits to mbarriers
+//   warp 0      TMA: the Q tile once, then 64-key K and V blocks into 3-stage K and V rings
+//   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64, double-buffered in
+//               TMEM) and O += P V (M 128, N hd, V as an MN-major operand; O stays in TMEM for
+//               the whole key loop) and commits to mbarriers
 //   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
 //               per-thread loops; P is written as fp16 into shared memory in the 128-byte
-//               swizzled K-major layout the MMA reads; the running output O stays in registers
-//               and is rescaled by the online-softmax correction before each block's P V is added.
+//               swizzled K-major layout the MMA reads.
+// Online softmax with a lazily moved reference: P = 2^((s - m) log2(e)/sqrt(hd)) uses the row's
+// reference m, which moves to the block maximum only when that maximum exceeds m by more than
+// 8 / (log2(e)/sqrt(hd)) (so P <= 2^8 in fp16). Only then is the row of O in TMEM (and the row
+// sum l) scaled by 2^((m_old - m_new) ...), after the previous block's P V has completed; O / l is
+// the same softmax whatever the reference, and most blocks need no correction.
 // Key blocks are 64-aligned and visited in order 0, 1, ...; a block whose keys all lie past a
-// row's position leaves that row's state exactly unchanged (correction 1, P = 0). A decode step
+// row's position leaves that row's state exactly unchanged (no move, P = 0). A decode step
 // (one query row per window, keys from the cache) therefore reproduces the prefill row bit for
 // bit: the tensor cores' row results do not depend on the other rows of the tile.
 // Every mbarrier wait is bounded (~2 s), after which kErrLimit is recorded and the loops end.
@@ -26,7 +31,8 @@ namespace lmgc {
 namespace attn {
 
 constexpr int BQ = 128, BKV = 64;
-constexpr int kThreads = 320;  // TMA warp, MMA warp, 8 softmax warps
+constexpr int kThreads = 192;  // TMA warp, MMA warp, 4 softmax warps
+constexpr float kLazyLog2 = 8.f;  // reference moves when the block max exceeds it by 2^8 in P
 
 template <int HD>
 struct Shape {
@@ -38,8 +44,8 @@ struct Shape {
   static constexpr int KS = 3;                          // stages of the K ring and of the V ring
   static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB per P buffer (two)
   static constexpr uint32_t TMEM_S = 0;                 // S double buffer: columns 0..127
-  static constexpr uint32_t TMEM_O = 128;               // P V double buffer: 2 x HD columns
-  static constexpr uint32_t TMEM_COLS = (128 + 2 * HD <= 256) ? 256 : 512;
+  static constexpr uint32_t TMEM_O = 128;               // O: HD columns
+  static constexpr uint32_t TMEM_COLS = 256;
   static constexpr size_t SMEM = Q_BYTES + KS * (K_BYTES + V_BYTES) + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) |
@@ -151,6 +157,18 @@ __device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[3
       : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// 32 lanes x 32 columns of 32-bit back to TMEM (thread i writes lane base + i)
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),
+      "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),
+      "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -192,11 +210,9 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   uint8_t* p_gen = smem + (sp - sq);
   uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + 2 * S::P_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
-  float* red_m = reinterpret_cast<float*>(bars + 32);  // [2 parities][2 halves][128 rows]
-  float* red_l = red_m + 512;                          // [2 halves][128 rows]
-  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (256 arrivals) | 5-6 P V ready |
-  //           7-9 K stage loaded | 10-12 K stage free | 13-15 V stage loaded | 16-18 V stage free |
-  //           19-22 softmax warp pairs (64 arrivals)
+  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (128 arrivals) | 5-6 P V done (by the
+  //           parity of the block) | 7-9 K stage loaded | 10-12 K stage free | 13-15 V stage
+  //           loaded | 16-18 V stage free
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
   auto b_p = [&](int i) { return smem_u32(bars + 3 + i); };
@@ -221,7 +237,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 23; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 256 : (i >= 19 ? 64 : 1));
+    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 128 : 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -302,46 +318,22 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         // O_blk = P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
-          tc_mma(tmem + S::TMEM_O + st * HD, desc_kmajor(sp + st * S::P_BYTES + k * 32),
-                 desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, k > 0 ? 1u : 0u);
+          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + st * S::P_BYTES + k * 32),
+                 desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
         tc_commit(b_pv(st));
         tc_commit(b_vempty(ks));
       }
       __syncwarp();
     }
   } else {
-    // ---------------- softmax (warps 2..9): a row is shared by two warps with the same TMEM
-    // lanes (warp mod 4); half hf of them takes key columns [32 hf, 32 hf + 32) and output
-    // columns [hf hd/2, (hf + 1) hd/2). The pair exchanges its partial row maxima through shared
-    // memory behind an mbarrier of 64 arrivals; the two partial row sums are added at the end.
-    const int q4 = warp & 3, hf = (warp - 2) >> 2;
+    // ---------------- softmax (warps 2..5): thread r owns query row r = TMEM lane r ----------------
+    const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
     const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
-    constexpr int OH = HD / 2;
-    const uint32_t b_pair = smem_u32(bars + 19 + q4);
-    float m = -INFINITY, l = 0.f, corr_prev = 1.f;
-    uint64_t o2[OH / 2];  // output columns in packed pairs
-#pragma unroll
-    for (int i = 0; i < OH / 2; i++) o2[i] = 0ull;
-    // O = O * corr + (P V) of a block; deferred by one block so the P V MMA runs meanwhile
-    auto add_pv = [&](int kb, float corr) -> bool {
-      const int st = kb & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)(kb >> 1) & 1u, p.err))) return false;
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < OH / 32; c++) {
-        uint32_t pa[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_O + st * HD + hf * OH + c * 32, pa);
-        tmem_wait();
-        const uint64_t corr2 = f2pack(corr, corr);
-#pragma unroll
-        for (int j = 0; j < 16; j++)
-          o2[c * 16 + j] = ffma2(o2[c * 16 + j], corr2, f2pack(__uint_as_float(pa[2 * j]), __uint_as_float(pa[2 * j + 1])));
-      }
-      tc_fence_before();
-      return true;
-    };
+    const float c = p.scale_log2;
+    const float lazy = kLazyLog2 / c;  // the move threshold in score units
+    float m = -INFINITY, l = 0.f;
     // this row's P row in the swizzled layout: 8-row groups of 1024 B, rows of 128 B, 16-byte
     // chunk index XOR (row mod 8)
     const int prow_off = (r >> 3) * 1024 + (r & 7) * 128;
@@ -350,38 +342,64 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       const int st = kb & 1;
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(st), (uint32_t)(kb >> 1) & 1u, p.err)))) break;
       tc_fence_after();
-      float s[32];
+      float s[64];
       {
-        uint32_t a[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + hf * 32, a);
+        uint32_t a[32], b[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64, a);
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + 32, b);
         tmem_wait();
 #pragma unroll
-        for (int j = 0; j < 32; j++) s[j] = __uint_as_float(a[j]);
+        for (int j = 0; j < 32; j++) {
+          s[j] = __uint_as_float(a[j]);
+          s[32 + j] = __uint_as_float(b[j]);
+        }
       }
       // causal mask, only on blocks that reach past the tile's first position
       if ((int)(kb * BKV + BKV - 1) > pos0_i) {
 #pragma unroll
-        for (int j = 0; j < 32; j++)
-          if (kb * BKV + hf * 32 + j > qpos_i) s[j] = -INFINITY;
+        for (int j = 0; j < 64; j++)
+          if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
       }
-      float mx4[4];
+      float mx8[8];
 #pragma unroll
-      for (int i = 0; i < 4; i++) mx4[i] = s[i];
+      for (int i = 0; i < 8; i++) mx8[i] = s[i];
 #pragma unroll
-      for (int j = 4; j < 32; j++) mx4[j & 3] = fmaxf(mx4[j & 3], s[j]);
-      const float pm = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
-      red_m[(kb & 1) * 256 + hf * 128 + r] = pm;
-      mbar_arrive(b_pair);
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pair, (uint32_t)kb & 1u, p.err)))) break;
-      const float mx = fmaxf(pm, red_m[(kb & 1) * 256 + (1 - hf) * 128 + r]);
-      const float mn = fmaxf(m, mx);  // finite: key 0 is never masked
-      // exactly 1 when the maximum does not change (a fully masked block is then a no-op)
-      const float corr = ex2_approx((m - mn) * p.scale_log2);
-      const float nb = -mn * p.scale_log2;
-      const uint64_t c2 = f2pack(p.scale_log2, p.scale_log2), nb2 = f2pack(nb, nb);
+      for (int j = 8; j < 64; j++) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      // move the reference only for a large rise (always on the first block: m = -inf)
+      const bool move = mx > m + lazy;
+      float corr = 1.f;
+      if (move) {
+        corr = ex2_approx((m - mx) * c);  // 0 on the first block
+        l *= corr;
+        m = mx;
+      }
+      if (kb > 0 && __any_sync(0xffffffffu, move)) {
+        // scale this warp's rows of O (factor 1 for rows that did not move) once the previous
+        // block's P V has landed in TMEM
+        const int pst = (kb - 1) & 1;
+        if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(pst), (uint32_t)((kb - 1) >> 1) & 1u, p.err)))) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int cc = 0; cc < HD / 32; cc++) {
+          uint32_t o[32];
+          tmem_ld32_nowait(tmem + tl + S::TMEM_O + cc * 32, o);
+          tmem_wait();
+#pragma unroll
+          for (int j = 0; j < 32; j++) o[j] = __float_as_uint(__uint_as_float(o[j]) * corr);
+          tmem_st32(tmem + tl + S::TMEM_O + cc * 32, o);
+        }
+        tmem_st_wait();
+      }
+      // the P buffer of this block was last read by P V(kb - 2)
+      if (kb >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)((kb - 2) >> 1) & 1u, p.err))))
+        break;
+      const float nb = (m == -INFINITY) ? 0.f : -m * c;
+      const uint64_t c2 = f2pack(c, c), nb2 = f2pack(nb, nb);
       uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
 #pragma unroll
-      for (int j = 0; j < 32; j += 2) {
+      for (int j = 0; j < 64; j += 2) {
         float t0, t1;
         f2unpack(ffma2(f2pack(s[j], s[j + 1]), c2, nb2), t0, t1);
         s[j] = ex2_approx(t0);
@@ -392,48 +410,49 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       float a0, a1, a2, a3;
       f2unpack(acc0, a0, a1);
       f2unpack(acc1, a2, a3);
-      l = l * corr + ((a0 + a1) + (a2 + a3));
-      m = mn;
+      l += (a0 + a1) + (a2 + a3);
       uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
 #pragma unroll
-      for (int cc = 0; cc < 4; cc++) {
-        const int c = hf * 4 + cc;
+      for (int ch = 0; ch < 8; ch++) {
         uint32_t wv[4];
 #pragma unroll
         for (int t = 0; t < 4; t++) {
-          __half2 hb = __floats2half2_rn(s[8 * cc + 2 * t], s[8 * cc + 2 * t + 1]);
+          __half2 hb = __floats2half2_rn(s[8 * ch + 2 * t], s[8 * ch + 2 * t + 1]);
           wv[t] = *reinterpret_cast<uint32_t*>(&hb);
         }
-        *reinterpret_cast<uint4*>(prow + ((c ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        *reinterpret_cast<uint4*>(prow + ((ch ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
       mbar_arrive(b_p(st));
-      if (kb > 0 && !(ok = add_pv(kb - 1, corr_prev))) break;
-      corr_prev = corr;
     }
-    if (ok) ok = add_pv(nkb - 1, corr_prev);
+    // O / l once the last P V has completed
     if (ok) {
-      // row sum = half 0's partial + half 1's partial (the same order in both threads)
-      red_l[hf * 128 + r] = l;
-      mbar_arrive(b_pair);
-      ok = __all_sync(0xffffffffu, mbar_wait(b_pair, (uint32_t)nkb & 1u, p.err));
+      const int last = nkb - 1;
+      ok = __all_sync(0xffffffffu, mbar_wait(b_pv(last & 1), (uint32_t)(last >> 1) & 1u, p.err));
     }
-    if (ok && r < nrows) {
-      const float other = red_l[(1 - hf) * 128 + r];
-      const float inv = 1.f / (hf == 0 ? l + other : other + l);
-      __half* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD + hf * OH;
+    if (ok) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      __half* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
+#pragma unroll 1
+      for (int cc = 0; cc < HD / 32; cc++) {
+        uint32_t o[32];
+        tmem_ld32_nowait(tmem + tl + S::TMEM_O + cc * 32, o);
+        tmem_wait();
+        if (r < nrows) {
 #pragma unroll
-      for (int c = 0; c < OH / 8; c++) {
-        uint32_t wv[4];
+          for (int q = 0; q < 4; q++) {
+            uint32_t wv[4];
 #pragma unroll
-        for (int t = 0; t < 4; t++) {
-          float x0, x1;
-          f2unpack(o2[4 * c + t], x0, x1);
-          __half2 hb = __floats2half2_rn(x0 * inv, x1 * inv);
-          wv[t] = *reinterpret_cast<uint32_t*>(&hb);
+            for (int t = 0; t < 4; t++) {
+              __half2 hb = __floats2half2_rn(__uint_as_float(o[8 * q + 2 * t]) * inv,
+                                             __uint_as_float(o[8 * q + 2 * t + 1]) * inv);
+              wv[t] = *reinterpret_cast<uint32_t*>(&hb);
+            }
+            reinterpret_cast<uint4*>(dst + cc * 32)[q] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+          }
         }
-        reinterpret_cast<uint4*>(dst)[c] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
       }
     }
   }
