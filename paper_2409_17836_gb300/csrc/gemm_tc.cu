@@ -35,7 +35,11 @@ constexpr uint32_t A_BYTES = BM * BK * 2;  // 16 KiB
 constexpr uint32_t B_BYTES = BN * BK * 2;  // 32 KiB
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
-constexpr int GROUP_M = 16;
+// tile order: groups of group_m M-blocks, N-blocks swept inside a group (M fastest). A weight
+// operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy and groups are 16
+// M-blocks; a larger one (the vocabulary projection) streams instead, with groups of 64 M-blocks
+// so that it is re-read only once per 8192 rows.
+constexpr int64_t kKeepBBytes = 48ll << 20;
 // residual epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, row pitch 36 words so
 // that both the row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B
 constexpr int STG_PITCH = 36;
@@ -92,6 +96,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// the same with an L2 cache policy (createpolicy) attached to the read
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%3, "
+      "%4}], [%2], %5;" ::"r"(dst),
+      "l"((uint64_t)map), "r"(mbar), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_commit(uint32_t mbar) {
@@ -135,6 +149,7 @@ struct Params {
   void* C;
   int64_t M, N, K;
   int tiles_m, tiles_n, num_kb;
+  int group_m, keep_b;
   uint32_t* err;
   // kQKVRope: rotary embedding of columns [0, rope_cols) in heads of rope_hd; row m sits at
   // position rope_pos0 + m % rope_pos_mod; rope_cs[pos * rope_hd/2 + i] = (cos, sin)
@@ -160,10 +175,10 @@ __device__ __forceinline__ float row_scale(const Params& p, int64_t m) {
 }
 
 __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int& nb) {
-  const int per_group = GROUP_M * p.tiles_n;
+  const int per_group = p.group_m * p.tiles_n;
   const int g = t / per_group;
-  const int first_m = g * GROUP_M;
-  const int gm = min(p.tiles_m - first_m, GROUP_M);
+  const int first_m = g * p.group_m;
+  const int gm = min(p.tiles_m - first_m, p.group_m);
   const int r = t - g * per_group;
   mb = first_m + r % gm;
   nb = r / gm;
@@ -215,7 +230,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
           v.z += o[j].z;
           v.w += o[j].w;
         }
-        d[j] = v;
+        __stcs(d + j, v);
       }
     } else {
 #pragma unroll
@@ -268,6 +283,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
+    // the weight operand B is re-read by every group of M-blocks: keep it in L2 ahead of the
+    // streamed activations
+    uint64_t keep_b;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep_b));
     uint32_t g = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
@@ -281,7 +300,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
           mbar_expect_tx(full(s), STAGE_BYTES);
           tma_load_2d(sA(s), &tma_a, full(s), kb * BK, mb * BM);
-          tma_load_2d(sB(s), &tma_b, full(s), kb * BK, nb * BN);
+          if (p.keep_b) tma_load_2d_hint(sB(s), &tma_b, full(s), kb * BK, nb * BN, keep_b);
+          else tma_load_2d(sB(s), &tma_b, full(s), kb * BK, nb * BN);
         }
         __syncwarp();
       }
@@ -326,15 +346,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int a = i & 1;
       const uint32_t aph = (uint32_t)(i >> 1) & 1u;
       const int64_t m = (int64_t)mb * BM + q * 32 + lane;
-      if (EPI == kAddResidual && (p.N & 31) == 0) {
-        // pull the residual rows of this tile (first visit) and of the next one into L2 ahead of use
-        if (i == 0) prefetch_residual(p, m, nb);
-        if (t + (int)gridDim.x < n_tiles) {
-          int mb2, nb2;
-          tile_coords(t + (int)gridDim.x, p, mb2, nb2);
-          prefetch_residual(p, (int64_t)mb2 * BM + q * 32 + lane, nb2);
-        }
-      }
+      // pull this tile's residual rows into L2 while its accumulator is still being built
+      if (EPI == kAddResidual && (p.N & 31) == 0) prefetch_residual(p, m, nb);
       const float rs = row_scale(p, m);
       if (!__all_sync(0xffffffffu, mbar_wait(tfull(a), aph, p.err))) break;
       tc_fence_after();
@@ -439,7 +452,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 8; k++) {
             const int64_t gm = row0 + 4 * k + cr;
-            o[k] = gm < p.M ? *reinterpret_cast<const float4*>(xbase + gm * p.N) : make_float4(0.f, 0.f, 0.f, 0.f);
+            o[k] = gm < p.M ? __ldcs(reinterpret_cast<const float4*>(xbase + gm * p.N)) : make_float4(0.f, 0.f, 0.f, 0.f);
           }
 #pragma unroll
           for (int k = 0; k < 8; k++) {
@@ -451,11 +464,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             v.z = o[k].z + acc.z;
             v.w = o[k].w + acc.w;
             if (gm < p.M) {
-              *reinterpret_cast<float4*>(xbase + gm * p.N) = v;
+              __stcs(reinterpret_cast<float4*>(xbase + gm * p.N), v);
               if (p.xh) {
                 __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
-                *reinterpret_cast<uint2*>(p.xh + gm * p.N + n0 + cc) =
-                    make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1));
+                __stcs(reinterpret_cast<uint2*>(p.xh + gm * p.N + n0 + cc),
+                       make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1)));
               }
             }
             ssl[k] += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
@@ -560,6 +573,8 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.tiles_m = (int)((M + BM - 1) / BM);
   p.tiles_n = (int)((N + BN - 1) / BN);
   p.num_kb = (int)((K + BK - 1) / BK);
+  p.keep_b = N * K * 2 <= kKeepBBytes ? 1 : 0;
+  p.group_m = p.keep_b ? 16 : 64;
   p.err = err;
   p.rope_cs = rope ? rope->cs : nullptr;
   p.rope_cols = rope ? rope->cols : 0;
