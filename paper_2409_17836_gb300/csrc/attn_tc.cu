@@ -1,14 +1,18 @@
 // attn_tc.cu -- causal softmax attention of the LM prior (Eq. 2's Llama decoder) on the
 // 5th-generation tensor cores, fp16 inputs and probabilities, fp32 softmax and accumulation.
 //
-// One CTA per (128 query rows, query head, window); 192 threads:
-//   warp 0      TMA: the Q tile once, then 64-key K and V blocks into 3-stage K and V rings
-//   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64, double-buffered in
-//               TMEM) and O += P V (M 128, N hd, V as an MN-major operand; O stays in TMEM for
-//               the whole key loop) and commits to mbarriers
+// One CTA per (128 query rows, query head, window); 224 threads:
+//   warp 0      TMA: the Q tile once, then 64-key K blocks into a 3-stage ring
+//   warp 6      TMA: 64-key V blocks into a 2-stage ring
+//   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64) two blocks ahead into a
+//               3-deep ring in TMEM, and O += P V (M 128, N hd, V as an MN-major operand; O stays
+//               in TMEM for the whole key loop), and commits to mbarriers
 //   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
-//               per-thread loops; P is written as fp16 into shared memory in the 128-byte
-//               swizzled K-major layout the MMA reads.
+//               per-thread loops; P is written as fp16 into shared memory (3 buffers) in the
+//               128-byte swizzled K-major layout the MMA reads.
+// Issue order S(kb+2), P V(kb) means that S(kb) is issued after P V(kb-3); its completion (the
+// commit tracks every earlier tensor-core operation of the issuing thread) therefore also says
+// that P buffer kb mod 3 is free again, so the softmax waits on nothing else in steady state.
 // Online softmax with a lazily moved reference: P = 2^((s - m) log2(e)/sqrt(hd)) uses the row's
 // reference m, which moves to the block maximum only when that maximum exceeds m by more than
 // 8 / (log2(e)/sqrt(hd)) (so P <= 2^8 in fp16). Only then is the row of O in TMEM (and the row
@@ -31,7 +35,7 @@ namespace lmgc {
 namespace attn {
 
 constexpr int BQ = 128, BKV = 64;
-constexpr int kThreads = 192;  // TMA warp, MMA warp, 4 softmax warps
+constexpr int kThreads = 224;  // K TMA warp, MMA warp, 4 softmax warps, V TMA warp
 constexpr float kLazyLog2 = 8.f;  // reference moves when the block max exceeds it by 2^8 in P
 
 template <int HD>
@@ -41,12 +45,13 @@ struct Shape {
   static constexpr uint32_t KV_CHUNK = BKV * 128;       // one 64x64 bf16 chunk (8 KiB)
   static constexpr uint32_t K_BYTES = BKV * HD * 2;
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
-  static constexpr int KS = 3;                          // stages of the K ring and of the V ring
-  static constexpr uint32_t P_BYTES = BQ * BKV * 2;     // 16 KiB per P buffer (two)
-  static constexpr uint32_t TMEM_S = 0;                 // S double buffer: columns 0..127
-  static constexpr uint32_t TMEM_O = 128;               // O: HD columns
-  static constexpr uint32_t TMEM_COLS = 256;
-  static constexpr size_t SMEM = Q_BYTES + KS * (K_BYTES + V_BYTES) + 2 * P_BYTES + 1024 + 256 + 3 * 1024;
+  static constexpr int KSK = 3, KSV = 2;                // stages of the K ring and of the V ring
+  static constexpr int NP = 3;                          // P buffers (16 KiB each)
+  static constexpr uint32_t P_BYTES = BQ * BKV * 2;
+  static constexpr uint32_t TMEM_S = 0;                 // S ring: columns 0..191
+  static constexpr uint32_t TMEM_O = HD == 64 ? 192 : 256;  // O: HD columns
+  static constexpr uint32_t TMEM_COLS = HD == 64 ? 256 : 512;
+  static constexpr size_t SMEM = Q_BYTES + KSK * K_BYTES + KSV * V_BYTES + NP * P_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
@@ -66,11 +71,10 @@ __device__ __forceinline__ void mbar_arrive(uint32_t a) {
 }
 __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
   uint32_t ok;
-  // the suspend-time hint lets a waiting warp sleep until the phase completes instead of spinning
   asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(a), "r"(parity), "r"(0x989680u)
+      : "r"(a), "r"(parity)
       : "memory");
   return ok != 0;
 }
@@ -205,22 +209,22 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   const uint32_t sq = smem_u32(smem);
   const uint32_t sk = sq + S::Q_BYTES;                // K ring
-  const uint32_t sv = sk + S::KS * S::K_BYTES;         // V ring
-  const uint32_t sp = sv + S::KS * S::V_BYTES;         // two P buffers
+  const uint32_t sv = sk + S::KSK * S::K_BYTES;        // V ring
+  const uint32_t sp = sv + S::KSV * S::V_BYTES;        // P buffers
   uint8_t* p_gen = smem + (sp - sq);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + 2 * S::P_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + S::NP * S::P_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
-  // barriers: 0 Q loaded | 1-2 S ready | 3-4 P written (128 arrivals) | 5-6 P V done (by the
-  //           parity of the block) | 7-9 K stage loaded | 10-12 K stage free | 13-15 V stage
-  //           loaded | 16-18 V stage free
+  // barriers: 0 Q loaded | 1-3 S ready | 4-6 P written (128 arrivals) | 7-8 P V done (by the
+  //           parity of the block) | 9-11 K stage loaded | 12-14 K stage free | 15-16 V stage
+  //           loaded | 17-18 V stage free
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
-  auto b_p = [&](int i) { return smem_u32(bars + 3 + i); };
-  auto b_pv = [&](int i) { return smem_u32(bars + 5 + i); };
-  auto b_kfull = [&](int i) { return smem_u32(bars + 7 + i); };
-  auto b_kempty = [&](int i) { return smem_u32(bars + 10 + i); };
-  auto b_vfull = [&](int i) { return smem_u32(bars + 13 + i); };
-  auto b_vempty = [&](int i) { return smem_u32(bars + 16 + i); };
+  auto b_p = [&](int i) { return smem_u32(bars + 4 + i); };
+  auto b_pv = [&](int i) { return smem_u32(bars + 7 + i); };
+  auto b_kfull = [&](int i) { return smem_u32(bars + 9 + i); };
+  auto b_kempty = [&](int i) { return smem_u32(bars + 12 + i); };
+  auto b_vfull = [&](int i) { return smem_u32(bars + 15 + i); };
+  auto b_vempty = [&](int i) { return smem_u32(bars + 17 + i); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -237,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i == 3 || i == 4) ? 128 : 1);
+    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -253,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
+    // ---------------- TMA producer: Q, then K blocks ----------------
     if (lane == 0) {
       mbar_expect_tx(b_q, S::Q_BYTES);
 #pragma unroll
@@ -261,9 +265,8 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     }
     __syncwarp();
     for (int kb = 0; kb < nkb; kb++) {
-      const int ks = kb % S::KS;
-      const uint32_t ph = (uint32_t)(kb / S::KS) & 1u;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kempty(ks), ph ^ 1u, p.err))) break;
+      const int ks = kb % S::KSK;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kempty(ks), ((uint32_t)(kb / S::KSK) & 1u) ^ 1u, p.err))) break;
       if (lane == 0) {
         mbar_expect_tx(b_kfull(ks), S::K_BYTES);
 #pragma unroll
@@ -272,22 +275,27 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
                       kv_row0 + kb * BKV);
       }
       __syncwarp();
-      if (!__all_sync(0xffffffffu, mbar_wait(b_vempty(ks), ph ^ 1u, p.err))) break;
+    }
+  } else if (warp == 6) {
+    // ---------------- TMA producer: V blocks ----------------
+    for (int kb = 0; kb < nkb; kb++) {
+      const int vs = kb % S::KSV;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_vempty(vs), ((uint32_t)(kb / S::KSV) & 1u) ^ 1u, p.err))) break;
       if (lane == 0) {
-        mbar_expect_tx(b_vfull(ks), S::V_BYTES);
+        mbar_expect_tx(b_vfull(vs), S::V_BYTES);
 #pragma unroll
         for (int c = 0; c < S::KCH; c++)
-          tma_load_2d(sv + ks * S::V_BYTES + c * S::KV_CHUNK, &tkv, b_vfull(ks), p.v_col0 + kvh * HD + 64 * c,
+          tma_load_2d(sv + vs * S::V_BYTES + c * S::KV_CHUNK, &tkv, b_vfull(vs), p.v_col0 + kvh * HD + 64 * c,
                       kv_row0 + kb * BKV);
       }
       __syncwarp();
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer: S(kb+1) is issued before P V(kb) so the softmax of block kb
-    // overlaps the tensor cores; a K stage is released as soon as its S is done ----------------
+    // ---------------- MMA issuer: S(kb+2) is issued before P V(kb), so the softmax of block kb
+    // never waits for the other rows' P(kb-1); a K stage is released as soon as its S is done ----------------
     auto issue_s = [&](int kb) -> bool {
-      const int ks = kb % S::KS;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KS) & 1u, p.err))) return false;
+      const int ks = kb % S::KSK, sb = kb % 3;
+      if (!__all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KSK) & 1u, p.err))) return false;
       tc_fence_after();
       if (lane == 0) {
         const uint32_t kbase = sk + ks * S::K_BYTES;
@@ -295,10 +303,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
 #pragma unroll
         for (int k = 0; k < HD / 16; k++) {
           const int c = k >> 2, o = (k & 3) * 32;
-          tc_mma(tmem + S::TMEM_S + (kb & 1) * 64, desc_kmajor(sq + c * (BQ * 128) + o),
+          tc_mma(tmem + S::TMEM_S + sb * 64, desc_kmajor(sq + c * (BQ * 128) + o),
                  desc_kmajor(kbase + c * S::KV_CHUNK + o), S::IDESC_S, k > 0 ? 1u : 0u);
         }
-        tc_commit(b_s(kb & 1));
+        tc_commit(b_s(sb));
         tc_commit(b_kempty(ks));
       }
       __syncwarp();
@@ -306,22 +314,23 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     };
     bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
     if (ok) ok = issue_s(0);
+    if (ok && nkb > 1) ok = issue_s(1);
     for (int kb = 0; kb < nkb && ok; kb++) {
-      const int st = kb & 1, ks = kb % S::KS;
-      if (kb + 1 < nkb && !(ok = issue_s(kb + 1))) break;
-      ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(ks), (uint32_t)(kb / S::KS) & 1u, p.err));
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(st), (uint32_t)(kb >> 1) & 1u, p.err));
+      const int pb = kb % S::NP, vs = kb % S::KSV;
+      if (kb + 2 < nkb && !(ok = issue_s(kb + 2))) break;
+      ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(vs), (uint32_t)(kb / S::KSV) & 1u, p.err));
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(pb), (uint32_t)(kb / S::NP) & 1u, p.err));
       if (!ok) break;
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t vbase = sv + ks * S::V_BYTES;
-        // O_blk = P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
+        const uint32_t vbase = sv + vs * S::V_BYTES;
+        // O += P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
-          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + st * S::P_BYTES + k * 32),
+          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + pb * S::P_BYTES + k * 32),
                  desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
-        tc_commit(b_pv(st));
-        tc_commit(b_vempty(ks));
+        tc_commit(b_pv(kb & 1));
+        tc_commit(b_vempty(vs));
       }
       __syncwarp();
     }
@@ -339,14 +348,15 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     const int prow_off = (r >> 3) * 1024 + (r & 7) * 128;
     bool ok = true;
     for (int kb = 0; kb < nkb; kb++) {
-      const int st = kb & 1;
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(st), (uint32_t)(kb >> 1) & 1u, p.err)))) break;
+      const int sb = kb % 3;
+      // S(kb) done: also P V(kb-3) done, so P buffer kb mod 3 is free
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / 3) & 1u, p.err)))) break;
       tc_fence_after();
       float s[64];
       {
         uint32_t a[32], b[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64, a);
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + st * 64 + 32, b);
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64, a);
+        tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64 + 32, b);
         tmem_wait();
 #pragma unroll
         for (int j = 0; j < 32; j++) {
@@ -377,7 +387,8 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       }
       if (kb > 0 && __any_sync(0xffffffffu, move)) {
         // scale this warp's rows of O (factor 1 for rows that did not move) once the previous
-        // block's P V has landed in TMEM
+        // block's P V has landed in TMEM (its barrier is read by parity: P V(kb-3) has completed,
+        // as S(kb) has)
         const int pst = (kb - 1) & 1;
         if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(pst), (uint32_t)((kb - 1) >> 1) & 1u, p.err)))) break;
         tc_fence_after();
@@ -392,9 +403,6 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         }
         tmem_st_wait();
       }
-      // the P buffer of this block was last read by P V(kb - 2)
-      if (kb >= 2 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(st), (uint32_t)((kb - 2) >> 1) & 1u, p.err))))
-        break;
       const float nb = (m == -INFINITY) ? 0.f : -m * c;
       const uint64_t c2 = f2pack(c, c), nb2 = f2pack(nb, nb);
       uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
@@ -411,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       f2unpack(acc0, a0, a1);
       f2unpack(acc1, a2, a3);
       l += (a0 + a1) + (a2 + a3);
-      uint8_t* prow = p_gen + st * S::P_BYTES + prow_off;
+      uint8_t* prow = p_gen + sb * S::P_BYTES + prow_off;
 #pragma unroll
       for (int ch = 0; ch < 8; ch++) {
         uint32_t wv[4];
@@ -424,13 +432,13 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
-      mbar_arrive(b_p(st));
+      mbar_arrive(b_p(sb));
     }
     // O / l once the last P V has completed
-    if (ok) {
-      const int last = nkb - 1;
-      ok = __all_sync(0xffffffffu, mbar_wait(b_pv(last & 1), (uint32_t)(last >> 1) & 1u, p.err));
-    }
+    // (P V(j)'s barrier is read by parity, which is only meaningful once P V(j-2) has completed:
+    // S(last) implies P V(last-3), so P V(last-1) is awaited before P V(last))
+    for (int j = nkb >= 2 ? nkb - 2 : 0; j < nkb && ok; j++)
+      ok = __all_sync(0xffffffffu, mbar_wait(b_pv(j & 1), (uint32_t)(j >> 1) & 1u, p.err));
     if (ok) {
       tc_fence_after();
       const float inv = 1.f / l;
