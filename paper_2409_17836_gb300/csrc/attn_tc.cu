@@ -143,6 +143,12 @@ __device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
+// max of three (one instruction on sm_100 and later)
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
 // 2^x on the special-function unit (flushes subnormal results to zero; ex2(-inf) = 0)
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -370,13 +376,12 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         for (int j = 0; j < 64; j++)
           if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
       }
-      float mx8[8];
+      float mx4[4];
 #pragma unroll
-      for (int i = 0; i < 8; i++) mx8[i] = s[i];
+      for (int i = 0; i < 4; i++) mx4[i] = s[i];
 #pragma unroll
-      for (int j = 8; j < 64; j++) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      for (int j = 4; j < 64; j += 2) mx4[(j >> 1) & 3] = fmax3(mx4[(j >> 1) & 3], s[j], s[j + 1]);
+      const float mx = fmaxf(fmax3(mx4[0], mx4[1], mx4[2]), mx4[3]);
       // move the reference only for a large rise (always on the first block: m = -inf)
       const bool move = mx > m + lazy;
       float corr = 1.f;
