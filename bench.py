@@ -248,6 +248,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="convnet-tinyllama", choices=WORKLOADS)
     ap.add_argument("--batch-windows", type=int, default=0)
+    # a model with fewer layers, for small profiler captures only (the config line names it)
+    ap.add_argument("--layers", type=int, default=0)
     ap.add_argument("--ref-positions", type=int, default=12)
     ap.add_argument("--cpu-target-s", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -275,6 +277,8 @@ def main():
     cfg, vals = workload(args.workload)
     if args.batch_windows:
         cfg = configs.with_(cfg, batch_windows=args.batch_windows)
+    if args.layers:
+        cfg = configs.with_(cfg, n_layers=args.layers)
     ctx = L.Context(cfg)
     tpv = ctx.tpv
     per_step = (cfg.batch_windows * cfg.window) // tpv  # values filling one model batch

@@ -52,14 +52,17 @@ constexpr int kAMax = 40 * 65536;
 __device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t* __restrict__ H,
                                                const uint32_t* __restrict__ L) {
   const float C = (float)(65536.0 * 1.4426950408889634073599246810019);
-  float y = __fmul_rn(__fsub_rn(z, m), C);
-  // a = -rint(y) (ties to even), capped at 40 * 2^16; y below the cap is clamped before the
-  // conversion so that huge logit gaps cannot overflow it
-  int a = (y < -(float)kAMax) ? kAMax : -__float2int_rn(y);
-  a = min(max(a, 0), kAMax);
-  uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
-  uint64_t e = (hl + (1ull << 30)) >> 31;
-  return (uint32_t)(e >> (a >> 16));
+  const float y = __fmul_rn(__fsub_rn(z, m), C);  // <= 0: m is the row maximum
+  // a = -rint(y) (ties to even), capped at 40 * 2^16: y is clamped to -40 * 2^16 (an integer, so
+  // rint keeps it) before the conversion, which also keeps huge logit gaps from overflowing it
+  const int a = -__float2int_rn(fmaxf(y, -(float)kAMax));
+  // H, L <= 2^31, so (H L + 2^30) >> 31 <= 2^31 fits 32 bits; the final shift by a >> 16 (<= 40)
+  // uses shr.b32, which yields 0 for shifts of 32 or more
+  const uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
+  const uint32_t e31 = (uint32_t)((hl + (1ull << 30)) >> 31);
+  uint32_t e;
+  asm("shr.b32 %0, %1, %2;" : "=r"(e) : "r"(e31), "r"(a >> 16));
+  return e;
 }
 
 template <typename V>
@@ -124,7 +127,7 @@ struct RowStats {
 // S >= 2^31, the largest e being 2^31), and q0 S <= e Mq < 2^61, so one remainder test fixes it.
 __device__ __forceinline__ uint64_t gfloor(uint32_t e, const RowStats& st) {
   const uint64_t X = (uint64_t)e * st.Mq;
-  uint64_t q = ((uint64_t)e * st.F) >> 32;
+  uint64_t q = __umulhi(e, st.F);
   if (X - q * st.S >= st.S) q++;
   return q;
 }
