@@ -3,11 +3,14 @@
 // fp16 operands (the model's bf16-valued weights held exactly in fp16, fp16 activations), fp32
 // accumulation in tensor memory.
 //
-// Persistent, warp-specialised kernel, one CTA per SM (192 threads):
+// Persistent, warp-specialised kernel, one CTA per SM:
 //   warp 0      TMA producer: 128x64 A and 256x64 B tiles (128-byte swizzle) into a 4-stage ring
 //   warp 1      allocates 512 TMEM columns; one lane issues tcgen05.mma (M 128, N 256, K 16) and
 //               tcgen05.commit to the ring's empty barriers and to the accumulator-full barriers
-//   warps 2-5   epilogue: tcgen05.ld 32 lanes x 32 columns, convert / add, store to global
+//   warps 2..   epilogue: 4 warps (8 for the fp32 logits, whose stores dominate): warp w reads
+//               TMEM lanes 32 (w mod 4) .. and, with 8 warps, one column half of the tile;
+//               tcgen05.ld 32 lanes x 32 columns, convert / add, store to global (fp32 outputs
+//               through a shared-memory transpose)
 // Two 128x256 fp32 accumulators (2 x 256 TMEM columns) let the epilogue of one tile run under the
 // main loop of the next. Tiles are visited in groups of 16 M-blocks so the A and B tiles in
 // flight stay in L2.
@@ -30,7 +33,13 @@ namespace lmgc {
 namespace tc {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int kThreads = 192;
+// epilogue warps per epilogue kind, and the CTA size
+template <int EPI>
+struct EpiShape {
+  static constexpr int kWarps = EPI == kStoreF32 ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kWarps;
+  static constexpr uint32_t kStgBytes = kWarps == 8 ? 8 * 32 * 32 * 4 : 4 * 32 * 36 * 4;
+};
 constexpr uint32_t A_BYTES = BM * BK * 2;  // 16 KiB
 constexpr uint32_t B_BYTES = BN * BK * 2;  // 32 KiB
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
@@ -40,11 +49,18 @@ constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 // M-blocks; a larger one (the vocabulary projection) streams instead, with groups of 64 M-blocks
 // so that it is re-read only once per 8192 rows.
 constexpr int64_t kKeepBBytes = 48ll << 20;
-// residual epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, row pitch 36 words so
-// that both the row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B
-constexpr int STG_PITCH = 36;
-constexpr uint32_t STG_BYTES = 4 * 32 * STG_PITCH * 4;
-constexpr size_t SMEM_BYTES = (size_t)STAGES * STAGE_BYTES + 256 + STG_BYTES + 1024;
+// fp32 epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, laid out so that both the
+// row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B: with 4 warps a
+// row pitch of 36 words; with 8 warps (which need the space) a pitch of 32 words with the 16-byte
+// slot j of row r stored at slot j ^ (r mod 8)
+template <int NH>
+__device__ __forceinline__ int stg_off(int r, int j) {
+  return NH == 2 ? r * 32 + ((j ^ (r & 7)) << 2) : r * 36 + (j << 2);
+}
+template <int EPI>
+constexpr size_t smem_bytes() {
+  return (size_t)STAGES * STAGE_BYTES + 256 + EpiShape<EPI>::kStgBytes + 1024;
+}
 
 // instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B f16 (bits 7-9, 10-12 = 0),
 // both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28
@@ -184,11 +200,11 @@ __device__ __forceinline__ void tile_coords(int t, const Params& p, int& mb, int
   nb = r / gm;
 }
 
-// L2 prefetch of row m's BN residual columns starting at column block nb (N % 32 == 0)
-__device__ __forceinline__ void prefetch_residual(const Params& p, int64_t m, int nb) {
-  if (m >= p.M) return;
-  const char* xr = reinterpret_cast<const char*>(reinterpret_cast<const float*>(p.C) + m * p.N + (int64_t)nb * BN);
-  const int lines = (int)(min((int64_t)BN, p.N - (int64_t)nb * BN) * 4 / 128);
+// L2 prefetch of row m's fp32 residual, columns [n0, n0 + cnt) (N % 32 == 0, n0 % 32 == 0)
+__device__ __forceinline__ void prefetch_residual(const Params& p, int64_t m, int64_t n0, int cnt) {
+  if (m >= p.M || n0 >= p.N) return;
+  const char* xr = reinterpret_cast<const char*>(reinterpret_cast<const float*>(p.C) + m * p.N + n0);
+  const int lines = (int)(min((int64_t)cnt, p.N - n0) * 4 / 128);
   for (int j = 0; j < lines; j++) asm volatile("prefetch.global.L2 [%0];" ::"l"(xr + j * 128));
 }
 
@@ -241,7 +257,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
 }
 
 template <int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -264,7 +280,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; a++) {
       mbar_init(tfull(a), 1);
-      mbar_init(tempty(a), 128);
+      mbar_init(tempty(a), 32 * EpiShape<EPI>::kWarps);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -337,8 +353,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int q = warp & 3;  // TMEM lanes 32q .. 32q+31
+    // ---------------- epilogue (warps 2 ..) ----------------
+    constexpr int NH = EpiShape<EPI>::kWarps / 4;  // column parts of a tile
+    constexpr int HN = BN / NH;
+    const int q = warp & 3;            // TMEM lanes 32q .. 32q+31
+    const int hw = (warp - 2) >> 2;    // tile columns [HN hw, HN hw + HN)
+    float* stg = staging + (warp - 2) * (NH == 2 ? 32 * 32 : 32 * 36);
     int i = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
       int mb, nb;
@@ -346,21 +366,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int a = i & 1;
       const uint32_t aph = (uint32_t)(i >> 1) & 1u;
       const int64_t m = (int64_t)mb * BM + q * 32 + lane;
-      // pull this tile's residual rows into L2 while its accumulator is still being built
-      if (EPI == kAddResidual && (p.N & 31) == 0) prefetch_residual(p, m, nb);
+      const int64_t ncol0 = (int64_t)nb * BN + hw * HN;  // first output column of this half
+      // pull this half-tile's residual rows into L2 while its accumulator is still being built
+      if (EPI == kAddResidual && (p.N & 31) == 0) prefetch_residual(p, m, ncol0, HN);
       const float rs = row_scale(p, m);
       if (!__all_sync(0xffffffffu, mbar_wait(tfull(a), aph, p.err))) break;
       tc_fence_after();
-      const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);
+      const uint32_t tacc = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(a * BN);  // tile column 0
+      const uint32_t tbase = tacc + (uint32_t)(hw * HN);
       if (EPI == kQKVRope) {
-        // one head at a time: halves [0, hd/2) and [hd/2, hd) rotate pairwise by pos * theta_i
+        // one head at a time (a half holds HN / hd whole heads): halves [0, hd/2) and [hd/2, hd)
+        // rotate pairwise by pos * theta_i
         const int hd = p.rope_hd, hh = hd / 2;
         const int64_t pos = p.rope_pos0 + m % p.rope_pos_mod;
         const float2* cs = p.rope_cs + pos * hh;
 #pragma unroll 1
         for (int c = 0; c < hh / 32; ++c) {
           float ct[32], st[32];
-          const bool any_rot = (int64_t)nb * BN < p.rope_cols && m < p.M;
+          const bool any_rot = ncol0 < p.rope_cols && m < p.M;
           if (any_rot) {
             const float4* c4 = reinterpret_cast<const float4*>(cs + c * 32);
 #pragma unroll
@@ -373,8 +396,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
 #pragma unroll 1
-          for (int hs = 0; hs < BN / hd; ++hs) {
-            const int64_t col0 = (int64_t)nb * BN + hs * hd;
+          for (int hs = 0; hs < HN / hd; ++hs) {
+            const int64_t col0 = ncol0 + hs * hd;
             const bool rot = col0 < p.rope_cols;
             uint32_t a[32], b[32];
             tmem_ld32(tbase + (uint32_t)(hs * hd + c * 32), a);
@@ -400,12 +423,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       } else if (EPI == kSwiGLU) {
-        // columns [0, 128) of the tile are gate, [128, 256) the matching up columns
+        // columns [0, 128) of the tile are gate, [128, 256) the matching up columns; this warp
+        // writes output chunks [4 hw / NH, 4 (hw + 1) / NH) (32 columns each)
 #pragma unroll 1
-        for (int c = 0; c < BN / 64; ++c) {
+        for (int c = 4 * hw / NH; c < 4 * (hw + 1) / NH; ++c) {
           uint32_t g[32], u[32];
-          tmem_ld32(tbase + (uint32_t)(c * 32), g);
-          tmem_ld32(tbase + (uint32_t)(BN / 2 + c * 32), u);
+          tmem_ld32(tacc + (uint32_t)(c * 32), g);
+          tmem_ld32(tacc + (uint32_t)(BN / 2 + c * 32), u);
           if (m < p.M) {
             const int64_t half_n = p.N / 2;
             __half* dst = reinterpret_cast<__half*>(p.C) + m * half_n + (int64_t)nb * (BN / 2) + c * 32;
@@ -423,49 +447,59 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < 4; j++) d4[j] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
           }
         }
-      } else if (EPI == kAddResidual && (p.N & 31) == 0) {
-        // x += acc through a shared-memory transpose: the warp's 32 rows x 32 columns go in one row
-        // per thread and come out as 8 lanes per row, so each global access covers 4 full rows of
-        // 128 B. With xh set, fp16(x) is written too and ss_out[row * tiles_n + nb] receives the
-        // row's sum of squares over this tile's columns (fixed order: per lane over chunks, then
-        // a butterfly over the row's 8 lanes).
-        float* stg = staging + q * 32 * STG_PITCH;
-        const int cr = lane >> 3, cc = (lane & 7) * 4;
+      } else if ((EPI == kAddResidual || EPI == kStoreF32) && (p.N & 31) == 0) {
+        // fp32 output through a shared-memory transpose: the warp's 32 rows x 32 columns go in one
+        // row per thread and come out as 8 lanes per row, so each global access covers 4 full rows
+        // of 128 B. kAddResidual (4 epilogue warps, so a warp covers the whole tile) adds the stored
+        // x; with xh set it also writes fp16(x), and ss_out[row * tiles_n + nb] receives the row's
+        // sum of squares over the tile's columns (fixed order: per lane over chunks, then a
+        // butterfly over the row's 8 lanes).
+        const int cr = lane >> 3, sl = lane & 7, cc = sl * 4;
         const int64_t row0 = (int64_t)mb * BM + q * 32;
         float ssl[8];
 #pragma unroll
         for (int k = 0; k < 8; k++) ssl[k] = 0.f;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          const int64_t n0 = (int64_t)nb * BN + c * 32;
+        for (int c = 0; c < HN / 32; ++c) {
+          const int64_t n0 = ncol0 + c * 32;
           if (n0 >= p.N) break;
           uint32_t r[32];
           tmem_ld32(tbase + (uint32_t)(c * 32), r);
-          float4* srow = reinterpret_cast<float4*>(stg + lane * STG_PITCH);
+          if (p.row_ss) {
+#pragma unroll
+            for (int j = 0; j < 32; j++) r[j] = __float_as_uint(__uint_as_float(r[j]) * rs);
+          }
 #pragma unroll
           for (int j = 0; j < 8; j++)
-            srow[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
-                                  __uint_as_float(r[4 * j + 3]));
+            *reinterpret_cast<float4*>(stg + stg_off<NH>(lane, j)) =
+                make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
+                            __uint_as_float(r[4 * j + 3]));
           __syncwarp();
-          float* xbase = reinterpret_cast<float*>(p.C) + n0 + cc;
+          float* cbase = reinterpret_cast<float*>(p.C) + n0 + cc;
           float4 o[8];
+          if (EPI == kAddResidual) {
 #pragma unroll
-          for (int k = 0; k < 8; k++) {
-            const int64_t gm = row0 + 4 * k + cr;
-            o[k] = gm < p.M ? __ldcs(reinterpret_cast<const float4*>(xbase + gm * p.N)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int k = 0; k < 8; k++) {
+              const int64_t gm = row0 + 4 * k + cr;
+              o[k] = gm < p.M ? __ldcs(reinterpret_cast<const float4*>(cbase + gm * p.N))
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
           }
 #pragma unroll
           for (int k = 0; k < 8; k++) {
-            const int64_t gm = row0 + 4 * k + cr;
-            const float4 acc = *reinterpret_cast<const float4*>(stg + (4 * k + cr) * STG_PITCH + cc);
-            float4 v;
-            v.x = o[k].x + acc.x;
-            v.y = o[k].y + acc.y;
-            v.z = o[k].z + acc.z;
-            v.w = o[k].w + acc.w;
+            const int rr = 4 * k + cr;
+            const int64_t gm = row0 + rr;
+            const float4 acc = *reinterpret_cast<const float4*>(stg + stg_off<NH>(rr, sl));
+            float4 v = acc;
+            if (EPI == kAddResidual) {
+              v.x = o[k].x + acc.x;
+              v.y = o[k].y + acc.y;
+              v.z = o[k].z + acc.z;
+              v.w = o[k].w + acc.w;
+            }
             if (gm < p.M) {
-              __stcs(reinterpret_cast<float4*>(xbase + gm * p.N), v);
-              if (p.xh) {
+              __stcs(reinterpret_cast<float4*>(cbase + gm * p.N), v);
+              if (EPI == kAddResidual && p.xh) {
                 __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
                 __stcs(reinterpret_cast<uint2*>(p.xh + gm * p.N + n0 + cc),
                        make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1)));
@@ -475,7 +509,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           __syncwarp();
         }
-        if (p.xh) {
+        if (EPI == kAddResidual && p.xh) {
 #pragma unroll
           for (int k = 0; k < 8; k++) {
             float v = ssl[k];
@@ -488,10 +522,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       } else {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < HN / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(tbase + (uint32_t)(c * 32), r);
-          const int64_t n0 = (int64_t)nb * BN + c * 32;
+          const int64_t n0 = ncol0 + c * 32;
           if (p.row_ss) {
 #pragma unroll
             for (int j = 0; j < 32; j++) r[j] = __float_as_uint(__uint_as_float(r[j]) * rs);
@@ -529,11 +563,11 @@ static void init_once() {
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (major != 10) g_encode = nullptr;  // tcgen05 path only on Blackwell-class devices
-  cudaFuncSetAttribute(k_gemm_tc<kStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-  cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-  cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-  cudaFuncSetAttribute(k_gemm_tc<kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-  cudaFuncSetAttribute(k_gemm_tc<kQKVRope>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  cudaFuncSetAttribute(k_gemm_tc<kStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kStore>());
+  cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kAddResidual>());
+  cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kStoreF32>());
+  cudaFuncSetAttribute(k_gemm_tc<kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kSwiGLU>());
+  cudaFuncSetAttribute(k_gemm_tc<kQKVRope>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kQKVRope>());
 }
 
 static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t rows, uint32_t box_rows) {
@@ -590,11 +624,12 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   const int tiles = p.tiles_m * p.tiles_n;
   const int grid = std::max(1, std::min(tiles, g_num_sms));
   note_launch();
-  if (epi == kStore) k_gemm_tc<kStore><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else if (epi == kAddResidual) k_gemm_tc<kAddResidual><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else if (epi == kStoreF32) k_gemm_tc<kStoreF32><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else if (epi == kSwiGLU) k_gemm_tc<kSwiGLU><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
-  else k_gemm_tc<kQKVRope><<<grid, kThreads, SMEM_BYTES, s>>>(ma, mb, p);
+  if (epi == kStore) k_gemm_tc<kStore><<<grid, EpiShape<kStore>::kThreads, smem_bytes<kStore>(), s>>>(ma, mb, p);
+  else if (epi == kAddResidual)
+    k_gemm_tc<kAddResidual><<<grid, EpiShape<kAddResidual>::kThreads, smem_bytes<kAddResidual>(), s>>>(ma, mb, p);
+  else if (epi == kStoreF32) k_gemm_tc<kStoreF32><<<grid, EpiShape<kStoreF32>::kThreads, smem_bytes<kStoreF32>(), s>>>(ma, mb, p);
+  else if (epi == kSwiGLU) k_gemm_tc<kSwiGLU><<<grid, EpiShape<kSwiGLU>::kThreads, smem_bytes<kSwiGLU>(), s>>>(ma, mb, p);
+  else k_gemm_tc<kQKVRope><<<grid, EpiShape<kQKVRope>::kThreads, smem_bytes<kQKVRope>(), s>>>(ma, mb, p);
 }
 
 }  // namespace lmgc
