@@ -3,17 +3,23 @@
 // fp16 operands (the model's bf16-valued weights held exactly in fp16, fp16 activations), fp32
 // accumulation in tensor memory.
 //
-// Persistent, warp-specialised kernel, one CTA per SM:
-//   warp 0      TMA producer: 128x64 A and 256x64 B tiles (128-byte swizzle) into a 4-stage ring
-//   warp 1      allocates 512 TMEM columns; one lane issues tcgen05.mma (M 128, N 256, K 16) and
-//               tcgen05.commit to the ring's empty barriers and to the accumulator-full barriers
-//   warps 2..   epilogue: 4 warps (8 for the fp32 logits, whose stores dominate): warp w reads
-//               TMEM lanes 32 (w mod 4) .. and, with 8 warps, one column half of the tile;
+// Persistent, warp-specialised kernel on CTA pairs (clusters of 2, one CTA per SM): a pair computes
+// 256x256 output tiles with tcgen05.mma.cta_group::2 (M 256, N 256, K 16). CTA r of the pair
+// stages rows [128 r, 128 r + 128) of the tile's A block and rows [128 r, 128 r + 128) of its B
+// block (the N dimension), so each SM reads 8 KiB of operands per MMA instead of 12, and holds
+// its own 128 output rows in its tensor memory.
+//   warp 0      TMA producer (both CTAs): 128x64 A and 128x64 B tiles (128-byte swizzle) into a
+//               6-stage ring; both CTAs' copies complete on the leader CTA's full barrier
+//   warp 1      both CTAs allocate 512 TMEM columns together; in the leader one lane issues the
+//               MMAs and multicasts its commits to both CTAs' empty and accumulator-full barriers
+//   warps 2..   epilogue (both CTAs): 4 warps (8 for the fp32 logits, whose stores dominate): warp
+//               w reads TMEM lanes 32 (w mod 4) .. and, with 8 warps, one column half of the tile;
 //               tcgen05.ld 32 lanes x 32 columns, convert / add, store to global (fp32 outputs
-//               through a shared-memory transpose)
-// Two 128x256 fp32 accumulators (2 x 256 TMEM columns) let the epilogue of one tile run under the
-// main loop of the next. Tiles are visited in groups of 16 M-blocks so the A and B tiles in
-// flight stay in L2.
+//               through a shared-memory transpose); then arrive on the leader's accumulator-empty
+//               barrier
+// Two 128x256 fp32 accumulators per CTA (2 x 256 TMEM columns) let the epilogue of one tile run
+// under the main loop of the next. Tiles are visited in groups of M-blocks so the A and B tiles
+// in flight stay in L2.
 //
 // Row invariance (needed by the KV-cached decoder): every output element is accumulated over k
 // in the same order by the same MMA shape whatever M is; rows past M are zero-filled by TMA and
@@ -32,7 +38,9 @@
 namespace lmgc {
 namespace tc {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BM = 128;  // rows per CTA; a pair covers 2 BM = 256 rows of a tile
+constexpr int BN = 256, BK = 64, STAGES = 6;
+constexpr int TM = 2 * BM;  // tile rows
 // epilogue warps per epilogue kind, and the CTA size
 template <int EPI>
 struct EpiShape {
@@ -40,14 +48,14 @@ struct EpiShape {
   static constexpr int kThreads = 64 + 32 * kWarps;
   static constexpr uint32_t kStgBytes = kWarps == 8 ? 8 * 32 * 32 * 4 : 4 * 32 * 36 * 4;
 };
-constexpr uint32_t A_BYTES = BM * BK * 2;  // 16 KiB
-constexpr uint32_t B_BYTES = BN * BK * 2;  // 32 KiB
+constexpr uint32_t A_BYTES = BM * BK * 2;        // 16 KiB
+constexpr uint32_t B_BYTES = (BN / 2) * BK * 2;  // 16 KiB: this CTA's half of the B tile
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
-// tile order: groups of group_m M-blocks, N-blocks swept inside a group (M fastest). A weight
-// operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy and groups are 16
-// M-blocks; a larger one (the vocabulary projection) streams instead, with groups of 64 M-blocks
-// so that it is re-read only once per 8192 rows.
+// tile order: groups of group_m M-blocks (256 rows each), N-blocks swept inside a group (M
+// fastest). A weight operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy
+// and groups are 8 M-blocks; a larger one (the vocabulary projection) streams instead, with
+// groups of 32 M-blocks so that it is re-read only once per 8192 rows.
 constexpr int64_t kKeepBBytes = 48ll << 20;
 // fp32 epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, laid out so that both the
 // row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B: with 4 warps a
@@ -63,8 +71,8 @@ constexpr size_t smem_bytes() {
 }
 
 // instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B f16 (bits 7-9, 10-12 = 0),
-// both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28
-constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+// both K-major (15, 16 = 0), N >> 3 at bits 17-22, M >> 4 at bits 24-28 (M = 256: the pair)
+constexpr uint32_t IDESC = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TM >> 4) << 24);
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -104,32 +112,50 @@ __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t*
   return false;
 }
 
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y) {
+// tile copy into this CTA's shared memory that completes on a barrier of either CTA of the pair
+// (`mbar` is a shared::cluster address)
+__device__ __forceinline__ void tma_load_pair(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(
-          dst),
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(dst),
       "l"((uint64_t)map), "r"(mbar), "r"(x), "r"(y)
       : "memory");
 }
 
 // the same with an L2 cache policy (createpolicy) attached to the read
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y,
-                                                 uint64_t policy) {
+__device__ __forceinline__ void tma_load_pair_hint(uint32_t dst, const CUtensorMap* map, uint32_t mbar, int x, int y,
+                                                   uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1, {%3, "
-      "%4}], [%2], %5;" ::"r"(dst),
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
       "l"((uint64_t)map), "r"(mbar), "r"(x), "r"(y), "l"(policy)
       : "memory");
 }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_commit(uint32_t mbar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar) : "memory");
+// arrive on the barrier at this offset in both CTAs of the pair once the issued MMAs complete
+__device__ __forceinline__ void tc_commit_pair(uint32_t mbar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(mbar),
+      "h"((uint16_t)3)
+      : "memory");
+}
+// the same shared-memory offset in CTA `rank` of the cluster (a shared::cluster address)
+__device__ __forceinline__ uint32_t cluster_addr(uint32_t a, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_a) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_a) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
   asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
           d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(IDESC), "r"(accumulate)
       : "memory");
@@ -257,7 +283,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
 }
 
 template <int EPI>
-__global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThreads, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -273,29 +299,34 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
   auto tempty = [&](int a) { return smem_u32(bars + 2 * STAGES + 2 + a); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint32_t rank;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const bool leader = rank == 0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; s++) {
-      mbar_init(full(s), 1);
-      mbar_init(empty(s), 1);
+      mbar_init(full(s), 1);   // the leader's: its expect_tx arrival plus both CTAs' bytes
+      mbar_init(empty(s), 1);  // the leader's multicast commit
     }
     for (int a = 0; a < 2; a++) {
-      mbar_init(tfull(a), 1);
-      mbar_init(tempty(a), 32 * EpiShape<EPI>::kWarps);
+      mbar_init(tfull(a), 1);                           // the leader's multicast commit
+      mbar_init(tempty(a), 2 * 32 * EpiShape<EPI>::kWarps);  // the leader's: both CTAs' epilogues
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+    // one warp of each CTA of the pair allocates together (the same columns in both)
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(TMEM_COLS)
                  : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int n_tiles = p.tiles_m * p.tiles_n;
+  const int cid = (int)(blockIdx.x >> 1), ncl = (int)(gridDim.x >> 1);
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -305,7 +336,8 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep_b));
     uint32_t g = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    const int a_row = (int)rank * BM, b_row = (int)rank * (BN / 2);
+    for (int t = cid; t < n_tiles && ok; t += ncl) {
       int mb, nb;
       tile_coords(t, p, mb, nb);
       for (int kb = 0; kb < p.num_kb; ++kb, ++g) {
@@ -314,20 +346,21 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
         ok = __all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u, p.err));
         if (!ok) break;
         if (lane == 0) {
-          mbar_expect_tx(full(s), STAGE_BYTES);
-          tma_load_2d(sA(s), &tma_a, full(s), kb * BK, mb * BM);
-          if (p.keep_b) tma_load_2d_hint(sB(s), &tma_b, full(s), kb * BK, nb * BN, keep_b);
-          else tma_load_2d(sB(s), &tma_b, full(s), kb * BK, nb * BN);
+          const uint32_t lf = cluster_addr(full(s), 0);
+          if (leader) mbar_expect_tx(full(s), 2 * STAGE_BYTES);
+          tma_load_pair(sA(s), &tma_a, lf, kb * BK, mb * TM + a_row);
+          if (p.keep_b) tma_load_pair_hint(sB(s), &tma_b, lf, kb * BK, nb * BN + b_row, keep_b);
+          else tma_load_pair(sB(s), &tma_b, lf, kb * BK, nb * BN + b_row);
         }
         __syncwarp();
       }
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
+    // ---------------- MMA issuer (the leader CTA) ----------------
     uint32_t g = 0;
     int i = 0;
-    bool ok = true;
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++i) {
+    bool ok = leader;
+    for (int t = cid; t < n_tiles && ok; t += ncl, ++i) {
       const int a = i & 1;
       const uint32_t aph = (uint32_t)(i >> 1) & 1u;
       ok = __all_sync(0xffffffffu, mbar_wait(tempty(a), aph ^ 1u, p.err));
@@ -345,11 +378,11 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc_mma(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), (kb > 0 || k > 0) ? 1u : 0u);
-          tc_commit(empty(s));
+          tc_commit_pair(empty(s));
         }
         __syncwarp();
       }
-      if (lane == 0) tc_commit(tfull(a));
+      if (lane == 0) tc_commit_pair(tfull(a));
       __syncwarp();
     }
   } else {
@@ -360,12 +393,14 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
     const int hw = (warp - 2) >> 2;    // tile columns [HN hw, HN hw + HN)
     float* stg = staging + (warp - 2) * (NH == 2 ? 32 * 32 : 32 * 36);
     int i = 0;
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++i) {
+    const uint32_t tempty_leader0 = cluster_addr(tempty(0), 0), tempty_leader1 = cluster_addr(tempty(1), 0);
+    for (int t = cid; t < n_tiles; t += ncl, ++i) {
       int mb, nb;
       tile_coords(t, p, mb, nb);
       const int a = i & 1;
       const uint32_t aph = (uint32_t)(i >> 1) & 1u;
-      const int64_t m = (int64_t)mb * BM + q * 32 + lane;
+      const int64_t mrow0 = (int64_t)mb * TM + (int64_t)rank * BM;  // this CTA's first tile row
+      const int64_t m = mrow0 + q * 32 + lane;
       const int64_t ncol0 = (int64_t)nb * BN + hw * HN;  // first output column of this half
       // pull this half-tile's residual rows into L2 while its accumulator is still being built
       if (EPI == kAddResidual && (p.N & 31) == 0) prefetch_residual(p, m, ncol0, HN);
@@ -455,7 +490,7 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
         // sum of squares over the tile's columns (fixed order: per lane over chunks, then a
         // butterfly over the row's 8 lanes).
         const int cr = lane >> 3, sl = lane & 7, cc = sl * 4;
-        const int64_t row0 = (int64_t)mb * BM + q * 32;
+        const int64_t row0 = mrow0 + q * 32;
         float ssl[8];
 #pragma unroll
         for (int k = 0; k < 8; k++) ssl[k] = 0.f;
@@ -534,14 +569,15 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(tempty(a));
+      mbar_arrive_cluster(a ? tempty_leader1 : tempty_leader0);
     }
   }
+  // neither CTA leaves (or frees its tensor memory) while the pair's MMAs may still use it
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TMEM_COLS) : "memory");
   }
 }
 
@@ -549,6 +585,22 @@ __global__ void __launch_bounds__(EpiShape<EPI>::kThreads, 1)
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static std::once_flag g_once;
 static int g_num_sms = 0;
+static int g_max_clusters[5] = {0, 0, 0, 0, 0};  // co-resident CTA pairs, per epilogue kind
+
+template <int EPI>
+static void setup_kernel() {
+  cudaFuncSetAttribute(k_gemm_tc<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<EPI>());
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)std::max(2, g_num_sms & ~1), 1, 1);
+  cfg.blockDim = dim3(EpiShape<EPI>::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem_bytes<EPI>();
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<EPI>, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = g_num_sms / 2;
+  }
+  g_max_clusters[EPI] = std::max(1, n);
+}
 
 static void init_once() {
   cudaDriverEntryPointQueryResult q;
@@ -563,11 +615,12 @@ static void init_once() {
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (major != 10) g_encode = nullptr;  // tcgen05 path only on Blackwell-class devices
-  cudaFuncSetAttribute(k_gemm_tc<kStore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kStore>());
-  cudaFuncSetAttribute(k_gemm_tc<kAddResidual>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kAddResidual>());
-  cudaFuncSetAttribute(k_gemm_tc<kStoreF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kStoreF32>());
-  cudaFuncSetAttribute(k_gemm_tc<kSwiGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kSwiGLU>());
-  cudaFuncSetAttribute(k_gemm_tc<kQKVRope>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes<kQKVRope>());
+  if (!g_encode) return;
+  setup_kernel<kStore>();
+  setup_kernel<kAddResidual>();
+  setup_kernel<kStoreF32>();
+  setup_kernel<kSwiGLU>();
+  setup_kernel<kQKVRope>();
 }
 
 static bool make_map(CUtensorMap* map, const void* ptr, uint64_t k, uint64_t rows, uint32_t box_rows) {
@@ -595,7 +648,7 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   using namespace tc;
   std::call_once(g_once, init_once);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN)) {
+  if (!make_map(&ma, A, (uint64_t)K, (uint64_t)M, BM) || !make_map(&mb, B, (uint64_t)K, (uint64_t)N, BN / 2)) {
     set_thread_error("cuTensorMapEncodeTiled failed");
     return;
   }
@@ -604,11 +657,11 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.M = M;
   p.N = N;
   p.K = K;
-  p.tiles_m = (int)((M + BM - 1) / BM);
+  p.tiles_m = (int)((M + TM - 1) / TM);
   p.tiles_n = (int)((N + BN - 1) / BN);
   p.num_kb = (int)((K + BK - 1) / BK);
   p.keep_b = N * K * 2 <= kKeepBBytes ? 1 : 0;
-  p.group_m = p.keep_b ? 16 : 64;
+  p.group_m = p.keep_b ? 8 : 32;
   p.err = err;
   p.rope_cs = rope ? rope->cs : nullptr;
   p.rope_cols = rope ? rope->cols : 0;
@@ -622,7 +675,7 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.xh = norm ? norm->xh : nullptr;
   p.ss_out = norm ? norm->ss_out : nullptr;
   const int tiles = p.tiles_m * p.tiles_n;
-  const int grid = std::max(1, std::min(tiles, g_num_sms));
+  const int grid = 2 * std::max(1, std::min(tiles, g_max_clusters[epi]));  // CTA pairs
   note_launch();
   if (epi == kStore) k_gemm_tc<kStore><<<grid, EpiShape<kStore>::kThreads, smem_bytes<kStore>(), s>>>(ma, mb, p);
   else if (epi == kAddResidual)
