@@ -8,11 +8,10 @@
 //               3-deep ring in TMEM, and O += P V (M 128, N hd, V as an MN-major operand; O stays
 //               in TMEM for the whole key loop), and commits to mbarriers
 //   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
-//               per-thread loops; P is written as fp16 into shared memory (3 buffers) in the
-//               128-byte swizzled K-major layout the MMA reads.
-// Issue order S(kb+2), P V(kb) means that S(kb) is issued after P V(kb-3); its completion (the
-// commit tracks every earlier tensor-core operation of the issuing thread) therefore also says
-// that P buffer kb mod 3 is free again, so the softmax waits on nothing else in steady state.
+//               per-thread loops; P is written as fp16 pairs back into the first 32 columns of
+//               the block's own S buffer in TMEM, and the P V MMA reads its A operand from there.
+// S(kb+2) reuses the S buffer of block kb-1, so the issuer first waits for P V(kb-1), which read
+// P(kb-1) from it.
 // Online softmax with a lazily moved reference: P = 2^((s - m) log2(e)/sqrt(hd)) uses the row's
 // reference m, which moves to the block maximum only when that maximum exceeds m by more than
 // 8 / (log2(e)/sqrt(hd)) (so P <= 2^8 in fp16). Only then is the row of O in TMEM (and the row
@@ -46,12 +45,10 @@ struct Shape {
   static constexpr uint32_t K_BYTES = BKV * HD * 2;
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
   static constexpr int KSK = 3, KSV = 2;                // stages of the K ring and of the V ring
-  static constexpr int NP = 3;                          // P buffers (16 KiB each)
-  static constexpr uint32_t P_BYTES = BQ * BKV * 2;
-  static constexpr uint32_t TMEM_S = 0;                 // S ring: columns 0..191
+  static constexpr uint32_t TMEM_S = 0;                 // S ring: columns 0..191 (P in the first 32 of each)
   static constexpr uint32_t TMEM_O = HD == 64 ? 192 : 256;  // O: HD columns
   static constexpr uint32_t TMEM_COLS = HD == 64 ? 256 : 512;
-  static constexpr size_t SMEM = Q_BYTES + KSK * K_BYTES + KSV * V_BYTES + NP * P_BYTES + 1024 + 256 + 3 * 1024;
+  static constexpr size_t SMEM = Q_BYTES + KSK * K_BYTES + KSV * V_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) |
                                       ((uint32_t)(BQ >> 4) << 24);
@@ -111,6 +108,16 @@ __device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t a_desc, uint64_
       "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(
           d_tmem),
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// D (+)= A B with A read from tensor memory: row i in lane i, two fp16 per 32-bit column, K step
+// k of 16 at column offset 8k
+__device__ __forceinline__ void tc_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\ttcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 // K-major operand, 128-byte swizzle: 8-row groups 1024 B apart (SBO), LBO unused.
@@ -216,9 +223,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const uint32_t sq = smem_u32(smem);
   const uint32_t sk = sq + S::Q_BYTES;                // K ring
   const uint32_t sv = sk + S::KSK * S::K_BYTES;        // V ring
-  const uint32_t sp = sv + S::KSV * S::V_BYTES;        // P buffers
-  uint8_t* p_gen = smem + (sp - sq);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(p_gen + S::NP * S::P_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (sv + S::KSV * S::V_BYTES - sq));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   // barriers: 0 Q loaded | 1-3 S ready | 4-6 P written (128 arrivals) | 7-8 P V done (by the
   //           parity of the block) | 9-11 K stage loaded | 12-14 K stage free | 15-16 V stage
@@ -322,19 +327,26 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     if (ok) ok = issue_s(0);
     if (ok && nkb > 1) ok = issue_s(1);
     for (int kb = 0; kb < nkb && ok; kb++) {
-      const int pb = kb % S::NP, vs = kb % S::KSV;
-      if (kb + 2 < nkb && !(ok = issue_s(kb + 2))) break;
+      const int sb = kb % 3, vs = kb % S::KSV;
+      if (kb + 2 < nkb) {
+        // S(kb+2) overwrites the buffer from which P V(kb-1) read P(kb-1)
+        if (kb >= 1 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv((kb - 1) & 1), (uint32_t)((kb - 1) >> 1) & 1u,
+                                                                p.err))))
+          break;
+        if (!(ok = issue_s(kb + 2))) break;
+      }
       ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(vs), (uint32_t)(kb / S::KSV) & 1u, p.err));
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(pb), (uint32_t)(kb / S::NP) & 1u, p.err));
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(sb), (uint32_t)(kb / 3) & 1u, p.err));
       if (!ok) break;
       tc_fence_after();
       if (lane == 0) {
         const uint32_t vbase = sv + vs * S::V_BYTES;
-        // O += P V over the 64 keys in steps of 16: P advances 32 B, V advances 16 rows (2 KiB)
+        // O += P V over the 64 keys in steps of 16: P (in TMEM) advances 8 columns, V advances
+        // 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
-          tc_mma(tmem + S::TMEM_O, desc_kmajor(sp + pb * S::P_BYTES + k * 32),
-                 desc_mnmajor(vbase + k * 2048, S::KV_CHUNK), S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
+          tc_mma_ts(tmem + S::TMEM_O, tmem + S::TMEM_S + sb * 64 + 8 * k, desc_mnmajor(vbase + k * 2048, S::KV_CHUNK),
+                    S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
         tc_commit(b_pv(kb & 1));
         tc_commit(b_vempty(vs));
       }
@@ -349,13 +361,9 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     const float c = p.scale_log2;
     const float lazy = kLazyLog2 / c;  // the move threshold in score units
     float m = -INFINITY, l = 0.f;
-    // this row's P row in the swizzled layout: 8-row groups of 1024 B, rows of 128 B, 16-byte
-    // chunk index XOR (row mod 8)
-    const int prow_off = (r >> 3) * 1024 + (r & 7) * 128;
     bool ok = true;
     for (int kb = 0; kb < nkb; kb++) {
       const int sb = kb % 3;
-      // S(kb) done: also P V(kb-3) done, so P buffer kb mod 3 is free
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / 3) & 1u, p.err)))) break;
       tc_fence_after();
       float s[64];
@@ -424,18 +432,17 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       f2unpack(acc0, a0, a1);
       f2unpack(acc1, a2, a3);
       l += (a0 + a1) + (a2 + a3);
-      uint8_t* prow = p_gen + sb * S::P_BYTES + prow_off;
+      // P as fp16 pairs over the first 32 columns of this block's S buffer (already read)
+      {
+        uint32_t pw[32];
 #pragma unroll
-      for (int ch = 0; ch < 8; ch++) {
-        uint32_t wv[4];
-#pragma unroll
-        for (int t = 0; t < 4; t++) {
-          __half2 hb = __floats2half2_rn(s[8 * ch + 2 * t], s[8 * ch + 2 * t + 1]);
-          wv[t] = *reinterpret_cast<uint32_t*>(&hb);
+        for (int j = 0; j < 32; j++) {
+          __half2 hb = __floats2half2_rn(s[2 * j], s[2 * j + 1]);
+          pw[j] = *reinterpret_cast<uint32_t*>(&hb);
         }
-        *reinterpret_cast<uint4*>(prow + ((ch ^ (r & 7)) << 4)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        tmem_st32(tmem + tl + S::TMEM_S + sb * 64, pw);
+        tmem_st_wait();
       }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       tc_fence_before();
       mbar_arrive(b_p(sb));
     }
