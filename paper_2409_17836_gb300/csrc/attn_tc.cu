@@ -13,10 +13,11 @@
 // S(kb+2) reuses the S buffer of block kb-1, so the issuer first waits for P V(kb-1), which read
 // P(kb-1) from it.
 // Online softmax with a lazily moved reference: P = 2^((s - m) log2(e)/sqrt(hd)) uses the row's
-// reference m, which moves to the block maximum only when that maximum exceeds m by more than
-// 8 / (log2(e)/sqrt(hd)) (so P <= 2^8 in fp16). Only then is the row of O in TMEM (and the row
-// sum l) scaled by 2^((m_old - m_new) ...), after the previous block's P V has completed; O / l is
-// the same softmax whatever the reference, and most blocks need no correction.
+// reference m, which is set to the block maximum on the row's first block and moves again only
+// when a block's P sum against the current reference would exceed 2^12 (so P <= 2^12 in fp16);
+// the block is then recomputed, and the row of O in TMEM (and the row sum l) is scaled by
+// 2^((m_old - m_new) log2(e)/sqrt(hd)) after the previous block's P V has completed. O / l is the
+// same softmax whatever the reference, and most blocks need neither a maximum nor a correction.
 // Key blocks are 64-aligned and visited in order 0, 1, ...; a block whose keys all lie past a
 // row's position leaves that row's state exactly unchanged (no move, P = 0). A decode step
 // (one query row per window, keys from the cache) therefore reproduces the prefill row bit for
@@ -35,7 +36,7 @@ namespace attn {
 
 constexpr int BQ = 128, BKV = 64;
 constexpr int kThreads = 224;  // K TMA warp, MMA warp, 4 softmax warps, V TMA warp
-constexpr float kLazyLog2 = 8.f;  // reference moves when the block max exceeds it by 2^8 in P
+constexpr float kMaxBlockSum = 4096.f;  // the reference moves when a block's P sum would exceed 2^12
 
 template <int HD>
 struct Shape {
@@ -359,7 +360,6 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
     const float c = p.scale_log2;
-    const float lazy = kLazyLog2 / c;  // the move threshold in score units
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int kb = 0; kb < nkb; kb++) {
@@ -367,7 +367,9 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / 3) & 1u, p.err)))) break;
       tc_fence_after();
       float s[64];
-      {
+      // S row of this block into s[], causally masked (only on blocks that reach past the tile's
+      // first position)
+      auto load_s = [&]() {
         uint32_t a[32], b[32];
         tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64, a);
         tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64 + 32, b);
@@ -377,61 +379,74 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
           s[j] = __uint_as_float(a[j]);
           s[32 + j] = __uint_as_float(b[j]);
         }
-      }
-      // causal mask, only on blocks that reach past the tile's first position
-      if ((int)(kb * BKV + BKV - 1) > pos0_i) {
+        if ((int)(kb * BKV + BKV - 1) > pos0_i) {
 #pragma unroll
-        for (int j = 0; j < 64; j++)
-          if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
-      }
-      float mx4[4];
-#pragma unroll
-      for (int i = 0; i < 4; i++) mx4[i] = s[i];
-#pragma unroll
-      for (int j = 4; j < 64; j += 2) mx4[(j >> 1) & 3] = fmax3(mx4[(j >> 1) & 3], s[j], s[j + 1]);
-      const float mx = fmaxf(fmax3(mx4[0], mx4[1], mx4[2]), mx4[3]);
-      // move the reference only for a large rise (always on the first block: m = -inf)
-      const bool move = mx > m + lazy;
-      float corr = 1.f;
-      if (move) {
-        corr = ex2_approx((m - mx) * c);  // 0 on the first block
-        l *= corr;
-        m = mx;
-      }
-      if (kb > 0 && __any_sync(0xffffffffu, move)) {
-        // scale this warp's rows of O (factor 1 for rows that did not move) once the previous
-        // block's P V has landed in TMEM (its barrier is read by parity: P V(kb-3) has completed,
-        // as S(kb) has)
-        const int pst = (kb - 1) & 1;
-        if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(pst), (uint32_t)((kb - 1) >> 1) & 1u, p.err)))) break;
-        tc_fence_after();
-#pragma unroll 1
-        for (int cc = 0; cc < HD / 32; cc++) {
-          uint32_t o[32];
-          tmem_ld32_nowait(tmem + tl + S::TMEM_O + cc * 32, o);
-          tmem_wait();
-#pragma unroll
-          for (int j = 0; j < 32; j++) o[j] = __float_as_uint(__uint_as_float(o[j]) * corr);
-          tmem_st32(tmem + tl + S::TMEM_O + cc * 32, o);
+          for (int j = 0; j < 64; j++)
+            if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
         }
-        tmem_st_wait();
-      }
-      const float nb = (m == -INFINITY) ? 0.f : -m * c;
-      const uint64_t c2 = f2pack(c, c), nb2 = f2pack(nb, nb);
-      uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
+      };
+      // s[j] <- 2^((s[j] - m) c) in place; returns the block's sum (fixed order)
+      auto exp_block = [&]() -> float {
+        const float nb = -m * c;
+        const uint64_t c2 = f2pack(c, c), nb2 = f2pack(nb, nb);
+        uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
 #pragma unroll
-      for (int j = 0; j < 64; j += 2) {
-        float t0, t1;
-        f2unpack(ffma2(f2pack(s[j], s[j + 1]), c2, nb2), t0, t1);
-        s[j] = ex2_approx(t0);
-        s[j + 1] = ex2_approx(t1);
-        if ((j >> 1) & 1) acc1 = fadd2(acc1, f2pack(s[j], s[j + 1]));
-        else acc0 = fadd2(acc0, f2pack(s[j], s[j + 1]));
+        for (int j = 0; j < 64; j += 2) {
+          float t0, t1;
+          f2unpack(ffma2(f2pack(s[j], s[j + 1]), c2, nb2), t0, t1);
+          s[j] = ex2_approx(t0);
+          s[j + 1] = ex2_approx(t1);
+          if ((j >> 1) & 1) acc1 = fadd2(acc1, f2pack(s[j], s[j + 1]));
+          else acc0 = fadd2(acc0, f2pack(s[j], s[j + 1]));
+        }
+        float a0, a1, a2, a3;
+        f2unpack(acc0, a0, a1);
+        f2unpack(acc1, a2, a3);
+        return (a0 + a1) + (a2 + a3);
+      };
+      load_s();
+      // Common case: P against the current reference. The reference moves (to the block
+      // maximum) on a row's first block and whenever the block's P sum would exceed 2^12 (or is
+      // not finite); the block is then recomputed. A warp takes that path if any of its rows
+      // needs it, and its other rows recompute the same values.
+      float bsum = 0.f;
+      if (kb > 0) bsum = exp_block();
+      const bool move = kb == 0 || !(bsum <= kMaxBlockSum);
+      if (__any_sync(0xffffffffu, move)) {
+        if (kb > 0) load_s();
+        float corr = 1.f;
+        if (move) {
+          float mx4[4];
+#pragma unroll
+          for (int i = 0; i < 4; i++) mx4[i] = s[i];
+#pragma unroll
+          for (int j = 4; j < 64; j += 2) mx4[(j >> 1) & 3] = fmax3(mx4[(j >> 1) & 3], s[j], s[j + 1]);
+          const float mx = fmaxf(fmax3(mx4[0], mx4[1], mx4[2]), mx4[3]);  // finite: key 0 is unmasked
+          corr = kb == 0 ? 0.f : ex2_approx((m - mx) * c);
+          l *= corr;
+          m = mx;
+        }
+        if (kb > 0) {
+          // scale this warp's rows of O (factor 1 for rows that did not move) once the previous
+          // block's P V has landed in TMEM (its barrier is read by parity: P V(kb-3) has
+          // completed, as S(kb) has)
+          const int pst = (kb - 1) & 1;
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(pst), (uint32_t)((kb - 1) >> 1) & 1u, p.err)))) break;
+          tc_fence_after();
+#pragma unroll 1
+          for (int cc = 0; cc < HD / 32; cc++) {
+            uint32_t o[32];
+            tmem_ld32_nowait(tmem + tl + S::TMEM_O + cc * 32, o);
+            tmem_wait();
+#pragma unroll
+            for (int j = 0; j < 32; j++) o[j] = __float_as_uint(__uint_as_float(o[j]) * corr);
+            tmem_st32(tmem + tl + S::TMEM_O + cc * 32, o);
+          }
+          tmem_st_wait();
+        }
+        bsum = exp_block();
       }
-      float a0, a1, a2, a3;
-      f2unpack(acc0, a0, a1);
-      f2unpack(acc1, a2, a3);
-      l += (a0 + a1) + (a2 + a3);
+      l += bsum;
       // P as fp16 pairs over the first 32 columns of this block's S buffer (already read)
       {
         uint32_t pw[32];
