@@ -23,11 +23,14 @@ def gpu_logits(ctx, tok, first, n_win):
     return L.lmgc_lm_probs(ctx, d, first, n_win).cpu().numpy()
 
 
-def compare(cfg, tok, wins, n_pos, batch=None):
+def compare(cfg, tok, wins, n_pos, batch=None, scale_tol=False):
+    """Max-abs logit error against the oracle within TOL; with scale_tol the bound grows with the
+    logits' magnitude, TOL * max(1, max|logit| / 4): fp16 activations carry a relative error, and
+    the 5e-2 bound was set for the bench models, whose logits stay below 4."""
     ctx = L.Context(configs.with_(cfg, batch_windows=batch or len(wins)))
     oc = oracle_config(cfg, n_threads=cpu_threads())
     W = cfg.window
-    worst = 0.0
+    worst, tol = 0.0, TOL[cfg.dtype]
     for w in wins:
         g = gpu_logits(ctx, tok, w, 1)[0]
         seg = tok[w * W: (w + 1) * W]
@@ -35,9 +38,11 @@ def compare(cfg, tok, wins, n_pos, batch=None):
         ref = O.window_logits(oc, seg, n)
         err = np.abs(g[:n].astype(np.float64) - ref).max()
         worst = max(worst, err)
+        if scale_tol:
+            tol = max(tol, TOL[cfg.dtype] * np.abs(ref).max() / 4)
         assert np.all(np.isfinite(g[:n]))
     ctx.close()
-    assert worst <= TOL[cfg.dtype], worst
+    assert worst <= tol, (worst, tol)
     return worst
 
 
@@ -56,6 +61,30 @@ def test_small_bf16_ragged(hd, nkv):
     rng = np.random.default_rng(hd)
     tok = tokens(rng, 130 * 3 + 41)
     compare(cfg, tok, [0, 2, 3], 130, batch=2)
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_peaky_attention_reference_moves(hd):
+    """Large weights (init_std 0.25): attention scores spread over tens of units of log2, so
+    a row's softmax reference has to move on many key blocks after the first (the block P sum
+    would pass 2^12). Six key blocks per window (330 = 5*64 + 10); logits against the oracle
+    (magnitude-scaled bound: the logits reach 19), and an encode / KV-cached decode round trip
+    that needs prefill and decode to agree bit for bit through those moves."""
+    cfg = L.ModelConfig(n_layers=2, d_model=256, n_heads=256 // hd, n_kv_heads=2, d_ffn=384, vocab=300,
+                        dtype=L.BF16, window=330, cdf_bits=16, init_std=0.25)
+    rng = np.random.default_rng(300 + hd)
+    tok = tokens(rng, 330 * 2 + 17)
+    compare(cfg, tok, [0, 2], 330, batch=2, scale_tol=True)
+    ctx = L.Context(configs.with_(cfg, batch_windows=2))
+    from paper_2409_17836_gb300 import inputs as I
+    vals = I.tiny_gradient(hd)[:100]  # 900 tokens: windows of 330, 330 and 240
+    d = torch.from_numpy(vals.view(np.int32).copy()).cuda()
+    buf = L.lmgc_encode(ctx, d)
+    out = L.lmgc_decode(ctx, buf, [0, 1, 2]).cpu().numpy().view(np.uint16)
+    ref = O.serialize(vals, 0)
+    flat = np.concatenate([out[0], out[1], out[2, : ref.size - 660]])
+    assert np.array_equal(flat, ref)
+    ctx.close()
 
 
 def test_tinyllama_width_one_layer():
