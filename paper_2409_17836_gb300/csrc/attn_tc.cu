@@ -1,12 +1,17 @@
 // attn_tc.cu -- causal softmax attention of the LM prior (Eq. 2's Llama decoder) on the
 // 5th-generation tensor cores, fp16 inputs and probabilities, fp32 softmax and accumulation.
 //
-// One CTA per (128 query rows, query head, window); 224 threads:
-//   warp 0      TMA: the Q tile once, then 64-key K blocks into a 3-stage ring
-//   warp 6      TMA: 64-key V blocks into a 2-stage ring
+// One CTA per (128 query rows, query head, window); 256 threads:
+//   warp 0      TMA: the Q tile once, then 64-key K blocks into a 3-stage ring (a stage is reused
+//               once the S that read it is done)
+//   warp 6      TMA: 64-key V blocks into a 2-stage ring (reused once its P V is done)
 //   warp 1      TMEM allocation; one lane issues S = Q K^T (M 128, N 64) two blocks ahead into a
-//               3-deep ring in TMEM, and O += P V (M 128, N hd, V as an MN-major operand; O stays
-//               in TMEM for the whole key loop), and commits to mbarriers
+//               3-deep ring in TMEM and commits to the S-done barriers
+//   warp 7      one lane issues O += P V (M 128, N hd, V as an MN-major operand; O stays in TMEM
+//               for the whole key loop) and commits to the P V-done barriers
+// Issuing an MMA, committing and waiting on a barrier each cost tens to a hundred cycles in the
+// issuing thread; with small N (64) the two MMA streams are split over two warps so that neither
+// chain, rather than the tensor core or the softmax, sets the pace.
 //   warps 2-5   softmax: thread i owns query row i (TMEM lane i), so row max and row sum are
 //               per-thread loops; P is written as fp16 pairs back into the first 32 columns of
 //               the block's own S buffer in TMEM, and the P V MMA reads its A operand from there.
@@ -35,7 +40,7 @@ namespace lmgc {
 namespace attn {
 
 constexpr int BQ = 128, BKV = 64;
-constexpr int kThreads = 224;  // K TMA warp, MMA warp, 4 softmax warps, V TMA warp
+constexpr int kThreads = 256;  // K TMA warp, S-MMA warp, 4 softmax warps, V TMA warp, PV-MMA warp
 constexpr float kMaxBlockSum = 4096.f;  // the reference moves when a block's P sum would exceed 2^12
 
 template <int HD>
@@ -213,16 +218,13 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (sv + S::KSV * S::V_BYTES - sq));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   // barriers: 0 Q loaded | 1-3 S ready | 4-6 P written (128 arrivals) | 7-8 P V done (by the
-  //           parity of the block) | 9-11 K stage loaded | 12-14 K stage free | 15-16 V stage
-  //           loaded | 17-18 V stage free
+  //           parity of the block) | 9-11 K stage loaded | 15-16 V stage loaded
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
   auto b_p = [&](int i) { return smem_u32(bars + 4 + i); };
   auto b_pv = [&](int i) { return smem_u32(bars + 7 + i); };
   auto b_kfull = [&](int i) { return smem_u32(bars + 9 + i); };
-  auto b_kempty = [&](int i) { return smem_u32(bars + 12 + i); };
   auto b_vfull = [&](int i) { return smem_u32(bars + 15 + i); };
-  auto b_vempty = [&](int i) { return smem_u32(bars + 17 + i); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;
@@ -239,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int kv_row0 = (int)(w * p.W);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);
+    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);  // 12-14, 17-18 unused
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -263,8 +265,11 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     }
     __syncwarp();
     for (int kb = 0; kb < nkb; kb++) {
-      const int ks = kb % S::KSK;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kempty(ks), ((uint32_t)(kb / S::KSK) & 1u) ^ 1u, p.err))) break;
+      const int ks = kb % S::KSK;  // == kb % 3, the S buffer index of block kb
+      // stage free once S(kb - 3), which read it, is done
+      if (kb >= S::KSK &&
+          !__all_sync(0xffffffffu, mbar_wait(b_s(ks), (uint32_t)((kb - S::KSK) / 3) & 1u, p.err)))
+        break;
       if (lane == 0) {
         mbar_expect_tx(b_kfull(ks), S::K_BYTES);
 #pragma unroll
@@ -277,8 +282,11 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   } else if (warp == 6) {
     // ---------------- TMA producer: V blocks ----------------
     for (int kb = 0; kb < nkb; kb++) {
-      const int vs = kb % S::KSV;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_vempty(vs), ((uint32_t)(kb / S::KSV) & 1u) ^ 1u, p.err))) break;
+      const int vs = kb % S::KSV;  // == kb & 1, the P V-done barrier index of block kb
+      // stage free once P V(kb - 2), which read it, is done
+      if (kb >= S::KSV &&
+          !__all_sync(0xffffffffu, mbar_wait(b_pv(vs), (uint32_t)((kb - S::KSV) >> 1) & 1u, p.err)))
+        break;
       if (lane == 0) {
         mbar_expect_tx(b_vfull(vs), S::V_BYTES);
 #pragma unroll
@@ -289,11 +297,15 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
       __syncwarp();
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer: S(kb+2) is issued before P V(kb), so the softmax of block kb
-    // never waits for the other rows' P(kb-1); a K stage is released as soon as its S is done ----------------
-    auto issue_s = [&](int kb) -> bool {
+    // ---------------- S issuer: S(kb) = Q K(kb)^T two blocks ahead of the softmax ----------------
+    bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
+    for (int kb = 0; kb < nkb && ok; kb++) {
       const int ks = kb % S::KSK, sb = kb % 3;
-      if (!__all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KSK) & 1u, p.err))) return false;
+      // S(kb) overwrites the buffer from which P V(kb-3) read P(kb-3)
+      if (kb >= 3 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv((kb - 3) & 1), (uint32_t)((kb - 3) >> 1) & 1u,
+                                                              p.err))))
+        break;
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KSK) & 1u, p.err)))) break;
       tc_fence_after();
       if (lane == 0) {
         const uint32_t kbase = sk + ks * S::K_BYTES;
@@ -305,23 +317,14 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
                  desc_kmajor(kbase + c * S::KV_CHUNK + o), S::IDESC_S, k > 0 ? 1u : 0u);
         }
         tc_commit(b_s(sb));
-        tc_commit(b_kempty(ks));
       }
       __syncwarp();
-      return true;
-    };
-    bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
-    if (ok) ok = issue_s(0);
-    if (ok && nkb > 1) ok = issue_s(1);
+    }
+  } else if (warp == 7) {
+    // ---------------- P V issuer ----------------
+    bool ok = true;
     for (int kb = 0; kb < nkb && ok; kb++) {
       const int sb = kb % 3, vs = kb % S::KSV;
-      if (kb + 2 < nkb) {
-        // S(kb+2) overwrites the buffer from which P V(kb-1) read P(kb-1)
-        if (kb >= 1 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv((kb - 1) & 1), (uint32_t)((kb - 1) >> 1) & 1u,
-                                                                p.err))))
-          break;
-        if (!(ok = issue_s(kb + 2))) break;
-      }
       ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(vs), (uint32_t)(kb / S::KSV) & 1u, p.err));
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(sb), (uint32_t)(kb / 3) & 1u, p.err));
       if (!ok) break;
@@ -335,7 +338,6 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
           tc_mma_ts(tmem + S::TMEM_O, tmem + S::TMEM_S + sb * 64 + 8 * k, desc_mnmajor(vbase + k * 2048, S::KV_CHUNK),
                     S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
         tc_commit(b_pv(kb & 1));
-        tc_commit(b_vempty(vs));
       }
       __syncwarp();
     }
