@@ -8,8 +8,9 @@
 // stages rows [128 r, 128 r + 128) of the tile's A block and rows [128 r, 128 r + 128) of its B
 // block (the N dimension), so each SM reads 8 KiB of operands per MMA instead of 12, and holds
 // its own 128 output rows in its tensor memory.
-//   warp 0      TMA producer (both CTAs): 128x64 A and 128x64 B tiles (128-byte swizzle) into a
-//               6-stage ring; both CTAs' copies complete on the leader CTA's full barrier
+//   warp 0      TMA producer (both CTAs): 128x64 A and 128x64 B tiles (128-byte swizzle), two
+//               per operand and stage in a 3-stage ring (one in 6 stages for the fp32 logits);
+//               both CTAs' copies complete on the leader CTA's full barrier
 //   warp 1      both CTAs allocate 512 TMEM columns together; in the leader one lane issues the
 //               MMAs and multicasts its commits to both CTAs' empty and accumulator-full barriers
 //   warps 2..   epilogue (both CTAs): 4 warps (8 for the fp32 logits, whose stores dominate): warp
@@ -39,18 +40,23 @@ namespace lmgc {
 namespace tc {
 
 constexpr int BM = 128;  // rows per CTA; a pair covers 2 BM = 256 rows of a tile
-constexpr int BN = 256, BK = 64, STAGES = 6;
+constexpr int BN = 256, BK = 64;
 constexpr int TM = 2 * BM;  // tile rows
 // epilogue warps per epilogue kind, and the CTA size
 template <int EPI>
 struct EpiShape {
+  // k depth of a ring stage in 64-wide (128-byte swizzle) atoms, and stages: two atoms (8 MMAs
+  // per barrier wait and commit, which cost the MMA warp about as much as the MMAs themselves)
+  // in 3 stages; the fp32 logits keep one atom in 6 stages (their 8 epilogue warps and
+  // streamed weights do better with a finer ring)
+  static constexpr int kSub = EPI == kStoreF32 ? 1 : 2;
+  static constexpr int kStages = EPI == kStoreF32 ? 6 : 3;
   static constexpr int kWarps = EPI == kStoreF32 ? 8 : 4;
   static constexpr int kThreads = 64 + 32 * kWarps;
   static constexpr uint32_t kStgBytes = kWarps == 8 ? 8 * 32 * 32 * 4 : 4 * 32 * 36 * 4;
 };
-constexpr uint32_t A_BYTES = BM * BK * 2;        // 16 KiB
-constexpr uint32_t B_BYTES = (BN / 2) * BK * 2;  // 16 KiB: this CTA's half of the B tile
-constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t A_SUB = BM * BK * 2;        // 16 KiB per k atom
+constexpr uint32_t B_SUB = (BN / 2) * BK * 2;  // 16 KiB per k atom: this CTA's half of the B tile
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 // tile order: groups of group_m M-blocks (256 rows each), N-blocks swept inside a group (M
 // fastest). A weight operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy
@@ -67,7 +73,8 @@ __device__ __forceinline__ int stg_off(int r, int j) {
 }
 template <int EPI>
 constexpr size_t smem_bytes() {
-  return (size_t)STAGES * STAGE_BYTES + 256 + EpiShape<EPI>::kStgBytes + 1024;
+  return (size_t)EpiShape<EPI>::kStages * EpiShape<EPI>::kSub * (A_SUB + B_SUB) + 256 + EpiShape<EPI>::kStgBytes +
+         1024;
 }
 
 // instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A and B f16 (bits 7-9, 10-12 = 0),
@@ -97,9 +104,19 @@ __device__ __forceinline__ uint64_t gtimer() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+// non-blocking probe of a phase: cheaper than try_wait when the phase has already completed
+__device__ __forceinline__ bool mbar_test(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 // Bounded wait for the phase with the given parity; false (and kErrLimit) after ~2 s.
 __device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
-  if (mbar_try(a, parity)) return true;
+  if (mbar_test(a, parity) || mbar_try(a, parity)) return true;
   const uint64_t t0 = gtimer();
   for (uint32_t i = 1; i < (1u << 28); ++i) {
     if (mbar_try(a, parity)) return true;
@@ -282,6 +299,8 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
 template <int EPI>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThreads, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tma_a, const __grid_constant__ CUtensorMap tma_b, Params p) {
+  constexpr int STAGES = EpiShape<EPI>::kStages, KSUB = EpiShape<EPI>::kSub;
+  constexpr uint32_t A_BYTES = KSUB * A_SUB, STAGE_BYTES = KSUB * (A_SUB + B_SUB);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
@@ -345,9 +364,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
         if (lane == 0) {
           const uint32_t lf = cluster_addr(full(s), 0);
           if (leader) mbar_expect_tx(full(s), 2 * STAGE_BYTES);
-          tma_load_pair(sA(s), &tma_a, lf, kb * BK, mb * TM + a_row);
-          if (p.keep_b) tma_load_pair_hint(sB(s), &tma_b, lf, kb * BK, nb * BN + b_row, keep_b);
-          else tma_load_pair(sB(s), &tma_b, lf, kb * BK, nb * BN + b_row);
+#pragma unroll
+          for (int u = 0; u < KSUB; u++) {
+            const int kx = (kb * KSUB + u) * BK;
+            tma_load_pair(sA(s) + u * A_SUB, &tma_a, lf, kx, mb * TM + a_row);
+            if (p.keep_b) tma_load_pair_hint(sB(s) + u * B_SUB, &tma_b, lf, kx, nb * BN + b_row, keep_b);
+            else tma_load_pair(sB(s) + u * B_SUB, &tma_b, lf, kx, nb * BN + b_row);
+          }
         }
         __syncwarp();
       }
@@ -371,10 +394,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
         if (!ok) break;
         tc_fence_after();
         if (lane == 0) {
-          const uint64_t da = sw128_desc(sA(s)), db = sw128_desc(sB(s));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            tc_mma(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), (kb > 0 || k > 0) ? 1u : 0u);
+          for (int u = 0; u < KSUB; ++u) {
+            const uint64_t da = sw128_desc(sA(s) + u * A_SUB), db = sw128_desc(sB(s) + u * B_SUB);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              tc_mma(d, da + (uint64_t)(2 * k), db + (uint64_t)(2 * k), (kb > 0 || u > 0 || k > 0) ? 1u : 0u);
+          }
           tc_commit_pair(empty(s));
         }
         __syncwarp();
@@ -656,7 +682,8 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.K = K;
   p.tiles_m = (int)((M + TM - 1) / TM);
   p.tiles_n = (int)((N + BN - 1) / BN);
-  p.num_kb = (int)((K + BK - 1) / BK);
+  const int ksub = epi == kStoreF32 ? EpiShape<kStoreF32>::kSub : EpiShape<kStore>::kSub;
+  p.num_kb = (int)((K + ksub * BK - 1) / (ksub * BK));  // ring stages along K
   p.keep_b = N * K * 2 <= kKeepBBytes ? 1 : 0;
   p.group_m = p.keep_b ? 8 : 32;
   p.err = err;
