@@ -59,9 +59,9 @@ constexpr uint32_t A_SUB = BM * BK * 2;        // 16 KiB per k atom
 constexpr uint32_t B_SUB = (BN / 2) * BK * 2;  // 16 KiB per k atom: this CTA's half of the B tile
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 // tile order: groups of group_m M-blocks (256 rows each), N-blocks swept inside a group (M
-// fastest). A weight operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy
-// and groups are 8 M-blocks; a larger one (the vocabulary projection) streams instead, with
-// groups of 32 M-blocks so that it is re-read only once per 8192 rows.
+// fastest). A weight operand that fits in L2 (<= kKeepBBytes) is read with an evict-last policy;
+// groups are 8 M-blocks for narrow GEMMs and 32 (8192 rows) for wide ones and for a weight that
+// streams (the vocabulary projection), which is then read once per 8192 rows.
 constexpr int64_t kKeepBBytes = 48ll << 20;
 // fp32 epilogue staging: per epilogue warp 32 rows x 32 fp32 columns, laid out so that both the
 // row-per-thread writes and the row-per-8-lanes reads take 4 wavefronts per 512 B: with 4 warps a
@@ -685,7 +685,9 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   const int ksub = epi == kStoreF32 ? EpiShape<kStoreF32>::kSub : EpiShape<kStore>::kSub;
   p.num_kb = (int)((K + ksub * BK - 1) / (ksub * BK));  // ring stages along K
   p.keep_b = N * K * 2 <= kKeepBBytes ? 1 : 0;
-  p.group_m = p.keep_b ? 8 : 32;
+  // wide GEMMs (many N tiles) sweep the weight fewer times with 32 pair tiles per group; narrow
+  // ones keep 8 so that a wave of 76 pairs spans whole groups
+  p.group_m = (p.keep_b && p.tiles_n < 16) ? 8 : 32;
   p.err = err;
   p.rope_cs = rope ? rope->cs : nullptr;
   p.rope_cols = rope ? rope->cols : 0;
