@@ -30,7 +30,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "raw gradient MB/s encoded (1 GB300); LM tensor-pipe % of bf16 peak; coder HBM GB/s"
-WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama")
+WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama", "laplace-tinyllama")
 
 
 def peaks():
@@ -108,6 +108,8 @@ def workload(name: str):
         return configs.TINYLLAMA_LOSSY, inputs.lossy_codes(inputs.convnet_gradient(0))
     if name == "tiny":
         return configs.TINY, inputs.tiny_gradient(0)
+    if name == "laplace-tinyllama":  # 64M-value Laplace mixture; window batch set by --batch-windows
+        return configs.TINYLLAMA, inputs.laplace_gradient()
     raise ValueError(name)
 
 
