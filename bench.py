@@ -113,6 +113,48 @@ def workload(name: str):
     raise ValueError(name)
 
 
+def run_full(args, cfg, ctx, vals):
+    """One lmgc_encode of the whole workload (inputs resident on the device), timed with CUDA
+    events; then the first, middle and last windows are decoded (KV-cached) and compared with the
+    serialised input tokens."""
+    import numpy as np
+    import torch
+
+    import oracle as O
+    from paper_2409_17836_gb300 import lmgc as L
+
+    d = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()
+    out = torch.empty(L.lmgc_encode_bound(ctx, vals.size), dtype=torch.uint8, device="cuda")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with Clocks(torch.cuda.current_device()) as clk:
+        e0.record()
+        buf = L.lmgc_encode(ctx, d, out)
+        e1.record()
+        torch.cuda.synchronize()
+    sec = e0.elapsed_time(e1) / 1e3
+    W = cfg.window
+    n_tok = vals.size * ctx.tpv
+    n_win = -(-n_tok // W)
+    ids = [0, n_win // 2, n_win - 1]
+    toks = L.lmgc_decode(ctx, buf, ids).cpu().numpy().view(np.uint16)
+    ok = True
+    for i, w in enumerate(ids):
+        n = min(W, n_tok - w * W)
+        v0, v1 = (w * W) // ctx.tpv, -(-min(n_tok, (w + 1) * W) // ctx.tpv)
+        ref = O.serialize(vals[v0:v1], cfg.sep_mode)[w * W - v0 * ctx.tpv:][:n]
+        ok = ok and bool(np.array_equal(toks[i, :n], ref))
+    bpv = 4 if vals.dtype == np.float32 else 1
+    print(json.dumps({"mode": "full", "workload": args.workload, "values": int(vals.size), "windows": int(n_win),
+                      "batch_windows": cfg.batch_windows, "seconds": sec,
+                      "value": vals.size * bpv / sec / 1e6, "unit": "MB/s",
+                      "container_bytes": int(buf.numel()),
+                      "compression_rate_pct": 100.0 * buf.numel() / (vals.size * bpv),
+                      "decoded_windows": ids, "decoded_match": ok, "clocks": clk.summary()}), flush=True)
+    ctx.close()
+    return 0 if ok else 1
+
+
 def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
     """Oracle encode of the first `positions` tokens of window `win` (model + CDF + coder)."""
     import numpy as np
@@ -256,6 +298,9 @@ def main():
     ap.add_argument("--cpu-target-s", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-micro", action="store_true")
+    # encode the whole workload once (every window, in batches of --batch-windows), then decode
+    # the first, middle and last windows and check them; prints one JSON line of its own
+    ap.add_argument("--full", action="store_true")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -283,6 +328,8 @@ def main():
         cfg = configs.with_(cfg, n_layers=args.layers)
     ctx = L.Context(cfg)
     tpv = ctx.tpv
+    if args.full:
+        return run_full(args, cfg, ctx, vals)
     per_step = (cfg.batch_windows * cfg.window) // tpv  # values filling one model batch
     n_slices = max(1, vals.size // per_step)
     dev = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()
