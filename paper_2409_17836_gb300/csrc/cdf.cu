@@ -54,8 +54,10 @@ __device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t*
   const float C = (float)(65536.0 * 1.4426950408889634073599246810019);
   const float y = __fmul_rn(__fsub_rn(z, m), C);  // <= 0: m is the row maximum
   // a = -rint(y) (ties to even), capped at 40 * 2^16: y is clamped to -40 * 2^16 (an integer, so
-  // rint keeps it) before the conversion, which also keeps huge logit gaps from overflowing it
-  const int a = -__float2int_rn(fmaxf(y, -(float)kAMax));
+  // rint keeps it), and rint is taken by adding 1.5 * 2^23 in round-to-nearest-even: the sum lies
+  // in [2^23, 2^24), where fp32 spacing is 1, so its low mantissa bits are 2^22 + rint(y)
+  const float t = __fadd_rn(fmaxf(y, -(float)kAMax), 12582912.f);
+  const int a = (int)(0x4B400000u - __float_as_uint(t));
   // H, L <= 2^31, so (H L + 2^30) >> 31 <= 2^31 fits 32 bits; the final shift by a >> 16 (<= 40)
   // uses shr.b32, which yields 0 for shifts of 32 or more
   const uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
@@ -193,8 +195,13 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
     }
     const float* z = logits + r * (int64_t)V;
     RowStats st = row_stats(z, V, P, H, L, redf, redu);
+    // The remainder (T - V) - sum g goes to the argmax: it moves the symbol's start only when the
+    // argmax lies below the symbol and its freq only when it is the symbol, so the pass over the
+    // whole row that sums g is taken only then (block-uniform).
+    const bool need_resid = st.amax <= sym;
     uint64_t gall = 0;
-    for (int j = threadIdx.x; j < V; j += kCdfThreads) gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
+    if (need_resid)
+      for (int j = threadIdx.x; j < V; j += kCdfThreads) gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
     // g below the coded symbol and g of the symbol: only j <= sym, packed as (below << 32) + at
     // (each part < 2^31)
     uint64_t packed = 0;
@@ -202,7 +209,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
       const uint64_t g = gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
       packed += j < sym ? (g << 32) : g;
     }
-    gall = block_sum_u64(gall, redu);
+    if (need_resid) gall = block_sum_u64(gall, redu);
     packed = block_sum_u64(packed, redu);
     const uint64_t gbelow = packed >> 32, gsym = packed & 0xFFFFFFFFull;
     if (threadIdx.x == 0) {
