@@ -175,7 +175,7 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
     return dt, min(positions, seg.size)
 
 
-def microbenchmarks(L, ctx, pk, reps: int = 3) -> dict:
+def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> dict:
     """HBM-bound stages at sizes where bandwidth, not launch latency, decides: the serialiser on
     the 64M-value Laplace mixture, and the coder alone on 2^18 windows x 2048 tokens of seeded
     random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most likely)."""
@@ -201,14 +201,14 @@ def microbenchmarks(L, ctx, pk, reps: int = 3) -> dict:
     out["serialize"] = {"values": d.numel(), "ms": ms, "bytes": nbytes, "achieved": nbytes / ms / 1e6,
                         "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
     del d, tok
-    V, P, W, n_win = 32000, 24, 2048, 1 << 18
+    V, P, W, n_win = 32000, 24, 2048, coder_windows
     g = torch.Generator(device="cuda").manual_seed(5)
     z = torch.randn(256, V, generator=g, device="cuda") * torch.linspace(0.3, 6.0, 256, device="cuda")[:, None]
     cdf = L.lmgc_quantize_cdf(ctx, z).long()
     likely = torch.argmax(cdf[:, 1:] - cdf[:, :-1], dim=1)
     start = torch.empty((W, n_win), dtype=torch.int32, device="cuda")  # position-major
     freq = torch.empty_like(start)
-    step = 1 << 15
+    step = min(n_win, 1 << 15)
     for w0 in range(0, n_win, step):
         row = torch.randint(0, 256, (W, step), generator=g, device="cuda")
         sym = torch.randint(0, V, (W, step), generator=g, device="cuda")
@@ -301,6 +301,10 @@ def main():
     # encode the whole workload once (every window, in batches of --batch-windows), then decode
     # the first, middle and last windows and check them; prints one JSON line of its own
     ap.add_argument("--full", action="store_true")
+    # only the serialise and coder microbenchmarks (one JSON line), the coder on this many windows
+    # of 2048 tokens (small profiler captures use 2^16)
+    ap.add_argument("--micro-only", action="store_true")
+    ap.add_argument("--coder-windows", type=int, default=1 << 18)
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -330,6 +334,11 @@ def main():
     tpv = ctx.tpv
     if args.full:
         return run_full(args, cfg, ctx, vals)
+    if args.micro_only:
+        print(json.dumps({"mode": "micro", "microbench": microbenchmarks(L, ctx, peaks(), coder_windows=args.coder_windows)}),
+              flush=True)
+        ctx.close()
+        return 0
     per_step = (cfg.batch_windows * cfg.window) // tpv  # values filling one model batch
     n_slices = max(1, vals.size // per_step)
     dev = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()

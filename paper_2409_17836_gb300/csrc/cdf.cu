@@ -49,15 +49,21 @@ void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s) {
 constexpr int kCdfThreads = 512;
 constexpr int kAMax = 40 * 65536;
 
-__device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t* __restrict__ H,
-                                               const uint32_t* __restrict__ L) {
+// a = -rint(fp32(fp32(z - m) * C)) capped at 40 * 2^16: 2^(-a / 2^16) approximates exp(z - m).
+// a = 0 exactly where e reaches its maximum 2^31, so the row's lowest-index argmax of e is its
+// lowest index with a = 0.
+__device__ __forceinline__ int exp2_code(float z, float m) {
   const float C = (float)(65536.0 * 1.4426950408889634073599246810019);
   const float y = __fmul_rn(__fsub_rn(z, m), C);  // <= 0: m is the row maximum
-  // a = -rint(y) (ties to even), capped at 40 * 2^16: y is clamped to -40 * 2^16 (an integer, so
-  // rint keeps it), and rint is taken by adding 1.5 * 2^23 in round-to-nearest-even: the sum lies
-  // in [2^23, 2^24), where fp32 spacing is 1, so its low mantissa bits are 2^22 + rint(y)
+  // rint (ties to even) after clamping y to -40 * 2^16 (an integer, so rint keeps it), taken by
+  // adding 1.5 * 2^23 in round-to-nearest-even: the sum lies in [2^23, 2^24), where fp32 spacing
+  // is 1, so its low mantissa bits are 2^22 + rint(y)
   const float t = __fadd_rn(fmaxf(y, -(float)kAMax), 12582912.f);
-  const int a = (int)(0x4B400000u - __float_as_uint(t));
+  return (int)(0x4B400000u - __float_as_uint(t));
+}
+
+__device__ __forceinline__ uint32_t exp2_from_code(int a, const uint32_t* __restrict__ H,
+                                                   const uint32_t* __restrict__ L) {
   // H, L <= 2^31, so (H L + 2^30) >> 31 <= 2^31 fits 32 bits; the final shift by a >> 16 (<= 40)
   // uses shr.b32, which yields 0 for shifts of 32 or more
   const uint64_t hl = (uint64_t)H[(a >> 8) & 255] * (uint64_t)L[a & 255];
@@ -65,6 +71,11 @@ __device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t*
   uint32_t e;
   asm("shr.b32 %0, %1, %2;" : "=r"(e) : "r"(e31), "r"(a >> 16));
   return e;
+}
+
+__device__ __forceinline__ uint32_t exp2_fixed(float z, float m, const uint32_t* __restrict__ H,
+                                               const uint32_t* __restrict__ L) {
+  return exp2_from_code(exp2_code(z, m), H, L);
 }
 
 template <typename V>
@@ -98,24 +109,17 @@ __device__ __forceinline__ uint64_t block_sum_u64(uint64_t v, uint64_t* red) {
   return warp_sum(v);
 }
 
-// (value, index) max with the lowest index among equal values; packed as value << 32 | ~index
-__device__ __forceinline__ uint64_t block_argmax(uint64_t key, uint64_t* red) {
+__device__ __forceinline__ int block_min_int(int v, int* red) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    uint64_t k2 = __shfl_xor_sync(0xffffffffu, key, o);
-    key = k2 > key ? k2 : key;
-  }
+  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   __syncthreads();
-  if (lane == 0) red[w] = key;
+  if (lane == 0) red[w] = v;
   __syncthreads();
-  key = lane < (kCdfThreads / 32) ? red[lane] : 0ull;
+  v = lane < (kCdfThreads / 32) ? red[lane] : 0x7fffffff;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    uint64_t k2 = __shfl_xor_sync(0xffffffffu, key, o);
-    key = k2 > key ? k2 : key;
-  }
-  return key;
+  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
 }
 
 struct RowStats {
@@ -134,32 +138,70 @@ __device__ __forceinline__ uint64_t gfloor(uint32_t e, const RowStats& st) {
   return q;
 }
 
+// Rows whose start is 16-byte aligned and whose length is a multiple of 4 are read as float4.
+__device__ __forceinline__ bool row_vec4(const float* z, int V) {
+  return (V & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0;
+}
+
 // Passes 1 and 2 over a row: max, sum of e, lowest-index argmax of e.
 __device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V, int P, const uint32_t* H,
                                               const uint32_t* L, float* redf, uint64_t* redu) {
   RowStats st;
+  const bool vec = row_vec4(z, V);  // block-uniform
+  const float4* z4 = reinterpret_cast<const float4*>(z);
+  const int V4 = V >> 2;
   float m = -INFINITY;
-  for (int j = threadIdx.x; j < V; j += kCdfThreads) m = fmaxf(m, __ldg(z + j));
+  if (vec) {
+    for (int j = threadIdx.x; j < V4; j += kCdfThreads) {
+      const float4 v = __ldg(z4 + j);
+      m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
+    }
+  } else {
+    for (int j = threadIdx.x; j < V; j += kCdfThreads) m = fmaxf(m, __ldg(z + j));
+  }
   m = block_max(m, redf);
   uint64_t S = 0;
-  uint32_t best_e = 0;
-  int best_j = 0x7fffffff;
-  for (int j = threadIdx.x; j < V; j += kCdfThreads) {  // j increases: strict > keeps the lowest index
-    const uint32_t e = exp2_fixed(__ldg(z + j), m, H, L);
-    S += e;
-    if (e > best_e) {
-      best_e = e;
-      best_j = j;
+  int best_j = 0x7fffffff;  // a thread's indices increase, so its first a = 0 is its lowest
+  if (vec) {
+    for (int j = threadIdx.x; j < V4; j += kCdfThreads) {
+      const float4 v = __ldg(z4 + j);
+      const int a0 = exp2_code(v.x, m), a1 = exp2_code(v.y, m), a2 = exp2_code(v.z, m), a3 = exp2_code(v.w, m);
+      S += (uint64_t)exp2_from_code(a0, H, L) + (uint64_t)exp2_from_code(a1, H, L) +
+           (uint64_t)exp2_from_code(a2, H, L) + (uint64_t)exp2_from_code(a3, H, L);
+      if (min(min(a0, a1), min(a2, a3)) == 0 && best_j == 0x7fffffff)
+        best_j = 4 * j + (a0 == 0 ? 0 : a1 == 0 ? 1 : a2 == 0 ? 2 : 3);
+    }
+  } else {
+    for (int j = threadIdx.x; j < V; j += kCdfThreads) {
+      const int a = exp2_code(__ldg(z + j), m);
+      S += exp2_from_code(a, H, L);
+      if (a == 0 && best_j == 0x7fffffff) best_j = j;
     }
   }
   S = block_sum_u64(S, redu);
-  const uint64_t best = block_argmax(((uint64_t)best_e << 32) | (uint32_t)(~(uint32_t)best_j), redu);
   st.m = m;
   st.S = S;
   st.Mq = (1ull << P) - (uint64_t)V;
   st.F = (uint32_t)((st.Mq << 32) / S);
-  st.amax = (int)(~(uint32_t)(best & 0xFFFFFFFFu));
+  st.amax = block_min_int(best_j, reinterpret_cast<int*>(redu));
   return st;
+}
+
+// sum of g = floor(e (T - V) / S) over the row (this thread's part)
+__device__ __forceinline__ uint64_t row_gsum(const float* __restrict__ z, int V, const RowStats& st,
+                                             const uint32_t* H, const uint32_t* L) {
+  uint64_t gall = 0;
+  if (row_vec4(z, V)) {
+    const float4* z4 = reinterpret_cast<const float4*>(z);
+    for (int j = threadIdx.x; j < (V >> 2); j += kCdfThreads) {
+      const float4 v = __ldg(z4 + j);
+      gall += gfloor(exp2_fixed(v.x, st.m, H, L), st) + gfloor(exp2_fixed(v.y, st.m, H, L), st) +
+              gfloor(exp2_fixed(v.z, st.m, H, L), st) + gfloor(exp2_fixed(v.w, st.m, H, L), st);
+    }
+  } else {
+    for (int j = threadIdx.x; j < V; j += kCdfThreads) gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
+  }
+  return gall;
 }
 
 // mode 0: row r codes d_sym[r]; pair index r.
@@ -199,9 +241,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
     // argmax lies below the symbol and its freq only when it is the symbol, so the pass over the
     // whole row that sums g is taken only then (block-uniform).
     const bool need_resid = st.amax <= sym;
-    uint64_t gall = 0;
-    if (need_resid)
-      for (int j = threadIdx.x; j < V; j += kCdfThreads) gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
+    uint64_t gall = need_resid ? row_gsum(z, V, st, H, L) : 0ull;
     // g below the coded symbol and g of the symbol: only j <= sym, packed as (below << 32) + at
     // (each part < 2^31)
     uint64_t packed = 0;
@@ -274,10 +314,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_quantize_cdf(const float* __res
     const float* z = logits + r * (int64_t)V;
     uint32_t* c = cdf + r * (int64_t)(V + 1);
     RowStats st = row_stats(z, V, P, H, L, redf, redu);
-    uint64_t gall = 0;
-    for (int j = threadIdx.x; j < V; j += kCdfThreads)
-      gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
-    gall = block_sum_u64(gall, redu);
+    const uint64_t gall = block_sum_u64(row_gsum(z, V, st, H, L), redu);
     const uint64_t resid = st.Mq - gall;
     uint64_t run = 0;
     if (threadIdx.x == 0) c[0] = 0;
@@ -372,10 +409,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_dec_search(const float* __restr
   const uint64_t t = s.D / r;
   const float* z = logits + w * (int64_t)V;
   RowStats st = row_stats(z, V, P, H, L, redf, redu);
-  uint64_t gall = 0;
-  for (int j = threadIdx.x; j < V; j += kCdfThreads)
-    gall += gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
-  gall = block_sum_u64(gall, redu);
+  const uint64_t gall = block_sum_u64(row_gsum(z, V, st, H, L), redu);
   const uint64_t resid = st.Mq - gall;
   if (threadIdx.x == 0) found_s = -1;
   uint64_t run = 0;
