@@ -7,11 +7,12 @@
 // R >= 2^61), most significant bit first.
 //
 // The range R depends only on the freq sequence; L is the only unbounded quantity. A thread keeps
-// the low 62 bits of L in a register; the bits shifted above them are emitted into a 64-bit
-// accumulator and leave in 32-bit words to the stream's own scratch slot. A carry out of the
-// low 62 bits increments the emitted bits: in the accumulator, or -- when the accumulator was all
-// ones -- in the already written words of this stream's slot (never beyond word 0: L + R stays
-// below 2^(B+62)). The carry walk is bounded by the slot length.
+// the low 62 bits of L in a register (as 4 L, so that the carry out of them is the carry out of
+// a 64-bit add); the bits shifted above them collect in a 32-bit pending word and leave in 32-bit
+// words to the stream's own scratch slot. A carry out of the low 62 bits increments the emitted
+// bits: the pending ones, or -- when they were all ones -- the already written words of this
+// stream's slot (never beyond word 0: L + R stays below 2^(B+62)). The carry walk is bounded by
+// the slot length. All shifts are 32-bit funnel shifts by less than 32 (k <= P <= 30 per token).
 //
 // Layout: one stream per thread, 32 windows per warp. Pairs are read at
 // start[w*stride_win + i*stride_pos]; with the encode path's position-major layout
@@ -32,18 +33,36 @@ size_t slot_bytes(size_t win_tokens, int P) {
 
 __device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
 
-struct Emitter {
-  uint32_t* slot;   // stream words (stored big-endian so the bytes are in stream order)
-  uint32_t wpos;    // words written
-  uint32_t max_words;
-  uint64_t acc;     // pending emitted bits, right-aligned
-  int nacc;         // number of pending bits (< 32 after each flush)
+// 64-bit add with the carry out of bit 63
+__device__ __forceinline__ uint64_t add_carry(uint64_t a, uint64_t b, uint32_t& c) {
+  uint32_t lo, hi;
+  asm("add.cc.u32 %0, %3, %5;\n\taddc.cc.u32 %1, %4, %6;\n\taddc.u32 %2, 0, 0;"
+      : "=r"(lo), "=r"(hi), "=r"(c)
+      : "r"((uint32_t)a), "r"((uint32_t)(a >> 32)), "r"((uint32_t)b), "r"((uint32_t)(b >> 32)));
+  return ((uint64_t)hi << 32) | lo;
+}
+
+// One stream's coder state in 32-bit pieces. L is held as L4 = 4 L (its 62 bits at the top of a
+// 64-bit word, so a carry out of bit 62 of L is the carry out of the 64-bit add); the emitted bits
+// not yet written form `acc` (nacc < 32 bits, right-aligned). Every shift is a 32-bit (funnel)
+// shift by less than 32: k <= P <= 30 bits move per token.
+struct Coder {
+  uint32_t R_hi, R_lo;
+  uint64_t L4;
+  uint32_t acc, nacc, wpos, max_words;
+  uint32_t* slot;  // stream words, big-endian
   bool overflow;
 
+  __device__ __forceinline__ void write(uint32_t wv) {
+    if (wpos < max_words) slot[wpos] = bswap32(wv);
+    else overflow = true;
+    wpos++;
+  }
+  // +1 into the emitted bits: the pending ones, else (all ones) the written words
   __device__ __forceinline__ void carry() {
-    acc += 1;
-    if ((acc >> nacc) != 0) {  // pending bits were all ones: carry into written words
-      acc = 0;
+    acc += 1u;
+    if ((acc >> nacc) != 0u) {
+      acc = 0u;
       int64_t i = (int64_t)wpos - 1;
       for (; i >= 0; --i) {
         uint32_t v = bswap32(slot[i]) + 1u;
@@ -53,20 +72,48 @@ struct Emitter {
       if (i < 0) overflow = true;  // impossible for valid input; reported, not propagated
     }
   }
-  __device__ __forceinline__ void put(uint64_t bits, int k) {  // append k (<= 32) bits
-    acc = (acc << k) | bits;
+  // move the top k (< 32) bits of L4 to the pending bits; L4 and R shift left by k
+  __device__ __forceinline__ void shift_out(uint32_t k) {
+    const uint32_t l_hi = (uint32_t)(L4 >> 32), l_lo = (uint32_t)L4;
+    const uint32_t a_hi = __funnelshift_l(acc, 0u, k);            // acc >> (32 - k), 0 for k = 0
+    const uint32_t a_lo = (acc << k) | __funnelshift_l(l_hi, 0u, k);
+    L4 = ((uint64_t)__funnelshift_l(l_lo, l_hi, k) << 32) | (l_lo << k);
+    R_hi = __funnelshift_l(R_lo, R_hi, k);
+    R_lo <<= k;
     nacc += k;
-    if (nacc >= 32) {
-      uint32_t w = (uint32_t)(acc >> (nacc - 32));
-      if (wpos < max_words) slot[wpos] = bswap32(w);
-      else overflow = true;
-      wpos++;
-      nacc -= 32;
-      acc &= (nacc > 0) ? ((1ull << nacc) - 1ull) : 0ull;
+    if (nacc >= 32u) {
+      nacc -= 32u;
+      write(__funnelshift_r(a_lo, a_hi, nacc));  // the top 32 of the nacc + 32 pending bits
+      acc = a_lo & ((1u << nacc) - 1u);
+    } else {
+      acc = a_lo;  // a_hi = 0: fewer than 32 bits pending
     }
   }
 };
 
+// Per token (s = start, f = freq, T = 2^P): r = R >> P; L4 += 4 r s (carry -> emitted bits);
+// R = r f; k = max(0, clz(R) - 2); shift_out(k). R >= 2^(61 - P) after the multiply, so for
+// P <= 29 its high word is nonzero (HI32: a 32-bit count of leading zeros).
+template <bool HI32>
+__device__ __forceinline__ void code_token(Coder& c, uint32_t s, uint32_t f, int P, uint32_t T, bool& bad) {
+  // 0 < f <= T and s + f <= T; an invalid pair stops the stream after its group (the arithmetic
+  // stays bounded meanwhile: writes are slot-checked and the carry walk stops at word 0)
+  bad |= (f - 1u >= T) | (s > T - f);
+  const uint32_t r_lo = __funnelshift_r(c.R_lo, c.R_hi, (uint32_t)P), r_hi = c.R_hi >> P;
+  const uint64_t r = ((uint64_t)r_hi << 32) | r_lo;
+  uint32_t cy;
+  c.L4 = add_carry(c.L4, r * (uint64_t)(s << 2), cy);  // r s < 2^62, so 4 r s < 2^64
+  if (cy) c.carry();
+  const uint64_t Rn = r * (uint64_t)f;
+  c.R_hi = (uint32_t)(Rn >> 32);
+  c.R_lo = (uint32_t)Rn;
+  int k = (HI32 ? __clz((int)c.R_hi) : __clzll((long long)Rn)) - 2;
+  k = max(k, 0);                // R = 2^62 (f = T) needs no shift
+  if (!HI32) k = min(k, 31);    // only an invalid f = 0 reaches past P
+  c.shift_out((uint32_t)k);
+}
+
+template <bool HI32>
 __global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict__ start,
                                                       const uint32_t* __restrict__ freq, int P, int64_t n_win,
                                                       int64_t win_tokens, const uint32_t* __restrict__ win_len,
@@ -75,76 +122,70 @@ __global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict
   const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (w >= n_win) return;
   const int64_t n = win_len ? (int64_t)win_len[w] : win_tokens;
-  const uint64_t mask62 = (1ull << 62) - 1ull;
-  const uint64_t T = 1ull << P;
-  Emitter em;
-  em.slot = reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz);
-  em.wpos = 0;
-  em.max_words = (uint32_t)(slot_sz / 4);
-  em.acc = 0;
-  em.nacc = 0;
-  em.overflow = false;
-  uint64_t R = 1ull << 62, L = 0, B = 0;
+  const uint32_t T = 1u << P;
+  Coder c;
+  c.R_hi = 1u << 30;  // R = 2^62
+  c.R_lo = 0u;
+  c.L4 = 0ull;
+  c.acc = 0u;
+  c.nacc = 0u;
+  c.wpos = 0u;
+  c.max_words = (uint32_t)(slot_sz / 4);
+  c.slot = reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz);
+  c.overflow = false;
   bool bad = n > win_tokens;
-  const uint32_t* ps = start + w * stride_win;
-  const uint32_t* pf = freq + w * stride_win;
-  // the pairs of the next kPre tokens are loaded ahead so their latency overlaps the serial chain
+  // the pairs of the next kPre tokens are loaded ahead so their latency overlaps the serial chain;
+  // the load pointers advance by the position stride
   constexpr int kPre = 8;
+  const uint32_t* qs = start + w * stride_win;
+  const uint32_t* qf = freq + w * stride_win;
   uint32_t bs[kPre], bf[kPre];
 #pragma unroll
   for (int j = 0; j < kPre; j++) {
-    bs[j] = j < n ? __ldcs(ps + j * stride_pos) : 0u;
-    bf[j] = j < n ? __ldcs(pf + j * stride_pos) : 1u;
+    bs[j] = j < n ? __ldcs(qs) : 0u;
+    bf[j] = j < n ? __ldcs(qf) : 1u;
+    qs += stride_pos;
+    qf += stride_pos;
   }
   for (int64_t i0 = 0; i0 < n && !bad; i0 += kPre) {
     uint32_t cs[kPre], cf[kPre];
+    const bool full_next = i0 + 2 * kPre <= n;
 #pragma unroll
     for (int j = 0; j < kPre; j++) {
       cs[j] = bs[j];
       cf[j] = bf[j];
-      const int64_t nx = i0 + kPre + j;
-      bs[j] = nx < n ? __ldcs(ps + nx * stride_pos) : 0u;
-      bf[j] = nx < n ? __ldcs(pf + nx * stride_pos) : 1u;
+      if (full_next || i0 + kPre + j < n) {
+        bs[j] = __ldcs(qs);
+        bf[j] = __ldcs(qf);
+      } else {
+        bs[j] = 0u;
+        bf[j] = 1u;
+      }
+      qs += stride_pos;
+      qf += stride_pos;
     }
+    if (i0 + kPre <= n) {
 #pragma unroll
-  for (int j = 0; j < kPre; j++) {
-    if (i0 + j >= n) break;
-    const uint64_t s = cs[j];
-    const uint64_t f = cf[j];
-    if (f == 0 || s + f > T) {
-      bad = true;
-      break;
+      for (int j = 0; j < kPre; j++) code_token<HI32>(c, cs[j], cf[j], P, T, bad);
+    } else {
+      const int jn = (int)(n - i0);
+#pragma unroll
+      for (int j = 0; j < kPre; j++)
+        if (j < jn) code_token<HI32>(c, cs[j], cf[j], P, T, bad);
     }
-    const uint64_t r = R >> P;
-    L += r * s;  // < 2^63
-    if (L >> 62) {
-      L &= mask62;
-      em.carry();
-    }
-    R = r * f;
-    const int k = __clzll((long long)R) - 2;  // 62 - bitlen(R) >= 0 since R < 2^62
-    if (k > 0) {
-      em.put(L >> (62 - k), k);
-      L = (L << k) & mask62;
-      R <<= k;
-      B += (uint64_t)k;
-    }
-  }
   }
   // termination: v = ceil(L / 2^60) * 2^60; emit its top 2 bits of the low 62
-  L += (1ull << 60) - 1ull;
-  if (L >> 62) {
-    L &= mask62;
-    em.carry();
+  {
+    uint32_t cy;
+    c.L4 = add_carry(c.L4, ((1ull << 60) - 1ull) << 2, cy);
+    if (cy) c.carry();
   }
-  em.put(L >> 60, 2);
-  if (em.nacc > 0) {
-    uint32_t wv = (uint32_t)(em.acc << (32 - em.nacc));
-    if (em.wpos < em.max_words) em.slot[em.wpos] = bswap32(wv);
-    else em.overflow = true;
-  }
-  bitlen[w] = (uint32_t)(B + 2);
-  if (bad || em.overflow) atomicOr(err, kErrCorrupt);
+  c.shift_out(2u);
+  // every emitted bit went through the pending bits: B + 2 bits in all
+  const uint64_t nbits = (uint64_t)c.wpos * 32u + c.nacc;
+  if (c.nacc > 0u) c.write(c.acc << (32u - c.nacc));
+  bitlen[w] = (uint32_t)nbits;
+  if (bad || c.overflow) atomicOr(err, kErrCorrupt);
 }
 
 void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
@@ -152,8 +193,14 @@ void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int
                          size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
   if (n_win <= 0) return;
   note_launch();
-  k_range_encode<<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
-                                                                  stride_win, stride_pos, slots, slot_sz, bitlen, err);
+  if (P <= 29)
+    k_range_encode<true><<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
+                                                                        stride_win, stride_pos, slots, slot_sz, bitlen,
+                                                                        err);
+  else
+    k_range_encode<false><<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
+                                                                         stride_win, stride_pos, slots, slot_sz, bitlen,
+                                                                         err);
 }
 
 // ------------------------------------------------------------------------------------------
