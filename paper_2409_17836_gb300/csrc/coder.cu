@@ -58,10 +58,10 @@ struct Coder {
     else overflow = true;
     wpos++;
   }
-  // +1 into the emitted bits: the pending ones, else (all ones) the written words
-  __device__ __forceinline__ void carry() {
-    acc += 1u;
-    if ((acc >> nacc) != 0u) {
+  // +cy (0 or 1) into the emitted bits: the pending ones, else (all ones) the written words
+  __device__ __forceinline__ void carry(uint32_t cy) {
+    acc += cy;
+    if ((acc >> nacc) != 0u) {  // only when cy = 1 and the pending bits were all ones
       acc = 0u;
       int64_t i = (int64_t)wpos - 1;
       for (; i >= 0; --i) {
@@ -80,14 +80,15 @@ struct Coder {
     L4 = ((uint64_t)__funnelshift_l(l_lo, l_hi, k) << 32) | (l_lo << k);
     R_hi = __funnelshift_l(R_lo, R_hi, k);
     R_lo <<= k;
-    nacc += k;
-    if (nacc >= 32u) {
-      nacc -= 32u;
-      write(__funnelshift_r(a_lo, a_hi, nacc));  // the top 32 of the nacc + 32 pending bits
-      acc = a_lo & ((1u << nacc) - 1u);
-    } else {
-      acc = a_lo;  // a_hi = 0: fewer than 32 bits pending
-    }
+    // a full word leaves when 32 or more bits are pending (a_hi = 0 otherwise); no branch
+    const bool full = nacc + k >= 32u;
+    nacc = full ? nacc + k - 32u : nacc + k;
+    const uint32_t wv = __funnelshift_r(a_lo, a_hi, nacc);  // the top 32 of the nacc + 32 pending bits
+    const bool in_slot = wpos < max_words;
+    if (full && in_slot) slot[wpos] = bswap32(wv);
+    overflow |= full && !in_slot;
+    wpos += full ? 1u : 0u;
+    acc = full ? (a_lo & ((1u << nacc) - 1u)) : a_lo;
   }
 };
 
@@ -103,7 +104,7 @@ __device__ __forceinline__ void code_token(Coder& c, uint32_t s, uint32_t f, int
   const uint64_t r = ((uint64_t)r_hi << 32) | r_lo;
   uint32_t cy;
   c.L4 = add_carry(c.L4, r * (uint64_t)(s << 2), cy);  // r s < 2^62, so 4 r s < 2^64
-  if (cy) c.carry();
+  c.carry(cy);
   const uint64_t Rn = r * (uint64_t)f;
   c.R_hi = (uint32_t)(Rn >> 32);
   c.R_lo = (uint32_t)Rn;
@@ -178,7 +179,7 @@ __global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict
   {
     uint32_t cy;
     c.L4 = add_carry(c.L4, ((1ull << 60) - 1ull) << 2, cy);
-    if (cy) c.carry();
+    c.carry(cy);
   }
   c.shift_out(2u);
   // every emitted bit went through the pending bits: B + 2 bits in all
