@@ -177,7 +177,16 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
       gemm(ctx, xh, L.wgu, ws.act, rows, 2 * (int64_t)F, d, kSwiGLU, s, nullptr, &consume);
       gemm(ctx, ws.act, L.wdown, ws.x, rows, d, F, kAddResidual, s, nullptr, &produce);
     }
-    gemm(ctx, xh, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s, nullptr, &consume);
+    // a prefill also leaves each logits row's maximum for the CDF kernel (the transposing fp32
+    // epilogue, which takes vocabularies that are multiples of 32, computes it)
+    NormArgs head = consume;
+    const bool with_max = !decode && c.vocab % 32 == 0;
+    if (with_max) {
+      cudaMemsetAsync(ctx->row_max, 0, (size_t)rows * 4, s);
+      head.row_max = ctx->row_max;
+    }
+    gemm(ctx, xh, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s, nullptr, &head);
+    ctx->row_max_valid = with_max;
     return;
   }
   for (int l = 0; l < c.n_layers; l++) {
@@ -222,6 +231,7 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
   }
   gemm(ctx, ws.n, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s);
+  ctx->row_max_valid = false;
 }
 
 // x = E[tok_in] for `rows` rows (and, on the fused-RMSNorm path, fp16(x) and its sums of squares)
@@ -311,7 +321,7 @@ lmgc_status lmgc_destroy(lmgc_ctx* ctx) {
   if (!ctx) return LMGC_OK;
   cudaDeviceSynchronize();
   void* ptrs[] = {ctx->weights_blob, ctx->rope_cs, ctx->exp2_tab, ctx->ws.x, ctx->ws.n, ctx->ws.qkv, ctx->ws.att,
-                  ctx->ws.act, ctx->ws.gu, ctx->ws.ss, ctx->ws.tok_in, ctx->logits, ctx->d_err, ctx->tok, ctx->pair_start,
+                  ctx->ws.act, ctx->ws.gu, ctx->ws.ss, ctx->ws.tok_in, ctx->logits, ctx->row_max, ctx->d_err, ctx->tok, ctx->pair_start,
                   ctx->win_len, ctx->host_in, ctx->host_out, ctx->kv_cache};
   for (void* p : ptrs)
     if (p) cudaFree(p);
@@ -441,6 +451,7 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (err == cudaSuccess && ctx->fused_norm) err = dmalloc(&ws.ss, R * (size_t)(d / 256) * 4);
   if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
   if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
+  if (err == cudaSuccess) err = dmalloc(&ctx->row_max, R * 4);
   for (int i = 0; i < 6 && err == cudaSuccess; i++) err = cudaEventCreate(&ctx->ev[i]);
   if (err == cudaSuccess) err = cudaDeviceSynchronize();
   if (err == cudaSuccess) err = cudaGetLastError();
@@ -633,7 +644,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
       const int64_t rows = nb * W;
       ProfScope ps(ctx, kCdf, (double)rows * ((double)c.vocab * 4 + 2 + 8), s);
       launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
-                       ctx->pair_start, ctx->pair_freq, 1, s, w_begin);
+                       ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
     }
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
   }

@@ -143,15 +143,19 @@ __device__ __forceinline__ bool row_vec4(const float* z, int V) {
   return (V & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0;
 }
 
-// Passes 1 and 2 over a row: max, sum of e, lowest-index argmax of e.
+// Passes 1 and 2 over a row: max, sum of e, lowest-index argmax of e. With mkey (the float_key
+// of the row's maximum, from the vocabulary GEMM's epilogue) the max pass is skipped.
 __device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V, int P, const uint32_t* H,
-                                              const uint32_t* L, float* redf, uint64_t* redu) {
+                                              const uint32_t* L, float* redf, uint64_t* redu,
+                                              const uint32_t* mkey = nullptr) {
   RowStats st;
   const bool vec = row_vec4(z, V);  // block-uniform
   const float4* z4 = reinterpret_cast<const float4*>(z);
   const int V4 = V >> 2;
   float m = -INFINITY;
-  if (vec) {
+  if (mkey) {
+    m = __uint_as_float(key_float_bits(*mkey));
+  } else if (vec) {
     for (int j = threadIdx.x; j < V4; j += kCdfThreads) {
       const float4 v = __ldg(z4 + j);
       m = fmaxf(m, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
@@ -159,7 +163,7 @@ __device__ __forceinline__ RowStats row_stats(const float* __restrict__ z, int V
   } else {
     for (int j = threadIdx.x; j < V; j += kCdfThreads) m = fmaxf(m, __ldg(z + j));
   }
-  m = block_max(m, redf);
+  if (!mkey) m = block_max(m, redf);
   uint64_t S = 0;
   int best_j = 0x7fffffff;  // a thread's indices increase, so its first a = 0 is its lowest
   if (vec) {
@@ -212,7 +216,8 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
                                                            const uint16_t* __restrict__ tok, int64_t n_tok, int W,
                                                            int64_t first_win, int64_t stride_pos,
                                                            uint32_t* __restrict__ start, uint32_t* __restrict__ freq,
-                                                           int mode, int64_t pair_win0) {
+                                                           int mode, int64_t pair_win0,
+                                                           const uint32_t* __restrict__ row_max) {
   __shared__ uint32_t H[256], L[256];
   __shared__ float redf[32];
   __shared__ uint64_t redu[32];
@@ -236,7 +241,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
       out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
     }
     const float* z = logits + r * (int64_t)V;
-    RowStats st = row_stats(z, V, P, H, L, redf, redu);
+    RowStats st = row_stats(z, V, P, H, L, redf, redu, row_max ? row_max + r : nullptr);
     // The remainder (T - V) - sum g goes to the argmax: it moves the symbol's start only when the
     // argmax lies below the symbol and its freq only when it is the symbol, so the pass over the
     // whole row that sums g is taken only then (block-uniform).
@@ -262,12 +267,12 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs(const float* __restri
 
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
                       int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0) {
+                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0, const uint32_t* row_max) {
   if (rows <= 0) return;
   unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
   note_launch();
   k_cdf_pairs<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win, pair_stride_pos,
-                                             start, freq, mode, pair_win0);
+                                             start, freq, mode, pair_win0, row_max);
 }
 
 // Block inclusive scan of one u64 per thread; returns the inclusive prefix; *total the tile sum.

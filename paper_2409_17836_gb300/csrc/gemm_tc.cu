@@ -220,6 +220,8 @@ struct Params {
   // kAddResidual: also write fp16(x) to xh and the tile's sum of squares to ss_out[m * tiles_n + nb]
   __half* xh;
   float* ss_out;
+  // kStoreF32: row_max[m] = max over the launch of float_key(C[m][n]) (atomic; zeroed beforehand)
+  uint32_t* row_max;
 };
 
 __device__ __forceinline__ float row_scale(const Params& p, int64_t m) {
@@ -514,6 +516,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
         // butterfly over the row's 8 lanes).
         const int cr = lane >> 3, sl = lane & 7, cc = sl * 4;
         const int64_t row0 = mrow0 + q * 32;
+        float rmax = -INFINITY;  // kStoreF32: this thread's row (m) over its columns
         float ssl[8];
 #pragma unroll
         for (int k = 0; k < 8; k++) ssl[k] = 0.f;
@@ -526,6 +529,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
           if (p.row_ss) {
 #pragma unroll
             for (int j = 0; j < 32; j++) r[j] = __float_as_uint(__uint_as_float(r[j]) * rs);
+          }
+          if (EPI == kStoreF32 && p.row_max) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) rmax = fmaxf(rmax, fmaxf(__uint_as_float(r[j]), __uint_as_float(r[j + 1])));
           }
 #pragma unroll
           for (int j = 0; j < 8; j++)
@@ -567,6 +574,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
           }
           __syncwarp();
         }
+        if (EPI == kStoreF32 && p.row_max && m < p.M && rmax != -INFINITY)
+          atomicMax(p.row_max + m, float_key(__float_as_uint(rmax)));
         if (EPI == kAddResidual && p.xh) {
 #pragma unroll
           for (int k = 0; k < 8; k++) {
@@ -700,6 +709,7 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   p.ss_eps = norm ? norm->eps : 0.f;
   p.xh = norm ? norm->xh : nullptr;
   p.ss_out = norm ? norm->ss_out : nullptr;
+  p.row_max = norm ? norm->row_max : nullptr;
   const int tiles = p.tiles_m * p.tiles_n;
   const int grid = 2 * std::max(1, std::min(tiles, g_max_clusters[epi]));  // CTA pairs
   note_launch();

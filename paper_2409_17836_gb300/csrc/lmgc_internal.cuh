@@ -73,6 +73,10 @@ struct lmgc_ctx {
   uint32_t* exp2_tab = nullptr;  // [512]: H then L
   lmgc::Workspace ws;
   float* logits = nullptr;     // [rows][V]
+  // [rows]: order-preserving key of each logits row's maximum, written by the vocabulary GEMM of
+  // a prefill (row_max_valid) and read by the CDF kernel in place of its max pass
+  uint32_t* row_max = nullptr;
+  bool row_max_valid = false;
   uint32_t* d_err = nullptr;   // device error word
   // encode staging
   uint16_t* tok = nullptr;
@@ -152,7 +156,16 @@ struct NormArgs {
   float inv_d, eps;
   __half* xh;
   float* ss_out;
+  uint32_t* row_max = nullptr;  // kStoreF32: atomic max of float_key(row values); zeroed by the caller
 };
+// Order-preserving map of fp32 (not NaN) to u32: a < b  <=>  float_key(a) < float_key(b); 0 is
+// below every key, so a zeroed buffer is the identity of the max.
+__host__ __device__ __forceinline__ uint32_t float_key(uint32_t bits) {
+  return (bits & 0x80000000u) ? ~bits : (bits | 0x80000000u);
+}
+__host__ __device__ __forceinline__ uint32_t key_float_bits(uint32_t key) {
+  return (key & 0x80000000u) ? (key & 0x7fffffffu) : ~key;
+}
 struct RopeArgs {
   const float2* cs;  // [W][hd/2] (cos, sin)
   int cols;          // columns [0, cols) are rotated: (n_heads + n_kv_heads) * hd
@@ -174,9 +187,11 @@ void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t ds
 // cdf.cu
 void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s);  // builds H and L on the host
 // mode 1: pair index i * pair_stride_pos + (window - pair_win0)
+// row_max (optional): float_key of each row's maximum, which replaces the kernel's max pass
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
                       int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0 = 0);
+                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0 = 0,
+                      const uint32_t* row_max = nullptr);
 void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
                          cudaStream_t s);
 void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,

@@ -66,6 +66,30 @@ def test_tiny_pairs_and_codes_given_gpu_logits():
     ctx.close()
 
 
+def test_tinyllama_shape_pairs_and_codes_given_gpu_logits():
+    """The tensor-core path (bf16, vocab 32000, P = 24, RMSNorm in the GEMMs, each row's maximum
+    taken in the vocabulary GEMM's epilogue): every window's code of lmgc_encode is bit-exact with
+    the oracle's CDF pairs and coder applied to the GPU's own logits of the same windows. One
+    layer keeps it short; three windows, the last partial, in two batches."""
+    cfg = configs.with_(configs.TINYLLAMA, n_layers=1, batch_windows=2)
+    ctx = L.Context(cfg)
+    W = cfg.window
+    vals = I.convnet_gradient(0)[: (2 * W + 700) // 9]
+    tok = O.serialize(vals, 0)
+    n_win = -(-tok.size // W)
+    assert n_win == 3
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    dtok = torch.from_numpy(tok.view(np.int16)).cuda()
+    for w in range(n_win):
+        n = min(W, tok.size - w * W)
+        lg = L.lmgc_lm_probs(ctx, dtok, w, 1)[0, :n].cpu().numpy()
+        st, fr = O.cdf_pairs(lg, tok[w * W: w * W + n], cfg.cdf_bits)
+        code, nbits = O.range_encode(st, fr, cfg.cdf_bits)
+        assert h["bitlen"][w] == nbits and buf[h["offsets"][w]: h["offsets"][w + 1]] == code, w
+    ctx.close()
+
+
 @pytest.mark.parametrize("n,sep,kind", [(1, 0, 0), (29, 2, 0), (1000, 4, 0), (777, 0, 1)])
 def test_tiny_edge_sizes_round_trip(n, sep, kind):
     cfg = configs.with_(configs.TINY, sep_mode=sep, input_kind=kind, batch_windows=3)
