@@ -126,7 +126,8 @@ static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M
   if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi))
     launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s, rope, norm);
   else
-    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi, s);  // kSwiGLU never reaches here
+    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi == kAddResidualWide ? (int)kAddResidual : epi,
+                     s);  // kSwiGLU never reaches here
 }
 
 static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, int64_t n_win, int64_t pos_first,
@@ -162,6 +163,8 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     __half* xh = (__half*)ws.n;
     const NormArgs consume{ws.ss, d / 256, 1.0f / (float)d, c.rms_eps, nullptr, nullptr};
     const NormArgs produce{nullptr, 0, 0.f, 0.f, xh, ws.ss};
+    const bool wide_o = qd <= 2048;  // measured: +5% at K = 2048, -2% at K = 4096
+    const NormArgs consume_o{ws.ss, d / 128, 1.0f / (float)d, c.rms_eps, nullptr, nullptr};
     for (int l = 0; l < c.n_layers; l++) {
       const Layer& L = ctx->layers[l];
       RopeArgs ra{ctx->rope_cs, (c.n_heads + c.n_kv_heads) * hd, hd, decode ? 1 : c.window, decode ? pos : 0};
@@ -173,8 +176,11 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
         launch_copy_rows(ws.qkv, ctx->qkv_dim, cache_l, W, pos, n_win, ctx->qkv_dim, c.dtype, s);
         attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s);
       }
-      gemm(ctx, ws.att, L.wo, ws.x, rows, d, qd, kAddResidual, s, nullptr, &produce);
-      gemm(ctx, xh, L.wgu, ws.act, rows, 2 * (int64_t)F, d, kSwiGLU, s, nullptr, &consume);
+      // the O projection (K = qd, a short main loop) takes the 8-warp residual epilogue, whose
+      // sums of squares come in 128-column parts; the choice depends on the shape only, so a
+      // decode makes the same one
+      gemm(ctx, ws.att, L.wo, ws.x, rows, d, qd, wide_o ? kAddResidualWide : kAddResidual, s, nullptr, &produce);
+      gemm(ctx, xh, L.wgu, ws.act, rows, 2 * (int64_t)F, d, kSwiGLU, s, nullptr, wide_o ? &consume_o : &consume);
       gemm(ctx, ws.act, L.wdown, ws.x, rows, d, F, kAddResidual, s, nullptr, &produce);
     }
     // a prefill also leaves each logits row's maximum for the CDF kernel (the transposing fp32
@@ -448,7 +454,7 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (err == cudaSuccess) err = dmalloc(&ws.act, R * F * e);
   if (err == cudaSuccess && !ctx->fused_swiglu) err = dmalloc(&ws.gu, R * 2 * F * e);
   ctx->fused_norm = ctx->fused_norm && ctx->fused_rope && ctx->fused_swiglu;
-  if (err == cudaSuccess && ctx->fused_norm) err = dmalloc(&ws.ss, R * (size_t)(d / 256) * 4);
+  if (err == cudaSuccess && ctx->fused_norm) err = dmalloc(&ws.ss, R * (size_t)(d / 128) * 4);
   if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
   if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
   if (err == cudaSuccess) err = dmalloc(&ctx->row_max, R * 4);
@@ -899,7 +905,8 @@ lmgc_status lmgc_launch_count(uint64_t* n) {
 lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
                       int epi, lmgc_stream stream) {
   if (!ctx || (M && N && (!d_a || !d_b || !d_c))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
-  if (K % 8 || epi < 0 || epi > 3) return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..3");
+  if (K % 8 || epi < 0 || (epi > 3 && epi != kAddResidualWide))
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..3 or 5");
   if (epi == kSwiGLU && !(ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi)))
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epi 3 needs the bf16 tensor-core path and N % 256 == 0");
   cudaStream_t s = (cudaStream_t)stream;

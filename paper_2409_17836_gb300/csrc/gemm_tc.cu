@@ -51,10 +51,11 @@ struct EpiShape {
   // streamed weights do better with a finer ring)
   static constexpr int kSub = EPI == kStoreF32 ? 1 : 2;
   static constexpr int kStages = EPI == kStoreF32 ? 6 : 3;
-  static constexpr int kWarps = EPI == kStoreF32 ? 8 : 4;
+  static constexpr int kWarps = (EPI == kStoreF32 || EPI == kAddResidualWide) ? 8 : 4;
   static constexpr int kThreads = 64 + 32 * kWarps;
   static constexpr uint32_t kStgBytes = kWarps == 8 ? 8 * 32 * 32 * 4 : 4 * 32 * 36 * 4;
 };
+constexpr bool is_resid(int epi) { return epi == kAddResidual || epi == kAddResidualWide; }
 constexpr uint32_t A_SUB = BM * BK * 2;        // 16 KiB per k atom
 constexpr uint32_t B_SUB = (BN / 2) * BK * 2;  // 16 KiB per k atom: this CTA's half of the B tile
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
@@ -217,7 +218,8 @@ struct Params {
   const float* row_ss;
   int ss_parts;
   float ss_inv_d, ss_eps;
-  // kAddResidual: also write fp16(x) to xh and the tile's sum of squares to ss_out[m * tiles_n + nb]
+  // kAddResidual(Wide): also write fp16(x) to xh and the row's sum of squares over each epilogue
+  // warp's columns to ss_out[m * tiles_n * NH + nb * NH + hw] (NH = 1, or 2 for the wide form)
   __half* xh;
   float* ss_out;
   // kStoreF32: row_max[m] = max over the launch of float_key(C[m][n]) (atomic; zeroed beforehand)
@@ -274,7 +276,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
     if (n0 + 32 <= p.N && (p.N & 3) == 0) {
       float4* d = reinterpret_cast<float4*>(c);
       float4 o[8];
-      if (EPI == kAddResidual) {
+      if (is_resid(EPI)) {
 #pragma unroll
         for (int j = 0; j < 8; j++) o[j] = d[j];  // all loads in flight before the first store
       }
@@ -282,7 +284,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
       for (int j = 0; j < 8; j++) {
         float4 v = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]), __uint_as_float(r[4 * j + 2]),
                                __uint_as_float(r[4 * j + 3]));
-        if (EPI == kAddResidual) {
+        if (is_resid(EPI)) {
           v.x += o[j].x;
           v.y += o[j].y;
           v.z += o[j].z;
@@ -293,7 +295,7 @@ __device__ __forceinline__ void store_chunk(const Params& p, int64_t m, int64_t 
     } else {
 #pragma unroll
       for (int j = 0; j < 32; j++)
-        if (n0 + j < p.N) c[j] = (EPI == kAddResidual ? c[j] : 0.f) + __uint_as_float(r[j]);
+        if (n0 + j < p.N) c[j] = (is_resid(EPI) ? c[j] : 0.f) + __uint_as_float(r[j]);
     }
   }
 }
@@ -428,7 +430,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
       const int64_t m = mrow0 + q * 32 + lane;
       const int64_t ncol0 = (int64_t)nb * BN + hw * HN;  // first output column of this half
       // pull this half-tile's residual rows into L2 while its accumulator is still being built
-      if (EPI == kAddResidual && (p.N & 31) == 0) prefetch_residual(p, m, ncol0, HN);
+      if (is_resid(EPI) && (p.N & 31) == 0) prefetch_residual(p, m, ncol0, HN);
       const float rs = row_scale(p, m);
       if (!__all_sync(0xffffffffu, mbar_wait(tfull(a), aph, p.err))) break;
       tc_fence_after();
@@ -507,13 +509,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
             for (int j = 0; j < 4; j++) d4[j] = make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
           }
         }
-      } else if ((EPI == kAddResidual || EPI == kStoreF32) && (p.N & 31) == 0) {
+      } else if ((is_resid(EPI) || EPI == kStoreF32) && (p.N & 31) == 0) {
         // fp32 output through a shared-memory transpose: the warp's 32 rows x 32 columns go in one
         // row per thread and come out as 8 lanes per row, so each global access covers 4 full rows
-        // of 128 B. kAddResidual (4 epilogue warps, so a warp covers the whole tile) adds the stored
-        // x; with xh set it also writes fp16(x), and ss_out[row * tiles_n + nb] receives the row's
-        // sum of squares over the tile's columns (fixed order: per lane over chunks, then a
-        // butterfly over the row's 8 lanes).
+        // of 128 B. The residual forms add the stored x; with xh set they also write fp16(x), and
+        // ss_out[row * tiles_n * NH + nb * NH + hw] receives the row's sum of squares over this
+        // warp's columns of the tile: all of them with 4 epilogue warps, half with 8 (fixed order:
+        // per lane over chunks, then a butterfly over the row's 8 lanes).
         const int cr = lane >> 3, sl = lane & 7, cc = sl * 4;
         const int64_t row0 = mrow0 + q * 32;
         float rmax = -INFINITY;  // kStoreF32: this thread's row (m) over its columns
@@ -542,7 +544,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
           __syncwarp();
           float* cbase = reinterpret_cast<float*>(p.C) + n0 + cc;
           float4 o[8];
-          if (EPI == kAddResidual) {
+          if (is_resid(EPI)) {
 #pragma unroll
             for (int k = 0; k < 8; k++) {
               const int64_t gm = row0 + 4 * k + cr;
@@ -556,7 +558,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
             const int64_t gm = row0 + rr;
             const float4 acc = *reinterpret_cast<const float4*>(stg + stg_off<NH>(rr, sl));
             float4 v = acc;
-            if (EPI == kAddResidual) {
+            if (is_resid(EPI)) {
               v.x = o[k].x + acc.x;
               v.y = o[k].y + acc.y;
               v.z = o[k].z + acc.z;
@@ -564,7 +566,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
             }
             if (gm < p.M) {
               __stcs(reinterpret_cast<float4*>(cbase + gm * p.N), v);
-              if (EPI == kAddResidual && p.xh) {
+              if (is_resid(EPI) && p.xh) {
                 __half2 h0 = __floats2half2_rn(v.x, v.y), h1 = __floats2half2_rn(v.z, v.w);
                 __stcs(reinterpret_cast<uint2*>(p.xh + gm * p.N + n0 + cc),
                        make_uint2(*reinterpret_cast<uint32_t*>(&h0), *reinterpret_cast<uint32_t*>(&h1)));
@@ -576,7 +578,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
         }
         if (EPI == kStoreF32 && p.row_max && m < p.M && rmax != -INFINITY)
           atomicMax(p.row_max + m, float_key(__float_as_uint(rmax)));
-        if (EPI == kAddResidual && p.xh) {
+        if (is_resid(EPI) && p.xh) {
 #pragma unroll
           for (int k = 0; k < 8; k++) {
             float v = ssl[k];
@@ -584,7 +586,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
             v += __shfl_xor_sync(0xffffffffu, v, 2);
             v += __shfl_xor_sync(0xffffffffu, v, 4);
             const int64_t gm = row0 + 4 * k + cr;
-            if ((lane & 7) == 0 && gm < p.M) p.ss_out[gm * p.tiles_n + nb] = v;
+            if ((lane & 7) == 0 && gm < p.M) p.ss_out[gm * (p.tiles_n * NH) + nb * NH + hw] = v;
           }
         }
       } else {
@@ -617,7 +619,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(EpiShape<EPI>::kThre
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 static std::once_flag g_once;
 static int g_num_sms = 0;
-static int g_max_clusters[5] = {0, 0, 0, 0, 0};  // co-resident CTA pairs, per epilogue kind
+static int g_max_clusters[6] = {0, 0, 0, 0, 0, 0};  // co-resident CTA pairs, per epilogue kind
 
 template <int EPI>
 static void setup_kernel() {
@@ -650,6 +652,7 @@ static void init_once() {
   if (!g_encode) return;
   setup_kernel<kStore>();
   setup_kernel<kAddResidual>();
+  setup_kernel<kAddResidualWide>();
   setup_kernel<kStoreF32>();
   setup_kernel<kSwiGLU>();
   setup_kernel<kQKVRope>();
@@ -716,6 +719,9 @@ void launch_gemm_tc(const void* A, const void* B, void* C, int64_t M, int64_t N,
   if (epi == kStore) k_gemm_tc<kStore><<<grid, EpiShape<kStore>::kThreads, smem_bytes<kStore>(), s>>>(ma, mb, p);
   else if (epi == kAddResidual)
     k_gemm_tc<kAddResidual><<<grid, EpiShape<kAddResidual>::kThreads, smem_bytes<kAddResidual>(), s>>>(ma, mb, p);
+  else if (epi == kAddResidualWide)
+    k_gemm_tc<kAddResidualWide>
+        <<<grid, EpiShape<kAddResidualWide>::kThreads, smem_bytes<kAddResidualWide>(), s>>>(ma, mb, p);
   else if (epi == kStoreF32) k_gemm_tc<kStoreF32><<<grid, EpiShape<kStoreF32>::kThreads, smem_bytes<kStoreF32>(), s>>>(ma, mb, p);
   else if (epi == kSwiGLU) k_gemm_tc<kSwiGLU><<<grid, EpiShape<kSwiGLU>::kThreads, smem_bytes<kSwiGLU>(), s>>>(ma, mb, p);
   else k_gemm_tc<kQKVRope><<<grid, EpiShape<kQKVRope>::kThreads, smem_bytes<kQKVRope>(), s>>>(ma, mb, p);

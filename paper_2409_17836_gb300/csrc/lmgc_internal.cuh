@@ -147,7 +147,10 @@ void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, i
 // kSwiGLU: B's rows are gate/up blocks interleaved 128 by 128 (rows 256t..256t+127 = gate rows
 // 128t.., rows 256t+128.. = up rows 128t..); C[m][128t + j] = silu(gate) * up, N/2 columns.
 // kQKVRope: kStore with the rotary embedding applied to the q and k heads (RopeArgs).
-enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3, kQKVRope = 4 };
+// kAddResidualWide: kAddResidual with 8 epilogue warps, each over half of a tile's columns, so
+// its sums of squares come in 128-column parts (for short-K GEMMs whose epilogue would outlast
+// the main loop).
+enum GemmEpi { kStore = 0, kAddResidual = 1, kStoreF32 = 2, kSwiGLU = 3, kQKVRope = 4, kAddResidualWide = 5 };
 // Fused RMSNorm (see gemm_tc.cu Params): consumers read row_ss (parts per row), residual
 // producers write xh and ss_out.
 struct NormArgs {

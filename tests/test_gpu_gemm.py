@@ -38,7 +38,7 @@ def run(ctx, M, N, K, epi, seed=0, scale=1.0):
     af, bf = a.float().numpy(), b.float().numpy()
     ref = O.gemm_nt(af, bf)
     bound = 2.0 ** -19 * O.gemm_nt(np.abs(af), np.abs(bf)) + 1e-30
-    if epi == 1:
+    if epi in (1, 5):
         ref = ref + c0.numpy().astype(np.float64)
         bound += 2.0 ** -23 * np.abs(ref)
     got = c.float().cpu().numpy().astype(np.float64)
@@ -56,6 +56,15 @@ def test_gemm_tc_shapes(ctx_f16, M, N, K, epi):
     if M * N > 2048 * 32000 // 2 and epi != 2:
         pytest.skip("the vocabulary shape is checked with the fp32 epilogue only")
     run(ctx_f16, M, N, K, epi, seed=M + N + K)
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 520, 136), (7, 2560, 2048), (1000, 2048, 2048)])
+def test_gemm_tc_wide_residual_epilogue(ctx_f16, M, N, K):
+    """epi 5 (the residual add through 8 epilogue warps) meets the epi 1 bound and equals epi 1
+    bit for bit: the same products accumulate in the same order, one fp32 add per element."""
+    c5 = run(ctx_f16, M, N, K, 5, seed=M + N + K)
+    c1 = run(ctx_f16, M, N, K, 1, seed=M + N + K)
+    assert torch.equal(c1, c5)
 
 
 def test_gemm_tc_row_invariance(ctx_f16):
