@@ -40,6 +40,9 @@ def lib():
             "orc_tokens_per_value": (i64, [i32, i32]),
             "orc_serialize": (i64, [i32, i32, vp, i64, vp]),
             "orc_deserialize": (i64, [i32, i32, vp, i64, vp]),
+            "orc_serial_tokens": (i64, [i32, i32, i32, i32, i64]),
+            "orc_serialize_grouped": (i64, [i32, i32, i32, i32, vp, i64, vp]),
+            "orc_deserialize_grouped": (i64, [i32, i32, i32, i32, vp, i64, vp]),
             "orc_splitmix64": (u64, [u64]),
             "orc_bf16_round": (f32, [f32]),
             "orc_weight": (f32, [u64, u32, u64, f32, i32]),
@@ -90,23 +93,40 @@ def tokens_per_value(input_kind: int, sep_mode: int) -> int:
     return int(lib().orc_tokens_per_value(input_kind, sep_mode))
 
 
-def serialize(values: np.ndarray, sep_mode: int = 0) -> np.ndarray:
+def serial_tokens(input_kind: int, sep_mode: int, n: int, byte_group: int = 0, byte_order: int = 0) -> int:
+    """Token count of n values (Sec. 3; byte grouping of Sec. 4.3)."""
+    return int(lib().orc_serial_tokens(input_kind, sep_mode, byte_group, byte_order, n))
+
+
+def serialize(values: np.ndarray, sep_mode: int = 0, byte_group: int = 0, byte_order: int = 0) -> np.ndarray:
+    """byte_group 0 and byte_order 0: one group per value, each value's nibbles most significant
+    first (Sec. 3). Otherwise the byte-grouped form (Sec. 4.3 "Byte grouping"): bytes in order
+    (fp32 most or least significant first), two digits each, a separator every byte_group bytes."""
     kind = 0 if values.dtype == np.float32 else 1
     if kind == 1 and values.dtype != np.uint8:
         raise TypeError("values must be float32 or uint8")
     v = np.ascontiguousarray(values)
-    out = np.empty(v.size * tokens_per_value(kind, sep_mode), dtype=np.uint16)
-    n = lib().orc_serialize(kind, sep_mode, _p(v), v.size, _p(out))
+    nt = serial_tokens(kind, sep_mode, v.size, byte_group, byte_order)
+    if nt < 0:
+        raise ValueError("bad serialisation arguments")
+    out = np.empty(max(nt, 1), dtype=np.uint16)
+    if byte_group == 0 and byte_order == 0:
+        n = lib().orc_serialize(kind, sep_mode, _p(v), v.size, _p(out))
+    else:
+        n = lib().orc_serialize_grouped(kind, sep_mode, byte_group, byte_order, _p(v), v.size, _p(out))
     if n < 0:
         raise ValueError("bad serialisation arguments")
     return out[:n]
 
 
-def deserialize(tokens: np.ndarray, input_kind: int, sep_mode: int = 0) -> np.ndarray:
+def deserialize(tokens: np.ndarray, input_kind: int, sep_mode: int = 0, byte_group: int = 0,
+                byte_order: int = 0) -> np.ndarray:
     t = np.ascontiguousarray(tokens, dtype=np.uint16)
-    per = tokens_per_value(input_kind, sep_mode)
-    out = np.empty(max(t.size // per, 1), dtype=np.float32 if input_kind == 0 else np.uint8)
-    n = lib().orc_deserialize(input_kind, sep_mode, _p(t), t.size, _p(out))
+    out = np.empty(max(t.size // 2, 1), dtype=np.float32 if input_kind == 0 else np.uint8)
+    if byte_group == 0 and byte_order == 0:
+        n = lib().orc_deserialize(input_kind, sep_mode, _p(t), t.size, _p(out))
+    else:
+        n = lib().orc_deserialize_grouped(input_kind, sep_mode, byte_group, byte_order, _p(t), t.size, _p(out))
     if n < 0:
         raise ValueError("malformed token stream")
     return out[:n]
@@ -151,6 +171,8 @@ class OracleConfig:
     sep_mode: int = 0
     input_kind: int = 0
     n_threads: int = 1
+    byte_group: int = 0  # bytes per separator group (Sec. 4.3); 0 = one group per value
+    byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
 
     def c(self) -> _Cfg:
         return _Cfg(self.n_layers, self.d_model, self.n_heads, self.n_kv_heads, self.d_ffn, self.vocab,
@@ -324,12 +346,14 @@ def crc32(b: bytes) -> int:
 # ------------------------------------------------------------------------------------------
 # Container (a build choice; the paper stores one code per window without a format).
 #   0  "LMGC"            4  u32 version (2)      8  u64 n_values       16 u64 n_tok
-#   24 u32 window        28 u32 cdf_bits         32 u32 input_kind     36 u32 sep_mode
+#   24 u32 window        28 u32 cdf_bits         32 u32 input_kind     36 u32 serialisation
 #   40 u32 vocab         44 u32 n_win            48 u64 weight_seed    56 u32 model crc
 #   60 u32 crc32 of bytes [0, 60)
 #   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | each window's code, ceil(bitlen/8) bytes, in
 #   window order. crc_tok[w] = crc32 of window w's token ids as little-endian u16 (its own
 #   length: W, or fewer for the last window), so that a decoder can check each window it restores.
+# serialisation = sep_mode | byte_group << 8 | byte_order << 16 (0 in the upper bits: the
+# default one group per value, most significant byte first).
 # model crc = crc32 of '<7i3f' (n_layers, d_model, n_heads, n_kv_heads, d_ffn, vocab, bf16,
 # init_std, rms_eps, rope_theta).
 # ------------------------------------------------------------------------------------------
@@ -353,10 +377,14 @@ def window_crcs(tok: np.ndarray, window: int, first: int = 0, count: int | None 
                     dtype=np.uint32)
 
 
+def serial_word(cfg: OracleConfig) -> int:
+    return cfg.sep_mode | cfg.byte_group << 8 | cfg.byte_order << 16
+
+
 def build_container(cfg: OracleConfig, n_values: int, n_tok: int, codes: list[tuple[bytes, int]],
                     crcs: np.ndarray) -> bytes:
     head = struct.pack("<4sIQQIIIIIIQI", b"LMGC", CONTAINER_VERSION, n_values, n_tok, cfg.window, cfg.cdf_bits,
-                       cfg.input_kind, cfg.sep_mode, cfg.vocab, len(codes), cfg.weight_seed, model_crc(cfg))
+                       cfg.input_kind, serial_word(cfg), cfg.vocab, len(codes), cfg.weight_seed, model_crc(cfg))
     head += struct.pack("<I", crc32(head))
     assert len(head) == HEADER_BYTES and len(crcs) == len(codes)
     table = np.array([bl for _, bl in codes], dtype="<u4").tobytes() + np.asarray(crcs, dtype="<u4").tobytes()
@@ -379,13 +407,13 @@ def parse_container(buf: bytes) -> dict:
     crc_tok = np.frombuffer(buf[64 + 4 * n_win: 64 + 8 * n_win], dtype="<u4").astype(np.uint32)
     offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)]) + 64 + 8 * n_win
     return dict(version=f[1], n_values=f[2], n_tok=f[3], window=f[4], cdf_bits=f[5], input_kind=f[6],
-                sep_mode=f[7], vocab=f[8], n_win=n_win, weight_seed=f[10], model_crc=f[11], bitlen=bl,
+                sep_mode=f[7] & 0xFF, byte_group=(f[7] >> 8) & 0xFF, byte_order=(f[7] >> 16) & 0xFF, vocab=f[8], n_win=n_win, weight_seed=f[10], model_crc=f[11], bitlen=bl,
                 crc_tok=crc_tok, offsets=offs)
 
 
 def encode(cfg: OracleConfig, values: np.ndarray, n_par: int = 1) -> bytes:
     """Full oracle encode of a gradient vector into the container (Sec. 3)."""
-    tok = serialize(values, cfg.sep_mode)
+    tok = serialize(values, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
     W = cfg.window
     n_win = (tok.size + W - 1) // W
     codes = encode_windows(cfg, tok, 0, n_win, n_par)

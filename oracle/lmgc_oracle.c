@@ -107,6 +107,80 @@ int64_t orc_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64
   return n;
 }
 
+/* Byte grouping (Sec. 4.3 "Byte grouping", Fig. 3: bytes per group BPG in {1, 2, 3, 4, 8} and
+ * none). The values' bytes are taken in order -- an fp32 value's four bytes most significant
+ * first (order 0) or least significant first (order 1), a uint8 code as its one byte -- and each
+ * byte becomes two hex digits, high nibble first. The separator follows every `group` bytes and
+ * also the last group when it is partial. group 0 means one group per value, which is
+ * orc_serialize's layout. Returns the token count of n values, or -1 for bad arguments. */
+static int64_t orc_bytes_per_value(int input_kind) { return input_kind == 0 ? 4 : (input_kind == 1 ? 1 : -1); }
+
+int64_t orc_serial_tokens(int input_kind, int sep_mode, int group, int order, int64_t n) {
+  uint16_t sep[2];
+  int ns = orc_sep_tokens(sep_mode, sep);
+  int64_t bv = orc_bytes_per_value(input_kind);
+  if (ns < 0 || bv < 0 || group < 0 || group > 8 || order < 0 || order > 1 || n < 0) return -1;
+  int64_t g = group ? group : bv, nbytes = n * bv;
+  return 2 * nbytes + ns * ((nbytes + g - 1) / g);
+}
+
+/* byte j (0-based, in stream order) of value i */
+static uint32_t orc_value_byte(int input_kind, int order, const void* in, int64_t i, int j) {
+  if (input_kind == 1) return ((const uint8_t*)in)[i];
+  uint32_t b = ((const uint32_t*)in)[i];
+  int shift = order == 0 ? 8 * (3 - j) : 8 * j;
+  return (b >> shift) & 0xFFu;
+}
+
+int64_t orc_serialize_grouped(int input_kind, int sep_mode, int group, int order, const void* in, int64_t n,
+                              uint16_t* out) {
+  uint16_t sep[2];
+  int ns = orc_sep_tokens(sep_mode, sep);
+  if (orc_serial_tokens(input_kind, sep_mode, group, order, n) < 0) return -1;
+  int64_t bv = orc_bytes_per_value(input_kind), g = group ? group : bv, nbytes = n * bv, t = 0;
+  for (int64_t k = 0; k < nbytes; k++) {
+    uint32_t byte = orc_value_byte(input_kind, order, in, k / bv, (int)(k % bv));
+    out[t++] = (uint16_t)(byte >> 4);
+    out[t++] = (uint16_t)(byte & 0xFu);
+    if ((k + 1) % g == 0 || k + 1 == nbytes)
+      for (int s = 0; s < ns; s++) out[t++] = sep[s];
+  }
+  return t;
+}
+
+/* Inverse of orc_serialize_grouped: the number of values, or -1 if no value count gives n_tok
+ * tokens or a token is out of place. */
+int64_t orc_deserialize_grouped(int input_kind, int sep_mode, int group, int order, const uint16_t* tok,
+                                int64_t n_tok, void* out) {
+  uint16_t sep[2];
+  int ns = orc_sep_tokens(sep_mode, sep);
+  if (orc_serial_tokens(input_kind, sep_mode, group, order, 0) < 0 || n_tok < 0) return -1;
+  int64_t bv = orc_bytes_per_value(input_kind), g = group ? group : bv;
+  /* the token count grows with n: find n by stepping (each value adds at least 2 tokens) */
+  int64_t n = n_tok / (2 * bv + ns * bv);
+  while (orc_serial_tokens(input_kind, sep_mode, group, order, n) < n_tok) n++;
+  if (orc_serial_tokens(input_kind, sep_mode, group, order, n) != n_tok) return -1;
+  int64_t nbytes = n * bv, t = 0;
+  if (input_kind == 0) memset(out, 0, (size_t)n * 4);
+  for (int64_t k = 0; k < nbytes; k++) {
+    uint16_t hi = tok[t++], lo = tok[t++];
+    if (hi > 15 || lo > 15) return -1;
+    uint32_t byte = (uint32_t)(hi << 4 | lo);
+    int64_t i = k / bv;
+    int j = (int)(k % bv);
+    if (input_kind == 1) {
+      ((uint8_t*)out)[i] = (uint8_t)byte;
+    } else {
+      int shift = order == 0 ? 8 * (3 - j) : 8 * j;
+      ((uint32_t*)out)[i] |= byte << shift;
+    }
+    if ((k + 1) % g == 0 || k + 1 == nbytes)
+      for (int s = 0; s < ns; s++)
+        if (tok[t++] != sep[s]) return -1;
+  }
+  return n;
+}
+
 /* ------------------------------------------------------------------------------------------ */
 /* Random-init weights. The paper uses pretrained checkpoints (Sec. 4.1); they are absent, so  */
 /* every weight is drawn from a counter-based generator: splitmix64 (Steele, Lea and Flood,    */

@@ -78,3 +78,74 @@ def test_tokens_per_value():
     assert O.tokens_per_value(0, 2) == 10
     assert O.tokens_per_value(0, 4) == 8
     assert O.tokens_per_value(1, 0) == 3
+
+
+# ---- byte grouping (Sec. 4.3 "Byte grouping": bytes per group BPG in {1, 2, 3, 4, 8}) ----
+
+def grouped_by_hex_string(vals: np.ndarray, sep_mode: int, group: int, order: int):
+    """The definition through Python's bytes.hex(): the byte stream (each fp32 big- or
+    little-endian, uint8 codes as is), two hex characters per byte, the separator after every
+    `group` bytes and after a final partial group."""
+    if vals.dtype == np.float32:
+        data = vals.astype(">f4" if order == 0 else "<f4").tobytes()
+    else:
+        data = vals.tobytes()
+    out = []
+    for k in range(0, len(data), group):
+        out += hex_tokens(data[k:k + group].hex()) + SEPS[sep_mode]
+    return out
+
+
+def test_grouped_worked_examples():
+    # 1.0f = 3f800000, -2.0f = c0000000
+    v = np.array([1.0, -2.0], dtype=np.float32)
+    assert O.serialize(v[:1], 0, 1, 0).tolist() == [3, 15, 16, 8, 0, 16, 0, 0, 16, 0, 0, 16]
+    assert O.serialize(v[:1], 0, 1, 1).tolist() == [0, 0, 16, 0, 0, 16, 8, 0, 16, 3, 15, 16]
+    # BPG 3 crosses the value boundary; the last group (2 bytes) is partial and still separated
+    assert O.serialize(v, 3, 3, 0).tolist() == [3, 15, 8, 0, 0, 0, 18, 0, 0, 12, 0, 0, 0, 18, 0, 0, 0, 0, 18]
+    # BPG 8: one separator per two values; H_{c+s} separators are two tokens
+    assert O.serialize(v, 2, 8, 0).tolist() == [3, 15, 8, 0, 0, 0, 0, 0, 12, 0, 0, 0, 0, 0, 0, 0, 17, 16]
+    assert O.serial_tokens(0, 2, 3, 8, 0) == 3 * 8 + 2 * 2
+
+
+def test_grouped_default_group_is_one_value():
+    # the paper's default BPG = 4 for fp32 (and 1 for uint8 codes) is the one-group-per-value layout
+    rng = np.random.default_rng(7)
+    vals = rng.integers(0, 2 ** 32, 3000, dtype=np.uint64).astype(np.uint32).view(np.float32)
+    codes = rng.integers(0, 256, 3000).astype(np.uint8)
+    for sep in range(5):
+        assert np.array_equal(O.serialize(vals, sep, 4, 0), O.serialize(vals, sep))
+        assert np.array_equal(O.serialize(codes, sep, 1, 0), O.serialize(codes, sep))
+
+
+@pytest.mark.parametrize("group", [1, 2, 3, 4, 8])
+@pytest.mark.parametrize("order", [0, 1])
+@pytest.mark.parametrize("sep_mode", [0, 2, 4])
+def test_grouped_against_hex_string_and_round_trip(group, order, sep_mode):
+    rng = np.random.default_rng(100 * group + 10 * order + sep_mode)
+    for n in (1, 2, 3, 5, 8, 333):
+        vals = rng.integers(0, 2 ** 32, n, dtype=np.uint64).astype(np.uint32).view(np.float32)
+        tok = O.serialize(vals, sep_mode, group, order)
+        assert tok.tolist() == grouped_by_hex_string(vals, sep_mode, group, order), n
+        assert tok.size == O.serial_tokens(0, sep_mode, n, group, order)
+        back = O.deserialize(tok, 0, sep_mode, group, order)
+        assert back.view(np.uint32).tolist() == vals.view(np.uint32).tolist()
+        codes = rng.integers(0, 256, n).astype(np.uint8)
+        tc = O.serialize(codes, sep_mode, group, 0)
+        assert tc.tolist() == grouped_by_hex_string(codes, sep_mode, group, 0)
+        assert np.array_equal(O.deserialize(tc, 1, sep_mode, group, 0), codes)
+
+
+def test_grouped_rejects_malformed_streams():
+    vals = np.array([1.0, -2.0, 3.5], dtype=np.float32)
+    tok = O.serialize(vals, 0, 3, 0)
+    with pytest.raises(ValueError):
+        O.deserialize(tok[:-1], 0, 0, 3, 0)  # no value count gives this length
+    bad = tok.copy()
+    bad[6] = 5  # a digit where the separator belongs
+    with pytest.raises(ValueError):
+        O.deserialize(bad, 0, 0, 3, 0)
+    bad = tok.copy()
+    bad[0] = 16  # a separator where a digit belongs
+    with pytest.raises(ValueError):
+        O.deserialize(bad, 0, 0, 3, 0)
