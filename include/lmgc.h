@@ -77,6 +77,10 @@ typedef struct {
   int32_t batch_windows; /* windows per model batch (workspace is sized for it) */
   uint64_t weight_seed;
   float init_std, rms_eps, rope_theta;
+  int32_t byte_group;    /* bytes per separator group (Sec. 4.3 "Byte grouping", BPG 1..8); 0 = one
+                            group per value (the default: BPG 4 for fp32, 1 for uint8 codes) */
+  int32_t byte_order;    /* fp32 bytes in the stream: 0 most significant first, 1 least significant
+                            first (uint8 codes: 0) */
 } lmgc_config;
 
 /* Create a context on the current CUDA device: validates the configuration, allocates the
@@ -92,19 +96,29 @@ lmgc_status lmgc_destroy(lmgc_ctx* ctx);
  * thread) into buf (NUL-terminated, truncated to len). */
 lmgc_status lmgc_last_error(const lmgc_ctx* ctx, char* buf, size_t len);
 
-/* Tokens per serialised value for the context's input kind and separator mode. */
+/* Tokens per serialised value for the context's input kind and separator mode. Errors: INVALID
+ * when byte groups cross values (byte_group 3, or 8 for fp32), so that no per-value count exists;
+ * lmgc_serial_tokens gives the count of any n then. */
 lmgc_status lmgc_tokens_per_value(const lmgc_ctx* ctx, size_t* tpv);
 
+/* Token count of n serialised values: 2 digits per byte plus the separator tokens of
+ * ceil(bytes / group) groups. Errors: INVALID. */
+lmgc_status lmgc_serial_tokens(const lmgc_ctx* ctx, size_t n, size_t* n_tok);
+
 /* Sec. 3 "Serialization" and Fig. 1: every 4 bits of a value become one hex digit, most
- * significant first (sign and exponent first), then the separator tokens.
+ * significant first (sign and exponent first), then the separator tokens. With byte_group or
+ * byte_order set (Sec. 4.3 "Byte grouping"): the values' bytes in order (fp32 bytes per
+ * byte_order), two hex digits per byte, high nibble first, and the separator after every
+ * byte_group bytes and after a final partial group.
  * d_in: n values (fp32 bit patterns or uint8 codes per the context's input kind).
- * d_tok: n * tpv uint16 token ids (capacity cap_tok). *n_tok receives n * tpv (host).
+ * d_tok: uint16 token ids (capacity cap_tok). *n_tok receives lmgc_serial_tokens(n) (host).
  * Errors: INVALID, NO_SPACE (cap_tok too small; *n_tok = required), CUDA. */
 lmgc_status lmgc_serialize(lmgc_ctx* ctx, const void* d_in, size_t n, uint16_t* d_tok, size_t cap_tok,
                            size_t* n_tok, lmgc_stream stream);
 
-/* Inverse of lmgc_serialize. d_out receives n_tok / tpv values (capacity cap_values).
- * Errors: CORRUPT if n_tok is not a multiple of tpv or a token is out of place; NO_SPACE. Syncs. */
+/* Inverse of lmgc_serialize. d_out receives the n values with lmgc_serial_tokens(n) = n_tok
+ * (capacity cap_values). Errors: CORRUPT if no n gives n_tok tokens or a token is out of place;
+ * NO_SPACE. Syncs. */
 lmgc_status lmgc_deserialize(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, void* d_out, size_t cap_values,
                              size_t* n_values, lmgc_stream stream);
 
@@ -186,7 +200,8 @@ lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);
 /* The whole encode path (Sec. 3): serialise -> windows from BOS -> model logits -> integer CDF
  * pairs -> one code per window -> container. Container layout (little-endian):
  *   0 "LMGC" | 4 u32 version=2 | 8 u64 n_values | 16 u64 n_tok | 24 u32 window | 28 u32 cdf_bits |
- *   32 u32 input_kind | 36 u32 sep_mode | 40 u32 vocab | 44 u32 n_win | 48 u64 weight_seed |
+ *   32 u32 input_kind | 36 u32 serialisation = sep_mode | byte_group << 8 | byte_order << 16 |
+ *   40 u32 vocab | 44 u32 n_win | 48 u64 weight_seed |
  *   56 u32 crc32 of the model shape | 60 u32 crc32 of bytes [0, 60) |
  *   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | codes, ceil(bitlen/8) bytes each, in window order.
  * crc_tok[w] is the CRC-32 (IEEE 802.3) of window w's token ids as little-endian u16 bytes (the

@@ -21,6 +21,11 @@ void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 void set_thread_error(const std::string& s) { g_thread_err = s; }
 
+// tokens of n serialised values under the context's layout (Sec. 3; byte grouping, Sec. 4.3)
+static int64_t n_tokens(const lmgc_ctx* ctx, int64_t n) {
+  return serial_tokens(ctx->cfg.input_kind, ctx->cfg.sep_mode, ctx->cfg.byte_group, n);
+}
+
 lmgc_status fail(lmgc_ctx* ctx, lmgc_status st, const std::string& msg) {
   if (ctx) ctx->err = msg;
   g_thread_err = msg;
@@ -319,7 +324,17 @@ lmgc_status lmgc_last_error(const lmgc_ctx* ctx, char* buf, size_t len) {
 
 lmgc_status lmgc_tokens_per_value(const lmgc_ctx* ctx, size_t* tpv) {
   if (!ctx || !tpv) return LMGC_ERR_INVALID;
-  *tpv = (size_t)ctx->tpv;
+  const lmgc_config& c = ctx->cfg;
+  const int64_t t1 = serial_tokens(c.input_kind, c.sep_mode, c.byte_group, 1);
+  if (serial_tokens(c.input_kind, c.sep_mode, c.byte_group, 8) != 8 * t1)
+    return fail(const_cast<lmgc_ctx*>(ctx), LMGC_ERR_INVALID, "byte groups cross values: no tokens-per-value count");
+  *tpv = (size_t)t1;
+  return LMGC_OK;
+}
+
+lmgc_status lmgc_serial_tokens(const lmgc_ctx* ctx, size_t n, size_t* n_tok) {
+  if (!ctx || !n_tok) return LMGC_ERR_INVALID;
+  *n_tok = (size_t)serial_tokens(ctx->cfg.input_kind, ctx->cfg.sep_mode, ctx->cfg.byte_group, (int64_t)n);
   return LMGC_OK;
 }
 
@@ -358,6 +373,8 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (c.dtype != LMGC_F32 && c.dtype != LMGC_BF16) return fail(nullptr, LMGC_ERR_INVALID, "bad dtype");
   int tpv = tokens_per_value(c.input_kind, c.sep_mode);
   if (tpv < 0) return fail(nullptr, LMGC_ERR_INVALID, "bad input kind or separator mode");
+  if (c.byte_group < 0 || c.byte_group > 8 || c.byte_order < 0 || c.byte_order > 1)
+    return fail(nullptr, LMGC_ERR_INVALID, "byte_group must be 0..8 and byte_order 0 or 1");
 
   lmgc_ctx* ctx = new lmgc_ctx();
   ctx->cfg = c;
@@ -473,11 +490,12 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
 lmgc_status lmgc_serialize(lmgc_ctx* ctx, const void* d_in, size_t n, uint16_t* d_tok, size_t cap_tok,
                            size_t* n_tok, lmgc_stream stream) {
   if (!ctx || !n_tok || (n && (!d_in || !d_tok))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
-  size_t need = n * (size_t)ctx->tpv;
+  const lmgc_config& c = ctx->cfg;
+  size_t need = (size_t)serial_tokens(c.input_kind, c.sep_mode, c.byte_group, (int64_t)n);
   *n_tok = need;
   if (cap_tok < need) return fail(ctx, LMGC_ERR_NO_SPACE, "token buffer too small");
   cudaStream_t s = (cudaStream_t)stream;
-  launch_serialize(ctx->cfg.input_kind, ctx->cfg.sep_mode, d_in, (int64_t)n, d_tok, s);
+  launch_serialize(c.input_kind, c.sep_mode, c.byte_group, c.byte_order, d_in, (int64_t)n, d_tok, s);
   LMGC_CUDA(ctx, cudaGetLastError());
   return LMGC_OK;
 }
@@ -485,12 +503,14 @@ lmgc_status lmgc_serialize(lmgc_ctx* ctx, const void* d_in, size_t n, uint16_t* 
 lmgc_status lmgc_deserialize(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, void* d_out, size_t cap_values,
                              size_t* n_values, lmgc_stream stream) {
   if (!ctx || !n_values || (n_tok && (!d_tok || !d_out))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
-  if (n_tok % (size_t)ctx->tpv) return fail(ctx, LMGC_ERR_CORRUPT, "token count not a multiple of tokens/value");
-  size_t nv = n_tok / (size_t)ctx->tpv;
+  const lmgc_config& c = ctx->cfg;
+  const int64_t nvs = serial_values(c.input_kind, c.sep_mode, c.byte_group, (int64_t)n_tok);
+  if (nvs < 0) return fail(ctx, LMGC_ERR_CORRUPT, "no value count serialises to this many tokens");
+  size_t nv = (size_t)nvs;
   *n_values = nv;
   if (cap_values < nv) return fail(ctx, LMGC_ERR_NO_SPACE, "value buffer too small");
   cudaStream_t s = (cudaStream_t)stream;
-  launch_deserialize(ctx->cfg.input_kind, ctx->cfg.sep_mode, d_tok, (int64_t)nv, d_out, ctx->d_err, s);
+  launch_deserialize(c.input_kind, c.sep_mode, c.byte_group, c.byte_order, d_tok, (int64_t)nv, d_out, ctx->d_err, s);
   LMGC_CUDA(ctx, cudaGetLastError());
   return check_err_word(ctx, s, "deserialize");
 }
@@ -590,7 +610,7 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
 
 lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes) {
   if (!ctx || !bytes) return LMGC_ERR_INVALID;
-  const size_t n_tok = n * (size_t)ctx->tpv, W = (size_t)ctx->cfg.window;
+  const size_t n_tok = (size_t)n_tokens(ctx, (int64_t)n), W = (size_t)ctx->cfg.window;
   const size_t n_win = (n_tok + W - 1) / W;
   *bytes = 64 + 8 * n_win + (n_tok * (size_t)ctx->cfg.cdf_bits + 2 * n_win + 7) / 8 + n_win;
   return LMGC_OK;
@@ -607,7 +627,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
                                 uint64_t* payload, cudaStream_t s) {
   const lmgc_config& c = ctx->cfg;
   const int64_t W = c.window, P = c.cdf_bits;
-  const int64_t n_tok = (int64_t)n * ctx->tpv;
+  const int64_t n_tok = n_tokens(ctx, (int64_t)n);
   const int64_t n_win = w_count;
   const size_t slot = slot_bytes((size_t)W, (int)P);
   // staging (grown on demand; reused across calls)
@@ -631,7 +651,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[0], s));
   {
     ProfScope ps(ctx, kSer, (double)n * (ctx->cfg.input_kind == LMGC_IN_F32 ? 4 : 1) + (double)n_tok * 2, s);
-    launch_serialize(c.input_kind, c.sep_mode, d_in, (int64_t)n, ctx->tok, s);
+    launch_serialize(c.input_kind, c.sep_mode, c.byte_group, c.byte_order, d_in, (int64_t)n, ctx->tok, s);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[1], s));
   const int64_t n_batches = (n_win + c.batch_windows - 1) / c.batch_windows;
@@ -703,9 +723,14 @@ static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bi
 
 constexpr uint32_t kContainerVersion = 2;  // 2: per-window token checksums after the bit lengths
 
+// header word at byte 36: the separator mode, and the byte grouping (0 for the default layout)
+static uint32_t serial_word(const lmgc_config& c) {
+  return (uint32_t)c.sep_mode | (uint32_t)c.byte_group << 8 | (uint32_t)c.byte_order << 16;
+}
+
 static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
   const lmgc_config& c = ctx->cfg;
-  const uint64_t n_tok = (uint64_t)n * (uint64_t)ctx->tpv;
+  const uint64_t n_tok = (uint64_t)n_tokens(ctx, (int64_t)n);
   const uint64_t n_win = (n_tok + (uint64_t)c.window - 1) / (uint64_t)c.window;
   memset(h, 0, 64);
   uint32_t u32;
@@ -717,7 +742,7 @@ static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
   u32 = (uint32_t)c.window; memcpy(h + 24, &u32, 4);
   u32 = (uint32_t)c.cdf_bits; memcpy(h + 28, &u32, 4);
   u32 = (uint32_t)c.input_kind; memcpy(h + 32, &u32, 4);
-  u32 = (uint32_t)c.sep_mode; memcpy(h + 36, &u32, 4);
+  u32 = serial_word(c); memcpy(h + 36, &u32, 4);
   u32 = (uint32_t)c.vocab; memcpy(h + 40, &u32, 4);
   u32 = (uint32_t)n_win; memcpy(h + 44, &u32, 4);
   u64 = c.weight_seed; memcpy(h + 48, &u64, 8);
@@ -735,7 +760,7 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
   if (n == 0) return fail(ctx, LMGC_ERR_INVALID, "empty input");
   cudaStream_t s = (cudaStream_t)stream;
   const int64_t W = ctx->cfg.window;
-  const int64_t n_win = ((int64_t)n * ctx->tpv + W - 1) / W;
+  const int64_t n_win = (n_tokens(ctx, (int64_t)n) + W - 1) / W;
   uint64_t payload = 0;
   lmgc_status st = encode_codes(ctx, d_in, n, 0, n_win, &payload, s);
   if (st != LMGC_OK) return st;
@@ -755,7 +780,7 @@ lmgc_status lmgc_encode_windows(lmgc_ctx* ctx, const void* d_in, size_t n, size_
   if (!ctx || !d_in || !payload_bytes || (n_win && (!d_bitlen || !d_crc)))
     return fail(ctx, LMGC_ERR_INVALID, "null argument");
   const int64_t W = ctx->cfg.window;
-  const int64_t total_win = ((int64_t)n * ctx->tpv + W - 1) / W;
+  const int64_t total_win = (n_tokens(ctx, (int64_t)n) + W - 1) / W;
   if (n == 0 || n_win == 0 || (int64_t)(first_win + n_win) > total_win)
     return fail(ctx, LMGC_ERR_INVALID, "window range outside the stream");
   cudaStream_t s = (cudaStream_t)stream;
@@ -817,7 +842,7 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   uint64_t seed;
   memcpy(&seed, h + 48, 8);
   if (ver != kContainerVersion || hW != (uint32_t)W || hP != (uint32_t)c.cdf_bits || kind != (uint32_t)c.input_kind ||
-      sep != (uint32_t)c.sep_mode || vocab != (uint32_t)c.vocab || mcrc != model_crc(c) || seed != c.weight_seed)
+      sep != serial_word(c) || vocab != (uint32_t)c.vocab || mcrc != model_crc(c) || seed != c.weight_seed)
     return fail(ctx, LMGC_ERR_CORRUPT, "container does not match this context's model or coder");
   if ((uint64_t)n_win != (n_tok + W - 1) / W || 64 + 8 * (size_t)n_win > in_bytes)
     return fail(ctx, LMGC_ERR_CORRUPT, "container window table truncated");

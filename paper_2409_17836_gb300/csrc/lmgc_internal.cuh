@@ -130,9 +130,15 @@ void note_launch();
 // ---- kernels' launchers (stream-ordered, no sync) ----
 // serialize.cu
 int tokens_per_value(int input_kind, int sep_mode);
-void launch_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* tok, cudaStream_t s);
-void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64_t n_values, void* out,
-                        uint32_t* err, cudaStream_t s);
+// Byte grouping (Sec. 4.3): tokens of n values; the n with that many tokens (or -1); whether the
+// layout is the default one group per value, most significant byte first.
+int64_t serial_tokens(int input_kind, int sep_mode, int byte_group, int64_t n);
+int64_t serial_values(int input_kind, int sep_mode, int byte_group, int64_t n_tok);
+bool serial_is_default(int input_kind, int byte_group, int byte_order);
+void launch_serialize(int input_kind, int sep_mode, int byte_group, int byte_order, const void* in, int64_t n,
+                      uint16_t* tok, cudaStream_t s);
+void launch_deserialize(int input_kind, int sep_mode, int byte_group, int byte_order, const uint16_t* tok,
+                        int64_t n_values, void* out, uint32_t* err, cudaStream_t s);
 
 // lm.cu
 // Canonical row r of tensor tid goes to dst row row_off + (r / rblk) * rstride + r % rblk

@@ -18,6 +18,32 @@ int tokens_per_value(int input_kind, int sep_mode) {
   return nd + ns;
 }
 
+// Byte grouping (Sec. 4.3): bytes per value, and the group size (0 = one group per value).
+static int64_t bytes_per_value(int input_kind) { return input_kind == LMGC_IN_F32 ? 4 : 1; }
+static int sep_count(int sep_mode) { return sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1); }
+
+int64_t serial_tokens(int input_kind, int sep_mode, int byte_group, int64_t n) {
+  const int64_t bv = bytes_per_value(input_kind), g = byte_group ? byte_group : bv, nb = n * bv;
+  return 2 * nb + sep_count(sep_mode) * ((nb + g - 1) / g);
+}
+
+int64_t serial_values(int input_kind, int sep_mode, int byte_group, int64_t n_tok) {
+  // the layout repeats every lcm(bytes per value, group) bytes = pv values = pt tokens, and the
+  // token count of q * pv + j values is q * pt + (the count of j values)
+  const int64_t bv = bytes_per_value(input_kind), g = byte_group ? byte_group : bv;
+  int64_t pb = bv;
+  while (pb % g) pb += bv;
+  const int64_t pv = pb / bv, pt = serial_tokens(input_kind, sep_mode, byte_group, pv);
+  const int64_t q = n_tok / pt;
+  for (int64_t j = 0; j < pv; j++)
+    if (serial_tokens(input_kind, sep_mode, byte_group, q * pv + j) == n_tok) return q * pv + j;
+  return -1;
+}
+
+bool serial_is_default(int input_kind, int byte_group, int byte_order) {
+  return (byte_group == 0 || byte_group == bytes_per_value(input_kind)) && byte_order == 0;
+}
+
 static void sep_ids(int sep_mode, uint16_t* s0, uint16_t* s1) {
   switch (sep_mode) {
     case LMGC_SEP_SPACE: *s0 = kTokSpace; *s1 = 0; break;
@@ -91,11 +117,44 @@ static void ser_dispatch(bool vec, const void* in, int64_t n, uint16_t* tok, uin
   else k_serialize<ND, NS, false><<<(unsigned)blocks, kSerThreads, 0, s>>>(in, n, tok, s0, s1);
 }
 
-void launch_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* tok, cudaStream_t s) {
+// Byte-grouped layout: one thread per group of g bytes (the group's 2g digits, then its separator
+// tokens). Byte b of the stream is byte b mod 4 of fp32 value b / 4 (most significant first, or
+// least with le) or uint8 code b.
+__global__ void k_serialize_grouped(const void* __restrict__ in, int64_t n, int bv, int g, int ns, int le,
+                                    uint16_t* __restrict__ tok, uint16_t sep0, uint16_t sep1) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t nb = n * bv;
+  if (k >= (nb + g - 1) / g) return;
+  const int64_t b0 = k * g, b1 = b0 + g < nb ? b0 + g : nb;
+  uint16_t* o = tok + 2 * b0 + ns * k;
+  for (int64_t b = b0; b < b1; b++) {
+    uint32_t byte;
+    if (bv == 1) {
+      byte = reinterpret_cast<const uint8_t*>(in)[b];
+    } else {
+      const int j = (int)(b & 3);
+      byte = (reinterpret_cast<const uint32_t*>(in)[b >> 2] >> (le ? 8 * j : 8 * (3 - j))) & 0xFFu;
+    }
+    *o++ = (uint16_t)(byte >> 4);
+    *o++ = (uint16_t)(byte & 0xFu);
+  }
+  if (ns >= 1) *o++ = sep0;
+  if (ns >= 2) *o = sep1;
+}
+
+void launch_serialize(int input_kind, int sep_mode, int byte_group, int byte_order, const void* in, int64_t n,
+                      uint16_t* tok, cudaStream_t s) {
   if (n <= 0) return;
   note_launch();
   uint16_t s0, s1;
   sep_ids(sep_mode, &s0, &s1);
+  if (!serial_is_default(input_kind, byte_group, byte_order)) {
+    const int bv = (int)bytes_per_value(input_kind), g = byte_group ? byte_group : bv;
+    const int64_t groups = (n * bv + g - 1) / g;
+    k_serialize_grouped<<<(unsigned)((groups + 255) / 256), 256, 0, s>>>(in, n, bv, g, sep_count(sep_mode),
+                                                                       byte_order, tok, s0, s1);
+    return;
+  }
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
   bool vec = (((uintptr_t)in) % 16 == 0) && (((uintptr_t)tok) % 16 == 0);
   if (input_kind == LMGC_IN_F32) {
@@ -130,11 +189,45 @@ __global__ void k_deserialize(const uint16_t* __restrict__ tok, int64_t n, int n
   else reinterpret_cast<uint8_t*>(out)[i] = (uint8_t)b;
 }
 
-void launch_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64_t n_values, void* out,
-                        uint32_t* err, cudaStream_t s) {
+// Inverse of k_serialize_grouped: one thread per group; each byte lands at its place in the
+// output (fp32 values are little-endian in memory); a malformed group sets kErrDeser.
+__global__ void k_deserialize_grouped(const uint16_t* __restrict__ tok, int64_t n, int bv, int g, int ns, int le,
+                                      uint16_t sep0, uint16_t sep1, uint8_t* __restrict__ out, uint32_t* err) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t nb = n * bv;
+  if (k >= (nb + g - 1) / g) return;
+  const int64_t b0 = k * g, b1 = b0 + g < nb ? b0 + g : nb;
+  const uint16_t* t = tok + 2 * b0 + ns * k;
+  bool bad = false;
+  for (int64_t b = b0; b < b1; b++) {
+    const uint16_t hi = *t++, lo = *t++;
+    bad |= hi > 15 || lo > 15;
+    const uint8_t byte = (uint8_t)(((hi & 0xFu) << 4) | (lo & 0xFu));
+    if (bv == 1) {
+      out[b] = byte;
+    } else {
+      const int j = (int)(b & 3), shift = le ? 8 * j : 8 * (3 - j);
+      out[(b >> 2) * 4 + shift / 8] = byte;
+    }
+  }
+  if (ns >= 1) bad |= *t++ != sep0;
+  if (ns >= 2) bad |= *t != sep1;
+  if (bad) atomicOr(err, kErrDeser);
+}
+
+void launch_deserialize(int input_kind, int sep_mode, int byte_group, int byte_order, const uint16_t* tok,
+                        int64_t n_values, void* out, uint32_t* err, cudaStream_t s) {
   if (n_values <= 0) return;
   uint16_t s0, s1;
   sep_ids(sep_mode, &s0, &s1);
+  if (!serial_is_default(input_kind, byte_group, byte_order)) {
+    const int bv = (int)bytes_per_value(input_kind), g = byte_group ? byte_group : bv;
+    const int64_t groups = (n_values * bv + g - 1) / g;
+    note_launch();
+    k_deserialize_grouped<<<(unsigned)((groups + 255) / 256), 256, 0, s>>>(
+        tok, n_values, bv, g, sep_count(sep_mode), byte_order, s0, s1, reinterpret_cast<uint8_t*>(out), err);
+    return;
+  }
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
   int nd = input_kind == LMGC_IN_F32 ? 8 : 2;
   note_launch();

@@ -33,7 +33,8 @@ class Config(C.Structure):
                 ("n_kv_heads", C.c_int32), ("d_ffn", C.c_int32), ("vocab", C.c_int32), ("dtype", C.c_int32),
                 ("window", C.c_int32), ("cdf_bits", C.c_int32), ("sep_mode", C.c_int32),
                 ("input_kind", C.c_int32), ("batch_windows", C.c_int32), ("weight_seed", C.c_uint64),
-                ("init_std", C.c_float), ("rms_eps", C.c_float), ("rope_theta", C.c_float)]
+                ("init_std", C.c_float), ("rms_eps", C.c_float), ("rope_theta", C.c_float),
+                ("byte_group", C.c_int32), ("byte_order", C.c_int32)]
 
 
 @dataclasses.dataclass
@@ -54,11 +55,14 @@ class ModelConfig:
     init_std: float = 0.02
     rms_eps: float = 1e-5
     rope_theta: float = 10000.0
+    byte_group: int = 0  # bytes per separator group (Sec. 4.3 byte grouping); 0 = one group per value
+    byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
 
     def c(self) -> Config:
         return Config(self.n_layers, self.d_model, self.n_heads, self.n_kv_heads, self.d_ffn, self.vocab, self.dtype,
                       self.window, self.cdf_bits, self.sep_mode, self.input_kind, self.batch_windows,
-                      self.weight_seed, self.init_std, self.rms_eps, self.rope_theta)
+                      self.weight_seed, self.init_std, self.rms_eps, self.rope_theta, self.byte_group,
+                      self.byte_order)
 
 
 _lib = None
@@ -68,6 +72,7 @@ SYMBOLS = {
     "lmgc_destroy": (C.c_int, [C.c_void_p]),
     "lmgc_last_error": (C.c_int, [C.c_void_p, C.c_char_p, C.c_size_t]),
     "lmgc_tokens_per_value": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "lmgc_serial_tokens": (C.c_int, [C.c_void_p, C.c_size_t, C.c_void_p]),
     "lmgc_serialize": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     "lmgc_deserialize": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p,
                                    C.c_void_p]),
@@ -161,8 +166,10 @@ class Context:
             pass
 
     @property
-    def tpv(self) -> int:
-        return lmgc_tokens_per_value(self)
+    def tpv(self) -> int | None:
+        """Tokens per value, or None when byte groups cross values (byte_group 3 or 8)."""
+        v = C.c_size_t()
+        return v.value if load().lmgc_tokens_per_value(self.handle, C.byref(v)) == OK else None
 
 
 # ---- entry points (same names as the C ABI) ----
@@ -173,10 +180,16 @@ def lmgc_tokens_per_value(ctx: Context) -> int:
     return v.value
 
 
+def lmgc_serial_tokens(ctx: Context, n: int) -> int:
+    v = C.c_size_t()
+    _check(ctx, load().lmgc_serial_tokens(ctx.handle, n, C.byref(v)))
+    return v.value
+
+
 def lmgc_serialize(ctx: Context, values: torch.Tensor, tokens: torch.Tensor | None = None, stream=None):
     n = values.numel()
     if tokens is None:
-        tokens = torch.empty(n * ctx.tpv, dtype=torch.int16, device=values.device)
+        tokens = torch.empty(lmgc_serial_tokens(ctx, n), dtype=torch.int16, device=values.device)
     n_tok = C.c_size_t()
     _check(ctx, load().lmgc_serialize(ctx.handle, _ptr(values), n, _ptr(tokens), tokens.numel(), C.byref(n_tok),
                                       _stream(stream)))

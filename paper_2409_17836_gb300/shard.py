@@ -60,7 +60,7 @@ def encode_sharded(ctx, values, rank: int, world: int, group=None) -> bytes | No
     `world` ranks; returns the container on rank 0."""
     from . import lmgc as L
 
-    n_win = -(-values.numel() * ctx.tpv // ctx.cfg.window)
+    n_win = -(-L.lmgc_serial_tokens(ctx, values.numel()) // ctx.cfg.window)
     first, count = window_ranges(n_win, world)[rank]
     if count:
         payload, bitlen, crc = L.lmgc_encode_windows(ctx, values, first, count)

@@ -12,7 +12,8 @@ def oracle_config(cfg, n_threads: int = 1) -> O.OracleConfig:
                           d_ffn=cfg.d_ffn, vocab=cfg.vocab, bf16=cfg.dtype == 1, window=cfg.window,
                           cdf_bits=cfg.cdf_bits, weight_seed=cfg.weight_seed, init_std=cfg.init_std,
                           rms_eps=cfg.rms_eps, rope_theta=cfg.rope_theta, sep_mode=cfg.sep_mode,
-                          input_kind=cfg.input_kind, n_threads=n_threads)
+                          input_kind=cfg.input_kind, n_threads=n_threads, byte_group=cfg.byte_group,
+                          byte_order=cfg.byte_order)
 
 
 def cpu_threads() -> int:

@@ -63,6 +63,53 @@ def test_serialize_unaligned_input_and_u8():
     ctx.close()
 
 
+@pytest.mark.parametrize("group,order", [(1, 0), (2, 1), (3, 0), (3, 1), (4, 1), (8, 0), (8, 1)])
+@pytest.mark.parametrize("sep_mode", [0, 2, 4])
+def test_serialize_byte_groups_bit_exact(group, order, sep_mode):
+    """Byte grouping (Sec. 4.3): tokens bit-exact with the oracle for fp32 values (either byte
+    order) and uint8 codes, ragged counts whose last group is partial; round trip; the token
+    count through lmgc_serial_tokens."""
+    ctx = ctx_for(sep_mode=sep_mode, byte_group=group, byte_order=order)
+    rng = np.random.default_rng(10 * group + order + sep_mode)
+    for n in (1, 2, 3, 1001, 65537):
+        bits = rng.integers(0, 2 ** 32, n, dtype=np.uint64).astype(np.uint32)
+        bits[: min(n, SPECIAL.size)] = SPECIAL[: min(n, SPECIAL.size)]
+        d = torch.from_numpy(bits.view(np.int32).copy()).cuda()
+        tok = L.lmgc_serialize(ctx, d)
+        ref = O.serialize(bits.view(np.float32), sep_mode, group, order)
+        assert L.lmgc_serial_tokens(ctx, n) == ref.size
+        assert np.array_equal(tok.cpu().numpy().view(np.uint16), ref), n
+        back = torch.zeros(n, dtype=torch.int32, device="cuda")
+        assert L.lmgc_deserialize(ctx, tok, back) == n
+        assert np.array_equal(back.cpu().numpy().view(np.uint32), bits), n
+    # a per-value token count exists unless groups cross values and carry separators
+    assert (ctx.tpv is None) == (group in (3, 8) and sep_mode != 4)
+    ctx.close()
+    ctx = ctx_for(sep_mode=sep_mode, byte_group=group, input_kind=L.IN_U8)
+    codes = rng.integers(0, 256, 4099).astype(np.uint8)
+    tok = L.lmgc_serialize(ctx, torch.from_numpy(codes).cuda())
+    assert np.array_equal(tok.cpu().numpy().view(np.uint16), O.serialize(codes, sep_mode, group, 0))
+    out = torch.empty(4099, dtype=torch.uint8, device="cuda")
+    assert L.lmgc_deserialize(ctx, tok, out) == 4099
+    assert np.array_equal(out.cpu().numpy(), codes)
+    ctx.close()
+
+
+def test_deserialize_byte_groups_rejects_malformed():
+    ctx = ctx_for(byte_group=3)
+    tok = L.lmgc_serialize(ctx, torch.ones(10, dtype=torch.float32, device="cuda"))
+    assert tok.numel() == 2 * 40 + 14
+    bad = tok.clone()
+    bad[6] = 5  # a digit where the first group's separator belongs
+    with pytest.raises(L.LmgcError) as e:
+        L.lmgc_deserialize(ctx, bad, torch.empty(10, device="cuda"))
+    assert e.value.status == L.ERR_CORRUPT
+    with pytest.raises(L.LmgcError) as e:
+        L.lmgc_deserialize(ctx, tok[:-1], torch.empty(10, device="cuda"))  # no count gives 93 tokens
+    assert e.value.status == L.ERR_CORRUPT
+    ctx.close()
+
+
 def test_deserialize_rejects_malformed(ctx_tiny):
     tok = L.lmgc_serialize(ctx_tiny, torch.ones(10, dtype=torch.float32, device="cuda"))
     bad = tok.clone()

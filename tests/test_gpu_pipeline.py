@@ -90,6 +90,42 @@ def test_tinyllama_shape_pairs_and_codes_given_gpu_logits():
     ctx.close()
 
 
+@pytest.mark.parametrize("group,order", [(3, 1), (8, 0), (1, 0)])
+def test_byte_grouped_encode_decode_and_codes(group, order):
+    """Byte grouping (Sec. 4.3) through the whole path: the container records the layout, every
+    window's code is bit-exact with the oracle's pairs and coder on the GPU's logits of the
+    oracle's token stream, and decoding restores the tokens and the values."""
+    cfg = configs.with_(configs.TINY, sep_mode=1, byte_group=group, byte_order=order, batch_windows=4)
+    ctx = L.Context(cfg)
+    vals = I.tiny_gradient(3)[:1111]
+    tok = O.serialize(vals, 1, group, order)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert (h["sep_mode"], h["byte_group"], h["byte_order"]) == (1, group, order)
+    assert h["n_tok"] == tok.size and h["n_values"] == vals.size
+    W = cfg.window
+    n_win = h["n_win"]
+    lg = L.lmgc_lm_probs(ctx, torch.from_numpy(tok.view(np.int16)).cuda(), 0, n_win).cpu().numpy()
+    for w in range(n_win):
+        n = min(W, tok.size - w * W)
+        st, fr = O.cdf_pairs(lg[w, :n], tok[w * W: w * W + n], cfg.cdf_bits)
+        code, nbits = O.range_encode(st, fr, cfg.cdf_bits)
+        assert h["bitlen"][w] == nbits and buf[h["offsets"][w]: h["offsets"][w + 1]] == code, w
+    toks = decode_all(ctx, buf, list(range(n_win)))
+    flat = np.concatenate([toks[w, :min(W, tok.size - w * W)] for w in range(n_win)])
+    assert np.array_equal(flat, tok)
+    back = torch.zeros(vals.size, dtype=torch.int32, device="cuda")
+    assert L.lmgc_deserialize(ctx, torch.from_numpy(flat.view(np.int16)).cuda(), back) == vals.size
+    assert back.cpu().numpy().tobytes() == vals.tobytes()
+    # a context with the default layout rejects this container
+    other = L.Context(configs.with_(configs.TINY, sep_mode=1, batch_windows=4))
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(other, buf, [0])
+    assert e.value.status == L.ERR_CORRUPT
+    other.close()
+    ctx.close()
+
+
 @pytest.mark.parametrize("n,sep,kind", [(1, 0, 0), (29, 2, 0), (1000, 4, 0), (777, 0, 1)])
 def test_tiny_edge_sizes_round_trip(n, sep, kind):
     cfg = configs.with_(configs.TINY, sep_mode=sep, input_kind=kind, batch_windows=3)
