@@ -177,12 +177,13 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
 
 def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> dict:
     """HBM-bound stages at sizes where bandwidth, not launch latency, decides: the serialiser on
-    the 64M-value Laplace mixture, and the coder alone on 2^18 windows x 2048 tokens of seeded
+    the 64M-value Laplace mixture (default layout, and byte groups of 3 that cross values), and
+    the coder alone on 2^18 windows x 2048 tokens of seeded
     random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most likely)."""
     import numpy as np
     import torch
 
-    from paper_2409_17836_gb300 import inputs
+    from paper_2409_17836_gb300 import configs, inputs
 
     out = {}
     vals = inputs.laplace_gradient()
@@ -200,6 +201,22 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> 
     nbytes = d.numel() * 4 + tok.numel() * 2
     out["serialize"] = {"values": d.numel(), "ms": ms, "bytes": nbytes, "achieved": nbytes / ms / 1e6,
                         "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
+    del tok
+    # the byte-grouped layout (Sec. 4.3): 3 bytes per group, fp32 bytes least significant first
+    gctx = L.Context(configs.with_(configs.TINY, byte_group=3, byte_order=1))
+    tok = torch.empty(L.lmgc_serial_tokens(gctx, d.numel()), dtype=torch.int16, device="cuda")
+    L.lmgc_serialize(gctx, d, tok)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(reps):
+        L.lmgc_serialize(gctx, d, tok)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    nbytes = d.numel() * 4 + tok.numel() * 2
+    out["serialize_grouped"] = {"values": d.numel(), "byte_group": 3, "byte_order": 1, "ms": ms, "bytes": nbytes,
+                                "achieved": nbytes / ms / 1e6, "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
+    gctx.close()
     del d, tok
     V, P, W, n_win = 32000, 24, 2048, coder_windows
     g = torch.Generator(device="cuda").manual_seed(5)

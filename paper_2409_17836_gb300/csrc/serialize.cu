@@ -117,29 +117,53 @@ static void ser_dispatch(bool vec, const void* in, int64_t n, uint16_t* tok, uin
   else k_serialize<ND, NS, false><<<(unsigned)blocks, kSerThreads, 0, s>>>(in, n, tok, s0, s1);
 }
 
-// Byte-grouped layout: one thread per group of g bytes (the group's 2g digits, then its separator
-// tokens). Byte b of the stream is byte b mod 4 of fp32 value b / 4 (most significant first, or
-// least with le) or uint8 code b.
-__global__ void k_serialize_grouped(const void* __restrict__ in, int64_t n, int bv, int g, int ns, int le,
-                                    uint16_t* __restrict__ tok, uint16_t sep0, uint16_t sep1) {
-  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t nb = n * bv;
-  if (k >= (nb + g - 1) / g) return;
-  const int64_t b0 = k * g, b1 = b0 + g < nb ? b0 + g : nb;
-  uint16_t* o = tok + 2 * b0 + ns * k;
-  for (int64_t b = b0; b < b1; b++) {
-    uint32_t byte;
-    if (bv == 1) {
-      byte = reinterpret_cast<const uint8_t*>(in)[b];
-    } else {
-      const int j = (int)(b & 3);
-      byte = (reinterpret_cast<const uint32_t*>(in)[b >> 2] >> (le ? 8 * j : 8 * (3 - j))) & 0xFFu;
+// Byte-grouped layout: a block takes kGrpTile consecutive groups of g bytes; each thread writes
+// its groups' 2g digits and separator tokens into shared memory, and the block stores the tile's
+// tokens as 16-byte vectors (a tile starts at token k0 (2g + ns), k0 a multiple of kGrpTile, so
+// on a 16-byte boundary). Byte b of the stream is byte b mod 4 of fp32 value b / 4 (most
+// significant first, or least with le) or uint8 code b.
+constexpr int kGrpThreads = 256, kGrpTile = 4 * kGrpThreads;
+
+__global__ void __launch_bounds__(kGrpThreads) k_serialize_grouped(const void* __restrict__ in, int64_t n, int bv,
+                                                                   int g, int ns, int le,
+                                                                   uint16_t* __restrict__ tok, uint16_t sep0,
+                                                                   uint16_t sep1, bool vec) {
+  __shared__ __align__(16) uint16_t buf[kGrpTile * (2 * 8 + 2)];
+  const int64_t nb = n * bv, n_groups = (nb + g - 1) / g;
+  const int64_t k0 = (int64_t)blockIdx.x * kGrpTile;
+  const int tpg = 2 * g + ns;
+  const int ng = n_groups - k0 < kGrpTile ? (int)(n_groups - k0) : kGrpTile;
+  for (int i = threadIdx.x; i < ng; i += kGrpThreads) {
+    const int64_t b0 = (k0 + i) * g, b1 = b0 + g < nb ? b0 + g : nb;
+    uint16_t* o = buf + i * tpg;
+    for (int64_t b = b0; b < b1; b++) {
+      uint32_t byte;
+      if (bv == 1) {
+        byte = reinterpret_cast<const uint8_t*>(in)[b];
+      } else {
+        const int j = (int)(b & 3);
+        byte = (reinterpret_cast<const uint32_t*>(in)[b >> 2] >> (le ? 8 * j : 8 * (3 - j))) & 0xFFu;
+      }
+      *o++ = (uint16_t)(byte >> 4);
+      *o++ = (uint16_t)(byte & 0xFu);
     }
-    *o++ = (uint16_t)(byte >> 4);
-    *o++ = (uint16_t)(byte & 0xFu);
+    if (ns >= 1) *o++ = sep0;
+    if (ns >= 2) *o = sep1;
   }
-  if (ns >= 1) *o++ = sep0;
-  if (ns >= 2) *o = sep1;
+  __syncthreads();
+  // the tile's tokens (the last group of the stream may be short)
+  const int64_t t0 = k0 * tpg;
+  const int64_t tend = 2 * nb + (int64_t)ns * n_groups;
+  const int nt = tend - t0 < (int64_t)kGrpTile * tpg ? (int)(tend - t0) : kGrpTile * tpg;
+  uint16_t* dst = tok + t0;
+  if (vec) {
+    const uint4* s4 = reinterpret_cast<const uint4*>(buf);
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    for (int q = threadIdx.x; q < nt / 8; q += kGrpThreads) __stcs(d4 + q, s4[q]);
+    for (int q = (nt / 8) * 8 + threadIdx.x; q < nt; q += kGrpThreads) dst[q] = buf[q];
+  } else {
+    for (int q = threadIdx.x; q < nt; q += kGrpThreads) dst[q] = buf[q];
+  }
 }
 
 void launch_serialize(int input_kind, int sep_mode, int byte_group, int byte_order, const void* in, int64_t n,
@@ -151,8 +175,9 @@ void launch_serialize(int input_kind, int sep_mode, int byte_group, int byte_ord
   if (!serial_is_default(input_kind, byte_group, byte_order)) {
     const int bv = (int)bytes_per_value(input_kind), g = byte_group ? byte_group : bv;
     const int64_t groups = (n * bv + g - 1) / g;
-    k_serialize_grouped<<<(unsigned)((groups + 255) / 256), 256, 0, s>>>(in, n, bv, g, sep_count(sep_mode),
-                                                                       byte_order, tok, s0, s1);
+    const bool vec = ((uintptr_t)tok) % 16 == 0;  // tiles start on 16-byte boundaries then
+    k_serialize_grouped<<<(unsigned)((groups + kGrpTile - 1) / kGrpTile), kGrpThreads, 0, s>>>(
+        in, n, bv, g, sep_count(sep_mode), byte_order, tok, s0, s1, vec);
     return;
   }
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);
