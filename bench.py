@@ -30,7 +30,8 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "raw gradient MB/s encoded (1 GB300); LM tensor-pipe % of bf16 peak; coder HBM GB/s"
-WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama", "laplace-tinyllama")
+WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama", "laplace-tinyllama",
+             "quant16-tinyllama", "quant1-tinyllama", "sparse50-tinyllama", "sparse25-tinyllama")
 
 
 def peaks():
@@ -110,7 +111,27 @@ def workload(name: str):
         return configs.TINY, inputs.tiny_gradient(0)
     if name == "laplace-tinyllama":  # 64M-value Laplace mixture; window batch set by --batch-windows
         return configs.TINYLLAMA, inputs.laplace_gradient()
+    # Sec. 5 compatibility settings one at a time: Eq. 4 indices of every value (16 bits as
+    # big-endian byte pairs, one separator per index; 1 bit as one byte each), or the top 50% / 25%
+    # of |v| still as fp32
+    if name in ("quant16-tinyllama", "quant1-tinyllama"):
+        b, group = inputs.code_bytes(inputs.quantized_codes(inputs.convnet_gradient(0), 16 if "16" in name else 1))
+        return configs.with_(configs.TINYLLAMA, input_kind=1, byte_group=group), b
+    if name in ("sparse50-tinyllama", "sparse25-tinyllama"):
+        return configs.TINYLLAMA, inputs.sparsified(inputs.convnet_gradient(0), 0.5 if "50" in name else 0.25)
     raise ValueError(name)
+
+
+def values_for_tokens(count, n_max: int, budget: int) -> int:
+    """The most values (<= n_max) whose serialisation fits in `budget` tokens; count(n) = tokens."""
+    lo, hi = 0, n_max
+    while lo < hi:
+        mid = (lo + hi + 1) // 2
+        if count(mid) <= budget:
+            lo = mid
+        else:
+            hi = mid - 1
+    return lo
 
 
 def run_full(args, cfg, ctx, vals):
@@ -134,15 +155,20 @@ def run_full(args, cfg, ctx, vals):
         torch.cuda.synchronize()
     sec = e0.elapsed_time(e1) / 1e3
     W = cfg.window
-    n_tok = vals.size * ctx.tpv
+    n_tok = L.lmgc_serial_tokens(ctx, vals.size)
     n_win = -(-n_tok // W)
     ids = [0, n_win // 2, n_win - 1]
     toks = L.lmgc_decode(ctx, buf, ids).cpu().numpy().view(np.uint16)
     ok = True
+    tpv = ctx.tpv
+    whole = None if tpv else O.serialize(vals, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
     for i, w in enumerate(ids):
         n = min(W, n_tok - w * W)
-        v0, v1 = (w * W) // ctx.tpv, -(-min(n_tok, (w + 1) * W) // ctx.tpv)
-        ref = O.serialize(vals[v0:v1], cfg.sep_mode)[w * W - v0 * ctx.tpv:][:n]
+        if tpv:
+            v0, v1 = (w * W) // tpv, -(-min(n_tok, (w + 1) * W) // tpv)
+            ref = O.serialize(vals[v0:v1], cfg.sep_mode, cfg.byte_group, cfg.byte_order)[w * W - v0 * tpv:][:n]
+        else:
+            ref = whole[w * W: w * W + n]
         ok = ok and bool(np.array_equal(toks[i, :n], ref))
     bpv = 4 if vals.dtype == np.float32 else 1
     print(json.dumps({"mode": "full", "workload": args.workload, "values": int(vals.size), "windows": int(n_win),
@@ -164,8 +190,9 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
     oc = O.OracleConfig(n_layers=cfg.n_layers, d_model=cfg.d_model, n_heads=cfg.n_heads, n_kv_heads=cfg.n_kv_heads,
                         d_ffn=cfg.d_ffn, vocab=cfg.vocab, bf16=cfg.dtype == 1, window=cfg.window,
                         cdf_bits=cfg.cdf_bits, weight_seed=cfg.weight_seed, init_std=cfg.init_std,
-                        sep_mode=cfg.sep_mode, input_kind=cfg.input_kind, n_threads=threads)
-    tok = O.serialize(vals, cfg.sep_mode)
+                        sep_mode=cfg.sep_mode, input_kind=cfg.input_kind, n_threads=threads,
+                        byte_group=cfg.byte_group, byte_order=cfg.byte_order)
+    tok = O.serialize(vals, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
     W = cfg.window
     seg = tok[win * W: win * W + W]
     t0 = time.perf_counter()
@@ -188,19 +215,21 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> 
     out = {}
     vals = inputs.laplace_gradient()
     d = torch.from_numpy(vals.view(np.int32)).cuda()
-    tok = torch.empty(d.numel() * ctx.tpv, dtype=torch.int16, device="cuda")
-    L.lmgc_serialize(ctx, d, tok)
+    sctx = L.Context(configs.TINY)  # fp32 values, one group per value, H_s
+    tok = torch.empty(L.lmgc_serial_tokens(sctx, d.numel()), dtype=torch.int16, device="cuda")
+    L.lmgc_serialize(sctx, d, tok)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     for _ in range(reps):
-        L.lmgc_serialize(ctx, d, tok)
+        L.lmgc_serialize(sctx, d, tok)
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / reps
     nbytes = d.numel() * 4 + tok.numel() * 2
     out["serialize"] = {"values": d.numel(), "ms": ms, "bytes": nbytes, "achieved": nbytes / ms / 1e6,
                         "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
+    sctx.close()
     del tok
     # the byte-grouped layout (Sec. 4.3): 3 bytes per group, fp32 bytes least significant first
     gctx = L.Context(configs.with_(configs.TINY, byte_group=3, byte_order=1))
@@ -279,9 +308,10 @@ def run_reference(args):
     O.lib()
     cfg, vals = workload(args.workload)
     threads = max(1, len(os.sched_getaffinity(0)))
-    tpv = O.tokens_per_value(cfg.input_kind, cfg.sep_mode)
+    n_tok = O.serial_tokens(cfg.input_kind, cfg.sep_mode, vals.size, cfg.byte_group, cfg.byte_order)
+    tpv = n_tok / vals.size  # tokens per value over the workload
     positions = args.ref_positions
-    n_win = -(-vals.size * tpv // cfg.window)
+    n_win = -(-n_tok // cfg.window)
     for i in range(args.warmup):
         oracle_sample(cfg, vals, 2, i % n_win, threads)
     total_t, total_tok = 0.0, 0
@@ -348,7 +378,7 @@ def main():
     if args.layers:
         cfg = configs.with_(cfg, n_layers=args.layers)
     ctx = L.Context(cfg)
-    tpv = ctx.tpv
+    tpv = L.lmgc_serial_tokens(ctx, vals.size) / vals.size  # tokens per value over the workload
     if args.full:
         return run_full(args, cfg, ctx, vals)
     if args.micro_only:
@@ -356,7 +386,8 @@ def main():
               flush=True)
         ctx.close()
         return 0
-    per_step = (cfg.batch_windows * cfg.window) // tpv  # values filling one model batch
+    # values filling one model batch
+    per_step = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, cfg.batch_windows * cfg.window)
     n_slices = max(1, vals.size // per_step)
     dev = torch.from_numpy(vals.view(np.int32) if vals.dtype == np.float32 else vals).cuda()
     slices = [dev[i * per_step:(i + 1) * per_step] for i in range(n_slices)]

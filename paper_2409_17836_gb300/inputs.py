@@ -13,6 +13,8 @@ not available, so seeded stand-ins of the same kind are used:
 * `lossy_codes`        Sec. 5 "Compatibility": top-10% magnitude sparsification followed by
                        8-bit linear quantisation (Eq. 4) of the kept values.
 * `laplace_gradient`   a 200-tensor Laplace mixture with log-uniform scales (throughput sweep).
+* `sparsified`, `quantized_codes`, `code_bytes`   the Sec. 5 compatibility inputs one at a time
+                     (sparsification 50/25/10% as fp32; 16/8/1-bit Eq. 4 indices).
 """
 from __future__ import annotations
 
@@ -47,6 +49,30 @@ def convnet_gradient(seed: int = 0, batch: int = 64) -> np.ndarray:
     loss.backward()
     grad = torch.cat([p.grad.reshape(-1) for p in net.parameters()])
     return grad.detach().numpy().astype(np.float32)
+
+
+def sparsified(grad: np.ndarray, keep: float) -> np.ndarray:
+    """Sec. 5 sparsification alone: the floor(keep*N) largest |v| (ties to the lower index) in
+    index order, still fp32 (the paper: sparsified gradients stay 32-bit floats)."""
+    g = np.asarray(grad, dtype=np.float32)
+    k = int(np.floor(keep * g.size))
+    order = np.lexsort((np.arange(g.size), -np.abs(g.astype(np.float64))))
+    return g[np.sort(order[:k])].copy()
+
+
+def quantized_codes(grad: np.ndarray, bits: int) -> np.ndarray:
+    """Sec. 5 quantisation alone: Eq. 4 over every value (n = 16, 8 or 1 bits; 1 bit is SignSGD's
+    setting); the indices are what is coded."""
+    return lossy_codes(grad, keep=1.0, bits=bits)
+
+
+def code_bytes(codes: np.ndarray) -> tuple[np.ndarray, int]:
+    """The byte stream of integer codes for the uint8 input kind, and the byte group that keeps one
+    code per separator group: uint16 codes as big-endian byte pairs (4 hex digits, most
+    significant first, then the separator: byte_group 2); uint8 codes as they are (group 0)."""
+    if codes.dtype == np.uint16:
+        return np.ascontiguousarray(codes.astype(">u2")).view(np.uint8), 2
+    return np.ascontiguousarray(codes, dtype=np.uint8), 0
 
 
 def lossy_codes(grad: np.ndarray, keep: float = 0.1, bits: int = 8) -> np.ndarray:

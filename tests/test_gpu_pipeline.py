@@ -126,6 +126,37 @@ def test_byte_grouped_encode_decode_and_codes(group, order):
     ctx.close()
 
 
+@pytest.mark.parametrize("setting", ["quant16", "quant1", "sparse50", "sparse25"])
+def test_compatibility_inputs_round_trip(setting):
+    """Sec. 5 compatibility inputs one at a time through the whole path: Eq. 4 indices of every
+    value (16 bits as big-endian byte pairs in 2-byte groups, 1 bit as bytes) or the top 50% /
+    25% of |v| kept as fp32. The restored tokens equal the oracle's serialisation of the same
+    input, the values come back exactly, and the container's size is within 0.5% of the
+    oracle's encode."""
+    g = I.tiny_gradient(4)
+    if setting.startswith("quant"):
+        vals, group = I.code_bytes(I.quantized_codes(g, 16 if setting == "quant16" else 1))
+        cfg = configs.with_(configs.TINY, input_kind=L.IN_U8, byte_group=group, batch_windows=8)
+        kind = 1
+    else:
+        vals, group = I.sparsified(g, 0.5 if setting == "sparse50" else 0.25), 0
+        cfg = configs.with_(configs.TINY, batch_windows=8)
+        kind = 0
+    ctx = L.Context(cfg)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    tok = O.serialize(vals, 0, group, 0)
+    assert h["n_tok"] == tok.size and h["byte_group"] == group
+    toks = decode_all(ctx, buf, list(range(h["n_win"])))
+    W = cfg.window
+    flat = np.concatenate([toks[w, :min(W, tok.size - w * W)] for w in range(h["n_win"])])
+    assert np.array_equal(flat, tok)
+    assert O.deserialize(flat, kind, 0, group, 0).tobytes() == vals.tobytes()
+    ref = O.encode(oracle_config(cfg), vals, n_par=cpu_threads())
+    assert abs(len(buf) - len(ref)) <= 0.005 * len(ref), (len(buf), len(ref))
+    ctx.close()
+
+
 @pytest.mark.parametrize("n,sep,kind", [(1, 0, 0), (29, 2, 0), (1000, 4, 0), (777, 0, 1)])
 def test_tiny_edge_sizes_round_trip(n, sep, kind):
     cfg = configs.with_(configs.TINY, sep_mode=sep, input_kind=kind, batch_windows=3)

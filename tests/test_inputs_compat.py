@@ -1,0 +1,35 @@
+"""The Sec. 5 compatibility inputs one at a time (the f3 sweep): Eq. 4 quantisation to 16, 8 and
+1 bits over every value, magnitude sparsification that keeps fp32 values, and the byte stream
+that carries 16-bit indices (4 hex digits per index through 2-byte groups). Worked by hand."""
+import numpy as np
+
+import oracle as O
+from paper_2409_17836_gb300 import inputs as I
+
+
+def test_eq4_worked_examples():
+    v = np.array([-1.0, 0.0, 3.0], dtype=np.float32)
+    # (v - min) / (max - min) * (2^n - 1): 0, 0.25, 1 of the range
+    assert I.quantized_codes(v, 16).tolist() == [0, 16384, 65535]  # 16383.75 rounds up
+    assert I.quantized_codes(v, 8).tolist() == [0, 64, 255]        # 63.75
+    assert I.quantized_codes(v, 16).dtype == np.uint16 and I.quantized_codes(v, 8).dtype == np.uint8
+    w = np.array([-2.0, 0.5, 3.0], dtype=np.float32)
+    assert I.quantized_codes(w, 1).tolist() == [0, 0, 1]             # 0.5 rounds to even
+
+
+def test_sparsified_keeps_largest_in_index_order():
+    g = np.array([0.1, -5.0, 2.0, 2.0, -2.0, 0.0, 7.0, -0.2], dtype=np.float32)
+    # |v| ranks: 7 (idx 6), 5 (idx 1), then the tie 2.0 / 2.0 / -2.0 at indices 2, 3, 4
+    assert I.sparsified(g, 0.5).tolist() == [-5.0, 2.0, 2.0, 7.0]   # keeps indices 1, 2, 3, 6
+    assert I.sparsified(g, 0.25).tolist() == [-5.0, 7.0]
+    assert I.sparsified(g, 0.5).dtype == np.float32
+
+
+def test_16bit_codes_as_byte_pairs():
+    b, group = I.code_bytes(np.array([0x1234, 0xABCD, 0x0007], dtype=np.uint16))
+    assert group == 2 and b.tolist() == [0x12, 0x34, 0xAB, 0xCD, 0x00, 0x07]
+    tok = O.serialize(b, 0, group, 0)
+    assert tok.tolist() == [1, 2, 3, 4, 16, 10, 11, 12, 13, 16, 0, 0, 0, 7, 16]
+    assert np.array_equal(O.deserialize(tok, 1, 0, group, 0), b)
+    c, g8 = I.code_bytes(np.array([5, 250], dtype=np.uint8))
+    assert g8 == 0 and c.tolist() == [5, 250]
