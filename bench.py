@@ -181,6 +181,49 @@ def run_full(args, cfg, ctx, vals):
     return 0 if ok else 1
 
 
+def run_decode(args, cfg, ctx, vals):
+    """lmgc_decode of every window of one encoded batch (batch_windows full windows), timed with
+    CUDA events around the call; the restored tokens are compared with the serialised input."""
+    import numpy as np
+    import torch
+
+    import oracle as O
+    from paper_2409_17836_gb300 import lmgc as L
+
+    W = cfg.window
+    n = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, cfg.batch_windows * W)
+    v = vals[:n]
+    d = torch.from_numpy(v.view(np.int32) if v.dtype == np.float32 else v).cuda()
+    buf = L.lmgc_encode(ctx, d)
+    n_tok = L.lmgc_serial_tokens(ctx, n)
+    n_win = -(-n_tok // W)
+    ids = list(range(n_win))
+    L.lmgc_decode(ctx, buf, ids[:1])  # warm-up
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with Clocks(torch.cuda.current_device()) as clk:
+        e0.record()
+        toks = L.lmgc_decode(ctx, buf, ids)
+        e1.record()
+        torch.cuda.synchronize()
+    sec = e0.elapsed_time(e1) / 1e3
+    # the same decode again with per-class kernel timing (CUDA events around each launch)
+    L.lmgc_profile(ctx, True)
+    L.lmgc_decode(ctx, buf, ids)
+    torch.cuda.synchronize()
+    st = L.lmgc_kernel_stats(ctx)
+    L.lmgc_profile(ctx, False)
+    classes = {k: {"launches": x["launches"], "ms": round(x["ms"], 1)} for k, x in st.items() if x["launches"]}
+    ref = O.serialize(v, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
+    got = toks.cpu().numpy().view(np.uint16).reshape(-1)[:n_tok]
+    print(json.dumps({"mode": "decode", "workload": args.workload, "windows": n_win, "tokens": n_tok,
+                      "seconds": sec, "tokens_per_s": n_tok / sec, "ms_per_position": 1e3 * sec / W,
+                      "match": bool(np.array_equal(got, ref)), "clocks": clk.summary(),
+                      "classes_profiled_run": classes}), flush=True)
+    ctx.close()
+    return 0
+
+
 def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
     """Oracle encode of the first `positions` tokens of window `win` (model + CDF + coder)."""
     import numpy as np
@@ -351,6 +394,9 @@ def main():
     # only the serialise and coder microbenchmarks (one JSON line), the coder on this many windows
     # of 2048 tokens (small profiler captures use 2^16)
     ap.add_argument("--micro-only", action="store_true")
+    # decode throughput: encode one batch of windows, then time lmgc_decode of all of them
+    # (KV-cached, one model step per position) and check the tokens; one JSON line of its own
+    ap.add_argument("--decode", action="store_true")
     ap.add_argument("--coder-windows", type=int, default=1 << 18)
     args = ap.parse_args()
     if args.impl == "reference":
@@ -381,6 +427,8 @@ def main():
     tpv = L.lmgc_serial_tokens(ctx, vals.size) / vals.size  # tokens per value over the workload
     if args.full:
         return run_full(args, cfg, ctx, vals)
+    if args.decode:
+        return run_decode(args, cfg, ctx, vals)
     if args.micro_only:
         print(json.dumps({"mode": "micro", "microbench": microbenchmarks(L, ctx, peaks(), coder_windows=args.coder_windows)}),
               flush=True)
