@@ -204,6 +204,9 @@ struct Params {
   int q_col0, k_col0, v_col0;  // column offsets of q head 0, k head 0, v head 0
   float scale_log2;            // log2(e) / sqrt(hd)
   uint32_t* err;
+  // decode packing: > 0 when each CTA takes the single query row (position pos_first) of every
+  // one of the `packed` query heads of KV head blockIdx.y, one per tile row
+  int packed;
 };
 
 template <int HD>
@@ -227,19 +230,26 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   auto b_vfull = [&](int i) { return smem_u32(bars + 15 + i); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.y;
+  const int h = blockIdx.y;  // query head; with packing, the KV head
   const int64_t w = blockIdx.z;
-  const int kvh = h / (p.nq / p.nkv);
+  const int kvh = p.packed ? h : h / (p.nq / p.nkv);
   // heavy (late) query tiles first
   const int qb = (int)gridDim.x - 1 - (int)blockIdx.x;
   const int64_t pos0 = p.pos_first + (int64_t)qb * BQ;  // position of tile row 0
   const int64_t rem = p.pos_first + p.n_pos - pos0;
-  const int nrows = rem < BQ ? (int)rem : BQ;  // valid rows
-  const int64_t last_pos = pos0 + nrows - 1;
+  const int nrows = p.packed ? p.packed : (rem < BQ ? (int)rem : BQ);  // valid rows
+  const int64_t last_pos = p.packed ? pos0 : pos0 + nrows - 1;
   const int nkb = (int)(last_pos / BKV) + 1;
   const int q_row0 = (int)(w * p.q_win_stride + (pos0 - p.pos_first));
   const int kv_row0 = (int)(w * p.W);
 
+  if (p.packed) {
+    // rows past the packed ones read zeros (their scores are then finite and need no moves)
+    uint4* q4 = reinterpret_cast<uint4*>(smem);
+    for (int i = threadIdx.x; i < S::KCH * BQ * 8; i += kThreads)
+      if ((i / 8) % BQ >= nrows) q4[i] = make_uint4(0u, 0u, 0u, 0u);
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);  // 12-14, 17-18 unused
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -259,9 +269,18 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   if (warp == 0) {
     // ---------------- TMA producer: Q, then K blocks ----------------
     if (lane == 0) {
-      mbar_expect_tx(b_q, S::Q_BYTES);
+      if (p.packed) {
+        // one 128-byte row per head and chunk (the tensor map's box is one row high)
+        mbar_expect_tx(b_q, (uint32_t)nrows * S::KCH * 128);
+        for (int j = 0; j < nrows; j++)
 #pragma unroll
-      for (int c = 0; c < S::KCH; c++) tma_load_2d(sq + c * (BQ * 128), &tq, b_q, p.q_col0 + h * HD + 64 * c, q_row0);
+          for (int c = 0; c < S::KCH; c++)
+            tma_load_2d(sq + c * (BQ * 128) + j * 128, &tq, b_q, p.q_col0 + (kvh * nrows + j) * HD + 64 * c, q_row0);
+      } else {
+        mbar_expect_tx(b_q, S::Q_BYTES);
+#pragma unroll
+        for (int c = 0; c < S::KCH; c++) tma_load_2d(sq + c * (BQ * 128), &tq, b_q, p.q_col0 + h * HD + 64 * c, q_row0);
+      }
     }
     __syncwarp();
     for (int kb = 0; kb < nkb; kb++) {
@@ -345,7 +364,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     // ---------------- softmax (warps 2..5): thread r owns query row r = TMEM lane r ----------------
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
-    const int pos0_i = (int)pos0, qpos_i = (int)pos0 + r;
+    const int pos0_i = (int)pos0, qpos_i = p.packed ? (int)pos0 : (int)pos0 + r;
+    // a warp whose rows are all past the valid ones only keeps the barrier protocol: it waits for
+    // each block's S (so its P arrivals stay in phase) and arrives without computing P
+    const bool live = q4 * 32 < nrows;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
     const float c = p.scale_log2;
     float m = -INFINITY, l = 0.f;
@@ -353,6 +375,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     for (int kb = 0; kb < nkb; kb++) {
       const int sb = kb % 3;
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / 3) & 1u, p.err)))) break;
+      if (!live) {
+        mbar_arrive(b_p(sb));
+        continue;
+      }
       tc_fence_after();
       float s[64];
       // S row of this block into s[], causally masked (only on blocks that reach past the tile's
@@ -454,10 +480,11 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     // S(last) implies P V(last-3), so P V(last-1) is awaited before P V(last))
     for (int j = nkb >= 2 ? nkb - 2 : 0; j < nkb && ok; j++)
       ok = __all_sync(0xffffffffu, mbar_wait(b_pv(j & 1), (uint32_t)(j >> 1) & 1u, p.err));
-    if (ok) {
+    if (ok && live) {
       tc_fence_after();
       const float inv = 1.f / l;
-      __half* dst = p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
+      __half* dst = p.packed ? p.out + (int64_t)q_row0 * p.out_stride + (int64_t)(kvh * nrows + r) * HD
+                             : p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
 #pragma unroll 1
       for (int cc = 0; cc < HD / 32; cc++) {
         uint32_t o[32];
@@ -546,7 +573,14 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
   p.v_col0 = v_off;
   p.scale_log2 = (float)(1.4426950408889634 / sqrt((double)hd));
   p.err = err;
-  dim3 grid((unsigned)((n_pos + BQ - 1) / BQ), (unsigned)nq, (unsigned)n_win);
+  // a decode step (one query row per window) packs the query heads of each KV head into one tile
+  const int group = nq / nkv;
+  p.packed = (n_pos == 1 && q_win_stride == 1 && group > 1 && group <= 32) ? group : 0;
+  if (p.packed && !make_map(&tq, q, (uint64_t)qkv_dim, (uint64_t)q_rows, 1)) {
+    set_thread_error("cuTensorMapEncodeTiled failed (attention)");
+    return;
+  }
+  dim3 grid((unsigned)((n_pos + BQ - 1) / BQ), (unsigned)(p.packed ? nkv : nq), (unsigned)n_win);
   note_launch();
   if (hd == 64) k_attn_tc<64><<<grid, kThreads, Shape<64>::SMEM, s>>>(tq, tkv, p);
   else k_attn_tc<128><<<grid, kThreads, Shape<128>::SMEM, s>>>(tq, tkv, p);
