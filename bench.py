@@ -182,8 +182,9 @@ def run_full(args, cfg, ctx, vals):
 
 
 def run_decode(args, cfg, ctx, vals):
-    """lmgc_decode of every window of one encoded batch (batch_windows full windows), timed with
-    CUDA events around the call; the restored tokens are compared with the serialised input."""
+    """lmgc_decode of every window of an encoded stream (--decode-windows full windows, default one
+    batch), timed with CUDA events around the call; the restored tokens are compared with the
+    serialised input. The library decodes as many windows per step as its KV cache budget holds."""
     import numpy as np
     import torch
 
@@ -191,7 +192,8 @@ def run_decode(args, cfg, ctx, vals):
     from paper_2409_17836_gb300 import lmgc as L
 
     W = cfg.window
-    n = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, cfg.batch_windows * W)
+    n_dec = args.decode_windows or cfg.batch_windows
+    n = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, n_dec * W)
     v = vals[:n]
     d = torch.from_numpy(v.view(np.int32) if v.dtype == np.float32 else v).cuda()
     buf = L.lmgc_encode(ctx, d)
@@ -397,6 +399,7 @@ def main():
     # decode throughput: encode one batch of windows, then time lmgc_decode of all of them
     # (KV-cached, one model step per position) and check the tokens; one JSON line of its own
     ap.add_argument("--decode", action="store_true")
+    ap.add_argument("--decode-windows", type=int, default=0)  # windows to decode (default: one batch)
     ap.add_argument("--coder-windows", type=int, default=1 << 18)
     args = ap.parse_args()
     if args.impl == "reference":

@@ -859,9 +859,16 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   if (off[n_win] > in_bytes) return fail(ctx, LMGC_ERR_CORRUPT, "container payload truncated");
   for (size_t i = 0; i < n_ids; i++)
     if (h_win_ids[i] >= n_win) return fail(ctx, LMGC_ERR_INVALID, "window id out of range");
-  // decode batch: as many windows as the workspace holds, with the KV cache kept under 16 GiB
   const size_t kv_per_win = (size_t)std::max(1, c.n_layers) * W * ctx->qkv_dim * ctx->elt;
-  const int64_t nd_max = std::max<int64_t>(1, std::min<int64_t>(c.batch_windows, (int64_t)((16ull << 30) / kv_per_win)));
+  // decode batch: as many of the requested windows as a KV cache of half the free device memory
+  // (at most 64 GiB) holds -- a step's GEMMs cost about the same for 64 rows as for 256
+  size_t free_b = 0, total_b = 0;
+  cudaMemGetInfo(&free_b, &total_b);
+  const size_t kv_budget = std::max<size_t>(ctx->kv_cap, std::min<size_t>(free_b / 2, 64ull << 30));
+  // (one workspace row per window: at most batch_windows * W of them)
+  const int64_t nd_max = std::max<int64_t>(
+      1, std::min<int64_t>(std::min<int64_t>((int64_t)std::max<size_t>(n_ids, 1), (int64_t)(kv_budget / kv_per_win)),
+                           (int64_t)c.batch_windows * W));
   const size_t kv_need = kv_per_win * (size_t)nd_max;
   if (ctx->kv_cap < kv_need || !ctx->kv_cache) {
     LMGC_CUDA(ctx, ensure(&ctx->kv_cache, &ctx->kv_cap, kv_need));
