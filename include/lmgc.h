@@ -236,7 +236,9 @@ lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t*
  * until the window is full). Decodes the windows h_win_ids[0 .. n_ids) (host array) of the
  * container d_in (device, in_bytes) into d_tok (device, [n_ids][W] uint16; a partial last window
  * fills only its length). Each decode step runs the same kernels as lmgc_encode on one row per
- * window, so its logits -- and hence its CDFs -- are bit-identical to the encoder's.
+ * window, so its logits -- and hence its CDFs -- are bit-identical to the encoder's. Windows
+ * are decoded in batches of as many as a KV cache of half the free device memory (at most
+ * 64 GiB) holds; the context keeps that cache for later calls (lmgc_destroy frees it).
  * Errors: CORRUPT (bad header, model mismatch, a code that leaves its interval, or a restored
  * window whose token checksum differs from the container's), INVALID
  * (window id out of range), NO_SPACE (cap_tok < n_ids * W), CUDA. Syncs. */
