@@ -209,7 +209,7 @@ struct Params {
   int packed;
 };
 
-template <int HD>
+template <int HD, bool PACKED>
 __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv, Params p) {
   using S = Shape<HD>;
@@ -232,18 +232,18 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;  // query head; with packing, the KV head
   const int64_t w = blockIdx.z;
-  const int kvh = p.packed ? h : h / (p.nq / p.nkv);
+  const int kvh = PACKED ? h : h / (p.nq / p.nkv);
   // heavy (late) query tiles first
   const int qb = (int)gridDim.x - 1 - (int)blockIdx.x;
   const int64_t pos0 = p.pos_first + (int64_t)qb * BQ;  // position of tile row 0
   const int64_t rem = p.pos_first + p.n_pos - pos0;
-  const int nrows = p.packed ? p.packed : (rem < BQ ? (int)rem : BQ);  // valid rows
-  const int64_t last_pos = p.packed ? pos0 : pos0 + nrows - 1;
+  const int nrows = PACKED ? p.packed : (rem < BQ ? (int)rem : BQ);  // valid rows
+  const int64_t last_pos = PACKED ? pos0 : pos0 + nrows - 1;
   const int nkb = (int)(last_pos / BKV) + 1;
   const int q_row0 = (int)(w * p.q_win_stride + (pos0 - p.pos_first));
   const int kv_row0 = (int)(w * p.W);
 
-  if (p.packed) {
+  if (PACKED) {
     // rows past the packed ones read zeros (their scores are then finite and need no moves)
     uint4* q4 = reinterpret_cast<uint4*>(smem);
     for (int i = threadIdx.x; i < S::KCH * BQ * 8; i += kThreads)
@@ -269,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   if (warp == 0) {
     // ---------------- TMA producer: Q, then K blocks ----------------
     if (lane == 0) {
-      if (p.packed) {
+      if (PACKED) {
         // one 128-byte row per head and chunk (the tensor map's box is one row high)
         mbar_expect_tx(b_q, (uint32_t)nrows * S::KCH * 128);
         for (int j = 0; j < nrows; j++)
@@ -364,10 +364,11 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     // ---------------- softmax (warps 2..5): thread r owns query row r = TMEM lane r ----------------
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
-    const int pos0_i = (int)pos0, qpos_i = p.packed ? (int)pos0 : (int)pos0 + r;
-    // a warp whose rows are all past the valid ones only keeps the barrier protocol: it waits for
-    // each block's S (so its P arrivals stay in phase) and arrives without computing P
-    const bool live = q4 * 32 < nrows;
+    const int pos0_i = (int)pos0, qpos_i = PACKED ? (int)pos0 : (int)pos0 + r;
+    // with packing, a warp whose rows are all past the packed ones only keeps the barrier
+    // protocol: it waits for each block's S (so its P arrivals stay in phase) and arrives without
+    // computing P
+    const bool live = !PACKED || q4 * 32 < nrows;
     const uint32_t tl = (uint32_t)(q4 * 32) << 16;
     const float c = p.scale_log2;
     float m = -INFINITY, l = 0.f;
@@ -483,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     if (ok && live) {
       tc_fence_after();
       const float inv = 1.f / l;
-      __half* dst = p.packed ? p.out + (int64_t)q_row0 * p.out_stride + (int64_t)(kvh * nrows + r) * HD
+      __half* dst = PACKED ? p.out + (int64_t)q_row0 * p.out_stride + (int64_t)(kvh * nrows + r) * HD
                              : p.out + ((int64_t)q_row0 + r) * p.out_stride + (int64_t)h * HD;
 #pragma unroll 1
       for (int cc = 0; cc < HD / 32; cc++) {
@@ -527,8 +528,10 @@ static void init_once() {
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
   if (major != 10) g_encode = nullptr;
-  cudaFuncSetAttribute(k_attn_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<64>::SMEM);
-  cudaFuncSetAttribute(k_attn_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<128>::SMEM);
+  cudaFuncSetAttribute(k_attn_tc<64, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<64>::SMEM);
+  cudaFuncSetAttribute(k_attn_tc<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<128>::SMEM);
+  cudaFuncSetAttribute(k_attn_tc<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<64>::SMEM);
+  cudaFuncSetAttribute(k_attn_tc<128, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Shape<128>::SMEM);
 }
 
 static bool make_map(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint32_t box_rows) {
@@ -582,8 +585,13 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
   }
   dim3 grid((unsigned)((n_pos + BQ - 1) / BQ), (unsigned)(p.packed ? nkv : nq), (unsigned)n_win);
   note_launch();
-  if (hd == 64) k_attn_tc<64><<<grid, kThreads, Shape<64>::SMEM, s>>>(tq, tkv, p);
-  else k_attn_tc<128><<<grid, kThreads, Shape<128>::SMEM, s>>>(tq, tkv, p);
+  if (p.packed) {
+    if (hd == 64) k_attn_tc<64, true><<<grid, kThreads, Shape<64>::SMEM, s>>>(tq, tkv, p);
+    else k_attn_tc<128, true><<<grid, kThreads, Shape<128>::SMEM, s>>>(tq, tkv, p);
+  } else {
+    if (hd == 64) k_attn_tc<64, false><<<grid, kThreads, Shape<64>::SMEM, s>>>(tq, tkv, p);
+    else k_attn_tc<128, false><<<grid, kThreads, Shape<128>::SMEM, s>>>(tq, tkv, p);
+  }
 }
 
 }  // namespace lmgc
