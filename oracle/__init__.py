@@ -86,7 +86,7 @@ def _p(a: np.ndarray):
 # sep_mode: 0 H_s (space), 1 H_c (comma), 2 H_{c+s}, 3 H_semi, 4 H_n (none). input_kind 0 = fp32,
 # 1 = uint8 codes (Eq. 4 indices).
 # ------------------------------------------------------------------------------------------
-TOK_BOS = 19
+TOK_SPACE, TOK_COMMA, TOK_SEMI, TOK_BOS = 16, 17, 18, 19
 
 
 def tokens_per_value(input_kind: int, sep_mode: int) -> int:
@@ -145,12 +145,19 @@ def weight_tensor(seed: int, tid: int, n: int, init_std: float, bf16: bool) -> n
     return out
 
 
+def alphabet_ids(sep_mode: int) -> list[int]:
+    """The ids a serialisation can emit (restricted-alphabet coding, a variant the paper does not
+    describe): the 16 hex digits and the separator ids of sep_mode, ascending."""
+    seps = {0: [TOK_SPACE], 1: [TOK_COMMA], 2: [TOK_COMMA, TOK_SPACE], 3: [TOK_SEMI], 4: []}[sep_mode]
+    return list(range(16)) + sorted(seps)
+
+
 class _Cfg(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("d_model", C.c_int32), ("n_heads", C.c_int32),
                 ("n_kv_heads", C.c_int32), ("d_ffn", C.c_int32), ("vocab", C.c_int32),
                 ("bf16", C.c_int32), ("window", C.c_int32), ("weight_seed", C.c_uint64),
                 ("init_std", C.c_float), ("rms_eps", C.c_float), ("rope_theta", C.c_float),
-                ("n_threads", C.c_int32)]
+                ("n_threads", C.c_int32), ("n_alpha", C.c_int32), ("alpha", C.c_uint16 * 32)]
 
 
 @dataclasses.dataclass
@@ -173,11 +180,14 @@ class OracleConfig:
     n_threads: int = 1
     byte_group: int = 0  # bytes per separator group (Sec. 4.3); 0 = one group per value
     byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
+    alphabet: int = 0    # 1: code over the ids the serialisation can emit (alphabet_ids) only
 
     def c(self) -> _Cfg:
+        ids = alphabet_ids(self.sep_mode) if self.alphabet else []
+        arr = (C.c_uint16 * 32)(*ids)
         return _Cfg(self.n_layers, self.d_model, self.n_heads, self.n_kv_heads, self.d_ffn, self.vocab,
                     int(self.bf16), self.window, self.weight_seed, self.init_std, self.rms_eps,
-                    self.rope_theta, self.n_threads)
+                    self.rope_theta, self.n_threads, len(ids), arr)
 
 
 class OracleLM:
@@ -352,8 +362,8 @@ def crc32(b: bytes) -> int:
 #   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | each window's code, ceil(bitlen/8) bytes, in
 #   window order. crc_tok[w] = crc32 of window w's token ids as little-endian u16 (its own
 #   length: W, or fewer for the last window), so that a decoder can check each window it restores.
-# serialisation = sep_mode | byte_group << 8 | byte_order << 16 (0 in the upper bits: the
-# default one group per value, most significant byte first).
+# serialisation = sep_mode | byte_group << 8 | byte_order << 16 | alphabet << 24 (0 in the upper
+# bits: the default one group per value, most significant byte first, the whole vocabulary).
 # model crc = crc32 of '<7i3f' (n_layers, d_model, n_heads, n_kv_heads, d_ffn, vocab, bf16,
 # init_std, rms_eps, rope_theta).
 # ------------------------------------------------------------------------------------------
@@ -378,7 +388,7 @@ def window_crcs(tok: np.ndarray, window: int, first: int = 0, count: int | None 
 
 
 def serial_word(cfg: OracleConfig) -> int:
-    return cfg.sep_mode | cfg.byte_group << 8 | cfg.byte_order << 16
+    return cfg.sep_mode | cfg.byte_group << 8 | cfg.byte_order << 16 | cfg.alphabet << 24
 
 
 def build_container(cfg: OracleConfig, n_values: int, n_tok: int, codes: list[tuple[bytes, int]],
@@ -407,7 +417,8 @@ def parse_container(buf: bytes) -> dict:
     crc_tok = np.frombuffer(buf[64 + 4 * n_win: 64 + 8 * n_win], dtype="<u4").astype(np.uint32)
     offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)]) + 64 + 8 * n_win
     return dict(version=f[1], n_values=f[2], n_tok=f[3], window=f[4], cdf_bits=f[5], input_kind=f[6],
-                sep_mode=f[7] & 0xFF, byte_group=(f[7] >> 8) & 0xFF, byte_order=(f[7] >> 16) & 0xFF, vocab=f[8], n_win=n_win, weight_seed=f[10], model_crc=f[11], bitlen=bl,
+                sep_mode=f[7] & 0xFF, byte_group=(f[7] >> 8) & 0xFF, byte_order=(f[7] >> 16) & 0xFF,
+                alphabet=(f[7] >> 24) & 0xFF, vocab=f[8], n_win=n_win, weight_seed=f[10], model_crc=f[11], bitlen=bl,
                 crc_tok=crc_tok, offsets=offs)
 
 

@@ -233,6 +233,11 @@ typedef struct {
   uint64_t weight_seed;
   float init_std, rms_eps, rope_theta;
   int32_t n_threads; /* OpenMP threads for the linear layers (1 = serial) */
+  /* restricted-alphabet coding (0 ids: the whole vocabulary): the integer CDF of a position is
+   * taken over the logits of these ids only (ascending), and the coded symbol is the token's
+   * index among them */
+  int32_t n_alpha;
+  uint16_t alpha[32];
 } orc_cfg;
 
 enum { ORC_WQ = 0, ORC_WK, ORC_WV, ORC_WO, ORC_WGATE, ORC_WUP, ORC_WDOWN };
@@ -646,21 +651,40 @@ int orc_dec_step(orc_dec* d, const uint32_t* cdf, int V, int P) {
 /* window (Sec. 3 "Compression": windows are coded independently, each from a fresh BOS).     */
 /* ------------------------------------------------------------------------------------------ */
 
+/* The integer CDF of one position: over the whole vocabulary, or over the restricted alphabet
+ * (the fp32 logits of its ids, in ascending id order). Returns the symbol count, or -1. */
+static int orc_position_cdf(const orc_cfg* c, const float* z, int P, float* zs, uint32_t* cdf) {
+  if (c->n_alpha <= 0) return orc_quantize_cdf(z, c->vocab, P, cdf) == 0 ? c->vocab : -1;
+  for (int j = 0; j < c->n_alpha; j++) zs[j] = z[c->alpha[j]];
+  return orc_quantize_cdf(zs, c->n_alpha, P, cdf) == 0 ? c->n_alpha : -1;
+}
+
+/* the coded symbol of token t: t itself, or its index in the restricted alphabet (-1: absent) */
+static int orc_symbol(const orc_cfg* c, uint16_t t) {
+  if (c->n_alpha <= 0) return t < c->vocab ? t : -1;
+  for (int j = 0; j < c->n_alpha; j++)
+    if (c->alpha[j] == t) return j;
+  return -1;
+}
+
 /* (start, freq) pairs of one window's n tokens, from the oracle LM. pairs_start/freq: [n]. */
 int orc_window_pairs(const orc_cfg* c, int P, const uint16_t* win_tok, int64_t n, uint32_t* pst, uint32_t* pfr,
                      float* logits_out /* optional [n][V] fp32 */) {
   int V = c->vocab;
   double* lg = (double*)malloc(sizeof(double) * (size_t)(n * V));
   float* z = (float*)malloc(sizeof(float) * (size_t)V);
+  float zs[32];
   uint32_t* cdf = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)(V + 1));
   int rc = orc_lm_window_logits(c, win_tok, n, lg);
   for (int64_t i = 0; rc == 0 && i < n; i++) {
     for (int j = 0; j < V; j++) z[j] = (float)lg[i * V + j];
     if (logits_out) memcpy(logits_out + i * V, z, sizeof(float) * (size_t)V);
-    rc = orc_quantize_cdf(z, V, P, cdf);
-    if (rc == 0) {
-      pst[i] = cdf[win_tok[i]];
-      pfr[i] = cdf[win_tok[i] + 1] - cdf[win_tok[i]];
+    const int sym = orc_symbol(c, win_tok[i]);
+    if (orc_position_cdf(c, z, P, zs, cdf) < 0 || sym < 0) {
+      rc = -1;
+    } else {
+      pst[i] = cdf[sym];
+      pfr[i] = cdf[sym + 1] - cdf[sym];
     }
   }
   free(lg);
@@ -711,6 +735,7 @@ int orc_decode_window(const orc_cfg* c, int P, const uint8_t* code, int64_t nbit
   double* lg = (double*)malloc(sizeof(double) * (size_t)V);
   float* z = (float*)malloc(sizeof(float) * (size_t)V);
   uint32_t* cdf = (uint32_t*)malloc(sizeof(uint32_t) * (size_t)(V + 1));
+  float zs[32];
   orc_dec d;
   orc_dec_init(&d, code, nbits);
   uint16_t cur = ORC_TOK_BOS;
@@ -719,15 +744,19 @@ int orc_decode_window(const orc_cfg* c, int P, const uint8_t* code, int64_t nbit
     rc = orc_lm_feed(s, &cur, 1, lg);
     if (rc) break;
     for (int j = 0; j < V; j++) z[j] = (float)lg[j];
-    rc = orc_quantize_cdf(z, V, P, cdf);
-    if (rc) break;
-    int sym = orc_dec_step(&d, cdf, V, P);
+    const int nsym = orc_position_cdf(c, z, P, zs, cdf);
+    if (nsym < 0) {
+      rc = -1;
+      break;
+    }
+    int sym = orc_dec_step(&d, cdf, nsym, P);
     if (sym < 0) {
       rc = -1;
       break;
     }
-    tok_out[i] = (uint16_t)sym;
-    cur = (uint16_t)sym;
+    const uint16_t t = c->n_alpha > 0 ? c->alpha[sym] : (uint16_t)sym;
+    tok_out[i] = t;
+    cur = t;
   }
   free(lg);
   free(z);
