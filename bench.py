@@ -31,7 +31,8 @@ sys.path.insert(0, ROOT)
 
 METRIC = "raw gradient MB/s encoded (1 GB300); LM tensor-pipe % of bf16 peak; coder HBM GB/s"
 WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama", "laplace-tinyllama",
-             "quant16-tinyllama", "quant1-tinyllama", "sparse50-tinyllama", "sparse25-tinyllama")
+             "quant16-tinyllama", "quant1-tinyllama", "sparse50-tinyllama", "sparse25-tinyllama",
+             "alpha-tinyllama")
 
 
 def peaks():
@@ -119,6 +120,8 @@ def workload(name: str):
         return configs.with_(configs.TINYLLAMA, input_kind=1, byte_group=group), b
     if name in ("sparse50-tinyllama", "sparse25-tinyllama"):
         return configs.TINYLLAMA, inputs.sparsified(inputs.convnet_gradient(0), 0.5 if "50" in name else 0.25)
+    if name == "alpha-tinyllama":  # integer CDFs over the 17 ids the space-separated stream can emit
+        return configs.with_(configs.TINYLLAMA, alphabet=1), inputs.convnet_gradient(0)
     raise ValueError(name)
 
 
@@ -236,7 +239,7 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
                         d_ffn=cfg.d_ffn, vocab=cfg.vocab, bf16=cfg.dtype == 1, window=cfg.window,
                         cdf_bits=cfg.cdf_bits, weight_seed=cfg.weight_seed, init_std=cfg.init_std,
                         sep_mode=cfg.sep_mode, input_kind=cfg.input_kind, n_threads=threads,
-                        byte_group=cfg.byte_group, byte_order=cfg.byte_order)
+                        byte_group=cfg.byte_group, byte_order=cfg.byte_order, alphabet=cfg.alphabet)
     tok = O.serialize(vals, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
     W = cfg.window
     seg = tok[win * W: win * W + W]

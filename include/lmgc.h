@@ -81,6 +81,11 @@ typedef struct {
                             group per value (the default: BPG 4 for fp32, 1 for uint8 codes) */
   int32_t byte_order;    /* fp32 bytes in the stream: 0 most significant first, 1 least significant
                             first (uint8 codes: 0) */
+  int32_t alphabet;      /* 0: each position's integer CDF spans the whole vocabulary (Sec. 3);
+                            1: it spans only the ids the serialisation can emit (the 16 hex digits
+                            and the separator ids of sep_mode), taken over those logits in
+                            ascending id order, and a token is coded as its index among them. A
+                            variant the paper does not describe. */
 } lmgc_config;
 
 /* Create a context on the current CUDA device: validates the configuration, allocates the
@@ -155,7 +160,10 @@ lmgc_status lmgc_quantize_cdf(lmgc_ctx* ctx, const float* d_logits, size_t rows,
 
 /* The coder's per-token input without materialising CDFs: for row r with symbol d_sym[r],
  * d_start[r] = cdf_r[sym] and d_freq[r] = cdf_r[sym + 1] - cdf_r[sym] under the quantiser of
- * lmgc_quantize_cdf. All arrays are indexed by row. Errors: INVALID, CUDA. */
+ * lmgc_quantize_cdf. All arrays are indexed by row. With alphabet 1 the quantiser runs over the
+ * restricted alphabet's logits of each row (V' ids), sym is the index of d_sym[r] among them,
+ * and the call syncs to report a d_sym[r] outside the alphabet (CORRUPT; its pair is (0, 1)).
+ * Errors: INVALID, CORRUPT, CUDA. */
 lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, const uint16_t* d_sym,
                            uint32_t* d_start, uint32_t* d_freq, lmgc_stream stream);
 
@@ -201,7 +209,7 @@ lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);
  * pairs -> one code per window -> container. Container layout (little-endian):
  *   0 "LMGC" | 4 u32 version=2 | 8 u64 n_values | 16 u64 n_tok | 24 u32 window | 28 u32 cdf_bits |
  *   32 u32 input_kind | 36 u32 serialisation = sep_mode | byte_group << 8 | byte_order << 16 |
- *   40 u32 vocab | 44 u32 n_win | 48 u64 weight_seed |
+ *   alphabet << 24 | 40 u32 vocab | 44 u32 n_win | 48 u64 weight_seed |
  *   56 u32 crc32 of the model shape | 60 u32 crc32 of bytes [0, 60) |
  *   64 u32 bitlen[n_win] | u32 crc_tok[n_win] | codes, ceil(bitlen/8) bytes each, in window order.
  * crc_tok[w] is the CRC-32 (IEEE 802.3) of window w's token ids as little-endian u16 bytes (the

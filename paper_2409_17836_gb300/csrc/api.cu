@@ -191,7 +191,7 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     // a prefill also leaves each logits row's maximum for the CDF kernel (the transposing fp32
     // epilogue, which takes vocabularies that are multiples of 32, computes it)
     NormArgs head = consume;
-    const bool with_max = !decode && c.vocab % 32 == 0;
+    const bool with_max = !decode && c.vocab % 32 == 0 && !c.alphabet;
     if (with_max) {
       cudaMemsetAsync(ctx->row_max, 0, (size_t)rows * 4, s);
       head.row_max = ctx->row_max;
@@ -375,9 +375,18 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   if (tpv < 0) return fail(nullptr, LMGC_ERR_INVALID, "bad input kind or separator mode");
   if (c.byte_group < 0 || c.byte_group > 8 || c.byte_order < 0 || c.byte_order > 1)
     return fail(nullptr, LMGC_ERR_INVALID, "byte_group must be 0..8 and byte_order 0 or 1");
+  if (c.alphabet != 0 && c.alphabet != 1) return fail(nullptr, LMGC_ERR_INVALID, "alphabet must be 0 or 1");
 
   lmgc_ctx* ctx = new lmgc_ctx();
   ctx->cfg = c;
+  if (c.alphabet) {
+    // the 16 hex digits, then the separator ids of sep_mode in ascending order
+    AlphaIds& a = ctx->alpha;
+    for (a.n = 0; a.n < 16; a.n++) a.id[a.n] = a.n;
+    if (c.sep_mode == LMGC_SEP_SPACE || c.sep_mode == LMGC_SEP_COMMA_SPACE) a.id[a.n++] = kTokSpace;
+    if (c.sep_mode == LMGC_SEP_COMMA || c.sep_mode == LMGC_SEP_COMMA_SPACE) a.id[a.n++] = kTokComma;
+    if (c.sep_mode == LMGC_SEP_SEMI) a.id[a.n++] = kTokSemi;
+  }
   cudaGetDevice(&ctx->device);
   ctx->hd = hd;
   ctx->qkv_dim = (c.n_heads + 2 * c.n_kv_heads) * hd;
@@ -549,6 +558,12 @@ lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, co
                            uint32_t* d_start, uint32_t* d_freq, lmgc_stream stream) {
   if (!ctx || (rows && (!d_logits || !d_sym || !d_start || !d_freq)))
     return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  if (ctx->cfg.alphabet) {
+    launch_cdf_pairs_alpha(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0,
+                           0, d_start, d_freq, 0, (cudaStream_t)stream, 0, ctx->alpha, ctx->d_err);
+    LMGC_CUDA(ctx, cudaGetLastError());
+    return check_err_word(ctx, (cudaStream_t)stream, "cdf_pairs");
+  }
   launch_cdf_pairs(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0, 0,
                    d_start, d_freq, 0, (cudaStream_t)stream);
   LMGC_CUDA(ctx, cudaGetLastError());
@@ -668,9 +683,16 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
     cudaEventRecord(ctx->batch_ev[2 * b + 1], s);
     {
       const int64_t rows = nb * W;
-      ProfScope ps(ctx, kCdf, (double)rows * ((double)c.vocab * 4 + 2 + 8), s);
-      launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
-                       ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
+      // per row: the logits the quantiser reads (the alphabet's ids only with alphabet 1), the
+      // token and the pair
+      const double cols = c.alphabet ? (double)ctx->alpha.n : (double)c.vocab;
+      ProfScope ps(ctx, kCdf, (double)rows * (cols * 4 + 2 + 8), s);
+      if (c.alphabet)
+        launch_cdf_pairs_alpha(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
+                               ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha, ctx->d_err);
+      else
+        launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
+                         ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
     }
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
   }
@@ -725,7 +747,8 @@ constexpr uint32_t kContainerVersion = 2;  // 2: per-window token checksums afte
 
 // header word at byte 36: the separator mode, and the byte grouping (0 for the default layout)
 static uint32_t serial_word(const lmgc_config& c) {
-  return (uint32_t)c.sep_mode | (uint32_t)c.byte_group << 8 | (uint32_t)c.byte_order << 16;
+  return (uint32_t)c.sep_mode | (uint32_t)c.byte_group << 8 | (uint32_t)c.byte_order << 16 |
+         (uint32_t)c.alphabet << 24;
 }
 
 static void container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h) {
@@ -908,8 +931,12 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
       k_dec_inputs<<<(unsigned)((nd + 127) / 128), 128, 0, s>>>(out, nd, W, pos, ctx->ws.tok_in);
       embed_rows(ctx, nd, s);
       forward_layers(ctx, nd, nd, true, pos, s);
-      launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
-                        ctx->d_err, s);
+      if (c.alphabet)
+        launch_dec_search_alpha(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos,
+                                d_len, ctx->alpha, ctx->d_err, s);
+      else
+        launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
+                          ctx->d_err, s);
     }
     // every restored window must reproduce the container's token checksum
     launch_window_crc(out, W, d_len, nd, d_crc, s);

@@ -466,3 +466,161 @@ void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint3
 }
 
 }  // namespace lmgc
+
+// ------------------------------------------------------------------------------------------
+// Restricted alphabet (a variant the paper does not describe): the integer CDF of a position is
+// taken over the logits of the na ids the serialisation can emit (ascending), and the coded
+// symbol is the token's index among them. One warp per row: lane j holds id alpha.id[j].
+// ------------------------------------------------------------------------------------------
+namespace lmgc {
+
+constexpr int kAlphaWarps = 8;
+
+// this lane's (start, freq) of the row's restricted CDF (lanes >= na: freq 0)
+__device__ __forceinline__ void alpha_cdf_lane(const float* __restrict__ z, const AlphaIds& alpha, int P,
+                                               const uint32_t* H, const uint32_t* L, uint32_t& start,
+                                               uint32_t& freq) {
+  const int lane = threadIdx.x & 31, na = alpha.n;
+  const bool in = lane < na;
+  const float zj = in ? __ldg(z + alpha.id[lane]) : -INFINITY;
+  float m = zj;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  const int a = in ? exp2_code(zj, m) : kAMax;
+  const uint32_t e = in ? exp2_from_code(a, H, L) : 0u;
+  RowStats st;
+  st.m = m;
+  st.S = warp_sum((uint64_t)e);
+  st.Mq = (1ull << P) - (uint64_t)na;
+  st.F = (uint32_t)((st.Mq << 32) / st.S);
+  const uint64_t g = in ? gfloor(e, st) : 0ull;
+  const uint64_t gall = warp_sum(g);
+  // the remainder goes to the lowest index whose exponent code is 0 (the largest e, 2^31)
+  const uint32_t top = __ballot_sync(0xffffffffu, in && a == 0);
+  const int amax = top ? __ffs(top) - 1 : -1;
+  uint32_t f = in ? (uint32_t)(1ull + g + (lane == amax ? st.Mq - gall : 0ull)) : 0u;
+  uint32_t inc = f;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  start = inc - f;
+  freq = f;
+}
+
+// the lane holding token t, or -1 (warp-uniform)
+__device__ __forceinline__ int alpha_index(const AlphaIds& alpha, int t) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t hit = __ballot_sync(0xffffffffu, lane < alpha.n && alpha.id[lane] == t);
+  return hit ? __ffs(hit) - 1 : -1;
+}
+
+// The pairs of k_cdf_pairs (same modes and output indexing) over the restricted alphabet.
+__global__ void __launch_bounds__(32 * kAlphaWarps) k_cdf_pairs_alpha(
+    const float* __restrict__ logits, int64_t rows, int V, int P, const uint32_t* __restrict__ tab,
+    const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win, int64_t stride_pos,
+    uint32_t* __restrict__ start, uint32_t* __restrict__ freq, int mode, int64_t pair_win0, AlphaIds alpha,
+    uint32_t* err) {
+  __shared__ uint32_t H[256], L[256];
+  for (int i = threadIdx.x; i < 256; i += 32 * kAlphaWarps) {
+    H[i] = tab[i];
+    L[i] = tab[256 + i];
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  for (int64_t r = (int64_t)blockIdx.x * kAlphaWarps + (threadIdx.x >> 5); r < rows;
+       r += (int64_t)gridDim.x * kAlphaWarps) {
+    int sym;
+    int64_t out_idx;
+    if (mode == 0) {
+      sym = tok[r];
+      out_idx = r;
+    } else {
+      const int64_t wl = r / W;
+      const int i = (int)(r - wl * W);
+      const int64_t gi = (first_win + wl) * W + i;
+      if (gi >= n_tok) continue;  // warp-uniform
+      sym = tok[gi];
+      out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
+    }
+    uint32_t st, fr;
+    alpha_cdf_lane(logits + r * (int64_t)V, alpha, P, H, L, st, fr);
+    const int s = alpha_index(alpha, sym);
+    if (s < 0) {
+      if (lane == 0) {
+        atomicOr(err, kErrCorrupt);  // a token outside the alphabet cannot be coded
+        start[out_idx] = 0;
+        freq[out_idx] = 1;
+      }
+    } else if (lane == s) {
+      start[out_idx] = st;
+      freq[out_idx] = fr;
+    }
+  }
+}
+
+void launch_cdf_pairs_alpha(const float* logits, int64_t rows, int V, int P, const uint32_t* tab,
+                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos,
+                            uint32_t* start, uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0,
+                            const AlphaIds& alpha, uint32_t* err) {
+  if (rows <= 0) return;
+  const int64_t blocks = std::min<int64_t>((rows + kAlphaWarps - 1) / kAlphaWarps, 152 * 16);
+  note_launch();
+  k_cdf_pairs_alpha<<<(unsigned)blocks, 32 * kAlphaWarps, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
+                                                                 pair_stride_pos, start, freq, mode, pair_win0, alpha,
+                                                                 err);
+}
+
+// k_dec_search over the restricted alphabet: one warp per decoding window.
+__global__ void __launch_bounds__(32 * kAlphaWarps) k_dec_search_alpha(
+    const float* __restrict__ logits, int64_t n, int V, int P, const uint32_t* __restrict__ tab,
+    DecState* __restrict__ states, const uint8_t* __restrict__ codes, uint16_t* __restrict__ sym_out,
+    int64_t sym_stride, int64_t pos, const uint32_t* __restrict__ win_len, AlphaIds alpha, uint32_t* err) {
+  __shared__ uint32_t H[256], L[256];
+  for (int i = threadIdx.x; i < 256; i += 32 * kAlphaWarps) {
+    H[i] = tab[i];
+    L[i] = tab[256 + i];
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int64_t w = (int64_t)blockIdx.x * kAlphaWarps + (threadIdx.x >> 5);
+  if (w >= n || (int64_t)win_len[w] <= pos) return;  // warp-uniform
+  DecState s = states[w];
+  const uint64_t r = s.R >> P;
+  const uint64_t t = s.D / r;
+  uint32_t st, fr;
+  alpha_cdf_lane(logits + w * (int64_t)V, alpha, P, H, L, st, fr);
+  const uint32_t hit = __ballot_sync(0xffffffffu, fr > 0 && (uint64_t)st <= t && t < (uint64_t)st + fr);
+  int j = hit ? __ffs(hit) - 1 : -1;
+  uint64_t lo = __shfl_sync(0xffffffffu, (uint64_t)st, j < 0 ? 0 : j);
+  uint64_t f = __shfl_sync(0xffffffffu, (uint64_t)fr, j < 0 ? 0 : j);
+  if (lane != 0) return;
+  if (t >= (1ull << P) || j < 0) {
+    atomicOr(err, kErrCorrupt);
+    j = 0;
+    lo = 0;
+    f = 1;
+  }
+  s.D -= r * lo;
+  s.R = r * f;
+  int k = __clzll((long long)s.R) - 2;
+  if (k < 0) k = 0;
+  const uint8_t* code = codes + s.code_off;
+  for (int i = 0; i < k; i++) s.D = (s.D << 1) | code_bit(code, s.nbits, s.bitpos + i);
+  s.bitpos += k;
+  s.R <<= k;
+  states[w] = s;
+  sym_out[w * sym_stride + pos] = alpha.id[j];
+}
+
+void launch_dec_search_alpha(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
+                             const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
+                             const uint32_t* win_len, const AlphaIds& alpha, uint32_t* err, cudaStream_t s) {
+  if (n <= 0) return;
+  note_launch();
+  k_dec_search_alpha<<<(unsigned)((n + kAlphaWarps - 1) / kAlphaWarps), 32 * kAlphaWarps, 0, s>>>(
+      logits, n, V, P, tab, (DecState*)dec_state, codes, sym_out, sym_stride, pos, win_len, alpha, err);
+}
+
+}  // namespace lmgc

@@ -58,6 +58,12 @@ struct Workspace {
   uint16_t* tok_in = nullptr;  // model input ids [rows]
 };
 
+// The restricted alphabet: ids id[0..n) ascending, 2 <= n <= 32, each < vocab.
+struct AlphaIds {
+  int32_t n;
+  int32_t id[32];
+};
+
 }  // namespace lmgc
 
 struct lmgc_ctx {
@@ -108,6 +114,7 @@ struct lmgc_ctx {
   bool fused_swiglu = false;  // gate/up interleaved, SwiGLU in the tcgen05 epilogue
   bool fused_rope = false;    // RoPE in the QKV tcgen05 epilogue
   bool fused_norm = false;    // RMSNorm folded into the GEMM epilogues (row scale + residual side outputs)
+  lmgc::AlphaIds alpha{};     // cfg.alphabet == 1: the ids the serialisation can emit
   std::string err;
 };
 
@@ -203,6 +210,15 @@ void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uin
                       const uint32_t* row_max = nullptr);
 void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
                          cudaStream_t s);
+// launch_cdf_pairs over the restricted alphabet (no row_max input); a token outside it sets
+// kErrCorrupt in *err and gets the pair (0, 1)
+void launch_cdf_pairs_alpha(const float* logits, int64_t rows, int V, int P, const uint32_t* tab,
+                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos,
+                            uint32_t* start, uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0,
+                            const AlphaIds& alpha, uint32_t* err);
+void launch_dec_search_alpha(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
+                             const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
+                             const uint32_t* win_len, const AlphaIds& alpha, uint32_t* err, cudaStream_t s);
 void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
                        const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
                        const uint32_t* win_len, uint32_t* err, cudaStream_t s);

@@ -34,7 +34,7 @@ class Config(C.Structure):
                 ("window", C.c_int32), ("cdf_bits", C.c_int32), ("sep_mode", C.c_int32),
                 ("input_kind", C.c_int32), ("batch_windows", C.c_int32), ("weight_seed", C.c_uint64),
                 ("init_std", C.c_float), ("rms_eps", C.c_float), ("rope_theta", C.c_float),
-                ("byte_group", C.c_int32), ("byte_order", C.c_int32)]
+                ("byte_group", C.c_int32), ("byte_order", C.c_int32), ("alphabet", C.c_int32)]
 
 
 @dataclasses.dataclass
@@ -57,12 +57,13 @@ class ModelConfig:
     rope_theta: float = 10000.0
     byte_group: int = 0  # bytes per separator group (Sec. 4.3 byte grouping); 0 = one group per value
     byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
+    alphabet: int = 0  # 1: integer CDFs over the ids the serialisation can emit only
 
     def c(self) -> Config:
         return Config(self.n_layers, self.d_model, self.n_heads, self.n_kv_heads, self.d_ffn, self.vocab, self.dtype,
                       self.window, self.cdf_bits, self.sep_mode, self.input_kind, self.batch_windows,
                       self.weight_seed, self.init_std, self.rms_eps, self.rope_theta, self.byte_group,
-                      self.byte_order)
+                      self.byte_order, self.alphabet)
 
 
 _lib = None

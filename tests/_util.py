@@ -13,7 +13,7 @@ def oracle_config(cfg, n_threads: int = 1) -> O.OracleConfig:
                           cdf_bits=cfg.cdf_bits, weight_seed=cfg.weight_seed, init_std=cfg.init_std,
                           rms_eps=cfg.rms_eps, rope_theta=cfg.rope_theta, sep_mode=cfg.sep_mode,
                           input_kind=cfg.input_kind, n_threads=n_threads, byte_group=cfg.byte_group,
-                          byte_order=cfg.byte_order)
+                          byte_order=cfg.byte_order, alphabet=cfg.alphabet)
 
 
 def cpu_threads() -> int:

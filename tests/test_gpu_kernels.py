@@ -201,3 +201,32 @@ def test_range_encode_rejects_bad_pairs():
     f = torch.zeros(4, dtype=torch.int32, device="cuda")  # freq 0 is invalid
     with pytest.raises(L.LmgcError):
         L.lmgc_range_encode(s, f, 16, 1, 4, None, 4, 1)
+
+
+@pytest.mark.parametrize("sep_mode,V,P", [(0, 32, 16), (2, 1000, 20), (4, 32000, 24)])
+def test_cdf_pairs_alphabet_bit_exact(sep_mode, V, P):
+    """Restricted-alphabet pairs: the quantiser over each row's alphabet logits (ascending ids)
+    and the token's index among them, bit-exact with the oracle's full quantiser applied to the
+    gathered columns; a token outside the alphabet is CORRUPT."""
+    ctx = L.Context(configs.with_(configs.TINY, vocab=V, cdf_bits=P, sep_mode=sep_mode, alphabet=1, batch_windows=1))
+    A = np.array(O.alphabet_ids(sep_mode))
+    rng = np.random.default_rng(V + sep_mode)
+    rows = 2000
+    z = logit_rows(rng, rows, V)
+    z[5, A[3]] = 50.0            # the alphabet's own maximum far above the rest of it
+    z[6, :] = -3.0
+    z[6, A[-1]] = 9.0            # ... at its last id
+    idx = rng.integers(0, A.size, rows)
+    idx[6] = A.size - 1
+    sym = A[idx].astype(np.uint16)
+    dz = torch.from_numpy(z).cuda()
+    st, fr = L.lmgc_cdf_pairs(ctx, dz, torch.from_numpy(sym.view(np.int16)).cuda())
+    rs, rf = O.cdf_pairs(np.ascontiguousarray(z[:, A]), idx.astype(np.uint16), P)
+    assert np.array_equal(st.cpu().numpy().view(np.uint32), rs)
+    assert np.array_equal(fr.cpu().numpy().view(np.uint32), rf)
+    bad = sym.copy()
+    bad[7] = 19  # BOS is context only, never coded
+    with pytest.raises(L.LmgcError) as e:
+        L.lmgc_cdf_pairs(ctx, dz, torch.from_numpy(bad.view(np.int16)).cuda())
+    assert e.value.status == L.ERR_CORRUPT
+    ctx.close()

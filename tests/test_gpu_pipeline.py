@@ -126,6 +126,47 @@ def test_byte_grouped_encode_decode_and_codes(group, order):
     ctx.close()
 
 
+@pytest.mark.parametrize("sep,group", [(0, 0), (2, 0), (4, 2)])
+def test_alphabet_encode_decode_and_codes(sep, group):
+    """Restricted-alphabet coding through the whole path: the container word carries the flag,
+    every window's code is bit-exact with the oracle's pairs over the alphabet columns of the
+    GPU's logits and its coder, decoding restores the tokens and values, the container is
+    within 0.5% of the oracle's own encode, no larger than the full-vocabulary container, and a
+    full-vocabulary context rejects it."""
+    cfg = configs.with_(configs.TINY, sep_mode=sep, byte_group=group, alphabet=1, batch_windows=4)
+    ctx = L.Context(cfg)
+    vals = I.tiny_gradient(6)[:1500]
+    tok = O.serialize(vals, sep, group, 0)
+    A = np.array(O.alphabet_ids(sep))
+    index = np.full(32, -1)
+    index[A] = np.arange(A.size)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert h["alphabet"] == 1 and h["sep_mode"] == sep and h["n_tok"] == tok.size
+    W = cfg.window
+    n_win = h["n_win"]
+    lg = L.lmgc_lm_probs(ctx, torch.from_numpy(tok.view(np.int16)).cuda(), 0, n_win).cpu().numpy()
+    for w in range(n_win):
+        n = min(W, tok.size - w * W)
+        t = tok[w * W: w * W + n]
+        st, fr = O.cdf_pairs(np.ascontiguousarray(lg[w, :n][:, A]), index[t].astype(np.uint16), cfg.cdf_bits)
+        code, nbits = O.range_encode(st, fr, cfg.cdf_bits)
+        assert h["bitlen"][w] == nbits and buf[h["offsets"][w]: h["offsets"][w + 1]] == code, w
+    toks = decode_all(ctx, buf, list(range(n_win)))
+    flat = np.concatenate([toks[w, :min(W, tok.size - w * W)] for w in range(n_win)])
+    assert np.array_equal(flat, tok)
+    assert O.deserialize(flat, 0, sep, group, 0).tobytes() == vals.tobytes()
+    ref = O.encode(oracle_config(cfg), vals, n_par=cpu_threads())
+    assert abs(len(buf) - len(ref)) <= 0.005 * len(ref), (len(buf), len(ref))
+    full = L.Context(configs.with_(cfg, alphabet=0))
+    assert len(buf) <= len(encode(full, vals))
+    with pytest.raises(L.LmgcError) as e:
+        decode_all(full, buf, [0])
+    assert e.value.status == L.ERR_CORRUPT
+    full.close()
+    ctx.close()
+
+
 @pytest.mark.parametrize("setting", ["quant16", "quant1", "sparse50", "sparse25"])
 def test_compatibility_inputs_round_trip(setting):
     """Sec. 5 compatibility inputs one at a time through the whole path: Eq. 4 indices of every
