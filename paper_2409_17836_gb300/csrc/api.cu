@@ -156,8 +156,13 @@ static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, i
 // One forward of the model over `rows` input rows already embedded into ws.x.
 //   prefill: rows = n_win * W, row r at position r mod W, keys/values from ws.qkv itself
 //   decode:  rows = n_win, every row at position pos; keys/values from the cache
-static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool decode, int64_t pos, cudaStream_t s) {
+// narrow: the vocabulary projection over the restricted alphabet's rows only (w_head_alpha,
+// logits [rows][kAlphaCols]) instead of all V rows.
+static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool decode, int64_t pos, cudaStream_t s,
+                           bool narrow = false) {
   const lmgc_config& c = ctx->cfg;
+  const void* w_head = narrow ? ctx->w_head_alpha : ctx->w_head;
+  const int64_t n_head = narrow ? kAlphaCols : c.vocab;
   const int d = c.d_model, F = c.d_ffn, hd = ctx->hd, qd = c.n_heads * hd;
   Workspace& ws = ctx->ws;
   const int64_t W = c.window;
@@ -191,12 +196,12 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     // a prefill also leaves each logits row's maximum for the CDF kernel (the transposing fp32
     // epilogue, which takes vocabularies that are multiples of 32, computes it)
     NormArgs head = consume;
-    const bool with_max = !decode && c.vocab % 32 == 0 && !c.alphabet;
+    const bool with_max = !decode && !narrow && c.vocab % 32 == 0;
     if (with_max) {
       cudaMemsetAsync(ctx->row_max, 0, (size_t)rows * 4, s);
       head.row_max = ctx->row_max;
     }
-    gemm(ctx, xh, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s, nullptr, &head);
+    gemm(ctx, xh, w_head, ctx->logits, rows, n_head, d, kStoreF32, s, nullptr, &head);
     ctx->row_max_valid = with_max;
     return;
   }
@@ -241,7 +246,7 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     ProfScope ps(ctx, kNorm, 0, s);
     launch_rmsnorm(ws.x, rows, d, c.rms_eps, ws.n, c.dtype, s);
   }
-  gemm(ctx, ws.n, ctx->w_head, ctx->logits, rows, c.vocab, d, kStoreF32, s);
+  gemm(ctx, ws.n, w_head, ctx->logits, rows, n_head, d, kStoreF32, s);
   ctx->row_max_valid = false;
 }
 
@@ -256,7 +261,7 @@ static void embed_rows(lmgc_ctx* ctx, int64_t rows, cudaStream_t s) {
 
 // Model logits for windows [first_win, first_win + nb) of a token stream, into ctx->logits.
 static void forward_windows(lmgc_ctx* ctx, const uint16_t* tok, int64_t n_tok, int64_t first_win, int64_t nb,
-                            cudaStream_t s) {
+                            cudaStream_t s, bool narrow = false) {
   const lmgc_config& c = ctx->cfg;
   const int64_t rows = nb * c.window;
   {
@@ -264,7 +269,7 @@ static void forward_windows(lmgc_ctx* ctx, const uint16_t* tok, int64_t n_tok, i
     launch_window_inputs(tok, n_tok, first_win, nb, c.window, ctx->ws.tok_in, s);
     embed_rows(ctx, rows, s);
   }
-  forward_layers(ctx, rows, nb, false, 0, s);
+  forward_layers(ctx, rows, nb, false, 0, s, narrow);
 }
 
 template <typename T>
@@ -343,7 +348,7 @@ lmgc_status lmgc_destroy(lmgc_ctx* ctx) {
   cudaDeviceSynchronize();
   void* ptrs[] = {ctx->weights_blob, ctx->rope_cs, ctx->exp2_tab, ctx->ws.x, ctx->ws.n, ctx->ws.qkv, ctx->ws.att,
                   ctx->ws.act, ctx->ws.gu, ctx->ws.ss, ctx->ws.tok_in, ctx->logits, ctx->row_max, ctx->d_err, ctx->tok, ctx->pair_start,
-                  ctx->win_len, ctx->host_in, ctx->host_out, ctx->kv_cache};
+                  ctx->win_len, ctx->host_in, ctx->host_out, ctx->kv_cache, ctx->w_head_alpha};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& e : ctx->ev)
@@ -454,6 +459,17 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
     launch_init_weights(L.wdown, dt, seed, t + 6, d, F, F, 0, c.init_std, s);
   }
   launch_init_weights(ctx->w_head, dt, seed, 1 + 7 * c.n_layers, V, d, d, 0, c.init_std, s);
+  if (c.alphabet) {
+    // the restricted alphabet's rows of the vocabulary weight in their order, zero rows after
+    const size_t row = (size_t)d * ctx->elt;
+    err = cudaMalloc(&ctx->w_head_alpha, kAlphaCols * row);
+    if (err == cudaSuccess) err = cudaMemsetAsync(ctx->w_head_alpha, 0, kAlphaCols * row, s);
+    for (int j = 0; j < ctx->alpha.n && err == cudaSuccess; j++)
+      err = cudaMemcpyAsync((char*)ctx->w_head_alpha + j * row, (const char*)ctx->w_head + ctx->alpha.id[j] * row, row,
+                            cudaMemcpyDeviceToDevice, s);
+    ctx->alpha_cols.n = ctx->alpha.n;
+    for (int j = 0; j < ctx->alpha.n; j++) ctx->alpha_cols.id[j] = j;
+  }
   // RoPE table: angle pos * theta^(-2i/hd) in binary64, stored as fp32 (cos, sin)
   {
     std::vector<float2> cs((size_t)c.window * (hd / 2));
@@ -482,7 +498,8 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->fused_norm = ctx->fused_norm && ctx->fused_rope && ctx->fused_swiglu;
   if (err == cudaSuccess && ctx->fused_norm) err = dmalloc(&ws.ss, R * (size_t)(d / 128) * 4);
   if (err == cudaSuccess) err = dmalloc(&ws.tok_in, R * 2);
-  if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * V * 4);
+  // [R][V], or [R][kAlphaCols] rows of the narrow head when that is wider
+  if (err == cudaSuccess) err = dmalloc(&ctx->logits, R * std::max<int64_t>(V, kAlphaCols) * 4);
   if (err == cudaSuccess) err = dmalloc(&ctx->row_max, R * 4);
   for (int i = 0; i < 6 && err == cudaSuccess; i++) err = cudaEventCreate(&ctx->ev[i]);
   if (err == cudaSuccess) err = cudaDeviceSynchronize();
@@ -679,7 +696,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   for (int64_t b = 0; b < n_batches; b++) {
     const int64_t w0 = w_begin + b * c.batch_windows;
     const int64_t nb = std::min<int64_t>(c.batch_windows, w_begin + n_win - w0);
-    forward_windows(ctx, ctx->tok, n_tok, w0, nb, s);
+    forward_windows(ctx, ctx->tok, n_tok, w0, nb, s, c.alphabet != 0);
     cudaEventRecord(ctx->batch_ev[2 * b + 1], s);
     {
       const int64_t rows = nb * W;
@@ -688,8 +705,8 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
       const double cols = c.alphabet ? (double)ctx->alpha.n : (double)c.vocab;
       ProfScope ps(ctx, kCdf, (double)rows * (cols * 4 + 2 + 8), s);
       if (c.alphabet)
-        launch_cdf_pairs_alpha(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
-                               ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha, ctx->d_err);
+        launch_cdf_pairs_alpha(ctx->logits, rows, kAlphaCols, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0,
+                               n_win, ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha_cols, ctx->d_err);
       else
         launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
                          ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
@@ -930,10 +947,10 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
       note_launch();
       k_dec_inputs<<<(unsigned)((nd + 127) / 128), 128, 0, s>>>(out, nd, W, pos, ctx->ws.tok_in);
       embed_rows(ctx, nd, s);
-      forward_layers(ctx, nd, nd, true, pos, s);
+      forward_layers(ctx, nd, nd, true, pos, s, c.alphabet != 0);
       if (c.alphabet)
-        launch_dec_search_alpha(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos,
-                                d_len, ctx->alpha, ctx->d_err, s);
+        launch_dec_search_alpha(ctx->logits, nd, kAlphaCols, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos,
+                                d_len, ctx->alpha_cols, ctx->d_err, s);
       else
         launch_dec_search(ctx->logits, nd, c.vocab, c.cdf_bits, ctx->exp2_tab, d_state, d_in, out, W, pos, d_len,
                           ctx->d_err, s);

@@ -58,6 +58,9 @@ struct Workspace {
   uint16_t* tok_in = nullptr;  // model input ids [rows]
 };
 
+// Columns of the restricted alphabet's logits rows (its ids, then zero-weight padding).
+constexpr int kAlphaCols = 32;
+
 // The restricted alphabet: ids id[0..n) ascending, 2 <= n <= 32, each < vocab.
 struct AlphaIds {
   int32_t n;
@@ -115,6 +118,8 @@ struct lmgc_ctx {
   bool fused_rope = false;    // RoPE in the QKV tcgen05 epilogue
   bool fused_norm = false;    // RMSNorm folded into the GEMM epilogues (row scale + residual side outputs)
   lmgc::AlphaIds alpha{};     // cfg.alphabet == 1: the ids the serialisation can emit
+  lmgc::AlphaIds alpha_cols{};  // the same as columns 0..n-1 of the narrow logits rows
+  void* w_head_alpha = nullptr;  // [kAlphaCols][d]: alpha's rows of w_head, then zero rows
   std::string err;
 };
 

@@ -167,6 +167,37 @@ def test_alphabet_encode_decode_and_codes(sep, group):
     ctx.close()
 
 
+def test_tinyllama_shape_alphabet_narrow_head():
+    """Restricted alphabet on the tensor-core path: encode and decode project onto the alphabet's
+    17 rows of the vocabulary weight only (a 32-column GEMM), and every window's code is
+    bit-exact with the oracle's pairs over those columns of the full 32,000-column logits of
+    lmgc_lm_probs, so the narrow projection reproduces the full one's columns exactly. The
+    partial last window decodes back to its tokens."""
+    cfg = configs.with_(configs.TINYLLAMA, n_layers=1, batch_windows=2, alphabet=1)
+    ctx = L.Context(cfg)
+    W = cfg.window
+    vals = I.convnet_gradient(1)[: (2 * W + 700) // 9]
+    tok = O.serialize(vals, 0)
+    n_win = -(-tok.size // W)
+    A = np.array(O.alphabet_ids(0))
+    index = np.full(32, -1)
+    index[A] = np.arange(A.size)
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert h["alphabet"] == 1 and h["n_win"] == n_win == 3
+    dtok = torch.from_numpy(tok.view(np.int16)).cuda()
+    for w in range(n_win):
+        n = min(W, tok.size - w * W)
+        lg = L.lmgc_lm_probs(ctx, dtok, w, 1)[0, :n].cpu().numpy()
+        t = tok[w * W: w * W + n]
+        st, fr = O.cdf_pairs(np.ascontiguousarray(lg[:, A]), index[t].astype(np.uint16), cfg.cdf_bits)
+        code, nbits = O.range_encode(st, fr, cfg.cdf_bits)
+        assert h["bitlen"][w] == nbits and buf[h["offsets"][w]: h["offsets"][w + 1]] == code, w
+    last = decode_all(ctx, buf, [n_win - 1])[0, : tok.size - (n_win - 1) * W]
+    assert np.array_equal(last, tok[(n_win - 1) * W:])
+    ctx.close()
+
+
 @pytest.mark.parametrize("setting", ["quant16", "quant1", "sparse50", "sparse25"])
 def test_compatibility_inputs_round_trip(setting):
     """Sec. 5 compatibility inputs one at a time through the whole path: Eq. 4 indices of every
