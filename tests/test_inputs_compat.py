@@ -33,3 +33,18 @@ def test_16bit_codes_as_byte_pairs():
     assert np.array_equal(O.deserialize(tok, 1, 0, group, 0), b)
     c, g8 = I.code_bytes(np.array([5, 250], dtype=np.uint8))
     assert g8 == 0 and c.tolist() == [5, 250]
+
+
+def test_lossy_codes_top_k_and_eq4_ends():
+    """The lossy input (top 10% by magnitude, then 8-bit Eq. 4 over the kept values): the kept
+    values stay in index order, a magnitude tie goes to the lower index, the kept minimum codes to
+    0 and the maximum to 255, and a value in between to rint of its place in the range."""
+    g = np.zeros(40, dtype=np.float32)
+    g[[3, 9, 17, 25, 31]] = [-4.0, 1.0, 6.0, -1.0, 2.0]  # |1.0| ties at indices 9 and 25
+    # k = floor(0.1 * 40) = 4: -4, 6, 2 and the lower-index 1.0 (index 9)
+    codes = I.lossy_codes(g, keep=0.1)
+    assert codes.dtype == np.uint8 and codes.tolist() == [0, 128, 255, 153]
+    # (1 + 4) / 10 * 255 = 127.5 -> 128 after rint (ties to even), (2 + 4) / 10 * 255 = 153
+    assert round((1 + 4) / 10 * 255) == 128 and np.rint(5 / 10 * 255) == 128
+    big = I.lossy_codes(I.convnet_gradient(0))
+    assert big.size == 29895 and big.min() == 0 and big.max() == 255

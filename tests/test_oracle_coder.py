@@ -83,6 +83,31 @@ def test_matches_bigint_spec_and_bound(P):
         assert [dec.step(c, P) for c in cdfs] == sym
 
 
+def test_ten_thousand_windows_against_bigint_spec():
+    """10^4 independent short windows with random P in 1..31, random lengths (empty included) and
+    random pairs drawn directly (any start in [0, T - freq], freq in [1, T], with runs of
+    probability-one tokens and of the smallest freq): each window's code from the C coder equals
+    the arbitrary-precision restatement bit for bit."""
+    rng = np.random.default_rng(2409)
+    for w in range(10_000):
+        P = int(rng.integers(1, 32))
+        T = 2 ** P
+        n = int(rng.integers(0, 24))
+        kind = w % 4
+        if kind == 0:
+            fr = rng.integers(1, T + 1, n)
+        elif kind == 1:  # long runs of the smallest freq: one renormalisation step per token
+            fr = np.ones(n, dtype=np.int64)
+        elif kind == 2:  # probability-one tokens mixed in
+            fr = np.where(rng.random(n) < 0.5, T, rng.integers(1, T + 1, n))
+        else:  # freq near T, start at the top of the range (the carry-heavy case)
+            fr = np.maximum(1, T - rng.integers(0, 4, n))
+        st = np.array([int(rng.integers(0, T - f + 1)) if kind != 3 else T - int(f) for f in fr], dtype=np.int64)
+        data, nbits = O.range_encode(st.astype(np.uint32), fr.astype(np.uint32), P)
+        code, nb = spec.encode(st.tolist(), fr.tolist(), P)
+        assert nb == nbits and data == spec.code_bytes(code, nb), (w, P, n)
+
+
 def test_uniform_closed_form():
     """V = 32 equiprobable symbols at P = 16: l = 5n + 1 and the first 5n bits are the
     symbols' 5-bit binary codes, concatenated."""

@@ -171,3 +171,57 @@ def test_zero_weights_give_zero_logits():
     c = cfg(init_std=0.0)
     lg = O.window_logits(c, np.arange(10, dtype=np.uint16), 10)
     assert np.all(lg == 0.0)
+
+
+def test_one_layer_one_head_two_positions_by_hand():
+    """A 1-layer, 1-head, W = 2 model written out scalar by scalar (plain Python floats, no
+    library routine): position 0 sees only itself, so its attention output is v_0; position 1
+    mixes v_0 and v_1 with the softmax of its two scaled scores; RoPE turns the pairs (i, i + hd/2)
+    of position 1 by 1 * theta^(-2i/hd) radians and leaves position 0 as it is."""
+    d, hd, Fd, V = 4, 4, 3, 20
+    c = cfg(n_layers=1, d_model=d, n_heads=1, n_kv_heads=1, d_ffn=Fd, vocab=V, window=2, init_std=0.5)
+    t0, t1 = 7, 3
+
+    def W(tid, rows, cols):
+        w = O.weight_tensor(c.weight_seed, tid, rows * cols, c.init_std, False).astype(np.float64).tolist()
+        return [w[r * cols:(r + 1) * cols] for r in range(rows)]
+
+    def matvec(M, x):
+        return [sum(M[r][j] * x[j] for j in range(len(x))) for r in range(len(M))]
+
+    def norm(x):
+        s = 1.0 / math.sqrt(sum(v * v for v in x) / len(x) + c.rms_eps)
+        return [v * s for v in x]
+
+    def rope(x, pos):
+        out = list(x)
+        for i in range(hd // 2):
+            ang = pos * c.rope_theta ** (-2.0 * i / hd)
+            a, b = x[i], x[i + hd // 2]
+            out[i] = a * math.cos(ang) - b * math.sin(ang)
+            out[i + hd // 2] = b * math.cos(ang) + a * math.sin(ang)
+        return out
+
+    E, Wq, Wk, Wv, Wo = W(0, V, d), W(1, hd, d), W(2, hd, d), W(3, hd, d), W(4, d, hd)
+    Wg, Wu, Wd, Wh = W(5, Fd, d), W(6, Fd, d), W(7, d, Fd), W(8, V, d)
+    xs = [list(E[O.TOK_BOS]), list(E[t0])]  # inputs: BOS, then the window's first token
+    ns = [norm(x) for x in xs]
+    q = [rope(matvec(Wq, ns[p]), p) for p in range(2)]
+    k = [rope(matvec(Wk, ns[p]), p) for p in range(2)]
+    v = [matvec(Wv, ns[p]) for p in range(2)]
+    s0 = sum(q[1][i] * k[0][i] for i in range(hd)) / math.sqrt(hd)
+    s1 = sum(q[1][i] * k[1][i] for i in range(hd)) / math.sqrt(hd)
+    w0 = 1.0 / (1.0 + math.exp(s1 - s0))
+    att = [v[0], [w0 * v[0][i] + (1.0 - w0) * v[1][i] for i in range(hd)]]
+    logits = []
+    for p in range(2):
+        x = [xs[p][i] + o for i, o in enumerate(matvec(Wo, att[p]))]
+        n2 = norm(x)
+        g, u = matvec(Wg, n2), matvec(Wu, n2)
+        a = [g[j] / (1.0 + math.exp(-g[j])) * u[j] for j in range(Fd)]
+        x = [x[i] + o for i, o in enumerate(matvec(Wd, a))]
+        logits.append(matvec(Wh, norm(x)))
+    lg = O.window_logits(c, np.array([t0, t1], dtype=np.uint16), 2)
+    # fp64 on both sides, different operation order: agreement to rounding (logits are O(1))
+    np.testing.assert_allclose(lg, np.array(logits), rtol=1e-10, atol=1e-12)
+    assert np.abs(lg).max() > 0.1
