@@ -68,11 +68,18 @@ def lib():
             "orc_decode_window": (i32, [vp, i32, vp, i64, i64, vp]),
             "orc_crc32": (u32, [vp, i64]),
             "orc_num_threads": (i32, []),
+            "orc_cfg_layout": (C.c_size_t, [vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
             fn.restype = res
             fn.argtypes = args
+        # the C struct this binding copies: its size and every field's offset but the last array
+        off = (C.c_size_t * 14)()
+        size = L.orc_cfg_layout(off)
+        names = [f for f, _ in _Cfg._fields_]
+        if size != C.sizeof(_Cfg) or [getattr(_Cfg, f).offset for f in names[:14]] != list(off):
+            raise RuntimeError("oracle: the binding's _Cfg does not match orc_cfg")
         _lib = L
     return _lib
 

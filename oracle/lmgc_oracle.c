@@ -27,6 +27,7 @@
  * Build: gcc -O2 -std=c11 -fPIC -shared -ffp-contract=off -fopenmp -o liblmgc_oracle.so
  */
 #include <math.h>
+#include <stddef.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -239,6 +240,18 @@ typedef struct {
   int32_t n_alpha;
   uint16_t alpha[32];
 } orc_cfg;
+
+/* sizeof(orc_cfg), and the offsets of its 14 fields in declaration order into off[0..13], so that
+ * a binding can check its copy of the struct */
+size_t orc_cfg_layout(size_t* off) {
+  const size_t o[14] = {offsetof(orc_cfg, n_layers),   offsetof(orc_cfg, d_model),   offsetof(orc_cfg, n_heads),
+                        offsetof(orc_cfg, n_kv_heads), offsetof(orc_cfg, d_ffn),     offsetof(orc_cfg, vocab),
+                        offsetof(orc_cfg, bf16),       offsetof(orc_cfg, window),    offsetof(orc_cfg, weight_seed),
+                        offsetof(orc_cfg, init_std),   offsetof(orc_cfg, rms_eps),   offsetof(orc_cfg, rope_theta),
+                        offsetof(orc_cfg, n_threads),  offsetof(orc_cfg, n_alpha)};
+  for (int i = 0; i < 14; i++) off[i] = o[i];
+  return sizeof(orc_cfg);
+}
 
 enum { ORC_WQ = 0, ORC_WK, ORC_WV, ORC_WO, ORC_WGATE, ORC_WUP, ORC_WDOWN };
 

@@ -28,3 +28,39 @@ def test_binding_names_match_header():
     assert sorted(lmgc.SYMBOLS) == declared_symbols()
     for s in declared_symbols():
         assert callable(getattr(lmgc, s)), s
+
+
+def test_config_layout_and_constants_match_header(tmp_path):
+    """The binding's lmgc_config matches the header's struct field by field (offsets, size), and
+    its status, dtype, separator and input-kind constants equal the header's enums: a C program
+    compiled against include/lmgc.h prints them."""
+    import subprocess
+
+    from paper_2409_17836_gb300 import lmgc as L
+
+    fields = [f for f, _ in L.Config._fields_]
+    consts = {"OK": "LMGC_OK", "ERR_INVALID": "LMGC_ERR_INVALID", "ERR_NO_SPACE": "LMGC_ERR_NO_SPACE",
+              "ERR_CUDA": "LMGC_ERR_CUDA", "ERR_CORRUPT": "LMGC_ERR_CORRUPT", "ERR_LIMIT": "LMGC_ERR_LIMIT",
+              "ERR_NOMEM": "LMGC_ERR_NOMEM", "F32": "LMGC_F32", "BF16": "LMGC_BF16", "SEP_SPACE": "LMGC_SEP_SPACE",
+              "SEP_COMMA": "LMGC_SEP_COMMA", "SEP_COMMA_SPACE": "LMGC_SEP_COMMA_SPACE", "SEP_SEMI": "LMGC_SEP_SEMI",
+              "SEP_NONE": "LMGC_SEP_NONE", "IN_F32": "LMGC_IN_F32", "IN_U8": "LMGC_IN_U8"}
+    src = ["#include <stdio.h>", "#include <stddef.h>", '#include "lmgc.h"', "int main(void) {",
+           '  printf("size %zu\\n", sizeof(lmgc_config));']
+    src += [f'  printf("off {f} %zu\\n", offsetof(lmgc_config, {f}));' for f in fields]
+    src += [f'  printf("const {k} %d\\n", (int){v});' for k, v in consts.items()]
+    src += ["  return 0;", "}"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(c), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    got = {}
+    for line in out:
+        if line:
+            kind, *rest = line.split()
+            got[(kind, rest[0]) if kind != "size" else ("size",)] = int(rest[-1])
+    assert got[("size",)] == ctypes.sizeof(L.Config)
+    for f in fields:
+        assert got[("off", f)] == getattr(L.Config, f).offset, f
+    for k in consts:
+        assert got[("const", k)] == getattr(L, k), k
