@@ -153,7 +153,9 @@ lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c
  * integers, Sec. 4.1). For a row z[0..V) with T = 2^P: m = max z; y_j = fp32(fp32(z_j - m) *
  * fp32(2^16 log2 e)); a_j = -rint(y_j) clamped to 40*2^16; e_j = 2^31 * 2^(-a_j/65536) in fixed
  * point from two 256-entry tables; g_j = floor(e_j (T - V) / sum e); freq_j = 1 + g_j with the
- * remainder added to the lowest-index largest e_j; cdf[0] = 0, cdf[V] = T.
+ * remainder added to the lowest-index largest e_j; cdf[0] = 0, cdf[V] = T. Rows always span the
+ * whole vocabulary: the restricted alphabet (lmgc_config.alphabet) does not apply here; its CDF
+ * is this one applied to the row's alphabet columns.
  * d_logits: fp32 [rows][V]; d_cdf: uint32 [rows][V+1]. Errors: INVALID, CUDA. */
 lmgc_status lmgc_quantize_cdf(lmgc_ctx* ctx, const float* d_logits, size_t rows, uint32_t* d_cdf,
                               lmgc_stream stream);
