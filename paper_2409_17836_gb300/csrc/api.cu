@@ -617,9 +617,9 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
     launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
     uint64_t total = 0;
     uint32_t herr = 0;
-    cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
-    cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
-    e = cudaStreamSynchronize(s);
+    e = cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) st = cuda_fail(nullptr, e, "range_encode");
     else if (herr) st = fail(nullptr, LMGC_ERR_INVALID, "range_encode: invalid (start, freq) or window length");
     else {
@@ -903,7 +903,7 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   // decode batch: as many of the requested windows as a KV cache of half the free device memory
   // (at most 64 GiB) holds -- a step's GEMMs cost about the same for 64 rows as for 256
   size_t free_b = 0, total_b = 0;
-  cudaMemGetInfo(&free_b, &total_b);
+  LMGC_CUDA(ctx, cudaMemGetInfo(&free_b, &total_b));
   const size_t kv_budget = std::max<size_t>(ctx->kv_cap, std::min<size_t>(free_b / 2, 64ull << 30));
   // (one workspace row per window: at most batch_windows * W of them)
   const int64_t nd_max = std::max<int64_t>(
