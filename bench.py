@@ -570,7 +570,9 @@ def main():
                           "parallelism": f"windows sharded over {world} GPU(s), no collective on the data path"},
                "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
                "stages": stages, "microbench": micro, "stage_ms_last_step": L.lmgc_stage_times(ctx),
-               "compression_rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv), "cpu_baseline": cpu}
+               "compression_rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv),
+               "bits_per_token": 8.0 * statistics.mean(sizes) / L.lmgc_serial_tokens(ctx, per_step),
+               "cpu_baseline": cpu}
         print(json.dumps(res), flush=True)
     ctx.close()
     if world > 1:
