@@ -13,7 +13,7 @@
  *                          only; decoding runs until the window is full.
  *   LM prior ............. Eq. 1 / Eq. 2 with a Llama-family decoder (Sec. 4.1 names
  *                          TinyLlama / OpenLLaMA / Llama 2), fp64 arithmetic.
- *   integer CDF .......... implied by "adapted the arithmetic coding from Torchac"
+ *   integer CDF .......... implied by the Torchac-based coder of Sec. 4.1 (integer CDFs)
  *                          (Sec. 4.1 "Implementation"): an integer-exact quantiser.
  *   arithmetic coder ..... Sec. 2 "Arithmetic coding" (interval subdivision, any number of
  *                          the final interval represents the message) in an exact integer form.
@@ -609,8 +609,8 @@ int64_t orc_range_encode(const uint32_t* start, const uint32_t* freq, int64_t n,
   return len;
 }
 
-/* Decoder (Sec. 2: "the decoder ... reconstructs the data by repeatedly looking up the
- * intervals"). D = first 62 bits of the code (zero padded). Per symbol: r = R >> P;
+/* Decoder (Sec. 2: decoding walks the same interval subdivision, finding at each step the
+ * symbol whose interval holds the code). D = first 62 bits of the code (zero padded). Per symbol: r = R >> P;
  * t = D / r (t >= T means a corrupt code); s with cdf[s] <= t < cdf[s+1]; D -= r * cdf[s];
  * R = r * f_s; renormalise by the same k as the encoder, shifting the next k code bits into D. */
 typedef struct {
