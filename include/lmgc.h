@@ -23,7 +23,8 @@
  *
  * Token alphabet (character-level reading of Sec. 3 / Fig. 1): hex digit v -> id v (0..15),
  * ' ' -> 16, ',' -> 17, ';' -> 18, BOS -> 19. The model's vocabulary has `vocab` >= 20 ids; the
- * coder codes over all of them (Eq. 2 is a distribution over the whole vocabulary).
+ * coder codes over all of them (Eq. 2 is a distribution over the whole vocabulary), or, with
+ * lmgc_config.alphabet = 1, over the ids the serialisation can emit only.
  */
 #ifndef LMGC_H
 #define LMGC_H
@@ -249,7 +250,8 @@ lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t*
  * window, so its logits -- and hence its CDFs -- are bit-identical to the encoder's. Windows
  * are decoded in batches of as many as a KV cache of half the free device memory (at most
  * 64 GiB) holds; the context keeps that cache for later calls (lmgc_destroy frees it).
- * Errors: CORRUPT (bad header, model mismatch, a code that leaves its interval, or a restored
+ * Errors: CORRUPT (bad header, a model or serialisation word -- separators, byte grouping and
+ * order, alphabet -- other than the context's, a code that leaves its interval, or a restored
  * window whose token checksum differs from the container's), INVALID
  * (window id out of range), NO_SPACE (cap_tok < n_ids * W), CUDA. Syncs. */
 lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, const uint32_t* h_win_ids,
