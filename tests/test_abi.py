@@ -64,3 +64,34 @@ def test_config_layout_and_constants_match_header(tmp_path):
         assert got[("off", f)] == getattr(L.Config, f).offset, f
     for k in consts:
         assert got[("const", k)] == getattr(L, k), k
+
+
+def test_create_rejects_bad_configs_before_any_cuda_call():
+    """lmgc_create validates the configuration before it touches the device, so every rejection
+    is checkable without a GPU: INVALID and a message naming the problem."""
+    from paper_2409_17836_gb300 import configs
+    from paper_2409_17836_gb300 import lmgc as L
+
+    lib = L.load()
+    cases = [
+        (dict(vocab=19), "bad model shape"),                              # the 20 reserved ids
+        (dict(n_heads=3), "bad model shape"),                             # d_model % n_heads
+        (dict(n_heads=4, n_kv_heads=3), "bad model shape"),               # n_heads % n_kv_heads
+        (dict(d_model=96, n_heads=2, n_kv_heads=2), "head dim"),          # hd 48
+        (dict(cdf_bits=31), "cdf_bits"),
+        (dict(vocab=70000, cdf_bits=16), "cdf_bits"),                     # 2^P must exceed V
+        (dict(dtype=7), "dtype"),
+        (dict(sep_mode=5), "separator mode"),
+        (dict(input_kind=2), "input kind"),
+        (dict(byte_group=9), "byte_group"),
+        (dict(byte_order=2), "byte_order"),
+        (dict(alphabet=2), "alphabet"),
+    ]
+    for kw, fragment in cases:
+        c = configs.with_(configs.TINY, **kw).c()
+        h = ctypes.c_void_p()
+        st = lib.lmgc_create(ctypes.byref(c), ctypes.byref(h))
+        assert st == L.ERR_INVALID and not h.value, (kw, st)
+        buf = ctypes.create_string_buffer(512)
+        lib.lmgc_last_error(None, buf, 512)
+        assert fragment in buf.value.decode(), (kw, buf.value)
