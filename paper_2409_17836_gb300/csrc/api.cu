@@ -124,11 +124,12 @@ static void prof_collect(lmgc_ctx* ctx) {
   ctx->prof.pending.clear();
 }
 
-// ---- GEMM dispatch: tcgen05 for bf16 when the shape fits, CUDA cores otherwise ----
+// ---- GEMM dispatch by the model's dtype: a bf16-weight model runs every contraction on the
+// tcgen05 kernel (lmgc_create rejects shapes it does not take), an fp32 model on CUDA cores ----
 static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi,
                  cudaStream_t s, const RopeArgs* rope = nullptr, const NormArgs* norm = nullptr) {
   ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
-  if (ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi))
+  if (ctx->cfg.dtype == LMGC_BF16)
     launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s, rope, norm);
   else
     launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi == kAddResidualWide ? (int)kAddResidual : epi,
@@ -143,7 +144,7 @@ static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, i
   for (int64_t p = pos_first; p < pos_first + n_pos; p++) pairs += (double)(p + 1);
   ProfScope ps(ctx, kAttn, 4.0 * ctx->hd * c.n_heads * pairs * (double)n_win, s);
   const int qd = c.n_heads * ctx->hd, kd = c.n_kv_heads * ctx->hd;
-  if (c.dtype == LMGC_BF16 && ctx->use_tc && tc_attention_supported(ctx->hd, ctx->qkv_dim)) {
+  if (c.dtype == LMGC_BF16) {  // lmgc_create admitted only head layouts the tcgen05 kernel takes
     const int64_t q_rows = q_win_stride == 1 ? n_win : n_win * c.window;
     launch_attention_tc(q, q_rows, kv, n_win * c.window, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads,
                         c.n_kv_heads, ctx->hd, c.window, n_win, pos_first, n_pos, q_win_stride, ctx->d_err, s);
@@ -372,6 +373,8 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
     return fail(nullptr, LMGC_ERR_INVALID, "bad model shape");
   const int hd = c.d_model / c.n_heads;
   if (hd != 32 && hd != 64 && hd != 128) return fail(nullptr, LMGC_ERR_INVALID, "head dim must be 32, 64 or 128");
+  if (c.dtype == LMGC_BF16 && hd == 32)
+    return fail(nullptr, LMGC_ERR_INVALID, "head dim of a bf16 model must be 64 or 128 (tcgen05 attention)");
   if (c.d_model % 8 || c.d_ffn % 8) return fail(nullptr, LMGC_ERR_INVALID, "d_model and d_ffn must be multiples of 8");
   if (c.cdf_bits < 1 || c.cdf_bits > 30 || (int64_t)c.vocab >= (1ll << c.cdf_bits))
     return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must satisfy vocab < 2^cdf_bits <= 2^30");
@@ -397,15 +400,24 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->qkv_dim = (c.n_heads + 2 * c.n_kv_heads) * hd;
   ctx->tpv = tpv;
   ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
-  const char* tc_env = getenv("LMGC_DISABLE_TC");
-  ctx->use_tc = !(tc_env && tc_env[0] == '1');
-  ctx->fused_rope = c.dtype == LMGC_BF16 && ctx->use_tc && (hd == 64 || hd == 128) &&
-                    tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kQKVRope);
-  ctx->fused_norm = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_model % 256 == 0 &&
+  if (c.dtype == LMGC_BF16) {
+    // a bf16 model has one backend, the tcgen05 kernels: without the tensor-map encoder (or on a
+    // device they do not run on) the context is refused instead of computing on CUDA cores
+    const bool tc = tc_attention_supported(hd, ctx->qkv_dim) &&
+                    tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kStore) &&
                     tc_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd, kAddResidual) &&
+                    tc_gemm_supported(1, 2 * (int64_t)c.d_ffn, c.d_model, kStore) &&
                     tc_gemm_supported(1, c.d_model, c.d_ffn, kAddResidual) &&
                     tc_gemm_supported(1, c.vocab, c.d_model, kStoreF32);
-  ctx->fused_swiglu = c.dtype == LMGC_BF16 && ctx->use_tc && c.d_ffn % 128 == 0 && tc_gemm_supported(1, 2 * c.d_ffn, c.d_model, kSwiGLU);
+    if (!tc) {
+      delete ctx;
+      return fail(nullptr, LMGC_ERR_INVALID,
+                  "bf16 models need the tcgen05 kernels: a Blackwell device and the driver's tensor-map encoder");
+    }
+  }
+  ctx->fused_rope = c.dtype == LMGC_BF16 && tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kQKVRope);
+  ctx->fused_norm = c.dtype == LMGC_BF16 && c.d_model % 256 == 0;
+  ctx->fused_swiglu = c.dtype == LMGC_BF16 && c.d_ffn % 128 == 0 && tc_gemm_supported(1, 2 * c.d_ffn, c.d_model, kSwiGLU);
   const int64_t d = c.d_model, F = c.d_ffn, V = c.vocab, qd = (int64_t)c.n_heads * hd;
   const size_t e = ctx->elt;
   // weights: one blob, every tensor 256-byte aligned
@@ -983,8 +995,10 @@ lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c
   if (!ctx || (M && N && (!d_a || !d_b || !d_c))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
   if (K % 8 || epi < 0 || (epi > 3 && epi != kAddResidualWide))
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: K must be a multiple of 8, epi 0..3 or 5");
-  if (epi == kSwiGLU && !(ctx->cfg.dtype == LMGC_BF16 && ctx->use_tc && tc_gemm_supported(M, N, K, epi)))
+  if (epi == kSwiGLU && !(ctx->cfg.dtype == LMGC_BF16 && tc_gemm_supported(M, N, K, epi)))
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epi 3 needs the bf16 tensor-core path and N % 256 == 0");
+  if (ctx->cfg.dtype == LMGC_BF16 && M && N && !tc_gemm_supported(M, N, K, epi))
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: shape outside the tcgen05 kernel");
   cudaStream_t s = (cudaStream_t)stream;
   gemm(ctx, d_a, d_b, d_c, (int64_t)M, (int64_t)N, (int64_t)K, epi, s);
   LMGC_CUDA(ctx, cudaGetLastError());

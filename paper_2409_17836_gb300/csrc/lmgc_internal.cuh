@@ -113,7 +113,6 @@ struct lmgc_ctx {
   cudaEvent_t ev[6] = {};
   std::vector<cudaEvent_t> batch_ev;
   lmgc::Profiler prof;
-  bool use_tc = true;        // tcgen05 GEMM for bf16 models when available
   bool fused_swiglu = false;  // gate/up interleaved, SwiGLU in the tcgen05 epilogue
   bool fused_rope = false;    // RoPE in the QKV tcgen05 epilogue
   bool fused_norm = false;    // RMSNorm folded into the GEMM epilogues (row scale + residual side outputs)

@@ -78,6 +78,7 @@ def test_create_rejects_bad_configs_before_any_cuda_call():
         (dict(n_heads=3), "bad model shape"),                             # d_model % n_heads
         (dict(n_heads=4, n_kv_heads=3), "bad model shape"),               # n_heads % n_kv_heads
         (dict(d_model=96, n_heads=2, n_kv_heads=2), "head dim"),          # hd 48
+        (dict(dtype=1), "head dim of a bf16 model"),                      # hd 32: no tcgen05 attention
         (dict(cdf_bits=31), "cdf_bits"),
         (dict(vocab=70000, cdf_bits=16), "cdf_bits"),                     # 2^P must exceed V
         (dict(dtype=7), "dtype"),
