@@ -198,10 +198,12 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * rounded up to 16, per window) lives in one fixed 64 MiB device array that every GPU loading the
  * library keeps until exit. Calls needing more than 64 MiB of scratch (about 10,900 windows of
  * 2048 tokens at cdf_bits 24) fail with INVALID and a message giving both sizes.
- * The first call on a device looks up the array's device address (once per device, with that
- * device current); make that first call before any stream capture. All calls share the array
- * and it keeps the last call's contents: calls that overlap on the GPU (other streams, other host
- * threads) race on it and must be serialised by the caller. Syncs. */
+ * Windows of more than 2^29 / cdf_bits tokens are rejected the same way.
+ * The first call on a device does the set-up: it looks up the array's device address (once per
+ * device, with that device current); make that first call before any stream capture begins.
+ * All calls share the array and it keeps the last call's contents: calls that overlap on the GPU
+ * (other streams, other host threads) race on it and must be serialised by the caller. Every
+ * call reads the total size back to the host and synchronises `stream` before it returns. */
 lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
                                       size_t win_tokens, const uint32_t* d_win_len, size_t stride_win,
                                       size_t stride_pos, uint8_t* d_out, size_t cap, size_t* out_bytes,

@@ -366,6 +366,12 @@ extern "C" lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const 
     return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: cdf_bits must be in 1..30");
   *out_bytes = 0;
   if (n_win == 0) return LMGC_OK;
+  // a window longer than this cannot fit in the array whatever n_win is; bounding it first also
+  // keeps slot_bytes' size arithmetic from wrapping
+  if (win_tokens > (kNoAllocScratchBytes * 8) / (size_t)cdf_bits)
+    return fail(nullptr, LMGC_ERR_INVALID,
+                "lmgc_range_encode_noalloc: win_tokens * cdf_bits exceeds the fixed maximum of " +
+                    std::to_string(kNoAllocScratchBytes) + " bytes of scratch");
   // scratch layout: [0, 256) error word | offsets [n_win + 1] u64 | one code slot per window
   const size_t slot = slot_bytes(win_tokens, cdf_bits);
   const size_t off_bytes = ((n_win + 1) * 8 + 255) / 256 * 256;
@@ -389,11 +395,14 @@ extern "C" lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const 
   launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
                       (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
   launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
+  // a failed launch must not let the previous call's total (still in the array) be read back
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: launch");
   uint64_t total = 0;
   uint32_t herr = 0;
-  cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
-  cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
-  e = cudaStreamSynchronize(s);
+  e = cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&herr, derr, 4, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc");
   if (herr) return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: invalid (start, freq) or window length");
   *out_bytes = total;

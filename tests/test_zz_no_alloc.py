@@ -57,3 +57,55 @@ def test_noalloc_rejects_more_than_its_fixed_scratch():
         L.lmgc_range_encode_noalloc(dummy, dummy, 24, 20000, 2048, None, 1, 20000, out, dummy)
     assert e.value.status == L.ERR_INVALID
     assert "fixed maximum" in str(e.value)
+
+
+def test_noalloc_runs_with_device_memory_exhausted():
+    """The point of the entry point: it still works when the caller has left it no device memory
+    to allocate. Torch claims all but a small margin of the free device memory (after one call has
+    loaded the module and found the array), then the call must succeed and reproduce the codes
+    computed beforehand. A version that quietly fell back to cudaMalloc for its 20 MB of slots
+    would fail here."""
+    rng = np.random.default_rng(77)
+    n_win, W, P = 3000, 2048, 24
+    start, freq, _ = random_pairs(rng, n_win, W, P)
+    s = torch.from_numpy(start.T.copy().view(np.int32)).cuda()
+    f = torch.from_numpy(freq.T.copy().view(np.int32)).cuda()
+    ref_out, ref_bl = L.lmgc_range_encode(s, f, P, n_win, W, None, 1, n_win)
+    out = torch.zeros(ref_out.numel() + 64, dtype=torch.uint8, device="cuda")
+    bitlen = torch.zeros(n_win, dtype=torch.int32, device="cuda")
+    L.lmgc_range_encode_noalloc(s, f, P, n_win, W, None, 1, n_win, out, bitlen)  # set-up call
+    out.zero_()
+    bitlen.zero_()
+    torch.cuda.synchronize()
+    margin = 16 << 20
+    hold = []
+    try:
+        while True:
+            free, _ = torch.cuda.mem_get_info()
+            if free <= 2 * margin:
+                break
+            try:
+                hold.append(torch.empty(min(free - margin, 1 << 30), dtype=torch.uint8, device="cuda"))
+            except torch.OutOfMemoryError:
+                break
+        free, _ = torch.cuda.mem_get_info()
+        assert free < 64 << 20, free  # less than the 64 MiB array itself: no room for a second one
+        nbytes = L.lmgc_range_encode_noalloc(s, f, P, n_win, W, None, 1, n_win, out, bitlen)
+        assert nbytes == ref_out.numel()
+        assert torch.equal(bitlen, ref_bl)
+        assert torch.equal(out[:nbytes], ref_out)
+    finally:
+        del hold
+        torch.cuda.empty_cache()
+
+
+def test_noalloc_rejects_windows_beyond_its_scratch():
+    """A window whose slot alone exceeds the array is refused before any size arithmetic that
+    could wrap."""
+    dummy = torch.zeros(16, dtype=torch.int32, device="cuda")
+    out = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    for W in [(1 << 29) // 24 + 1, 1 << 62]:
+        with pytest.raises(L.LmgcError) as e:
+            L.lmgc_range_encode_noalloc(dummy, dummy, 24, 1, W, None, 1, 1, out, dummy)
+        assert e.value.status == L.ERR_INVALID
+        assert "fixed maximum" in str(e.value)
