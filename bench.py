@@ -1,12 +1,14 @@
 """Throughput of the LM-GC encode path on GB300 (one JSON line on rank 0).
 
-Workload (default): gradients of a seeded random-init 4-layer ConvNet (298,954 values, 3x32x32
-Gaussian inputs, batch 64), serialised as 8 hex digits + a space per value, coded with a
-TinyLlama-1.1B-shaped model (22 layers, d 2048, 32/4 heads, FFN 5632, vocab 32000, random-init
-bf16 weights) over 2048-token windows, 64 windows per model batch, 24-bit integer CDFs.
-One step = lmgc_encode of one batch: 14,563 values (131,067 tokens, 64 windows) through
-serialise -> model -> CDF pairs -> range coder -> container. Step k encodes slice k mod 20 of the
-gradient; all slices are resident in HBM before timing.
+Workload (default, the largest single-GPU configuration): gradients of a seeded random-init
+4-layer ConvNet (298,954 values, 3x32x32 Gaussian inputs, batch 64), serialised as 8 hex digits +
+a space per value, coded with a Llama-2-7B-shaped model (32 layers, d 4096, 32 heads MHA, FFN
+11008, vocab 32000, random-init bf16 weights) over 4096-token windows, 32 windows per model
+batch, 24-bit integer CDFs. One step = lmgc_encode of one batch: 14,563 values (131,067 tokens,
+32 windows) through serialise -> model -> CDF pairs -> range coder -> container. Step k encodes
+slice k mod 20 of the gradient; all slices are resident in HBM before timing. The line also
+carries the TinyLlama-shaped step (22 layers, d 2048, 32/4 heads, FFN 5632, 2048-token windows,
+64 per batch) under "tinyllama_step".
 
 value     raw-gradient MB/s (4 bytes per value) over all ranks, device buffers, CUDA events
 e2e       the same through lmgc_encode_host (pinned host buffers; H2D + D2H inside the region)
@@ -30,6 +32,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "raw gradient MB/s encoded (1 GB300); LM tensor-pipe % of bf16 peak; coder HBM GB/s"
+DEFAULT_WORKLOAD = "convnet-llama2-7b"
 WORKLOADS = ("convnet-tinyllama", "tiny", "convnet-llama2-7b", "lossy-tinyllama", "laplace-tinyllama",
              "quant16-tinyllama", "quant1-tinyllama", "sparse50-tinyllama", "sparse25-tinyllama",
              "alpha-tinyllama")
@@ -252,25 +255,34 @@ def oracle_sample(cfg, vals, positions: int, win: int, threads: int):
 
 def cpu_baseline(cfg, vals, tpv: float, bpv: int, target_s: float) -> dict:
     """The oracle as it stands on the host's cores: a prefix of window 0 sized for about target_s
-    seconds with every core, then a prefix sized for about target_s / 4 on one thread."""
+    seconds with every core, then a prefix sized for about target_s / 4 on one thread. The
+    one-thread figure is left out when even its 4-position calibration would take longer than
+    target_s (estimated as the all-core calibration times the core count: the Llama-2-7B shape)."""
     threads = max(1, len(os.sched_getaffinity(0)))
-    runs = []
-    for n_threads, budget in ((threads, target_s), (1, target_s / 4)):
-        dt, n = oracle_sample(cfg, vals, 4, 0, n_threads)
-        positions = int(max(4, min(cfg.window, budget / max(dt / n, 1e-6))))
-        dt, n = oracle_sample(cfg, vals, positions, 0, n_threads)
-        runs.append((n / tpv * bpv / dt / 1e6, n, dt))
-    (mbs, n, dt), (mbs1, n1, dt1) = runs
     what = "oracle encode (fp64 model forward, integer CDF, range coder) of the first {} tokens of window 0, {:.1f} s"
-    return {"value": mbs, "unit": "MB/s", "cores": threads, "kind": "oracle", "sample": what.format(n, dt),
-            "single_thread": {"value": mbs1, "unit": "MB/s", "cores": 1, "sample": what.format(n1, dt1)}}
+    dt4, n4 = oracle_sample(cfg, vals, 4, 0, threads)
+    positions = int(max(4, min(cfg.window, target_s / max(dt4 / n4, 1e-6))))
+    dt, n = oracle_sample(cfg, vals, positions, 0, threads)
+    res = {"value": n / tpv * bpv / dt / 1e6, "unit": "MB/s", "cores": threads, "kind": "oracle",
+           "sample": what.format(n, dt)}
+    est1 = dt4 * threads
+    if est1 > target_s:
+        res["single_thread"] = {"skipped": f"a 4-position calibration on one thread would take about {est1:.0f} s"}
+        return res
+    dt1, n1 = oracle_sample(cfg, vals, 4, 0, 1)
+    positions = int(max(4, min(cfg.window, target_s / 4 / max(dt1 / n1, 1e-6))))
+    dt1, n1 = oracle_sample(cfg, vals, positions, 0, 1)
+    res["single_thread"] = {"value": n1 / tpv * bpv / dt1 / 1e6, "unit": "MB/s", "cores": 1,
+                            "sample": what.format(n1, dt1)}
+    return res
 
 
-def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> dict:
+def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> dict:
     """HBM-bound stages at sizes where bandwidth, not launch latency, decides: the serialiser on
     the 64M-value Laplace mixture (default layout, and byte groups of 3 that cross values), and
-    the coder alone on 2^18 windows x 2048 tokens of seeded
-    random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most likely)."""
+    the coder alone on 2^20 windows x 2048 tokens (the 64M-value sweep's coder microbenchmark) of
+    seeded random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most
+    likely); ctx supplies the integer CDFs (any context with vocab 32000 and P = 24)."""
     import numpy as np
     import torch
 
@@ -346,14 +358,28 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 18) -> 
     return out
 
 
-def profiled_traffic(workload: str, kernel: str):
-    """DRAM bytes per launch of a kernel class from the committed ncu launch-list summary of this
-    workload (profiles/launches_<workload>.md), or None when there is none."""
-    path = os.path.join(ROOT, "profiles", f"launches_{workload}.md")
+def micro_run(L, configs, pk, coder_windows: int) -> dict:
+    """The microbenchmarks with a small vocab-32000, P = 24 context (one layer, one window per
+    batch) that only supplies the coder's integer CDFs."""
+    ctx = L.Context(configs.with_(configs.TINYLLAMA, n_layers=1, batch_windows=1))
+    try:
+        return microbenchmarks(L, ctx, pk, coder_windows=coder_windows)
+    finally:
+        ctx.close()
+
+
+def profiled_traffic(workload: str, kernel: str, work_per_launch: float):
+    """DRAM bytes per launch of a kernel class, scaled from a small-case ncu capture of the same
+    kernels (profiles/traffic_<workload>-small.md: DRAM read + write bytes and algorithmic work
+    summed over the captured launches) by the algorithmic work of one launch here; None when there
+    is no capture. The scaling holds for the GEMMs, whose operand and output bytes grow with the
+    rows processed (the weight is read once per group of row tiles in both cases)."""
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}-small.md")
     try:
         text = open(path).read()
-        block = text.split("```json", 1)[1].split("```", 1)[0]
-        return json.loads(block)[kernel]["traffic_bytes_per_launch"], os.path.relpath(path, ROOT)
+        block = json.loads(text.split("```json", 1)[1].split("```", 1)[0])[kernel]
+        per_work = block["dram_bytes"] / block["work"]
+        return per_work * work_per_launch, os.path.relpath(path, ROOT)
     except Exception:
         return None, None
 
@@ -395,71 +421,20 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
-    ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="convnet-tinyllama", choices=WORKLOADS)
-    ap.add_argument("--batch-windows", type=int, default=0)
-    # a model with fewer layers, for small profiler captures only (the config line names it)
-    ap.add_argument("--layers", type=int, default=0)
-    ap.add_argument("--ref-positions", type=int, default=12)
-    ap.add_argument("--cpu-target-s", type=float, default=15.0)
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-micro", action="store_true")
-    # encode the whole workload once (every window, in batches of --batch-windows), then decode
-    # the first, middle and last windows and check them; prints one JSON line of its own
-    ap.add_argument("--full", action="store_true")
-    # only the serialise and coder microbenchmarks (one JSON line), the coder on this many windows
-    # of 2048 tokens (small profiler captures use 2^16)
-    ap.add_argument("--micro-only", action="store_true")
-    # decode throughput: encode one batch of windows, then time lmgc_decode of all of them
-    # (KV-cached, one model step per position) and check the tokens; one JSON line of its own
-    ap.add_argument("--decode", action="store_true")
-    ap.add_argument("--decode-windows", type=int, default=0)  # windows to decode (default: one batch)
-    ap.add_argument("--coder-windows", type=int, default=1 << 18)
-    args = ap.parse_args()
-    if args.impl == "reference":
-        return run_reference(args)
+def model_name(cfg) -> str:
+    return f"{cfg.n_layers}L d{cfg.d_model} {cfg.n_heads}/{cfg.n_kv_heads}h ffn{cfg.d_ffn} V{cfg.vocab}"
 
+
+def measure_steps(L, ctx, cfg, vals, args, world, rank, local, pk, name, e2e=True) -> dict:
+    """W warm-up and K timed steps of lmgc_encode (one model batch of the workload per step,
+    inputs resident in HBM), CUDA events on the launching stream, max over ranks; per-class kernel
+    times from the library's events inside the timed region; then, with e2e, the same K steps
+    through lmgc_encode_host (pinned host buffers, copies inside the timed region)."""
     import numpy as np
     import torch
     import torch.distributed as dist
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
-
-    import __graft_entry__
-
-    # one builder per node (the build writes in-tree files); the other ranks wait, then load
-    if local == 0:
-        __graft_entry__.build()
-    if world > 1:
-        dist.barrier()
-    from paper_2409_17836_gb300 import configs, lmgc as L
-
-    cfg, vals = workload(args.workload)
-    if args.batch_windows:
-        cfg = configs.with_(cfg, batch_windows=args.batch_windows)
-    if args.layers:
-        cfg = configs.with_(cfg, n_layers=args.layers)
-    ctx = L.Context(cfg)
     tpv = L.lmgc_serial_tokens(ctx, vals.size) / vals.size  # tokens per value over the workload
-    if args.full:
-        return run_full(args, cfg, ctx, vals)
-    if args.decode:
-        return run_decode(args, cfg, ctx, vals)
-    if args.micro_only:
-        print(json.dumps({"mode": "micro", "microbench": microbenchmarks(L, ctx, peaks(), coder_windows=args.coder_windows)}),
-              flush=True)
-        ctx.close()
-        return 0
     # values filling one model batch
     per_step = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, cfg.batch_windows * cfg.window)
     n_slices = max(1, vals.size // per_step)
@@ -496,39 +471,39 @@ def main():
         ms = float(t.item())
         dist.barrier()
     bpv = bytes_per_value(cfg)
-    raw_bytes = per_step * bpv * args.steps * world
-    value = raw_bytes / (ms / 1e3) / 1e6
+    value = per_step * bpv * args.steps * world / (ms / 1e3) / 1e6
+    del slices, dev
 
-    # end to end through host buffers
-    hin = [torch.from_numpy((vals.view(np.int32) if vals.dtype == np.float32 else vals)[i * per_step:(i + 1) *
-                                                                                          per_step].copy()).pin_memory()
-           for i in range(min(n_slices, 4))]
-    hout = torch.empty(L.lmgc_encode_bound(ctx, per_step), dtype=torch.uint8).pin_memory()
-    L.lmgc_encode_host(ctx, hin[0], hout)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    d2h = 0
-    t0 = time.perf_counter()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for k in range(args.steps):
-        d2h += L.lmgc_encode_host(ctx, hin[k % len(hin)], hout)
-    e1.record()
-    torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:  # the slowest rank's time, as for the device-timed value
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": per_step * bpv * args.steps * world / (e2e_ms / 1e3) / 1e6, "unit": "MB/s",
-           "h2d_bytes_per_step": per_step * bpv, "d2h_bytes_per_step": int(d2h / args.steps),
-           "wall_s": time.perf_counter() - t0}
+    e2e_res = None
+    if e2e:  # end to end through host buffers
+        src = vals.view(np.int32) if vals.dtype == np.float32 else vals
+        hin = [torch.from_numpy(src[i * per_step:(i + 1) * per_step].copy()).pin_memory()
+               for i in range(min(n_slices, 4))]
+        hout = torch.empty(L.lmgc_encode_bound(ctx, per_step), dtype=torch.uint8).pin_memory()
+        L.lmgc_encode_host(ctx, hin[0], hout)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        d2h = 0
+        t0 = time.perf_counter()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for k in range(args.steps):
+            d2h += L.lmgc_encode_host(ctx, hin[k % len(hin)], hout)
+        e1.record()
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1)
+        if world > 1:  # the slowest rank's time, as for the device-timed value
+            t = torch.tensor([e2e_ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e_res = {"value": per_step * bpv * args.steps * world / (e2e_ms / 1e3) / 1e6, "unit": "MB/s",
+                   "h2d_bytes_per_step": per_step * bpv, "d2h_bytes_per_step": int(d2h / args.steps),
+                   "wall_s": time.perf_counter() - t0}
 
-    pk = peaks()
     g = stats["gemm"]
     gemm_tflops = g["work"] / (g["ms"] / 1e3) / 1e12 if g["ms"] > 0 else 0.0
-    traffic, traffic_src = profiled_traffic(args.workload, "gemm_tc")
+    traffic, traffic_src = profiled_traffic(name, "gemm_tc", g["work"] / max(1, g["launches"]))
     roofline = {"bound": "tensor", "kernel": "gemm (all linear layers and the vocabulary projection)",
                 "achieved": gemm_tflops, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
                 "frac": gemm_tflops / pk["bf16_sus"],
@@ -538,43 +513,127 @@ def main():
                 "traffic": traffic, "traffic_unit": "bytes per launch (DRAM read + write)",
                 "traffic_source": traffic_src}
     stages = {}
-    for name, st in stats.items():
+    for cls, st in stats.items():
         if st["launches"] == 0:
             continue
         e = {"launches": st["launches"], "ms": st["ms"], "share": st["ms"] / ms if ms else None}
-        if name in ("gemm", "attention") and st["ms"] > 0:
+        if cls in ("gemm", "attention") and st["ms"] > 0:
             e.update(achieved=st["work"] / (st["ms"] / 1e3) / 1e12, unit="TFLOP/s")
             e["frac"] = e["achieved"] / pk["bf16_sus"]
-        elif name in ("cdf_pairs", "range_encode", "serialize") and st["ms"] > 0:
+        elif cls in ("cdf_pairs", "range_encode", "serialize") and st["ms"] > 0:
             e.update(achieved=st["work"] / (st["ms"] / 1e3) / 1e9, unit="GB/s")
             e["frac"] = e["achieved"] / pk["hbm"]
-        stages[name] = e
+        stages[cls] = e
+    return {"value": value, "ms": ms, "per_step": per_step, "tpv": tpv, "bpv": bpv, "clocks": clk.summary(),
+            "launches": launches, "roofline": roofline, "stages": stages, "e2e": e2e_res,
+            "stage_ms": L.lmgc_stage_times(ctx), "rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv),
+            "bits_per_token": 8.0 * statistics.mean(sizes) / L.lmgc_serial_tokens(ctx, per_step)}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=WORKLOADS)
+    ap.add_argument("--batch-windows", type=int, default=0)
+    # a model with fewer layers, for small profiler captures only (the config line names it)
+    ap.add_argument("--layers", type=int, default=0)
+    ap.add_argument("--ref-positions", type=int, default=12)
+    ap.add_argument("--cpu-target-s", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-micro", action="store_true")
+    # encode the whole workload once (every window, in batches of --batch-windows), then decode
+    # the first, middle and last windows and check them; prints one JSON line of its own
+    ap.add_argument("--full", action="store_true")
+    # only the serialise and coder microbenchmarks (one JSON line), the coder on this many windows
+    # of 2048 tokens (small profiler captures use 2^16)
+    ap.add_argument("--micro-only", action="store_true")
+    # decode throughput: encode one batch of windows, then time lmgc_decode of all of them
+    # (KV-cached, one model step per position) and check the tokens; one JSON line of its own
+    ap.add_argument("--decode", action="store_true")
+    ap.add_argument("--decode-windows", type=int, default=0)  # windows to decode (default: one batch)
+    ap.add_argument("--coder-windows", type=int, default=1 << 20)
+    # the default workload's line also carries the TinyLlama-shaped step; this leaves it out
+    ap.add_argument("--no-extra", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    import __graft_entry__
+
+    # one builder per node (the build writes in-tree files); the other ranks wait, then load
+    if local == 0:
+        __graft_entry__.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2409_17836_gb300 import configs, lmgc as L
+
+    cfg, vals = workload(args.workload)
+    if args.batch_windows:
+        cfg = configs.with_(cfg, batch_windows=args.batch_windows)
+    if args.layers:
+        cfg = configs.with_(cfg, n_layers=args.layers)
+    if args.micro_only:
+        print(json.dumps({"mode": "micro", "microbench": micro_run(L, configs, peaks(), args.coder_windows)}),
+              flush=True)
+        return 0
+    ctx = L.Context(cfg)
+    if args.full:
+        return run_full(args, cfg, ctx, vals)
+    if args.decode:
+        return run_decode(args, cfg, ctx, vals)
+    pk = peaks()
+    m = measure_steps(L, ctx, cfg, vals, args, world, rank, local, pk, args.workload)
+    ctx.close()
+    extra = None
+    if args.workload == DEFAULT_WORKLOAD and not args.no_extra:
+        # the TinyLlama-shaped step (2048-token windows, 64 per batch) beside the headline
+        tcfg, tvals = workload("convnet-tinyllama")
+        tctx = L.Context(tcfg)
+        t = measure_steps(L, tctx, tcfg, tvals, args, world, rank, local, pk, "convnet-tinyllama", e2e=False)
+        tctx.close()
+        extra = {"workload": "convnet-tinyllama", "value": t["value"], "unit": "MB/s",
+                 "ms_per_step": t["ms"] / args.steps, "model": model_name(tcfg), "window": tcfg.window,
+                 "batch_windows": tcfg.batch_windows, "values_per_step": t["per_step"], "clocks": t["clocks"],
+                 "roofline": t["roofline"], "stages": t["stages"], "gpu_launches": t["launches"]}
+    ctx = None
     micro = None
     if rank == 0 and not args.no_micro and cfg.vocab == 32000:
-        micro = microbenchmarks(L, ctx, pk)
+        micro = micro_run(L, configs, pk, args.coder_windows)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(cfg, vals, tpv, bpv, args.cpu_target_s)
+        cpu = cpu_baseline(cfg, vals, m["tpv"], m["bpv"], args.cpu_target_s)
     if rank == 0:
-        res = {"metric": METRIC, "value": value, "unit": "MB/s", "n_gpus": world, "steps": args.steps,
-               "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
-               "vs_baseline": None, "dtype": "f16" if cfg.dtype == L.BF16 else "f32",
+        res = {"metric": METRIC, "value": m["value"], "unit": "MB/s", "n_gpus": world, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": m["ms"] / args.steps, "higher_is_better": True,
+               "scaling": "weak", "vs_baseline": None, "dtype": "f16" if cfg.dtype == L.BF16 else "f32",
                "data": "synthetic (seeded random-init ConvNet gradients on Gaussian inputs; random-init model)",
-               "config": {"workload": args.workload, "values_per_step": per_step, "window": cfg.window,
-                          "batch_windows": cfg.batch_windows, "cdf_bits": cfg.cdf_bits,
-                          "model": f"{cfg.n_layers}L d{cfg.d_model} {cfg.n_heads}/{cfg.n_kv_heads}h "
-                                   f"ffn{cfg.d_ffn} V{cfg.vocab}",
+               "config": {"workload": args.workload, "values_per_step": m["per_step"], "window": cfg.window,
+                          "batch_windows": cfg.batch_windows, "cdf_bits": cfg.cdf_bits, "model": model_name(cfg),
                           "weights": "bf16 values (random init), held in fp16; fp16 activations, fp32 accumulation"
                           if cfg.dtype == L.BF16 else "fp32",
                           "l2": "no flush: each step reads > L2 (model weights and per-batch logits)",
                           "parallelism": f"windows sharded over {world} GPU(s), no collective on the data path"},
-               "clocks": clk.summary(), "e2e": e2e, "gpu_launches": launches, "roofline": roofline,
-               "stages": stages, "microbench": micro, "stage_ms_last_step": L.lmgc_stage_times(ctx),
-               "compression_rate_pct": 100.0 * statistics.mean(sizes) / (per_step * bpv),
-               "bits_per_token": 8.0 * statistics.mean(sizes) / L.lmgc_serial_tokens(ctx, per_step),
+               "clocks": m["clocks"], "e2e": m["e2e"], "gpu_launches": m["launches"], "roofline": m["roofline"],
+               "stages": m["stages"], "microbench": micro, "stage_ms_last_step": m["stage_ms"],
+               "compression_rate_pct": m["rate_pct"], "bits_per_token": m["bits_per_token"],
                "cpu_baseline": cpu}
+        if extra is not None:
+            res["tinyllama_step"] = extra
         print(json.dumps(res), flush=True)
-    ctx.close()
     if world > 1:
         dist.destroy_process_group()
 
