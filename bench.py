@@ -115,7 +115,7 @@ def workload(name: str):
         return configs.TINY, inputs.tiny_gradient(0)
     if name == "laplace-tinyllama":  # 64M-value Laplace mixture; window batch set by --batch-windows
         return configs.TINYLLAMA, inputs.laplace_gradient()
-    # Sec. 5 compatibility settings one at a time: Eq. 4 indices of every value (16 bits as
+    # Sec. 5.4 compatibility settings one at a time: Eq. 4 indices of every value (16 bits as
     # big-endian byte pairs, one separator per index; 1 bit as one byte each), or the top 50% / 25%
     # of |v| still as fp32
     if name in ("quant16-tinyllama", "quant1-tinyllama"):
@@ -307,7 +307,7 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> 
                         "unit": "GB/s", "frac": nbytes / ms / 1e6 / pk["hbm"]}
     sctx.close()
     del tok
-    # the byte-grouped layout (Sec. 4.3): 3 bytes per group, fp32 bytes least significant first
+    # the byte-grouped layout (Sec. 5.3): 3 bytes per group, fp32 bytes least significant first
     gctx = L.Context(configs.with_(configs.TINY, byte_group=3, byte_order=1))
     tok = torch.empty(L.lmgc_serial_tokens(gctx, d.numel()), dtype=torch.int16, device="cuda")
     L.lmgc_serialize(gctx, d, tok)

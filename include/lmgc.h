@@ -2,10 +2,10 @@
  * lmgc.h -- C ABI of liblmgc.so, the GB300 (sm_103a) encode path of LM-GC
  * ("Language Models as Zero-shot Lossless Gradient Compressors", arXiv 2409.17836).
  *
- * The method (Sec. 3): serialise fp32 gradients into hex-digit text with separators, feed it in
+ * The method (Sec. 4): serialise fp32 gradients into hex-digit text with separators, feed it in
  * fixed windows, each starting from BOS, to a causal language model whose next-token
- * distributions (Eq. 2) drive an arithmetic coder (Sec. 2). Decoding runs the model token by token
- * from BOS until the window is full (Sec. 3 "Compression").
+ * distributions (Eq. 2) drive an arithmetic coder (Sec. 3). Decoding runs the model token by token
+ * from BOS until the window is full (Sec. 4 "Compression").
  *
  * Conventions for every call:
  *  - Pointers named d_* are DEVICE pointers owned by the caller (allocated on the device the
@@ -21,7 +21,7 @@
  *    size pointer and no output.
  *  - Results are deterministic: the same input and configuration give the same bytes.
  *
- * Token alphabet (character-level reading of Sec. 3 / Fig. 1): hex digit v -> id v (0..15),
+ * Token alphabet (character-level reading of Sec. 4 / Fig. 1): hex digit v -> id v (0..15),
  * ' ' -> 16, ',' -> 17, ';' -> 18, BOS -> 19. The model's vocabulary has `vocab` >= 20 ids; the
  * coder codes over all of them (Eq. 2 is a distribution over the whole vocabulary), or, with
  * lmgc_config.alphabet = 1, over the ids the serialisation can emit only.
@@ -54,12 +54,12 @@ enum { LMGC_F32 = 0, LMGC_BF16 = 1 };
 /* Separator modes (Table 1 serialisations): H_s, H_c, H_{c+s}, H_semi, H_n. */
 enum { LMGC_SEP_SPACE = 0, LMGC_SEP_COMMA = 1, LMGC_SEP_COMMA_SPACE = 2, LMGC_SEP_SEMI = 3, LMGC_SEP_NONE = 4 };
 
-/* Input kinds: fp32 gradient values (8 hex digits each, Sec. 3) or uint8 codes of the
- * lossy-compatible setting (Sec. 5, Eq. 4; 2 hex digits each). */
+/* Input kinds: fp32 gradient values (8 hex digits each, Sec. 4) or uint8 codes of the
+ * lossy-compatible setting (Sec. 5.4, Eq. 4; 2 hex digits each). */
 enum { LMGC_IN_F32 = 0, LMGC_IN_U8 = 1 };
 
 /* Model and coder configuration. The model is a Llama-family decoder (the paper's LLMs,
- * Sec. 4.1): token embedding; per layer x += Wo Attn(RoPE(Wq n), RoPE(Wk n), Wv n) with
+ * Sec. 5.1): token embedding; per layer x += Wo Attn(RoPE(Wq n), RoPE(Wk n), Wv n) with
  * n = RMSNorm(x) and x += Wdown (silu(Wgate n') * Wup n') with n' = RMSNorm(x); a final RMSNorm;
  * logits = Wvocab x. Grouped-query attention when n_kv_heads < n_heads. Pretrained weights
  * are not available: every weight is drawn from splitmix64(weight_seed ^ (tensor_id << 40) ^
@@ -71,18 +71,18 @@ typedef struct {
                             computed with fp16 activations and fp16 x fp16 -> fp32 MMAs (every bf16
                             value >= 2^-17 in magnitude is exact in fp16, smaller ones round to
                             the 2^-24 grid) */
-  int32_t window;        /* W: tokens per independently coded window (Sec. 4.3 "Context window size") */
+  int32_t window;        /* W: tokens per independently coded window (Sec. 5.3 "Context window size") */
   int32_t cdf_bits;      /* P: the integer CDFs sum to 2^P; 2^P > vocab, P <= 30 */
   int32_t sep_mode;      /* LMGC_SEP_* */
   int32_t input_kind;    /* LMGC_IN_* */
   int32_t batch_windows; /* windows per model batch (workspace is sized for it) */
   uint64_t weight_seed;
   float init_std, rms_eps, rope_theta;
-  int32_t byte_group;    /* bytes per separator group (Sec. 4.3 "Byte grouping", BPG 1..8); 0 = one
+  int32_t byte_group;    /* bytes per separator group (Sec. 5.3 "Byte grouping", BPG 1..8); 0 = one
                             group per value (the default: BPG 4 for fp32, 1 for uint8 codes) */
   int32_t byte_order;    /* fp32 bytes in the stream: 0 most significant first, 1 least significant
                             first (uint8 codes: 0) */
-  int32_t alphabet;      /* 0: each position's integer CDF spans the whole vocabulary (Sec. 3);
+  int32_t alphabet;      /* 0: each position's integer CDF spans the whole vocabulary (Sec. 4);
                             1: it spans only the ids the serialisation can emit (the 16 hex digits
                             and the separator ids of sep_mode), taken over those logits in
                             ascending id order, and a token is coded as its index among them. A
@@ -114,9 +114,9 @@ lmgc_status lmgc_tokens_per_value(const lmgc_ctx* ctx, size_t* tpv);
  * ceil(bytes / group) groups. Errors: INVALID. */
 lmgc_status lmgc_serial_tokens(const lmgc_ctx* ctx, size_t n, size_t* n_tok);
 
-/* Sec. 3 "Serialization" and Fig. 1: every 4 bits of a value become one hex digit, most
+/* Sec. 4 "Serialization" and Fig. 1: every 4 bits of a value become one hex digit, most
  * significant first (sign and exponent first), then the separator tokens. With byte_group or
- * byte_order set (Sec. 4.3 "Byte grouping"): the values' bytes in order (fp32 bytes per
+ * byte_order set (Sec. 5.3 "Byte grouping"): the values' bytes in order (fp32 bytes per
  * byte_order), two hex digits per byte, high nibble first, and the separator after every
  * byte_group bytes and after a final partial group.
  * d_in: n values (fp32 bit patterns or uint8 codes per the context's input kind).
@@ -154,7 +154,7 @@ lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c
                       int epi, lmgc_stream stream);
 
 /* Integer CDF of each logit row (the coder input; the paper adapts Torchac, whose CDFs are
- * integers, Sec. 4.1). For a row z[0..V) with T = 2^P: m = max z; y_j = fp32(fp32(z_j - m) *
+ * integers, Sec. 5.1). For a row z[0..V) with T = 2^P: m = max z; y_j = fp32(fp32(z_j - m) *
  * fp32(2^16 log2 e)); a_j = -rint(y_j) clamped to 40*2^16; e_j = 2^31 * 2^(-a_j/65536) in fixed
  * point from two 256-entry tables; g_j = floor(e_j (T - V) / sum e); freq_j = 1 + g_j with the
  * remainder added to the lowest-index largest e_j; cdf[0] = 0, cdf[V] = T. Rows always span the
@@ -173,7 +173,7 @@ lmgc_status lmgc_quantize_cdf(lmgc_ctx* ctx, const float* d_logits, size_t rows,
 lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, const uint16_t* d_sym,
                            uint32_t* d_start, uint32_t* d_freq, lmgc_stream stream);
 
-/* Arithmetic coder (Sec. 2 "Arithmetic coding"), one independent stream per window, in an exact
+/* Arithmetic coder (Sec. 3 "Arithmetic coding"), one independent stream per window, in an exact
  * integer form: R = 2^62, L = 0, B = 0; per token r = R >> P, L += r*start, R = r*freq,
  * k = max(0, 62 - bitlen(R)), R <<= k, L <<= k, B += k; the code is the top B + 2 bits of
  * ceil(L / 2^60) * 2^60, most significant bit first, padded with zeros to a byte.
@@ -213,7 +213,7 @@ lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const uint32_t* d
  * tables + the coder's worst case of cdf_bits bits per token + 2 bits per window). */
 lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes);
 
-/* The whole encode path (Sec. 3): serialise -> windows from BOS -> model logits -> integer CDF
+/* The whole encode path (Sec. 4): serialise -> windows from BOS -> model logits -> integer CDF
  * pairs -> one code per window -> container. Container layout (little-endian):
  *   0 "LMGC" | 4 u32 version=2 | 8 u64 n_values | 16 u64 n_tok | 24 u32 window | 28 u32 cdf_bits |
  *   32 u32 input_kind | 36 u32 serialisation = sep_mode | byte_group << 8 | byte_order << 16 |
@@ -228,7 +228,7 @@ lmgc_status lmgc_encode(lmgc_ctx* ctx, const void* d_in, size_t n, uint8_t* d_ou
                         lmgc_stream stream);
 
 /* The windows [first_win, first_win + n_win) of lmgc_encode's container, for encoding a stream
- * sharded over several GPUs (windows are independent, Sec. 3 "Compression"): all n values are
+ * sharded over several GPUs (windows are independent, Sec. 4 "Compression"): all n values are
  * serialised, only the given windows are modelled and coded. d_payload receives their codes
  * byte-aligned in window order (the container's payload slice), d_bitlen and d_crc (device, n_win
  * each) their bit lengths and token checksums, *payload_bytes (host) the slice size. A container
@@ -248,7 +248,7 @@ lmgc_status lmgc_container_header(const lmgc_ctx* ctx, size_t n, uint8_t* h_head
 lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t* h_out, size_t cap,
                              size_t* out_bytes, lmgc_stream stream);
 
-/* The KV-cached autoregressive inverse (Sec. 3 "Compression": decoding starts from BOS and runs
+/* The KV-cached autoregressive inverse (Sec. 4 "Compression": decoding starts from BOS and runs
  * until the window is full). Decodes the windows h_win_ids[0 .. n_ids) (host array) of the
  * container d_in (device, in_bytes) into d_tok (device, [n_ids][W] uint16; a partial last window
  * fills only its length). Each decode step runs the same kernels as lmgc_encode on one row per

@@ -6,11 +6,11 @@ this package. The CUDA path never imports it and shares none of its code.
 This module wraps the plain C oracle (`lmgc_oracle.c`, built with gcc) through ctypes and adds
 the container layout in plain Python. Every function names the passage it follows:
 
-* `serialize` / `deserialize`      Sec. 3 "Serialization", Fig. 1 (hex digits + separators)
+* `serialize` / `deserialize`      Sec. 4 "Serialization", Fig. 1 (hex digits + separators)
 * `OracleLM`, `window_logits`      Eq. 1 / Eq. 2 (next-token distributions after BOS), fp64
-* `quantize_cdf`, `cdf_pair`       integer CDF for the Torchac-style coder of Sec. 4.1
-* `range_encode`, `Decoder`        Sec. 2 "Arithmetic coding" in exact integer form
-* `encode`, `decode_window`        Sec. 3 "Compression" (independent windows, BOS not coded)
+* `quantize_cdf`, `cdf_pair`       integer CDF for the Torchac-style coder of Sec. 5.1
+* `range_encode`, `Decoder`        Sec. 3 "Arithmetic coding" in exact integer form
+* `encode`, `decode_window`        Sec. 4 "Compression" (independent windows, BOS not coded)
 * `compression_rate`               Eq. 3
 
 Parity unpinned: the bit-level values of the LM logits (the paper prints none; they are pinned
@@ -89,7 +89,7 @@ def _p(a: np.ndarray):
 
 
 # ------------------------------------------------------------------------------------------
-# Serialisation (Sec. 3, Fig. 1). Token ids: hex digit -> 0..15, ' ' 16, ',' 17, ';' 18, BOS 19.
+# Serialisation (Sec. 4, Fig. 1). Token ids: hex digit -> 0..15, ' ' 16, ',' 17, ';' 18, BOS 19.
 # sep_mode: 0 H_s (space), 1 H_c (comma), 2 H_{c+s}, 3 H_semi, 4 H_n (none). input_kind 0 = fp32,
 # 1 = uint8 codes (Eq. 4 indices).
 # ------------------------------------------------------------------------------------------
@@ -101,13 +101,13 @@ def tokens_per_value(input_kind: int, sep_mode: int) -> int:
 
 
 def serial_tokens(input_kind: int, sep_mode: int, n: int, byte_group: int = 0, byte_order: int = 0) -> int:
-    """Token count of n values (Sec. 3; byte grouping of Sec. 4.3)."""
+    """Token count of n values (Sec. 4; byte grouping of Sec. 5.3)."""
     return int(lib().orc_serial_tokens(input_kind, sep_mode, byte_group, byte_order, n))
 
 
 def serialize(values: np.ndarray, sep_mode: int = 0, byte_group: int = 0, byte_order: int = 0) -> np.ndarray:
     """byte_group 0 and byte_order 0: one group per value, each value's nibbles most significant
-    first (Sec. 3). Otherwise the byte-grouped form (Sec. 4.3 "Byte grouping"): bytes in order
+    first (Sec. 4). Otherwise the byte-grouped form (Sec. 5.3 "Byte grouping"): bytes in order
     (fp32 most or least significant first), two digits each, a separator every byte_group bytes."""
     kind = 0 if values.dtype == np.float32 else 1
     if kind == 1 and values.dtype != np.uint8:
@@ -185,7 +185,7 @@ class OracleConfig:
     sep_mode: int = 0
     input_kind: int = 0
     n_threads: int = 1
-    byte_group: int = 0  # bytes per separator group (Sec. 4.3); 0 = one group per value
+    byte_group: int = 0  # bytes per separator group (Sec. 5.3); 0 = one group per value
     byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
     alphabet: int = 0    # 1: code over the ids the serialisation can emit (alphabet_ids) only
 
@@ -266,7 +266,7 @@ def swiglu(g: np.ndarray, u: np.ndarray) -> np.ndarray:
 
 
 # ------------------------------------------------------------------------------------------
-# Integer CDF (Torchac-style coder input, Sec. 4.1) and the arithmetic coder (Sec. 2).
+# Integer CDF (Torchac-style coder input, Sec. 5.1) and the arithmetic coder (Sec. 3).
 # ------------------------------------------------------------------------------------------
 def exp2_tables() -> tuple[np.ndarray, np.ndarray]:
     H = np.empty(256, dtype=np.uint32)
@@ -430,7 +430,7 @@ def parse_container(buf: bytes) -> dict:
 
 
 def encode(cfg: OracleConfig, values: np.ndarray, n_par: int = 1) -> bytes:
-    """Full oracle encode of a gradient vector into the container (Sec. 3)."""
+    """Full oracle encode of a gradient vector into the container (Sec. 4)."""
     tok = serialize(values, cfg.sep_mode, cfg.byte_group, cfg.byte_order)
     W = cfg.window
     n_win = (tok.size + W - 1) // W

@@ -1,6 +1,6 @@
 """Arbitrary-precision restatements of the arithmetic coder (test infrastructure only).
 
-* `interval_code` -- the real-interval recursion of Sec. 2 "Arithmetic coding" in exact
+* `interval_code` -- the real-interval recursion of Sec. 3 "Arithmetic coding" in exact
   rationals: start from [0, 1), give each symbol the sub-interval of its cumulative
   probability (symbol order low to high) and keep the chosen one; any number of the final
   interval represents the message. Used for the paper's worked example (a message "AAAB"
@@ -19,7 +19,7 @@ W_C = 62
 
 
 def interval_code(message: list[int], probs: list[Fraction]) -> list[tuple[Fraction, Fraction]]:
-    """Intervals [low, high) after each symbol of the real-interval recursion (Sec. 2)."""
+    """Intervals [low, high) after each symbol of the real-interval recursion (Sec. 3)."""
     cum = [Fraction(0)]
     for p in probs:
         cum.append(cum[-1] + p)

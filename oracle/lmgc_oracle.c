@@ -7,15 +7,15 @@
  * generator with the CUDA path, and it never calls into it.
  *
  * What it computes, step by step, and the passage each step follows:
- *   serialisation ........ Sec. 3 "Serialization" and Fig. 1: every 4 bits of an fp32 become
+ *   serialisation ........ Sec. 4 "Serialization" and Fig. 1: every 4 bits of an fp32 become
  *                          one hex digit, 8 digits per value, then a separator.
- *   windows + BOS ........ Sec. 3 "Compression", Eq. 2: p(t_k | BOS, t_<k); BOS is context
+ *   windows + BOS ........ Sec. 4 "Compression", Eq. 2: p(t_k | BOS, t_<k); BOS is context
  *                          only; decoding runs until the window is full.
- *   LM prior ............. Eq. 1 / Eq. 2 with a Llama-family decoder (Sec. 4.1 names
+ *   LM prior ............. Eq. 1 / Eq. 2 with a Llama-family decoder (Sec. 5.1 names
  *                          TinyLlama / OpenLLaMA / Llama 2), fp64 arithmetic.
- *   integer CDF .......... implied by the Torchac-based coder of Sec. 4.1 (integer CDFs)
- *                          (Sec. 4.1 "Implementation"): an integer-exact quantiser.
- *   arithmetic coder ..... Sec. 2 "Arithmetic coding" (interval subdivision, any number of
+ *   integer CDF .......... implied by the Torchac-based coder of Sec. 5.1 (integer CDFs)
+ *                          (Sec. 5.1 "Implementation"): an integer-exact quantiser.
+ *   arithmetic coder ..... Sec. 3 "Arithmetic coding" (interval subdivision, any number of
  *                          the final interval represents the message) in an exact integer form.
  *
  * Readings where the paper is silent are the ones listed in the design notes of the
@@ -39,7 +39,7 @@
 #endif
 
 /* ------------------------------------------------------------------------------------------ */
-/* Token alphabet (reading of Sec. 3 / Fig. 1 with a character-level tokeniser):              */
+/* Token alphabet (reading of Sec. 4 / Fig. 1 with a character-level tokeniser):              */
 /* hex digit v -> id v (0..15); ' ' -> 16, ',' -> 17, ';' -> 18; BOS -> 19.                  */
 /* ------------------------------------------------------------------------------------------ */
 #define ORC_TOK_SPACE 16
@@ -59,7 +59,7 @@ static int orc_sep_tokens(int sep_mode, uint16_t sep[2]) {
   }
 }
 
-/* Hex digits per value: 8 for an fp32 value (4 bytes), 2 for a uint8 code (Sec. 5 Eq. 4). */
+/* Hex digits per value: 8 for an fp32 value (4 bytes), 2 for a uint8 code (Sec. 5.4 Eq. 4). */
 static int orc_digits(int input_kind) { return input_kind == 0 ? 8 : (input_kind == 1 ? 2 : -1); }
 
 int64_t orc_tokens_per_value(int input_kind, int sep_mode) {
@@ -69,7 +69,7 @@ int64_t orc_tokens_per_value(int input_kind, int sep_mode) {
   return nd + ns;
 }
 
-/* Sec. 3 "Serialization": the bits of each value, split into 4-bit groups, most significant
+/* Sec. 4 "Serialization": the bits of each value, split into 4-bit groups, most significant
  * group first (sign and exponent first), each group one hex digit, then the separator. */
 int64_t orc_serialize(int input_kind, int sep_mode, const void* in, int64_t n, uint16_t* out) {
   uint16_t sep[2];
@@ -108,7 +108,7 @@ int64_t orc_deserialize(int input_kind, int sep_mode, const uint16_t* tok, int64
   return n;
 }
 
-/* Byte grouping (Sec. 4.3 "Byte grouping", Fig. 3: bytes per group BPG in {1, 2, 3, 4, 8} and
+/* Byte grouping (Sec. 5.3 "Byte grouping", Fig. 3: bytes per group BPG in {1, 2, 3, 4, 8} and
  * none). The values' bytes are taken in order -- an fp32 value's four bytes most significant
  * first (order 0) or least significant first (order 1), a uint8 code as its one byte -- and each
  * byte becomes two hex digits, high nibble first. The separator follows every `group` bytes and
@@ -183,7 +183,7 @@ int64_t orc_deserialize_grouped(int input_kind, int sep_mode, int group, int ord
 }
 
 /* ------------------------------------------------------------------------------------------ */
-/* Random-init weights. The paper uses pretrained checkpoints (Sec. 4.1); they are absent, so  */
+/* Random-init weights. The paper uses pretrained checkpoints (Sec. 5.1); they are absent, so  */
 /* every weight is drawn from a counter-based generator: splitmix64 (Steele, Lea and Flood,    */
 /* "Fast splittable pseudorandom number generators", OOPSLA 2014; the mixing function of       */
 /* Vigna's splitmix64.c) applied to seed ^ (tensor_id << 40) ^ index. The top 24 bits u give  */
@@ -446,7 +446,7 @@ int orc_lm_window_logits(const orc_cfg* c, const uint16_t* win_tok, int64_t n_po
 }
 
 /* ------------------------------------------------------------------------------------------ */
-/* Integer CDF (reading of the Torchac-based coder of Sec. 4.1; the paper does not say how    */
+/* Integer CDF (reading of the Torchac-based coder of Sec. 5.1; the paper does not say how    */
 /* the LM probabilities were made integer). T = 2^P, row z[0..V) of fp32 logits:               */
 /*  (i)   m = max z                                                                            */
 /*  (ii)  y_j = fp32(fp32(z_j - m) * C), C = fp32(2^16 * log2 e)   (round to nearest, no FMA) */
@@ -522,7 +522,7 @@ int orc_cdf_pair(const float* z, int V, int P, int sym, uint32_t* start, uint32_
 }
 
 /* ------------------------------------------------------------------------------------------ */
-/* Arithmetic coder (Sec. 2 "Arithmetic coding": the interval is split by P_AC per symbol,    */
+/* Arithmetic coder (Sec. 3 "Arithmetic coding": the interval is split by P_AC per symbol,    */
 /* symbol order low-to-high; any number of the final interval stands for the message).        */
 /* Exact integer form: range R (62 bits), low L (unbounded), B = bits shifted so far.          */
 /* Start R = 2^62, L = 0, B = 0. Per symbol (s = start, f = freq, T = 2^P):                    */
@@ -609,7 +609,7 @@ int64_t orc_range_encode(const uint32_t* start, const uint32_t* freq, int64_t n,
   return len;
 }
 
-/* Decoder (Sec. 2: decoding walks the same interval subdivision, finding at each step the
+/* Decoder (Sec. 3: decoding walks the same interval subdivision, finding at each step the
  * symbol whose interval holds the code). D = first 62 bits of the code (zero padded). Per symbol: r = R >> P;
  * t = D / r (t >= T means a corrupt code); s with cdf[s] <= t < cdf[s+1]; D -= r * cdf[s];
  * R = r * f_s; renormalise by the same k as the encoder, shifting the next k code bits into D. */
@@ -661,7 +661,7 @@ int orc_dec_step(orc_dec* d, const uint32_t* cdf, int V, int P) {
 
 /* ------------------------------------------------------------------------------------------ */
 /* Whole windows: LM forward -> fp32 logits -> integer CDF -> (start, freq) -> one code per    */
-/* window (Sec. 3 "Compression": windows are coded independently, each from a fresh BOS).     */
+/* window (Sec. 4 "Compression": windows are coded independently, each from a fresh BOS).     */
 /* ------------------------------------------------------------------------------------------ */
 
 /* The integer CDF of one position: over the whole vocabulary, or over the restricted alphabet

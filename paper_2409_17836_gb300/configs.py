@@ -1,8 +1,8 @@
-"""Model and coder shapes of the workloads (the paper's LLMs, Sec. 4.1, with random-init weights).
+"""Model and coder shapes of the workloads (the paper's LLMs, Sec. 5.1, with random-init weights).
 
 * TINY        2 layers, d 128, 4 heads, FFN 512, vocab 32, fp32, 256-token windows, P = 16
 * TINYLLAMA   TinyLlama-1.1B shape: 22 layers, d 2048, 32 Q / 4 KV heads, SwiGLU 5632, vocab 32000,
-              bf16, 2048-token windows (the paper's default window, Sec. 4.1), P = 24
+              bf16, 2048-token windows (the paper's default window, Sec. 5.1), P = 24
 * LLAMA2_7B   Llama-2-7B shape: 32 layers, d 4096, 32 heads (MHA), FFN 11008, vocab 32000, bf16,
               4096-token windows, P = 24
 P = 24 for vocab 32000 because at P = 16 the floor of one count per symbol would take 32000 of

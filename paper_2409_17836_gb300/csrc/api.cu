@@ -1,6 +1,6 @@
 // api.cu -- the C ABI of liblmgc.so (include/lmgc.h): context, model forward orchestration,
-// the encode pipeline (Sec. 3: serialise -> windows from BOS -> LM -> integer CDF -> one
-// arithmetic code per window -> container) and the KV-cached decode (Sec. 3 "Compression").
+// the encode pipeline (Sec. 4: serialise -> windows from BOS -> LM -> integer CDF -> one
+// arithmetic code per window -> container) and the KV-cached decode (Sec. 4 "Compression").
 #include <math.h>
 #include <stdio.h>
 #include <string.h>
@@ -21,7 +21,7 @@ void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 void set_thread_error(const std::string& s) { g_thread_err = s; }
 
-// tokens of n serialised values under the context's layout (Sec. 3; byte grouping, Sec. 4.3)
+// tokens of n serialised values under the context's layout (Sec. 4; byte grouping, Sec. 5.3)
 static int64_t n_tokens(const lmgc_ctx* ctx, int64_t n) {
   return serial_tokens(ctx->cfg.input_kind, ctx->cfg.sep_mode, ctx->cfg.byte_group, n);
 }

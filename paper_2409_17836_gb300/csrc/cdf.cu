@@ -1,8 +1,8 @@
 // cdf.cu -- logits -> integer CDF -> (start, freq) of the coded token, plus the decoder's
 // symbol search.
 //
-// The coder of Sec. 2 needs the model's distribution p(t | BOS, t_<) (Eq. 2) as an integer CDF
-// (the paper adapts Torchac, whose CDFs are integers; Sec. 4.1). For a row z[0..V), T = 2^P:
+// The coder of Sec. 3 needs the model's distribution p(t | BOS, t_<) (Eq. 2) as an integer CDF
+// (the paper adapts Torchac, whose CDFs are integers; Sec. 5.1). For a row z[0..V), T = 2^P:
 //   m = max z; y_j = fp32(fp32(z_j - m) * C), C = fp32(2^16 log2 e); a_j = -rint(y_j) (<= 40*2^16)
 //   e_j = ((H[(a>>8)&255] * L[a&255] + 2^30) >> 31) >> (a >> 16),   H[h] = round(2^31 2^(-h/256)),
 //         L[l] = round(2^31 2^(-l/65536))  -- a fixed-point 2^31 * exp(z_j - m)
@@ -480,7 +480,7 @@ void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const 
 }
 
 // ------------------------------------------------------------------------------------------
-// Decoder step (Sec. 2: the decoder repeatedly looks up the interval holding the code value).
+// Decoder step (Sec. 3: the decoder repeatedly looks up the interval holding the code value).
 // State per window: R, D (62-bit window of the code value minus L), the code's bit position.
 // t = D / (R >> P); the symbol s has cdf[s] <= t < cdf[s+1]; then D -= r cdf[s], R = r freq_s,
 // k = 62 - bitlen(R), R <<= k, D = (D << k) | next k code bits.

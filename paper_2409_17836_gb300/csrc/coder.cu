@@ -1,5 +1,5 @@
-// coder.cu -- the arithmetic coder (Sec. 2 "Arithmetic coding") in exact integer form, one
-// independent stream per window (Sec. 3 "Compression": each window is coded from its own BOS).
+// coder.cu -- the arithmetic coder (Sec. 3 "Arithmetic coding") in exact integer form, one
+// independent stream per window (Sec. 4 "Compression": each window is coded from its own BOS).
 //
 // Per stream: R = 2^62, L = 0, B = 0; per token (s = start, f = freq, T = 2^P):
 //   r = R >> P;  L += r*s;  R = r*f;  k = max(0, 62 - bitlen(R));  R <<= k;  L <<= k;  B += k

@@ -1,4 +1,4 @@
-// lm.cu -- the LM prior of Eq. 2 (a Llama-family decoder, Sec. 4.1): weight generation,
+// lm.cu -- the LM prior of Eq. 2 (a Llama-family decoder, Sec. 5.1): weight generation,
 // embedding, RMSNorm, RoPE, causal GQA attention, SwiGLU, and a CUDA-core GEMM.
 //
 // Every kernel here is row-invariant: a row's result depends only on that row's inputs (and, for

@@ -13,7 +13,7 @@
 
 namespace lmgc {
 
-// Token ids (character-level reading of Sec. 3 / Fig. 1).
+// Token ids (character-level reading of Sec. 4 / Fig. 1).
 constexpr int kTokSpace = 16, kTokComma = 17, kTokSemi = 18, kTokBos = 19;
 
 // Device error word bits (set by bounded device loops instead of spinning or trapping).
@@ -141,7 +141,7 @@ void note_launch();
 // ---- kernels' launchers (stream-ordered, no sync) ----
 // serialize.cu
 int tokens_per_value(int input_kind, int sep_mode);
-// Byte grouping (Sec. 4.3): tokens of n values; the n with that many tokens (or -1); whether the
+// Byte grouping (Sec. 5.3): tokens of n values; the n with that many tokens (or -1); whether the
 // layout is the default one group per value, most significant byte first.
 int64_t serial_tokens(int input_kind, int sep_mode, int byte_group, int64_t n);
 int64_t serial_values(int input_kind, int sep_mode, int byte_group, int64_t n_tok);

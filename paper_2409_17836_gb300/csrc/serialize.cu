@@ -1,6 +1,6 @@
 // serialize.cu -- fp32 / uint8 values -> hex-digit token ids with separators, and back.
 //
-// Sec. 3 "Serialization" and Fig. 1: each value's bits are cut into 4-bit groups, most
+// Sec. 4 "Serialization" and Fig. 1: each value's bits are cut into 4-bit groups, most
 // significant first (for fp32: the sign and exponent nibbles lead), each group becomes one hex
 // digit (token id = digit value 0..15), and a separator follows every value (' ' = 16,
 // ',' = 17, ', ' = 17 16, ';' = 18, or none).
@@ -18,7 +18,7 @@ int tokens_per_value(int input_kind, int sep_mode) {
   return nd + ns;
 }
 
-// Byte grouping (Sec. 4.3): bytes per value, and the group size (0 = one group per value).
+// Byte grouping (Sec. 5.3): bytes per value, and the group size (0 = one group per value).
 static int64_t bytes_per_value(int input_kind) { return input_kind == LMGC_IN_F32 ? 4 : 1; }
 static int sep_count(int sep_mode) { return sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1); }
 

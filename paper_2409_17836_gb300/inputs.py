@@ -4,16 +4,16 @@ This module holds input generators only (no step of the encode path). Both the C
 tests and the oracle's tests draw their inputs from here.
 
 The paper compresses gradients of networks trained on MNIST / CIFAR-10 / TinyImageNet
-(Sec. 4.1 "Datasets and models", "Evaluation protocols"). Those datasets and training runs are
+(Sec. 5.1 "Datasets and models", "Evaluation protocols"). Those datasets and training runs are
 not available, so seeded stand-ins of the same kind are used:
 
 * `tiny_gradient`      4,096 values = 4 tensors x 1,024, N(0, s_l^2), s_l = 10^(-3 + 2l/3).
 * `convnet_gradient`   the gradient of one cross-entropy step of a seeded random-init
                        4-layer ConvNet (298,954 parameters) on Gaussian 3x32x32 inputs.
-* `lossy_codes`        Sec. 5 "Compatibility": top-10% magnitude sparsification followed by
+* `lossy_codes`        Sec. 5.4 "Compatibility": top-10% magnitude sparsification followed by
                        8-bit linear quantisation (Eq. 4) of the kept values.
 * `laplace_gradient`   a 200-tensor Laplace mixture with log-uniform scales (throughput sweep).
-* `sparsified`, `quantized_codes`, `code_bytes`   the Sec. 5 compatibility inputs one at a time
+* `sparsified`, `quantized_codes`, `code_bytes`   the Sec. 5.4 compatibility inputs one at a time
                      (sparsification 50/25/10% as fp32; 16/8/1-bit Eq. 4 indices).
 """
 from __future__ import annotations
@@ -52,7 +52,7 @@ def convnet_gradient(seed: int = 0, batch: int = 64) -> np.ndarray:
 
 
 def sparsified(grad: np.ndarray, keep: float) -> np.ndarray:
-    """Sec. 5 sparsification alone: the floor(keep*N) largest |v| (ties to the lower index) in
+    """Sec. 5.4 sparsification alone: the floor(keep*N) largest |v| (ties to the lower index) in
     index order, still fp32 (the paper: sparsified gradients stay 32-bit floats)."""
     g = np.asarray(grad, dtype=np.float32)
     k = int(np.floor(keep * g.size))
@@ -61,7 +61,7 @@ def sparsified(grad: np.ndarray, keep: float) -> np.ndarray:
 
 
 def quantized_codes(grad: np.ndarray, bits: int) -> np.ndarray:
-    """Sec. 5 quantisation alone: Eq. 4 over every value (n = 16, 8 or 1 bits; 1 bit is SignSGD's
+    """Sec. 5.4 quantisation alone: Eq. 4 over every value (n = 16, 8 or 1 bits; 1 bit is SignSGD's
     setting); the indices are what is coded."""
     return lossy_codes(grad, keep=1.0, bits=bits)
 
@@ -76,7 +76,7 @@ def code_bytes(codes: np.ndarray) -> tuple[np.ndarray, int]:
 
 
 def lossy_codes(grad: np.ndarray, keep: float = 0.1, bits: int = 8) -> np.ndarray:
-    """Sec. 5: keep the floor(keep*N) largest |v| (ties to the lower index) in index order,
+    """Sec. 5.4: keep the floor(keep*N) largest |v| (ties to the lower index) in index order,
     then v_bar = (v - min v) / (max v - min v) * (2^bits - 1) (Eq. 4) over the kept values,
     rounded to nearest and clamped; the codes are what would be transmitted."""
     g = np.asarray(grad, dtype=np.float32)

@@ -55,7 +55,7 @@ class ModelConfig:
     init_std: float = 0.02
     rms_eps: float = 1e-5
     rope_theta: float = 10000.0
-    byte_group: int = 0  # bytes per separator group (Sec. 4.3 byte grouping); 0 = one group per value
+    byte_group: int = 0  # bytes per separator group (Sec. 5.3 byte grouping); 0 = one group per value
     byte_order: int = 0  # fp32 bytes most (0) or least (1) significant first
     alphabet: int = 0  # 1: integer CDFs over the ids the serialisation can emit only
 

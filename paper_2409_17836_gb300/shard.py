@@ -1,4 +1,4 @@
-"""Encoding one gradient on several GPUs: windows are independent (Sec. 3 "Compression": every
+"""Encoding one gradient on several GPUs: windows are independent (Sec. 4 "Compression": every
 window is coded from its own BOS), so each rank codes a contiguous range of windows with no data
 exchange. The one exchange step builds the container: the ranks all-gather their windows' bit
 lengths and token checksums (8 bytes per window) and payload slices; an exclusive scan of the

@@ -1,13 +1,13 @@
 """Edge cases and the largest configurations, through the C ABI:
 
 * empty inputs at every entry point that takes a count;
-* degenerate coder windows of 0, 1 and 2 tokens against the oracle (Sec. 2 coder);
+* degenerate coder windows of 0, 1 and 2 tokens against the oracle (Sec. 3 coder);
 * the 64M-value Laplace configuration: its serialisation sampled against the oracle, and
   windows at the start, middle and end of its 294,912-window stream coded in place and matched
   against a standalone encode of the same tokens, then decoded back (lossless);
 * the coder at the size of the coder-only benchmark (2^20 windows x 2048 tokens, vocabulary
   32000, P = 24): sampled windows bit-exact against the oracle, and every window's length within
-  the Sec. 2 bound J + 1 - eps < l <= J + 2 + eps."""
+  the Sec. 3 bound J + 1 - eps < l <= J + 2 + eps."""
 import numpy as np
 import pytest
 import torch

@@ -1,5 +1,5 @@
 """GPU parity of the integer stages against the oracle, through the C ABI:
-serialisation (Sec. 3), integer CDF given identical logits, and the arithmetic coder (Sec. 2)
+serialisation (Sec. 4), integer CDF given identical logits, and the arithmetic coder (Sec. 3)
 given identical (start, freq) pairs -- all bit-exact."""
 import numpy as np
 import pytest
@@ -66,7 +66,7 @@ def test_serialize_unaligned_input_and_u8():
 @pytest.mark.parametrize("group,order", [(1, 0), (2, 1), (3, 0), (3, 1), (4, 1), (8, 0), (8, 1)])
 @pytest.mark.parametrize("sep_mode", [0, 2, 4])
 def test_serialize_byte_groups_bit_exact(group, order, sep_mode):
-    """Byte grouping (Sec. 4.3): tokens bit-exact with the oracle for fp32 values (either byte
+    """Byte grouping (Sec. 5.3): tokens bit-exact with the oracle for fp32 values (either byte
     order) and uint8 codes, ragged counts whose last group is partial; round trip; the token
     count through lmgc_serial_tokens."""
     ctx = ctx_for(sep_mode=sep_mode, byte_group=group, byte_order=order)

@@ -1,4 +1,4 @@
-"""The synthetic input recipes (stand-ins for the paper's gradients, Sec. 4.1): sizes, scales and
+"""The synthetic input recipes (stand-ins for the paper's gradients, Sec. 5.1): sizes, scales and
 determinism as stated, so that every test and bench line draws the same inputs."""
 import numpy as np
 

@@ -1,4 +1,4 @@
-"""The Sec. 5 compatibility inputs one at a time (the f3 sweep): Eq. 4 quantisation to 16, 8 and
+"""The Sec. 5.4 compatibility inputs one at a time (the f3 sweep): Eq. 4 quantisation to 16, 8 and
 1 bits over every value, magnitude sparsification that keeps fp32 values, and the byte stream
 that carries 16-bit indices (4 hex digits per index through 2-byte groups). Worked by hand."""
 import numpy as np

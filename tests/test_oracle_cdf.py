@@ -1,4 +1,4 @@
-"""Pins of the oracle's integer CDF (the coder input of the Torchac-based coder, Sec. 4.1; the
+"""Pins of the oracle's integer CDF (the coder input of the Torchac-based coder, Sec. 5.1; the
 paper does not say how probabilities were made integer, so the quantiser is a reading pinned by
 exact table checks, closed forms, invariants and agreement with the softmax it approximates)."""
 import math

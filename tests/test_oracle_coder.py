@@ -1,4 +1,4 @@
-"""Pins of the oracle's arithmetic coder (Sec. 2 "Arithmetic coding" and its worked example):
+"""Pins of the oracle's arithmetic coder (Sec. 3 "Arithmetic coding" and its worked example):
 the paper's AAAB intervals and code, the entropy bound, the uniform closed form, brute force on
 tiny alphabets, and bit-equality with the arbitrary-precision restatement."""
 import itertools
@@ -33,7 +33,7 @@ def test_aaab_worked_example():
 @pytest.mark.parametrize("P", [8, 16, 20, 24])
 def test_integer_coder_code_lies_in_exact_interval(P):
     """The integer coder's code, read as a binary fraction, lies in the real interval of the
-    recursion of Sec. 2 computed with the same (quantised) probabilities."""
+    recursion of Sec. 3 computed with the same (quantised) probabilities."""
     T = 2 ** P
     fA = round(0.8 * T)
     starts, freqs = [0, 0, 0, fA], [fA, fA, fA, T - fA]
@@ -73,7 +73,7 @@ def test_matches_bigint_spec_and_bound(P):
         data, nbits = O.range_encode(np.array(st, dtype=np.uint32), np.array(fr, dtype=np.uint32), P)
         code, nb = spec.encode(st, fr, P)
         assert nb == nbits and data == spec.code_bytes(code, nb)
-        # entropy bound of Sec. 2 in its textbook form: J + 1 - eps < l <= J + 2 + eps
+        # entropy bound of Sec. 3 in its textbook form: J + 1 - eps < l <= J + 2 + eps
         J = -sum(math.log2(f / 2 ** P) for f in fr)
         eps = n * 2.0 ** (P - 60) * 1.45 + 1e-9
         assert J + 1 - eps < nbits <= J + 2 + eps

@@ -1,4 +1,4 @@
-"""Pins of the oracle LM prior (Eq. 1 / Eq. 2 with a Llama-family decoder, Sec. 4.1).
+"""Pins of the oracle LM prior (Eq. 1 / Eq. 2 with a Llama-family decoder, Sec. 5.1).
 
 The paper prints no logits, so the oracle is pinned by: the published splitmix64 test vector;
 torch library routines (rms_norm, scaled_dot_product_attention, silu, linear, embedding) in

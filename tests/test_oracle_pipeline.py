@@ -1,5 +1,5 @@
-"""Oracle end to end (Sec. 3): serialise -> windows with BOS -> LM -> integer CDF -> one code per
-window -> container; decoding each window token by token (KV-cached, Sec. 3 "Compression")
+"""Oracle end to end (Sec. 4): serialise -> windows with BOS -> LM -> integer CDF -> one code per
+window -> container; decoding each window token by token (KV-cached, Sec. 4 "Compression")
 must return the serialised tokens, and deserialising must return the input bits (lossless)."""
 import zlib
 

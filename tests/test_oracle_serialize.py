@@ -1,4 +1,4 @@
-"""Pins of the oracle's serialisation (Sec. 3 "Serialization", Fig. 1) against IEEE-754 closed
+"""Pins of the oracle's serialisation (Sec. 4 "Serialization", Fig. 1) against IEEE-754 closed
 forms, Python's struct/hex library routines, and a round-trip sweep of fp32 bit patterns."""
 import json
 import os
@@ -80,7 +80,7 @@ def test_tokens_per_value():
     assert O.tokens_per_value(1, 0) == 3
 
 
-# ---- byte grouping (Sec. 4.3 "Byte grouping": bytes per group BPG in {1, 2, 3, 4, 8}) ----
+# ---- byte grouping (Sec. 5.3 "Byte grouping": bytes per group BPG in {1, 2, 3, 4, 8}) ----
 
 def grouped_by_hex_string(vals: np.ndarray, sep_mode: int, group: int, order: int):
     """The definition through Python's bytes.hex(): the byte stream (each fp32 big- or
