@@ -280,9 +280,10 @@ def cpu_baseline(cfg, vals, tpv: float, bpv: int, target_s: float) -> dict:
 def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> dict:
     """HBM-bound stages at sizes where bandwidth, not launch latency, decides: the serialiser on
     the 64M-value Laplace mixture (default layout, and byte groups of 3 that cross values), and
-    the coder alone on 2^20 windows x 2048 tokens (the 64M-value sweep's coder microbenchmark) of
-    seeded random integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most
-    likely); ctx supplies the integer CDFs (any context with vocab 32000 and P = 24)."""
+    the coder alone (lmgc_range_encode_tiled, pairs in the window tiles the encode path uses) on
+    2^20 windows x 2048 tokens (the 64M-value sweep's coder microbenchmark) of seeded random
+    integer CDFs over vocab 32000 at P = 24 (half the symbols the row's most likely); ctx supplies
+    the integer CDFs (any context with vocab 32000 and P = 24)."""
     import numpy as np
     import torch
 
@@ -328,22 +329,28 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> 
     z = torch.randn(256, V, generator=g, device="cuda") * torch.linspace(0.3, 6.0, 256, device="cuda")[:, None]
     cdf = L.lmgc_quantize_cdf(ctx, z).long()
     likely = torch.argmax(cdf[:, 1:] - cdf[:, :-1], dim=1)
-    start = torch.empty((W, n_win), dtype=torch.int32, device="cuda")  # position-major
+    # window tiles, the encode path's layout: [window block][position group][window][position]
+    assert n_win % 32 == 0 and W % 8 == 0
+    NB, G = n_win // 32, W // 8
+    start = torch.empty((NB, G, 32, 8), dtype=torch.int32, device="cuda")
     freq = torch.empty_like(start)
-    step = min(n_win, 1 << 15)
-    for w0 in range(0, n_win, step):
-        row = torch.randint(0, 256, (W, step), generator=g, device="cuda")
-        sym = torch.randint(0, V, (W, step), generator=g, device="cuda")
-        sym = torch.where(torch.rand((W, step), generator=g, device="cuda") < 0.5, likely[row], sym)
+    step = min(NB, 1 << 10)  # 32,768 windows at a time
+    for b0 in range(0, NB, step):
+        nb = min(step, NB - b0)
+        row = torch.randint(0, 256, (W, nb * 32), generator=g, device="cuda")
+        sym = torch.randint(0, V, (W, nb * 32), generator=g, device="cuda")
+        sym = torch.where(torch.rand((W, nb * 32), generator=g, device="cuda") < 0.5, likely[row], sym)
         st = cdf[row, sym]
-        start[:, w0:w0 + step] = st.int()
-        freq[:, w0:w0 + step] = (cdf[row, sym + 1] - st).int()
-        del row, sym, st
-    payload, _ = L.lmgc_range_encode(start, freq, P, n_win, W, None, 1, n_win)
+        fr = cdf[row, sym + 1] - st
+        # [position][window] -> [block][group][window in block][position in group]
+        start[b0:b0 + nb] = st.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
+        freq[b0:b0 + nb] = fr.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
+        del row, sym, st, fr
+    payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None)
     torch.cuda.synchronize()
     L.lmgc_profile(None, True)
     for _ in range(reps):
-        payload, _ = L.lmgc_range_encode(start, freq, P, n_win, W, None, 1, n_win, out=payload)
+        payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None, out=payload)
     st = L.lmgc_kernel_stats(None)["range_encode"]
     L.lmgc_profile(None, False)
     kms = st["ms"] / max(1, st["launches"])

@@ -177,7 +177,8 @@ lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, co
  * integer form: R = 2^62, L = 0, B = 0; per token r = R >> P, L += r*start, R = r*freq,
  * k = max(0, 62 - bitlen(R)), R <<= k, L <<= k, B += k; the code is the top B + 2 bits of
  * ceil(L / 2^60) * 2^60, most significant bit first, padded with zeros to a byte.
- * Token i of window w is read at d_start[w*stride_win + i*stride_pos] (same for d_freq);
+ * Token i of window w is read at d_start[w*stride_win + i*stride_pos] (same for d_freq; every
+ * pair is checked: 0 < freq, start + freq <= 2^cdf_bits);
  * window w has d_win_len[w] tokens (device array), or win_tokens tokens when d_win_len is NULL.
  * d_out receives the codes of windows 0..n_win-1 back to back, each starting on a byte;
  * d_bitlen[w] (device) receives each code's bit length; *out_bytes (host) the total bytes.
@@ -188,6 +189,22 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
                               size_t win_tokens, const uint32_t* d_win_len, size_t stride_win, size_t stride_pos,
                               uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
                               lmgc_stream stream);
+
+/* lmgc_range_encode with the pairs in window tiles, the layout the encode path hands its coder:
+ * the pairs of 32 consecutive windows and 8 consecutive positions form one tile of 256 elements,
+ * tiles ordered by window block and then by position group. With G = ceil(win_tokens / 8), token
+ * i of window w is element ((w / 32) * G + i / 8) * 256 + (w % 32) * 8 + i % 8 of d_start (and of
+ * d_freq), arrays of lmgc_pair_tile_elems(n_win, win_tokens) elements, 16-byte aligned (elements
+ * past a window's length or past n_win are read but not used). Each thread codes one window and
+ * reads its 8 tokens of a group as two 16-byte vectors. Same arithmetic, output, scratch and
+ * errors as lmgc_range_encode. Syncs. */
+lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                                    size_t win_tokens, const uint32_t* d_win_len, uint8_t* d_out, size_t cap,
+                                    size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream);
+
+/* Elements of one window-tiled pair array for n_win windows of win_tokens positions
+ * (ceil(n_win / 32) * ceil(win_tokens / 8) * 256). */
+lmgc_status lmgc_pair_tile_elems(size_t n_win, size_t win_tokens, size_t* elems);
 
 /* lmgc_range_encode for callers that cannot allocate device memory (for example a process whose
  * device memory is held entirely by another allocator, or a latency-critical path where

@@ -589,20 +589,24 @@ lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, co
     return fail(ctx, LMGC_ERR_INVALID, "null argument");
   if (ctx->cfg.alphabet) {
     launch_cdf_pairs_alpha(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0,
-                           0, d_start, d_freq, 0, (cudaStream_t)stream, 0, ctx->alpha, ctx->d_err);
+                           d_start, d_freq, 0, (cudaStream_t)stream, 0, ctx->alpha, ctx->d_err);
     LMGC_CUDA(ctx, cudaGetLastError());
     return check_err_word(ctx, (cudaStream_t)stream, "cdf_pairs");
   }
-  launch_cdf_pairs(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0, 0,
+  launch_cdf_pairs(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0,
                    d_start, d_freq, 0, (cudaStream_t)stream);
   LMGC_CUDA(ctx, cudaGetLastError());
   return LMGC_OK;
 }
 
-lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
-                              size_t win_tokens, const uint32_t* d_win_len, size_t stride_win, size_t stride_pos,
-                              uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
-                              lmgc_stream stream) {
+}  // extern "C"
+
+// lmgc_range_encode and lmgc_range_encode_tiled: the coder over a caller's pairs (validated),
+// with stream-ordered scratch
+static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                                    size_t win_tokens, const uint32_t* d_win_len, size_t stride_win,
+                                    size_t stride_pos, bool tiled, uint8_t* d_out, size_t cap, size_t* out_bytes,
+                                    uint32_t* d_bitlen, lmgc_stream stream) {
   if (!out_bytes || (n_win && (!d_start || !d_freq || !d_bitlen)))
     return fail(nullptr, LMGC_ERR_INVALID, "null argument");
   if (cdf_bits < 1 || cdf_bits > 30) return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must be in 1..30");
@@ -624,7 +628,7 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
     {
       ProfScope ps(nullptr, kCoder, 8.0 * (double)n_win * (double)win_tokens, s);
       launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
-                          (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
+                          (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s, tiled, true);
     }
     launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
     uint64_t total = 0;
@@ -652,6 +656,29 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
   return st;
 }
 
+extern "C" {
+
+lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                              size_t win_tokens, const uint32_t* d_win_len, size_t stride_win, size_t stride_pos,
+                              uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
+                              lmgc_stream stream) {
+  return range_encode_any(d_start, d_freq, cdf_bits, n_win, win_tokens, d_win_len, stride_win, stride_pos, false,
+                          d_out, cap, out_bytes, d_bitlen, stream);
+}
+
+lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
+                                    size_t win_tokens, const uint32_t* d_win_len, uint8_t* d_out, size_t cap,
+                                    size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream) {
+  return range_encode_any(d_start, d_freq, cdf_bits, n_win, win_tokens, d_win_len, 0, 0, true, d_out, cap,
+                          out_bytes, d_bitlen, stream);
+}
+
+lmgc_status lmgc_pair_tile_elems(size_t n_win, size_t win_tokens, size_t* elems) {
+  if (!elems) return LMGC_ERR_INVALID;
+  *elems = (size_t)pair_tile_elems((int64_t)n_win, (int64_t)win_tokens);
+  return LMGC_OK;
+}
+
 lmgc_status lmgc_encode_bound(const lmgc_ctx* ctx, size_t n, size_t* bytes) {
   if (!ctx || !bytes) return LMGC_ERR_INVALID;
   const size_t n_tok = (size_t)n_tokens(ctx, (int64_t)n), W = (size_t)ctx->cfg.window;
@@ -676,9 +703,10 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   const size_t slot = slot_bytes((size_t)W, (int)P);
   // staging (grown on demand; reused across calls)
   LMGC_CUDA(ctx, ensure(&ctx->tok, &ctx->tok_cap, (size_t)n_tok * 2 + 16));
-  const size_t pair_need = (size_t)(W * n_win) * 4;
-  LMGC_CUDA(ctx, ensure(&ctx->pair_start, &ctx->pair_cap, 2 * pair_need));
-  ctx->pair_freq = ctx->pair_start + (size_t)(W * n_win);
+  // (start, freq) pairs in the coder's window tiles (whole tiles: 32-window blocks, 8-position groups)
+  const size_t pair_elems = (size_t)pair_tile_elems(n_win, W);
+  LMGC_CUDA(ctx, ensure(&ctx->pair_start, &ctx->pair_cap, 2 * pair_elems * 4));
+  ctx->pair_freq = ctx->pair_start + pair_elems;
   // win_len [n_win] u32 | bitlen [n_win] u32 | token crc [n_win] u32 | offsets [n_win+1] u64 | slots
   const size_t tbl = ((size_t)n_win * 4 + 255) / 256 * 256;
   const size_t wl_off = 0, bl_off = tbl, cr_off = 2 * tbl, of_off = 3 * tbl,
@@ -718,9 +746,9 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
       ProfScope ps(ctx, kCdf, (double)rows * (cols * 4 + 2 + 8), s);
       if (c.alphabet)
         launch_cdf_pairs_alpha(ctx->logits, rows, kAlphaCols, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0,
-                               n_win, ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha_cols, ctx->d_err);
+                               ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha_cols, ctx->d_err);
       else
-        launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0, n_win,
+        launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0,
                          ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
     }
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
@@ -731,8 +759,9 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   launch_window_crc(ctx->tok + w_begin * W, W, d_wl, n_win, ctx->enc_crc, s);
   {
     ProfScope ps(ctx, kCoder, (double)n_win * (double)W * 8, s);
-    launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 1, n_win, ctx->enc_slots, slot,
-                        ctx->enc_bl, ctx->d_err, s);
+    // the pairs come from the CDF kernels, valid by construction: no per-pair check
+    launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 0, 0, ctx->enc_slots, slot,
+                        ctx->enc_bl, ctx->d_err, s, true, false);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[3], s));
   launch_pack_codes(ctx->enc_slots, slot, ctx->enc_bl, n_win, ctx->enc_off, nullptr, s);

@@ -218,13 +218,14 @@ __device__ __forceinline__ uint64_t row_gsum(const float* __restrict__ z, int V,
 // it is the argmax: only then is the pass summing g over the whole row taken.
 // mode 0: row r codes d_sym[r]; pair index r.
 // mode 1: rows are positions of windows first_win + r / W; the coded token is tok[w*W + i];
-//         rows past the stream end are skipped; pair index i * stride_pos + w.
+//         rows past the stream end are skipped; the pair goes to window w - pair_win0's element
+//         of the coder's window tiles (pair_tile_index).
 // ------------------------------------------------------------------------------------------
 constexpr int kPairWarps = 8;
 
 __global__ void __launch_bounds__(32 * kPairWarps, 6) k_cdf_pairs(
     const float* __restrict__ logits, int64_t rows, int V, int P, const uint32_t* __restrict__ tab,
-    const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win, int64_t stride_pos,
+    const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win,
     uint32_t* __restrict__ start, uint32_t* __restrict__ freq, int mode, int64_t pair_win0,
     const uint32_t* __restrict__ row_max) {
   __shared__ uint32_t H[256], L[256];
@@ -249,7 +250,7 @@ __global__ void __launch_bounds__(32 * kPairWarps, 6) k_cdf_pairs(
       const int64_t gi = (first_win + wl) * W + i;
       if (gi >= n_tok) continue;  // warp-uniform
       sym = tok[gi];
-      out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
+      out_idx = pair_tile_index(first_win + wl - pair_win0, i, pair_tile_groups(W));
     }
     const float* z = logits + r * (int64_t)V;
     const bool vec = row_vec4(z, V);  // warp-uniform
@@ -329,7 +330,7 @@ __global__ void __launch_bounds__(32 * kPairWarps, 6) k_cdf_pairs(
 __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs_block(const float* __restrict__ logits, int64_t rows,
                                                                  int V, int P, const uint32_t* __restrict__ tab,
                                                            const uint16_t* __restrict__ tok, int64_t n_tok, int W,
-                                                           int64_t first_win, int64_t stride_pos,
+                                                           int64_t first_win,
                                                            uint32_t* __restrict__ start, uint32_t* __restrict__ freq,
                                                            int mode, int64_t pair_win0,
                                                            const uint32_t* __restrict__ row_max) {
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs_block(const float* __
       int64_t g = (first_win + wl) * W + i;
       if (g >= n_tok) continue;  // block-uniform
       sym = tok[g];
-      out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
+      out_idx = pair_tile_index(first_win + wl - pair_win0, i, pair_tile_groups(W));
     }
     const float* z = logits + r * (int64_t)V;
     RowStats st = row_stats(z, V, P, H, L, redf, redu, row_max ? row_max + r : nullptr);
@@ -381,7 +382,7 @@ __global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs_block(const float* __
 }
 
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
-                      int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
+                      int64_t n_tok, int W, int64_t first_win, uint32_t* start,
                       uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0, const uint32_t* row_max) {
   if (rows <= 0) return;
   if (!row_max) {
@@ -390,7 +391,7 @@ void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uin
     const unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
     note_launch();
     k_cdf_pairs_block<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
-                                                     pair_stride_pos, start, freq, mode, pair_win0, nullptr);
+                                                     start, freq, mode, pair_win0, nullptr);
     return;
   }
   // one wave of resident blocks, each warp walking rows
@@ -405,7 +406,7 @@ void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uin
   const int64_t blocks = std::min<int64_t>((rows + kPairWarps - 1) / kPairWarps, resident);
   note_launch();
   k_cdf_pairs<<<(unsigned)blocks, 32 * kPairWarps, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
-                                                          pair_stride_pos, start, freq, mode, pair_win0, row_max);
+                                                          start, freq, mode, pair_win0, row_max);
 }
 
 // Block inclusive scan of one u64 per thread; returns the inclusive prefix; *total the tile sum.
@@ -652,7 +653,7 @@ __device__ __forceinline__ int alpha_index(const AlphaIds& alpha, int t) {
 // The pairs of k_cdf_pairs (same modes and output indexing) over the restricted alphabet.
 __global__ void __launch_bounds__(32 * kAlphaWarps) k_cdf_pairs_alpha(
     const float* __restrict__ logits, int64_t rows, int V, int P, const uint32_t* __restrict__ tab,
-    const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win, int64_t stride_pos,
+    const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win,
     uint32_t* __restrict__ start, uint32_t* __restrict__ freq, int mode, int64_t pair_win0, AlphaIds alpha,
     uint32_t* err) {
   __shared__ uint32_t H[256], L[256];
@@ -675,7 +676,7 @@ __global__ void __launch_bounds__(32 * kAlphaWarps) k_cdf_pairs_alpha(
       const int64_t gi = (first_win + wl) * W + i;
       if (gi >= n_tok) continue;  // warp-uniform
       sym = tok[gi];
-      out_idx = (int64_t)i * stride_pos + (first_win + wl - pair_win0);
+      out_idx = pair_tile_index(first_win + wl - pair_win0, i, pair_tile_groups(W));
     }
     uint32_t st, fr;
     alpha_cdf_lane(logits + r * (int64_t)V, alpha, P, H, L, st, fr);
@@ -694,14 +695,14 @@ __global__ void __launch_bounds__(32 * kAlphaWarps) k_cdf_pairs_alpha(
 }
 
 void launch_cdf_pairs_alpha(const float* logits, int64_t rows, int V, int P, const uint32_t* tab,
-                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos,
+                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win,
                             uint32_t* start, uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0,
                             const AlphaIds& alpha, uint32_t* err) {
   if (rows <= 0) return;
   const int64_t blocks = std::min<int64_t>((rows + kAlphaWarps - 1) / kAlphaWarps, 152 * 16);
   note_launch();
   k_cdf_pairs_alpha<<<(unsigned)blocks, 32 * kAlphaWarps, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
-                                                                 pair_stride_pos, start, freq, mode, pair_win0, alpha,
+                                                                 start, freq, mode, pair_win0, alpha,
                                                                  err);
 }
 

@@ -6,17 +6,27 @@
 // and the code is the top B + 2 bits of v = ceil(L / 2^60) * 2^60 (v lies in [L, L + R) because
 // R >= 2^61), most significant bit first.
 //
-// The range R depends only on the freq sequence; L is the only unbounded quantity. A thread keeps
-// the low 62 bits of L in a register (as 4 L, so that the carry out of them is the carry out of
-// a 64-bit add); the bits shifted above them collect in a 32-bit pending word and leave in 32-bit
-// words to the stream's own scratch slot. A carry out of the low 62 bits increments the emitted
-// bits: the pending ones, or -- when they were all ones -- the already written words of this
-// stream's slot (never beyond word 0: L + R stays below 2^(B+62)). The carry walk is bounded by
-// the slot length. All shifts are 32-bit funnel shifts by less than 32 (k <= P <= 30 per token).
+// Form computed here (the same integers, no shift of L). R depends only on the freq sequence, and
+// only r = R >> P is kept: after R = r f and the shift by k, the next r is (r f) >> (P - k), with
+// k = clz(r f) - 2 over 64 bits (0 for r f = 2^62). In stream coordinates (bit j of the code has
+// weight 2^-(j+1)) token i's addend r s occupies bits [B_i, B_i + 62), B_i being the shift total
+// before it, so L is the sum of the addends at their positions. A thread keeps stream bits
+// [32 w, 32 w + 96) in three registers a0:a1:a2 and adds each addend at offset off = B - 32 w,
+// which stays in [3, 34] between tokens (sh = 34 - off is a funnel-shift count below 32). Word a0
+// is complete when off reaches 35: it leaves, the window moves one word on. A carry out of a0
+// increments the completed words before it (never beyond word 0: L + R stays below 2^(B+62)).
 //
-// Layout: one stream per thread, 32 windows per warp. Pairs are read at
-// start[w*stride_win + i*stride_pos]; with the encode path's position-major layout
-// (stride_win = 1) a warp's 32 loads of token i are one 128-byte transaction.
+// Per token: two 32x32->64 multiply-adds per product, three funnel shifts, a three-word add with
+// carry, a count of leading zeros and a handful of selects (the step is inline PTX so that each
+// operation is one instruction). Completed words go to a per-thread ring in shared memory and
+// leave for the stream's slot in 16-byte chunks, at most two per 8 tokens: scattered 4-byte
+// stores from 32 lanes to 32 slots would cost one memory transaction each.
+//
+// Layout: one stream per thread, 32 windows per warp. Pairs are read from window tiles (the
+// encode path; a warp reads one contiguous kilobyte per array per 8 tokens) or at
+// start[w*stride_win + i*stride_pos] (lmgc_range_encode's general layout, 8 tokens ahead).
+// Slot words are stored in native byte order; the pack step writes the bytes most significant
+// first.
 #include <algorithm>
 #include <mutex>
 #include <string>
@@ -25,188 +35,273 @@
 
 namespace lmgc {
 
+// ceil((W P + 2) / 32) + 1 words, rounded up to 16 bytes (whole 16-byte chunks)
 size_t slot_bytes(size_t win_tokens, int P) {
   size_t bits = win_tokens * (size_t)P + 2;
   size_t words = (bits + 31) / 32 + 1;
   return ((words * 4 + 15) / 16) * 16;
 }
 
-__device__ __forceinline__ uint32_t bswap32(uint32_t x) { return __byte_perm(x, 0, 0x0123); }
+constexpr int kRingWords = 16;   // completed words not yet written (at most 3 + 8 between flushes)
+constexpr int kRingStride = 20;  // words per thread in shared memory: 16-byte aligned, few bank conflicts
+constexpr int kCoderThreads = 128;
 
-// 64-bit add with the carry out of bit 63
-__device__ __forceinline__ uint64_t add_carry(uint64_t a, uint64_t b, uint32_t& c) {
-  uint32_t lo, hi;
-  asm("add.cc.u32 %0, %3, %5;\n\taddc.cc.u32 %1, %4, %6;\n\taddc.u32 %2, 0, 0;"
-      : "=r"(lo), "=r"(hi), "=r"(c)
-      : "r"((uint32_t)a), "r"((uint32_t)(a >> 32)), "r"((uint32_t)b), "r"((uint32_t)(b >> 32)));
-  return ((uint64_t)hi << 32) | lo;
-}
-
-// One stream's coder state in 32-bit pieces. L is held as L4 = 4 L (its 62 bits at the top of a
-// 64-bit word, so a carry out of bit 62 of L is the carry out of the 64-bit add); the emitted bits
-// not yet written form `acc` (nacc < 32 bits, right-aligned). Every shift is a 32-bit (funnel)
-// shift by less than 32: k <= P <= 30 bits move per token.
-struct Coder {
-  uint32_t R_hi, R_lo;
-  uint64_t L4;
-  uint32_t acc, nacc, wpos, max_words;
-  uint32_t* slot;  // stream words, big-endian
+struct Stream {
+  uint32_t rlo, rhi;   // r = R >> P
+  uint32_t a0, a1, a2; // stream bits [32 w, 32 w + 96)
+  int32_t sh;          // 34 - (B - 32 w), in [0, 31] between tokens
+  int32_t w;           // word index of a0 (-1 before the first word completes)
+  int32_t fw;          // words [0, fw) are in the slot, [fw, w) only in the ring
+  uint32_t chk;        // OR of s | (f - 1) | (s + f - 1) over the tokens: >= T iff a pair was invalid
+  uint32_t max_words;
+  uint32_t* slot;
+  uint32_t* ring;
   bool overflow;
 
-  __device__ __forceinline__ void write(uint32_t wv) {
-    if (wpos < max_words) slot[wpos] = bswap32(wv);
-    else overflow = true;
-    wpos++;
+  __device__ __forceinline__ void init(int P, uint32_t* sl, uint32_t mw, uint32_t* rg) {
+    const uint64_t r0 = 1ull << (62 - P);  // R = 2^62
+    rlo = (uint32_t)r0;
+    rhi = (uint32_t)(r0 >> 32);
+    a0 = a1 = a2 = 0u;
+    sh = 2;  // B = 0 at w = -1: off = 32
+    w = -1;
+    fw = 0;
+    chk = 0u;
+    max_words = mw;
+    slot = sl;
+    ring = rg;
+    overflow = false;
   }
-  // +cy (0 or 1) into the emitted bits: the pending ones, else (all ones) the written words
-  __device__ __forceinline__ void carry(uint32_t cy) {
-    acc += cy;
-    if ((acc >> nacc) != 0u) {  // only when cy = 1 and the pending bits were all ones
-      acc = 0u;
-      int64_t i = (int64_t)wpos - 1;
-      for (; i >= 0; --i) {
-        uint32_t v = bswap32(slot[i]) + 1u;
-        slot[i] = bswap32(v);
-        if (v != 0u) break;
+  // +1 into the completed words before a0 (ring or slot); a carry past word 0 cannot happen for
+  // valid input and is reported
+  __device__ __forceinline__ void carry() {
+    for (int32_t i = w - 1; i >= 0; --i) {
+      uint32_t v;
+      if (i >= fw) {
+        v = ring[i & (kRingWords - 1)] + 1u;
+        ring[i & (kRingWords - 1)] = v;
+      } else {
+        if ((uint32_t)i >= max_words) break;
+        v = slot[i] + 1u;
+        slot[i] = v;
       }
-      if (i < 0) overflow = true;  // impossible for valid input; reported, not propagated
+      if (v != 0u) return;
+    }
+    overflow = true;
+  }
+  // a0:a1:a2 += chi:clo placed with its bit 61 at stream position B; returns the carry out of a0
+  __device__ __forceinline__ uint32_t add(uint32_t clo, uint32_t chi) {
+    uint32_t cy;
+    asm("{\n\t.reg .u32 x0, x1, x2;\n\t"
+        "shf.l.wrap.b32 x2, 0, %4, %6;\n\t"
+        "shf.l.wrap.b32 x1, %4, %5, %6;\n\t"
+        "shf.l.wrap.b32 x0, %5, 0, %6;\n\t"
+        "add.cc.u32 %2, %2, x2;\n\t"
+        "addc.cc.u32 %1, %1, x1;\n\t"
+        "addc.cc.u32 %0, %0, x0;\n\t"
+        "addc.u32 %3, 0, 0;\n\t}"
+        : "+r"(a0), "+r"(a1), "+r"(a2), "=r"(cy)
+        : "r"(clo), "r"(chi), "r"(sh));
+    return cy;
+  }
+  // one token; a completed word goes to the ring
+  template <bool CHECK>
+  __device__ __forceinline__ void token(uint32_t s, uint32_t f, int P) {
+    if (CHECK) {
+      const uint32_t u = f - 1u;
+      chk |= s | u | (s + u);
+    }
+    uint32_t clo, chi, plo, phi;
+    asm("{\n\t.reg .u64 c;\n\tmul.wide.u32 c, %2, %3;\n\tmov.b64 {%0, %1}, c;\n\tmad.lo.u32 %1, %4, %3, %1;\n\t}"
+        : "=r"(clo), "=r"(chi)
+        : "r"(rlo), "r"(s), "r"(rhi));
+    if (add(clo, chi)) carry();
+    asm("{\n\t.reg .u64 c;\n\tmul.wide.u32 c, %2, %3;\n\tmov.b64 {%0, %1}, c;\n\tmad.lo.u32 %1, %4, %3, %1;\n\t}"
+        : "=r"(plo), "=r"(phi)
+        : "r"(rlo), "r"(f), "r"(rhi));
+    // k = 62 - bitlen(r f): clz of the high word less 2, plus 1 for r f = 2^62 (f = T). For any
+    // input k lies in [0, 30], so sh and w stay bounded whatever the pairs hold.
+    int32_t k;
+    asm("{\n\t.reg .u32 z, t;\n\tclz.b32 z, %1;\n\tshr.u32 t, %1, 30;\n\tadd.u32 z, z, t;\n\tsub.s32 %0, z, 2;\n\t}"
+        : "=r"(k)
+        : "r"(phi));
+    const int32_t s2 = P - k;  // in [0, P] for valid pairs
+    asm("shf.r.wrap.b32 %0, %1, %2, %3;" : "=r"(rlo) : "r"(plo), "r"(phi), "r"(s2));
+    asm("shr.u32 %0, %1, %2;" : "=r"(rhi) : "r"(phi), "r"(s2));
+    sh -= k;
+    const bool full = sh < 0;
+    if (full) ring[w & (kRingWords - 1)] = a0;
+    a0 = full ? a1 : a0;
+    a1 = full ? a2 : a1;
+    a2 = full ? 0u : a2;
+    sh += full ? 32 : 0;
+    w += full ? 1 : 0;
+  }
+  // the completed 16-byte chunks of the ring to the slot: k <= 30 per token, so at most 8 words
+  // complete per 8 tokens and two chunks leave at most 3 + 8 - 8 words behind
+  template <int CHUNKS>
+  __device__ __forceinline__ void flush() {
+#pragma unroll
+    for (int q = 0; q < CHUNKS; q++) {
+      if (w - fw >= 4) {
+        const uint4 v = *reinterpret_cast<const uint4*>(ring + (fw & (kRingWords - 1)));
+        if ((uint32_t)(fw + 3) < max_words) *reinterpret_cast<uint4*>(slot + fw) = v;
+        fw += 4;
+      }
     }
   }
-  // move the top k (< 32) bits of L4 to the pending bits; L4 and R shift left by k
-  __device__ __forceinline__ void shift_out(uint32_t k) {
-    const uint32_t l_hi = (uint32_t)(L4 >> 32), l_lo = (uint32_t)L4;
-    const uint32_t a_hi = __funnelshift_l(acc, 0u, k);            // acc >> (32 - k), 0 for k = 0
-    const uint32_t a_lo = (acc << k) | __funnelshift_l(l_hi, 0u, k);
-    L4 = ((uint64_t)__funnelshift_l(l_lo, l_hi, k) << 32) | (l_lo << k);
-    R_hi = __funnelshift_l(R_lo, R_hi, k);
-    R_lo <<= k;
-    // a full word leaves when 32 or more bits are pending (a_hi = 0 otherwise); no branch
-    const bool full = nacc + k >= 32u;
-    nacc = full ? nacc + k - 32u : nacc + k;
-    const uint32_t wv = __funnelshift_r(a_lo, a_hi, nacc);  // the top 32 of the nacc + 32 pending bits
-    const bool in_slot = wpos < max_words;
-    if (full && in_slot) slot[wpos] = bswap32(wv);
-    overflow |= full && !in_slot;
-    wpos += full ? 1u : 0u;
-    acc = full ? (a_lo & ((1u << nacc) - 1u)) : a_lo;
+  // termination: v = ceil(L / 2^60) * 2^60, i.e. add 2^60 - 1 at B and keep the top B + 2 bits;
+  // returns B + 2 and writes every remaining word
+  __device__ __forceinline__ uint64_t finish() {
+    if (add(0xFFFFFFFFu, 0x0FFFFFFFu)) carry();
+    const int32_t off = 34 - sh;
+    int32_t nrem;  // bits of the code in a0 (and a1)
+    uint64_t nbits;
+    if (w < 0) {  // B < 3: a0 holds stream bits [-32, 0), zero for valid input
+      overflow |= a0 != 0u;
+      a0 = a1;
+      a1 = a2;
+      w = 0;
+      nrem = off - 30;
+      nbits = (uint64_t)nrem;
+    } else {
+      nrem = off + 2;
+      nbits = (uint64_t)w * 32u + (uint64_t)nrem;
+    }
+    for (int32_t i = fw; i < w; i++)
+      if ((uint32_t)i < max_words) slot[i] = ring[i & (kRingWords - 1)];
+    if ((uint32_t)w < max_words) slot[w] = nrem >= 32 ? a0 : a0 & ~(0xFFFFFFFFu >> nrem);
+    if (nrem > 32 && (uint32_t)(w + 1) < max_words) slot[w + 1] = a1 & ~(0xFFFFFFFFu >> (nrem - 32));
+    return nbits;
   }
 };
 
-// Per token (s = start, f = freq, T = 2^P): r = R >> P; L4 += 4 r s (carry -> emitted bits);
-// R = r f; k = max(0, clz(R) - 2); shift_out(k). R >= 2^(61 - P) after the multiply, so for
-// P <= 29 its high word is nonzero (HI32: a 32-bit count of leading zeros).
-template <bool HI32>
-__device__ __forceinline__ void code_token(Coder& c, uint32_t s, uint32_t f, int P, uint32_t T, bool& bad) {
-  // 0 < f <= T and s + f <= T; an invalid pair stops the stream after its group (the arithmetic
-  // stays bounded meanwhile: writes are slot-checked and the carry walk stops at word 0)
-  bad |= (f - 1u >= T) | (s > T - f);
-  const uint32_t r_lo = __funnelshift_r(c.R_lo, c.R_hi, (uint32_t)P), r_hi = c.R_hi >> P;
-  const uint64_t r = ((uint64_t)r_hi << 32) | r_lo;
-  uint32_t cy;
-  c.L4 = add_carry(c.L4, r * (uint64_t)(s << 2), cy);  // r s < 2^62, so 4 r s < 2^64
-  c.carry(cy);
-  const uint64_t Rn = r * (uint64_t)f;
-  c.R_hi = (uint32_t)(Rn >> 32);
-  c.R_lo = (uint32_t)Rn;
-  int k = (HI32 ? __clz((int)c.R_hi) : __clzll((long long)Rn)) - 2;
-  k = max(k, 0);                // R = 2^62 (f = T) needs no shift
-  if (!HI32) k = min(k, 31);    // only an invalid f = 0 reaches past P
-  c.shift_out((uint32_t)k);
-}
-
-template <bool HI32>
-__global__ void __launch_bounds__(128) k_range_encode(const uint32_t* __restrict__ start,
-                                                      const uint32_t* __restrict__ freq, int P, int64_t n_win,
-                                                      int64_t win_tokens, const uint32_t* __restrict__ win_len,
-                                                      int64_t stride_win, int64_t stride_pos, uint8_t* __restrict__ slots,
-                                                      size_t slot_sz, uint32_t* __restrict__ bitlen, uint32_t* err) {
+// One stream per thread. TILED: pairs in window tiles (vector loads, 8 tokens a group);
+// otherwise at start[w*stride_win + i*stride_pos], loaded 8 tokens ahead. PT: P at compile
+// time (0: P_rt). CHECK: validate the pairs (a window stops after the group holding an invalid
+// pair, and the error word reports it).
+template <int PT, bool CHECK, bool TILED>
+__global__ void __launch_bounds__(kCoderThreads) k_range_encode(
+    const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
+    int64_t win_tokens, const uint32_t* __restrict__ win_len, int64_t stride_win, int64_t stride_pos,
+    uint8_t* __restrict__ slots, size_t slot_sz, uint32_t* __restrict__ bitlen, uint32_t* err) {
+  __shared__ __align__(16) uint32_t rings[kCoderThreads * kRingStride];
+  const int P = PT ? PT : P_rt;
+  const uint32_t T = 1u << P;
   const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (w >= n_win) return;
-  const int64_t n = win_len ? (int64_t)win_len[w] : win_tokens;
-  const uint32_t T = 1u << P;
-  Coder c;
-  c.R_hi = 1u << 30;  // R = 2^62
-  c.R_lo = 0u;
-  c.L4 = 0ull;
-  c.acc = 0u;
-  c.nacc = 0u;
-  c.wpos = 0u;
-  c.max_words = (uint32_t)(slot_sz / 4);
-  c.slot = reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz);
-  c.overflow = false;
+  int64_t n = win_len ? (int64_t)win_len[w] : win_tokens;
   bool bad = n > win_tokens;
-  // the pairs of the next kPre tokens are loaded ahead so their latency overlaps the serial chain;
-  // the load pointers advance by the position stride
-  constexpr int kPre = 8;
-  const uint32_t* qs = start + w * stride_win;
-  const uint32_t* qf = freq + w * stride_win;
-  uint32_t bs[kPre], bf[kPre];
+  if (bad) n = 0;  // a window longer than its slot is not coded
+  Stream c;
+  c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz), (uint32_t)(slot_sz / 4),
+         rings + threadIdx.x * kRingStride);
+  if (TILED) {
+    const int64_t groups = pair_tile_groups(win_tokens);
+    const int64_t g_end = (n + 7) >> 3;
+    const int64_t e0 = pair_tile_index(w, 0, groups);
+    const uint4* qs = reinterpret_cast<const uint4*>(start + e0);
+    const uint4* qf = reinterpret_cast<const uint4*>(freq + e0);
+    uint4 s0 = make_uint4(0, 0, 0, 0), s1 = s0, f0 = s0, f1 = s0;
+    if (g_end > 0) {
+      s0 = __ldcs(qs); s1 = __ldcs(qs + 1); f0 = __ldcs(qf); f1 = __ldcs(qf + 1);
+    }
+    for (int64_t g = 0; g < g_end; g++) {
+      const uint32_t cs[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+      const uint32_t cf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+      if (g + 1 < g_end) {  // the next tile of this window block: 256 elements on
+        qs += 64;
+        qf += 64;
+        s0 = __ldcs(qs); s1 = __ldcs(qs + 1); f0 = __ldcs(qf); f1 = __ldcs(qf + 1);
+      }
+      if (8 * g + 8 <= n) {
 #pragma unroll
-  for (int j = 0; j < kPre; j++) {
-    bs[j] = j < n ? __ldcs(qs) : 0u;
-    bf[j] = j < n ? __ldcs(qf) : 1u;
-    qs += stride_pos;
-    qf += stride_pos;
-  }
-  for (int64_t i0 = 0; i0 < n && !bad; i0 += kPre) {
-    uint32_t cs[kPre], cf[kPre];
-    const bool full_next = i0 + 2 * kPre <= n;
+        for (int j = 0; j < 8; j++) c.template token<CHECK>(cs[j], cf[j], P);
+      } else {
+        const int jn = (int)(n - 8 * g);
+#pragma unroll
+        for (int j = 0; j < 8; j++)
+          if (j < jn) c.template token<CHECK>(cs[j], cf[j], P);
+      }
+      c.template flush<2>();
+      if (CHECK && c.chk >= T) break;
+    }
+  } else {
+    constexpr int kPre = 8;
+    const uint32_t* qs = start + w * stride_win;
+    const uint32_t* qf = freq + w * stride_win;
+    uint32_t bs[kPre], bf[kPre];
 #pragma unroll
     for (int j = 0; j < kPre; j++) {
-      cs[j] = bs[j];
-      cf[j] = bf[j];
-      if (full_next || i0 + kPre + j < n) {
-        bs[j] = __ldcs(qs);
-        bf[j] = __ldcs(qf);
-      } else {
-        bs[j] = 0u;
-        bf[j] = 1u;
-      }
+      bs[j] = j < n ? __ldcs(qs) : 0u;
+      bf[j] = j < n ? __ldcs(qf) : 1u;
       qs += stride_pos;
       qf += stride_pos;
     }
-    if (i0 + kPre <= n) {
+    for (int64_t i0 = 0; i0 < n; i0 += kPre) {
+      uint32_t cs[kPre], cf[kPre];
+      const bool full_next = i0 + 2 * kPre <= n;
 #pragma unroll
-      for (int j = 0; j < kPre; j++) code_token<HI32>(c, cs[j], cf[j], P, T, bad);
-    } else {
-      const int jn = (int)(n - i0);
+      for (int j = 0; j < kPre; j++) {
+        cs[j] = bs[j];
+        cf[j] = bf[j];
+        if (full_next || i0 + kPre + j < n) {
+          bs[j] = __ldcs(qs);
+          bf[j] = __ldcs(qf);
+        }
+        qs += stride_pos;
+        qf += stride_pos;
+      }
+      if (i0 + kPre <= n) {
 #pragma unroll
-      for (int j = 0; j < kPre; j++)
-        if (j < jn) code_token<HI32>(c, cs[j], cf[j], P, T, bad);
+        for (int j = 0; j < kPre; j++) c.template token<CHECK>(cs[j], cf[j], P);
+      } else {
+        const int jn = (int)(n - i0);
+#pragma unroll
+        for (int j = 0; j < kPre; j++)
+          if (j < jn) c.template token<CHECK>(cs[j], cf[j], P);
+      }
+      c.template flush<2>();
+      if (CHECK && c.chk >= T) break;
     }
   }
-  // termination: v = ceil(L / 2^60) * 2^60; emit its top 2 bits of the low 62
-  {
-    uint32_t cy;
-    c.L4 = add_carry(c.L4, ((1ull << 60) - 1ull) << 2, cy);
-    c.carry(cy);
-  }
-  c.shift_out(2u);
-  // every emitted bit went through the pending bits: B + 2 bits in all
-  const uint64_t nbits = (uint64_t)c.wpos * 32u + c.nacc;
-  if (c.nacc > 0u) c.write(c.acc << (32u - c.nacc));
-  bitlen[w] = (uint32_t)nbits;
-  if (bad || c.overflow) atomicOr(err, kErrCorrupt);
+  bitlen[w] = (uint32_t)c.finish();
+  if (bad || c.overflow || (CHECK && c.chk >= T)) atomicOr(err, kErrCorrupt);
+}
+
+template <bool CHECK, bool TILED>
+static void launch_coder(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
+                         const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
+                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
+  const unsigned g = (unsigned)((n_win + kCoderThreads - 1) / kCoderThreads);
+  if (P == 24)
+    k_range_encode<24, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                                 stride_pos, slots, slot_sz, bitlen, err);
+  else if (P == 16)
+    k_range_encode<16, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                                 stride_pos, slots, slot_sz, bitlen, err);
+  else
+    k_range_encode<0, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                                stride_pos, slots, slot_sz, bitlen, err);
 }
 
 void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
                          const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
-                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
+                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s, bool tiled, bool check) {
   if (n_win <= 0) return;
   note_launch();
-  if (P <= 29)
-    k_range_encode<true><<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
-                                                                        stride_win, stride_pos, slots, slot_sz, bitlen,
-                                                                        err);
-  else
-    k_range_encode<false><<<(unsigned)((n_win + 127) / 128), 128, 0, s>>>(start, freq, P, n_win, win_tokens, win_len,
-                                                                         stride_win, stride_pos, slots, slot_sz, bitlen,
-                                                                         err);
+  if (tiled) {
+    if (check) launch_coder<true, true>(start, freq, P, n_win, win_tokens, win_len, 0, 0, slots, slot_sz, bitlen, err, s);
+    else launch_coder<false, true>(start, freq, P, n_win, win_tokens, win_len, 0, 0, slots, slot_sz, bitlen, err, s);
+  } else {
+    launch_coder<true, false>(start, freq, P, n_win, win_tokens, win_len, stride_win, stride_pos, slots, slot_sz,
+                              bitlen, err, s);
+  }
 }
 
 // ------------------------------------------------------------------------------------------
 // Container payload: exclusive scan of the code byte lengths (one block), then each window's
-// ceil(bitlen/8) bytes copied from its slot to its offset.
+// ceil(bitlen/8) bytes copied from its slot (words in native order) to its offset.
 // ------------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_scan_lengths(const uint32_t* __restrict__ bitlen, int64_t n,
                                                        uint64_t* __restrict__ off) {
@@ -251,7 +346,8 @@ __global__ void k_copy_codes(const uint8_t* __restrict__ slots, size_t slot_sz, 
     const uint32_t nb = (bitlen[w] + 7u) / 8u;
     const uint8_t* src = slots + (size_t)w * slot_sz;
     uint8_t* dst = out + off[w];
-    for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x) dst[b] = src[b];
+    // slot words are in native (little-endian) byte order; the code's bytes go most significant first
+    for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x) dst[b] = src[b ^ 3u];
   }
 }
 

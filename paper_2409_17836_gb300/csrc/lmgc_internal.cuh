@@ -209,7 +209,7 @@ void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s);  // builds H and L on 
 // mode 1: pair index i * pair_stride_pos + (window - pair_win0)
 // row_max (optional): float_key of each row's maximum, which replaces the kernel's max pass
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
-                      int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos, uint32_t* start,
+                      int64_t n_tok, int W, int64_t first_win, uint32_t* start,
                       uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0 = 0,
                       const uint32_t* row_max = nullptr);
 void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
@@ -217,8 +217,7 @@ void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const 
 // launch_cdf_pairs over the restricted alphabet (no row_max input); a token outside it sets
 // kErrCorrupt in *err and gets the pair (0, 1)
 void launch_cdf_pairs_alpha(const float* logits, int64_t rows, int V, int P, const uint32_t* tab,
-                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win, int64_t pair_stride_pos,
-                            uint32_t* start, uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0,
+                            const uint16_t* tok, int64_t n_tok, int W, int64_t first_win, uint32_t* start, uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0,
                             const AlphaIds& alpha, uint32_t* err);
 void launch_dec_search_alpha(const float* logits, int64_t n, int V, int P, const uint32_t* tab, void* dec_state,
                              const uint8_t* codes, uint16_t* sym_out, int64_t sym_stride, int64_t pos,
@@ -228,10 +227,26 @@ void launch_dec_search(const float* logits, int64_t n, int V, int P, const uint3
                        const uint32_t* win_len, uint32_t* err, cudaStream_t s);
 
 // coder.cu
+// Window tiles: the coder's input layout on the encode path. The (start, freq) pairs of 32
+// consecutive windows and 8 consecutive positions form one tile of 256 elements, element
+// (w % 32) * 8 + i % 8; tiles follow each other by window block, then by position group, with
+// G = ceil(W / 8) groups per window. A thread reading its window's 8 tokens of a group reads two
+// 16-byte vectors, and a warp's 32 threads one contiguous kilobyte per array.
+__host__ __device__ __forceinline__ int64_t pair_tile_groups(int64_t W) { return (W + 7) >> 3; }
+__host__ __device__ __forceinline__ int64_t pair_tile_index(int64_t w, int64_t i, int64_t groups) {
+  return (((w >> 5) * groups + (i >> 3)) << 8) + ((w & 31) << 3) + (i & 7);
+}
+// elements of a tiled pair array for n_win windows of W positions (whole tiles)
+__host__ __device__ __forceinline__ int64_t pair_tile_elems(int64_t n_win, int64_t W) {
+  return ((n_win + 31) >> 5) * pair_tile_groups(W) * 256;
+}
 size_t slot_bytes(size_t win_tokens, int P);
+// pairs at start[w * stride_win + i * stride_pos] (tiled = false) or in window tiles (tiled =
+// true, strides ignored); check: validate every pair (entry points taking a caller's pairs)
 void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
                          const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
-                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s);
+                         size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s, bool tiled = false,
+                         bool check = true);
 void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win,
                        uint64_t* offsets /* [n_win+1] scratch */, uint8_t* out, cudaStream_t s);
 // crc32 of the little-endian bytes of tok[w * stride .. w * stride + len[w]) for each w < n_win

@@ -43,3 +43,13 @@ def random_pairs(rng, n_win, W, P, lens=None, V=32000, layout="pos"):
     if lens is None:
         lens = np.full(n_win, W, dtype=np.uint32)
     return start, freq, lens
+
+
+def to_pair_tiles(a: np.ndarray) -> np.ndarray:
+    """A [n_win][W] (window-major) pair array in the coder's window tiles: 32 windows x 8 positions
+    per 256-element tile, tiles by window block then by position group, padding zero."""
+    n_win, W = a.shape
+    nb, G = -(-n_win // 32), -(-W // 8)
+    pad = np.zeros((nb * 32, G * 8), dtype=a.dtype)
+    pad[:n_win, :W] = a
+    return np.ascontiguousarray(pad.reshape(nb, 32, G, 8).transpose(0, 2, 1, 3)).reshape(-1)

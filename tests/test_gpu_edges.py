@@ -14,7 +14,7 @@ import torch
 
 import oracle as O
 from paper_2409_17836_gb300 import configs, inputs as I, lmgc as L
-from tests._util import random_pairs
+from tests._util import random_pairs, to_pair_tiles
 
 pytestmark = pytest.mark.gpu
 
@@ -39,17 +39,24 @@ def test_empty_inputs():
     ctx.close()
 
 
+@pytest.mark.parametrize("tiled", [False, True])
 @pytest.mark.parametrize("P", [16, 24])
-def test_degenerate_window_lengths(P):
-    """Windows of 0, 1, 2 and W tokens in one call: each code equals the oracle's code of the
-    same prefix (a window of no tokens codes to the 2 termination bits)."""
+def test_degenerate_window_lengths(P, tiled):
+    """Windows of 0, 1, 2, 7, 8, 9 and W tokens in one call (row-major strides, or window tiles
+    whose 8-position groups end mid-window): each code equals the oracle's code of the same prefix
+    (a window of no tokens codes to the 2 termination bits)."""
     rng = np.random.default_rng(P)
     W = 64
-    lens = np.array([0, 1, 2, W, 1, 0], dtype=np.uint32)
+    lens = np.array([0, 1, 2, W, 1, 0, 7, 8, 9], dtype=np.uint32)
     start, freq, _ = random_pairs(rng, lens.size, W, P, V=32 if P == 16 else 32000, layout="row")
-    out, bitlen = L.lmgc_range_encode(torch.from_numpy(start.view(np.int32)).cuda(),
-                                      torch.from_numpy(freq.view(np.int32)).cuda(), P, lens.size, W,
-                                      torch.from_numpy(lens.view(np.int32)).cuda(), W, 1)
+    wl = torch.from_numpy(lens.view(np.int32)).cuda()
+    if tiled:
+        out, bitlen = L.lmgc_range_encode_tiled(torch.from_numpy(to_pair_tiles(start).view(np.int32)).cuda(),
+                                                torch.from_numpy(to_pair_tiles(freq).view(np.int32)).cuda(), P,
+                                                lens.size, W, wl)
+    else:
+        out, bitlen = L.lmgc_range_encode(torch.from_numpy(start.view(np.int32)).cuda(),
+                                          torch.from_numpy(freq.view(np.int32)).cuda(), P, lens.size, W, wl, W, 1)
     bl = bitlen.cpu().numpy().astype(np.int64)
     payload = out.cpu().numpy().tobytes()
     off = 0
@@ -110,10 +117,12 @@ def test_laplace_64m_windows_in_place_and_round_trip(laplace):
 
 def test_range_encode_coder_benchmark_size():
     """2^20 windows x 2048 tokens (2^31 tokens) over 256 random integer CDFs of vocabulary 32000
-    at P = 24, position-major: sampled windows bit-exact against the oracle, and every window's
-    bit length within the coding bound of its own (start, freq) stream."""
+    at P = 24, in the window tiles the encode path and the coder microbenchmark use: sampled
+    windows bit-exact against the oracle, and every window's bit length within the coding bound of
+    its own (start, freq) stream."""
     n_win, W, P, V = 1 << 20, 2048, 24, 32000
     T = 1 << P
+    G, NB = W // 8, n_win // 32
     rng = np.random.default_rng(2048)
     cdfs = []
     for _ in range(256):
@@ -123,30 +132,34 @@ def test_range_encode_coder_benchmark_size():
         cdfs.append(np.concatenate([[0], np.cumsum(f)]))
     cdf = torch.from_numpy(np.array(cdfs, dtype=np.int32)).cuda()  # [256][V + 1]
     g = torch.Generator(device="cuda").manual_seed(2048)
-    start = torch.empty((W, n_win), dtype=torch.int32, device="cuda")
-    freq = torch.empty((W, n_win), dtype=torch.int32, device="cuda")
-    for p0 in range(0, W, 128):  # position chunks keep the temporaries small
+    # tiles as [window block][position group][window in block][position in group]
+    start = torch.empty((NB, G, 32, 8), dtype=torch.int32, device="cuda")
+    freq = torch.empty((NB, G, 32, 8), dtype=torch.int32, device="cuda")
+    assert start.numel() == L.lmgc_pair_tile_elems(n_win, W)
+    flat = cdf.view(-1)
+    for g0 in range(0, G, 16):  # 128 positions at a time keep the temporaries small
         row = torch.randint(0, 256, (128, n_win), device="cuda", generator=g)
         sym = torch.randint(0, V, (128, n_win), device="cuda", generator=g)
-        flat = cdf.view(-1)
         lo = flat[row * (V + 1) + sym]
-        start[p0:p0 + 128] = lo
-        freq[p0:p0 + 128] = flat[row * (V + 1) + sym + 1] - lo
-        del row, sym, lo
-    out, bitlen = L.lmgc_range_encode(start, freq, P, n_win, W, None, 1, n_win)
+        fr = flat[row * (V + 1) + sym + 1] - lo
+        # [position][window] -> [block][group][window in block][position in group]
+        start[:, g0:g0 + 16] = lo.view(16, 8, NB, 32).permute(2, 0, 3, 1)
+        freq[:, g0:g0 + 16] = fr.view(16, 8, NB, 32).permute(2, 0, 3, 1)
+        del row, sym, lo, fr
+    out, bitlen = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None)
     bl = bitlen.cpu().numpy().astype(np.int64)
     # the bound for every window: J = -sum log2(freq / T), eps <= n 2^(P-60) 1.45
-    J = torch.zeros(n_win, dtype=torch.float64, device="cuda")
-    for p0 in range(0, W, 128):
-        J -= torch.log2(freq[p0:p0 + 128].double() / T).sum(0)
-    J = J.cpu().numpy()
+    J = torch.zeros((NB, 32), dtype=torch.float64, device="cuda")
+    for g0 in range(0, G, 16):
+        J -= torch.log2(freq[:, g0:g0 + 16].double() / T).sum(dim=(1, 3))
+    J = J.view(-1).cpu().numpy()
     eps = W * 2.0 ** (P - 60) * 1.45
     assert np.all(bl > J + 1 - eps) and np.all(bl <= J + 2 + eps)
     offs = np.concatenate([[0], np.cumsum((bl + 7) // 8)])
     assert offs[-1] == out.numel()
     for w in [0, 1, 31, 32, n_win // 2, n_win - 1] + rng.integers(0, n_win, 8).tolist():
-        s = start[:, w].cpu().numpy().view(np.uint32)
-        f = freq[:, w].cpu().numpy().view(np.uint32)
+        s = start[w // 32, :, w % 32, :].reshape(-1).cpu().numpy().view(np.uint32)
+        f = freq[w // 32, :, w % 32, :].reshape(-1).cpu().numpy().view(np.uint32)
         code, nbits = O.range_encode(s, f, P)
         assert bl[w] == nbits, w
         assert out[offs[w]: offs[w + 1]].cpu().numpy().tobytes() == code, w

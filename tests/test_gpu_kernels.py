@@ -7,7 +7,7 @@ import torch
 
 import oracle as O
 from paper_2409_17836_gb300 import configs, lmgc as L
-from tests._util import random_pairs
+from tests._util import random_pairs, to_pair_tiles
 
 pytestmark = pytest.mark.gpu
 
@@ -152,30 +152,72 @@ def test_cdf_bit_exact(V, P, rows):
     ctx.close()
 
 
-@pytest.mark.parametrize("P,layout", [(16, "row"), (24, "pos"), (24, "row"), (30, "pos")])
-def test_range_encode_bit_exact(P, layout):
-    rng = np.random.default_rng(P)
-    n_win, W = 70, 300
-    V = 32 if P == 16 else 1000
-    start, freq, lens = random_pairs(rng, n_win, W, P, V=V)
-    lens = rng.integers(1, W + 1, n_win).astype(np.uint32)
-    lens[0], lens[1], lens[-1] = W, 1, 17
+def coder(start, freq, P, n_win, W, lens, layout):
+    """The GPU coder on [n_win][W] pairs passed in the given layout: row-major and position-major
+    through lmgc_range_encode's strides, window tiles through lmgc_range_encode_tiled."""
+    wl = torch.from_numpy(lens.view(np.int32)).cuda() if lens is not None else None
+    if layout == "tile":
+        st, fr = to_pair_tiles(start), to_pair_tiles(freq)
+        assert st.size == L.lmgc_pair_tile_elems(n_win, W)
+        return L.lmgc_range_encode_tiled(torch.from_numpy(st.view(np.int32)).cuda(),
+                                         torch.from_numpy(fr.view(np.int32)).cuda(), P, n_win, W, wl)
     if layout == "row":
         s_dev, f_dev, sw, sp = start, freq, W, 1
     else:
         s_dev, f_dev, sw, sp = start.T.copy(), freq.T.copy(), 1, n_win
-    out, bitlen = L.lmgc_range_encode(torch.from_numpy(s_dev.view(np.int32)).cuda(),
-                                      torch.from_numpy(f_dev.view(np.int32)).cuda(), P, n_win, W,
-                                      torch.from_numpy(lens.view(np.int32)).cuda(), sw, sp)
+    return L.lmgc_range_encode(torch.from_numpy(s_dev.view(np.int32)).cuda(),
+                               torch.from_numpy(f_dev.view(np.int32)).cuda(), P, n_win, W, wl, sw, sp)
+
+
+def check_codes(out, bitlen, start, freq, P, lens):
     payload = out.cpu().numpy().tobytes()
     bl = bitlen.cpu().numpy()
     off = 0
-    for w in range(n_win):
+    for w in range(start.shape[0]):
         code, nbits = O.range_encode(start[w, :lens[w]], freq[w, :lens[w]], P)
         assert bl[w] == nbits, w
         assert payload[off: off + len(code)] == code, w
         off += len(code)
     assert off == len(payload)
+
+
+@pytest.mark.parametrize("P,layout", [(16, "row"), (24, "pos"), (24, "row"), (30, "pos"), (16, "tile"), (24, "tile"),
+                                      (30, "tile"), (7, "tile")])
+def test_range_encode_bit_exact(P, layout):
+    """Ragged windows (lengths 1..300, one of 17) over random integer CDFs, 70 windows (two full
+    32-window blocks and a partial one), W = 300 (not a multiple of the 8-position tile group)."""
+    rng = np.random.default_rng(P)
+    n_win, W = 70, 300
+    V = 32 if P <= 16 else 1000
+    if P == 7:
+        V = 100
+    start, freq, lens = random_pairs(rng, n_win, W, P, V=V)
+    lens = rng.integers(1, W + 1, n_win).astype(np.uint32)
+    lens[0], lens[1], lens[-1] = W, 1, 17
+    out, bitlen = coder(start, freq, P, n_win, W, lens, layout)
+    check_codes(out, bitlen, start, freq, P, lens)
+
+
+@pytest.mark.parametrize("layout", ["tile", "pos"])
+@pytest.mark.parametrize("P", [16, 24])
+def test_range_encode_carry_heavy(P, layout):
+    """Streams built to carry: mostly tokens at the top of the range (start = T - freq) with small
+    freq, so L's low bits fill with ones and additions carry into already completed words, some
+    through whole words of ones; plus probability-one tokens (freq = T), which shift nothing."""
+    rng = np.random.default_rng(100 + P)
+    T = 1 << P
+    n_win, W = 64, 512
+    freq = rng.integers(1, 6, (n_win, W)).astype(np.int64)
+    start = T - freq - rng.integers(0, 2, (n_win, W))
+    low = rng.random((n_win, W)) < 0.08  # an occasional low symbol
+    start = np.where(low, rng.integers(0, T // 2, (n_win, W)), start)
+    one = rng.random((n_win, W)) < 0.05
+    freq = np.where(one, T, freq)
+    start = np.where(one, 0, np.clip(start, 0, T - freq))
+    start, freq = start.astype(np.uint32), freq.astype(np.uint32)
+    lens = np.full(n_win, W, np.uint32)
+    out, bitlen = coder(start, freq, P, n_win, W, lens, layout)
+    check_codes(out, bitlen, start, freq, P, lens)
 
 
 def test_range_encode_many_windows_sampled():
@@ -201,6 +243,16 @@ def test_range_encode_rejects_bad_pairs():
     f = torch.zeros(4, dtype=torch.int32, device="cuda")  # freq 0 is invalid
     with pytest.raises(L.LmgcError):
         L.lmgc_range_encode(s, f, 16, 1, 4, None, 4, 1)
+    # window tiles: freq 0, freq above T, start + freq above T, each in its own window of a block
+    T = 1 << 16
+    for bad in [(0, 0), (0, T + 1), (T - 3, 4), (0xFFFFFFFF, 2)]:
+        st = np.zeros((3, 20), np.uint32)
+        fr = np.full((3, 20), 2, np.uint32)
+        st[1, 13], fr[1, 13] = bad
+        with pytest.raises(L.LmgcError) as e:
+            L.lmgc_range_encode_tiled(torch.from_numpy(to_pair_tiles(st).view(np.int32)).cuda(),
+                                      torch.from_numpy(to_pair_tiles(fr).view(np.int32)).cuda(), 16, 3, 20, None)
+        assert e.value.status == L.ERR_INVALID, bad
 
 
 @pytest.mark.parametrize("sep_mode,V,P", [(0, 32, 16), (2, 1000, 20), (4, 32000, 24)])
