@@ -194,10 +194,10 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * the pairs of 32 consecutive windows and 8 consecutive positions form one tile of 256 elements,
  * tiles ordered by window block and then by position group. With G = ceil(win_tokens / 8), token
  * i of window w is element ((w / 32) * G + i / 8) * 256 + (w % 32) * 8 + i % 8 of d_start (and of
- * d_freq), arrays of lmgc_pair_tile_elems(n_win, win_tokens) elements, 16-byte aligned (elements
- * past a window's length or past n_win are read but not used). Each thread codes one window and
- * reads its 8 tokens of a group as two 16-byte vectors. Same arithmetic, output, scratch and
- * errors as lmgc_range_encode. Syncs. */
+ * d_freq), arrays of lmgc_pair_tile_elems(n_win, win_tokens) elements, 16-byte aligned (INVALID
+ * otherwise; elements past a window's length or past n_win are read but not used). Each thread
+ * codes one window; a warp stages its 32 windows' tiles through shared memory with bulk copies.
+ * Same arithmetic, output, scratch and errors as lmgc_range_encode. Syncs. */
 lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
                                     size_t win_tokens, const uint32_t* d_win_len, uint8_t* d_out, size_t cap,
                                     size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream);

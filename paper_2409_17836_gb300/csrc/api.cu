@@ -593,9 +593,16 @@ lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, co
     LMGC_CUDA(ctx, cudaGetLastError());
     return check_err_word(ctx, (cudaStream_t)stream, "cdf_pairs");
   }
+  // the encode's kernel, with each row's maximum from a pass of its own (stream-ordered scratch)
+  cudaStream_t s = (cudaStream_t)stream;
+  if (rows == 0) return LMGC_OK;
+  uint32_t* keys = nullptr;
+  LMGC_CUDA(ctx, cudaMallocAsync((void**)&keys, rows * 4, s));
   launch_cdf_pairs(d_logits, (int64_t)rows, ctx->cfg.vocab, ctx->cfg.cdf_bits, ctx->exp2_tab, d_sym, 0, 1, 0,
-                   d_start, d_freq, 0, (cudaStream_t)stream);
-  LMGC_CUDA(ctx, cudaGetLastError());
+                   d_start, d_freq, 0, s, 0, keys, false);
+  const cudaError_t e = cudaGetLastError();
+  cudaFreeAsync(keys, s);
+  LMGC_CUDA(ctx, e);
   return LMGC_OK;
 }
 
@@ -612,6 +619,9 @@ static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_f
   if (cdf_bits < 1 || cdf_bits > 30) return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must be in 1..30");
   *out_bytes = 0;
   if (n_win == 0) return LMGC_OK;
+  // the tiles are staged by bulk copies, whose sources must be 16-byte aligned
+  if (tiled && (((uintptr_t)d_start | (uintptr_t)d_freq) & 15))
+    return fail(nullptr, LMGC_ERR_INVALID, "range_encode_tiled: pair arrays must be 16-byte aligned");
   cudaStream_t s = (cudaStream_t)stream;
   const size_t slot = slot_bytes(win_tokens, cdf_bits);
   uint8_t* slots = nullptr;
@@ -749,7 +759,7 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
                                ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->alpha_cols, ctx->d_err);
       else
         launch_cdf_pairs(ctx->logits, rows, c.vocab, (int)P, ctx->exp2_tab, ctx->tok, n_tok, (int)W, w0,
-                         ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max_valid ? ctx->row_max : nullptr);
+                         ctx->pair_start, ctx->pair_freq, 1, s, w_begin, ctx->row_max, ctx->row_max_valid);
     }
     cudaEventRecord(ctx->batch_ev[2 * b + 2], s);
   }

@@ -210,35 +210,131 @@ __device__ __forceinline__ uint64_t row_gsum(const float* __restrict__ z, int V,
 
 // ------------------------------------------------------------------------------------------
 // Pairs of the coded tokens, one warp per row (the encode path). Per row the work is one read of
-// the logits: the maximum comes from the vocabulary GEMM (row_max: the float_key of each row's
-// maximum), then one pass forms e_j, S = sum e_j and the lowest index with exponent code 0 (the
-// argmax of e). The
+// the logits: the maximum comes with them (row_max: the float_key of each row's maximum, from the
+// vocabulary GEMM's epilogue or from k_row_max_key), then one pass forms e_j and S = sum e_j. The
 // symbol's start needs g_j = floor(e_j (T - V) / S) for j below the symbol only, plus the
-// remainder (T - V) - sum g when the argmax lies below it, and its freq needs that remainder when
-// it is the argmax: only then is the pass summing g over the whole row taken.
+// remainder (T - V) - sum g when the argmax of e (its lowest index with exponent code 0) lies
+// below it, and its freq needs that remainder when the argmax is the symbol. So the pass over
+// j <= sym also looks for code 0 there (the first one found is the argmax), and only then is the
+// pass summing g over the whole row taken.
+//
+// Tables: H and L are held once per lane in shared memory, so a warp's 32 lookups fall in 32
+// distinct banks whatever the indices (one wavefront each, against about three for one shared
+// copy with random indices). Entry i of both tables sits at byte 256 i: lane c's copy of H2[i] at
+// + 4c, of L[i] at + 128 + 4c, so each byte offset is one logic or byte-permute operation on a.
+// H2[h] = 2 H[h] for h >= 1 and H2[0] = 2^32 - 1 (2 H[0] = 2^32 does not fit); then
+// (H2 L + 2^31) >> 32 = (H L + 2^30) >> 31 for every (h, l) (for h = 0 because L <= 2^31), so
+// the rounded product is the high word of one 32 x 32 + 64-bit multiply-add.
+// The exponent code is not clamped: where the clamp would act (y < -40 * 2^16) the unclamped code
+// is at least 40 * 2^16 as well, or (y < -2^22, -inf or NaN, where the rounding add leaves its
+// exact range) at least 2^22 modulo 2^32, and e = 0 for both; a = 0 iff y rounds to 0 either way.
+// Loads: 4 float4 per lane per stage and two stages in flight (the next stage is issued before
+// the current one is reduced); the next row's first stage is issued before this row's epilogue.
 // mode 0: row r codes d_sym[r]; pair index r.
 // mode 1: rows are positions of windows first_win + r / W; the coded token is tok[w*W + i];
 //         rows past the stream end are skipped; the pair goes to window w - pair_win0's element
 //         of the coder's window tiles (pair_tile_index).
 // ------------------------------------------------------------------------------------------
-constexpr int kPairWarps = 8;
+constexpr int kPairWarps = 16;
+constexpr int kPairSmem = 256 * 256;  // 256 entries x (32 copies of H2, 32 copies of L), u32
 
-__global__ void __launch_bounds__(32 * kPairWarps, 6) k_cdf_pairs(
+// a = -rint(fp32(fp32(z - m) * C)) modulo 2^32 without the clamp (see above); mone = 2^32 - 1,
+// passed at run time so that the subtraction is a multiply-add
+__device__ __forceinline__ uint32_t exp2_code_u(float z, float m, uint32_t mone) {
+  const float C = (float)(65536.0 * 1.4426950408889634073599246810019);
+  const float t = __fadd_rn(__fmul_rn(__fsub_rn(z, m), C), 12582912.f);
+  uint32_t a;
+  asm("mad.lo.u32 %0, %1, %2, 0x4B400000;" : "=r"(a) : "r"(__float_as_uint(t)), "r"(mone));
+  return a;
+}
+
+// e of exp2_from_code through this lane's table copies (tb: the tables' base; l4 = 4 lane,
+// l4h = 4 lane + 128)
+__device__ __forceinline__ uint32_t exp2_rep(uint32_t a, const char* tb, uint32_t l4, uint32_t l4h) {
+  const uint32_t h2 = *reinterpret_cast<const uint32_t*>(tb + ((a & 0xFF00u) | l4));
+  const uint32_t l = *reinterpret_cast<const uint32_t*>(tb + __byte_perm(a, l4h, 0x5504));
+  const uint32_t e31 = (uint32_t)(((uint64_t)h2 * (uint64_t)l + 0x80000000ull) >> 32);
+  uint32_t e;
+  asm("shr.b32 %0, %1, %2;" : "=r"(e) : "r"(e31), "r"(a >> 16));
+  return e;
+}
+
+struct TabLane {
+  const char* tb;
+  uint32_t l4, l4h, one, mone;
+  __device__ __forceinline__ uint32_t code(float z, float m) const { return exp2_code_u(z, m, mone); }
+  __device__ __forceinline__ uint32_t e(uint32_t a) const { return exp2_rep(a, tb, l4, l4h); }
+  // S += e as one multiply-add by a 1 known only at run time
+  __device__ __forceinline__ void acc(uint64_t& S, uint32_t x) const {
+    asm("mad.wide.u32 %0, %1, %2, %0;" : "+l"(S) : "r"(x), "r"(one));
+  }
+  __device__ __forceinline__ void acc4(uint64_t& S, const float4& v, float m) const {
+    acc(S, e(code(v.x, m)));
+    acc(S, e(code(v.y, m)));
+    acc(S, e(code(v.z, m)));
+    acc(S, e(code(v.w, m)));
+  }
+  __device__ __forceinline__ uint64_t g4(const float4& v, float m, const RowStats& st) const {
+    return gfloor(e(code(v.x, m)), st) + gfloor(e(code(v.y, m)), st) + gfloor(e(code(v.z, m)), st) +
+           gfloor(e(code(v.w, m)), st);
+  }
+};
+
+__device__ __forceinline__ float4 ld_stream4(const float4* p) {
+  float4 v;
+  asm("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+      : "l"(p));
+  return v;
+}
+
+struct Stage4 {
+  float4 v0, v1, v2, v3;
+  __device__ __forceinline__ void load(const float4* p) {  // p: this lane's first float4 of the stage
+    v0 = ld_stream4(p);
+    v1 = ld_stream4(p + 32);
+    v2 = ld_stream4(p + 64);
+    v3 = ld_stream4(p + 96);
+  }
+  __device__ __forceinline__ void acc(uint64_t& S, float m, const TabLane& t) const {
+    t.acc4(S, v0, m);
+    t.acc4(S, v1, m);
+    t.acc4(S, v2, m);
+    t.acc4(S, v3, m);
+  }
+};
+
+__global__ void __launch_bounds__(32 * kPairWarps, 2) k_cdf_pairs(
     const float* __restrict__ logits, int64_t rows, int V, int P, const uint32_t* __restrict__ tab,
     const uint16_t* __restrict__ tok, int64_t n_tok, int W, int64_t first_win,
     uint32_t* __restrict__ start, uint32_t* __restrict__ freq, int mode, int64_t pair_win0,
     const uint32_t* __restrict__ row_max) {
-  __shared__ uint32_t H[256], L[256];
-  for (int i = threadIdx.x; i < 256; i += 32 * kPairWarps) {
-    H[i] = tab[i];
-    L[i] = tab[256 + i];
+  extern __shared__ __align__(16) uint32_t rep_tab[];  // [256][64]: H2 x 32, L x 32
+  for (int i = threadIdx.x; i < 256 * 64; i += 32 * kPairWarps) {
+    const int j = i >> 6;
+    const uint32_t h = tab[j];
+    rep_tab[i] = (i & 32) ? tab[256 + j] : (h >= 0x80000000u ? 0xFFFFFFFFu : 2u * h);
   }
   __syncthreads();
   const int lane = threadIdx.x & 31;
+  TabLane tl;
+  tl.tb = reinterpret_cast<const char*>(rep_tab);
+  tl.l4 = 4u * (uint32_t)lane;
+  tl.l4h = tl.l4 | 128u;
+  tl.one = (uint32_t)(P > 0);
+  tl.mone = 0u - tl.one;
   const uint64_t Mq = (1ull << P) - (uint64_t)V;
-  const int V4 = V >> 2;
-  for (int64_t r = (int64_t)blockIdx.x * kPairWarps + (threadIdx.x >> 5); r < rows;
-       r += (int64_t)gridDim.x * kPairWarps) {
+  const int64_t step = (int64_t)gridDim.x * kPairWarps;
+  // rows start 16-byte aligned and hold whole float4s (kernel-uniform)
+  const bool vec = (V & 3) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0;
+  const int n4 = V >> 2;
+  const int ng = vec ? n4 >> 7 : 0;  // whole stages of 128 float4s per row
+  Stage4 A, B;
+  int64_t r = (int64_t)blockIdx.x * kPairWarps + (threadIdx.x >> 5);
+  if (r < rows && ng > 0) A.load(reinterpret_cast<const float4*>(logits + r * (int64_t)V) + lane);
+  for (; r < rows; r += step) {
+    const int64_t rn = r + step;
+    const float4* zn = reinterpret_cast<const float4*>(logits + rn * (int64_t)V) + lane;
     int sym;
     int64_t out_idx;
     if (mode == 0) {
@@ -248,165 +344,110 @@ __global__ void __launch_bounds__(32 * kPairWarps, 6) k_cdf_pairs(
       const int64_t wl = r / W;
       const int i = (int)(r - wl * W);
       const int64_t gi = (first_win + wl) * W + i;
-      if (gi >= n_tok) continue;  // warp-uniform
+      if (gi >= n_tok) {  // warp-uniform; stage 0 of the next row replaces this row's
+        if (rn < rows && ng > 0) A.load(zn);
+        continue;
+      }
       sym = tok[gi];
       out_idx = pair_tile_index(first_win + wl - pair_win0, i, pair_tile_groups(W));
     }
     const float* z = logits + r * (int64_t)V;
-    const bool vec = row_vec4(z, V);  // warp-uniform
-    const float4* z4 = reinterpret_cast<const float4*>(z);
+    const float4* z4 = reinterpret_cast<const float4*>(z) + lane;
     const float m = __uint_as_float(key_float_bits(row_max[r]));
     uint64_t S = 0;
-    int best = 0x7fffffff;  // a lane's indices increase, so its first code 0 is its lowest
     if (vec) {
-      int j = lane;
-      for (; j + 32 < V4; j += 64) {  // two loads in flight per lane
-        const float4 v = __ldg(z4 + j), u = __ldg(z4 + j + 32);
-        const int a0 = exp2_code(v.x, m), a1 = exp2_code(v.y, m), a2 = exp2_code(v.z, m), a3 = exp2_code(v.w, m);
-        const int b0 = exp2_code(u.x, m), b1 = exp2_code(u.y, m), b2 = exp2_code(u.z, m), b3 = exp2_code(u.w, m);
-        S += (uint64_t)exp2_from_code(a0, H, L) + (uint64_t)exp2_from_code(a1, H, L) +
-             (uint64_t)exp2_from_code(a2, H, L) + (uint64_t)exp2_from_code(a3, H, L);
-        S += (uint64_t)exp2_from_code(b0, H, L) + (uint64_t)exp2_from_code(b1, H, L) +
-             (uint64_t)exp2_from_code(b2, H, L) + (uint64_t)exp2_from_code(b3, H, L);
-        if (best == 0x7fffffff) {
-          if (min(min(a0, a1), min(a2, a3)) == 0)
-            best = 4 * j + (a0 == 0 ? 0 : a1 == 0 ? 1 : a2 == 0 ? 2 : 3);
-          else if (min(min(b0, b1), min(b2, b3)) == 0)
-            best = 4 * (j + 32) + (b0 == 0 ? 0 : b1 == 0 ? 1 : b2 == 0 ? 2 : 3);
-        }
+      int g = 0;
+      for (; g + 2 <= ng; g += 2) {
+        B.load(z4 + (g + 1) * 128);
+        A.acc(S, m, tl);
+        if (g + 2 < ng) A.load(z4 + (g + 2) * 128);
+        B.acc(S, m, tl);
       }
-      if (j < V4) {
-        const float4 v = __ldg(z4 + j);
-        const int a0 = exp2_code(v.x, m), a1 = exp2_code(v.y, m), a2 = exp2_code(v.z, m), a3 = exp2_code(v.w, m);
-        S += (uint64_t)exp2_from_code(a0, H, L) + (uint64_t)exp2_from_code(a1, H, L) +
-             (uint64_t)exp2_from_code(a2, H, L) + (uint64_t)exp2_from_code(a3, H, L);
-        if (best == 0x7fffffff && min(min(a0, a1), min(a2, a3)) == 0)
-          best = 4 * j + (a0 == 0 ? 0 : a1 == 0 ? 1 : a2 == 0 ? 2 : 3);
-      }
+      if (g < ng) A.acc(S, m, tl);
+      if (rn < rows && ng > 0) A.load(zn);
+      for (int j = ng * 128; j + lane < n4; j += 32) tl.acc4(S, ld_stream4(z4 + j), m);
     } else {
-      for (int j = lane; j < V; j += 32) {
-        const int a = exp2_code(__ldg(z + j), m);
-        S += exp2_from_code(a, H, L);
-        if (a == 0 && best == 0x7fffffff) best = j;
-      }
+      for (int j = lane; j < V; j += 32) tl.acc(S, tl.e(tl.code(__ldg(z + j), m)));
     }
     RowStats st;
     st.m = m;
     st.S = warp_sum(S);
     st.Mq = Mq;
-    st.F = (uint32_t)((Mq << 32) / st.S);
-    st.amax = (int)__reduce_min_sync(0xffffffffu, (unsigned)best);
-    const bool need_resid = st.amax <= sym;  // warp-uniform
+    st.F = st.S ? (uint32_t)((Mq << 32) / st.S) : 0u;  // S >= 2^31 when m is the row's maximum
+    // g below the coded symbol and g of the symbol, packed as (below << 32) + at (each < 2^31),
+    // and the lowest index <= sym with exponent code 0
+    uint64_t packed = 0;
+    int first0 = 0x7fffffff;
+    for (int j = lane; j <= sym && j < V; j += 32) {
+      const uint32_t a = tl.code(__ldg(z + j), m);
+      const uint64_t g = gfloor(tl.e(a), st);
+      packed += j < sym ? (g << 32) : g;
+      if (a == 0u && first0 == 0x7fffffff) first0 = j;
+    }
+    packed = warp_sum(packed);
+    const int amax = (int)__reduce_min_sync(0xffffffffu, (unsigned)first0);
     uint64_t gall = 0;
-    if (need_resid) {
+    if (amax <= sym) {  // warp-uniform: the argmax lies at or below the symbol
       if (vec) {
-        for (int j = lane; j < V4; j += 32) {
-          const float4 v = __ldg(z4 + j);
-          gall += gfloor(exp2_fixed(v.x, m, H, L), st) + gfloor(exp2_fixed(v.y, m, H, L), st) +
-                  gfloor(exp2_fixed(v.z, m, H, L), st) + gfloor(exp2_fixed(v.w, m, H, L), st);
-        }
+        for (int j = 0; j + lane < n4; j += 32) gall += tl.g4(__ldg(z4 + j), m, st);
       } else {
-        for (int j = lane; j < V; j += 32) gall += gfloor(exp2_fixed(__ldg(z + j), m, H, L), st);
+        for (int j = lane; j < V; j += 32) gall += gfloor(tl.e(tl.code(__ldg(z + j), m)), st);
       }
       gall = warp_sum(gall);
     }
-    // g below the coded symbol and g of the symbol, packed as (below << 32) + at (each < 2^31)
-    uint64_t packed = 0;
-    for (int j = lane; j <= sym && j < V; j += 32) {
-      const uint64_t g = gfloor(exp2_fixed(__ldg(z + j), m, H, L), st);
-      packed += j < sym ? (g << 32) : g;
-    }
-    packed = warp_sum(packed);
     if (lane == 0) {
       const uint64_t resid = Mq - gall;
-      start[out_idx] = (uint32_t)(sym + (packed >> 32) + (st.amax < sym ? resid : 0ull));
-      freq[out_idx] = (uint32_t)(1ull + (packed & 0xFFFFFFFFull) + (st.amax == sym ? resid : 0ull));
+      start[out_idx] = (uint32_t)(sym + (packed >> 32) + (amax < sym ? resid : 0ull));
+      freq[out_idx] = (uint32_t)(1ull + (packed & 0xFFFFFFFFull) + (amax == sym ? resid : 0ull));
     }
   }
 }
 
-// The same pairs with one block of kCdfThreads per row and the maximum taken in the kernel: the
-// second read of a row then comes from L2, as the rows in flight (4 per SM) fit in it.
-__global__ void __launch_bounds__(kCdfThreads) k_cdf_pairs_block(const float* __restrict__ logits, int64_t rows,
-                                                                 int V, int P, const uint32_t* __restrict__ tab,
-                                                           const uint16_t* __restrict__ tok, int64_t n_tok, int W,
-                                                           int64_t first_win,
-                                                           uint32_t* __restrict__ start, uint32_t* __restrict__ freq,
-                                                           int mode, int64_t pair_win0,
-                                                           const uint32_t* __restrict__ row_max) {
-  __shared__ uint32_t H[256], L[256];
-  __shared__ float redf[32];
-  __shared__ uint64_t redu[32];
-  for (int i = threadIdx.x; i < 256; i += kCdfThreads) {
-    H[i] = tab[i];
-    L[i] = tab[256 + i];
-  }
-  __syncthreads();
-  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x) {
-    int sym;
-    int64_t out_idx;
-    if (mode == 0) {
-      sym = tok[r];
-      out_idx = r;
-    } else {
-      int64_t wl = r / W;
-      int i = (int)(r - wl * W);
-      int64_t g = (first_win + wl) * W + i;
-      if (g >= n_tok) continue;  // block-uniform
-      sym = tok[g];
-      out_idx = pair_tile_index(first_win + wl - pair_win0, i, pair_tile_groups(W));
-    }
+// float_key of each row's maximum (one warp per row), for callers without the GEMM's maxima
+__global__ void __launch_bounds__(256) k_row_max_key(const float* __restrict__ logits, int64_t rows, int V,
+                                                     uint32_t* __restrict__ row_max) {
+  const int lane = threadIdx.x & 31;
+  const bool vec = (V & 3) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15) == 0;
+  for (int64_t r = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); r < rows; r += (int64_t)gridDim.x * 8) {
     const float* z = logits + r * (int64_t)V;
-    RowStats st = row_stats(z, V, P, H, L, redf, redu, row_max ? row_max + r : nullptr);
-    // The remainder (T - V) - sum g goes to the argmax: it moves the symbol's start only when the
-    // argmax lies below the symbol and its freq only when it is the symbol, so the pass over the
-    // whole row that sums g is taken only then (block-uniform).
-    const bool need_resid = st.amax <= sym;
-    uint64_t gall = need_resid ? row_gsum(z, V, st, H, L) : 0ull;
-    // g below the coded symbol and g of the symbol: only j <= sym, packed as (below << 32) + at
-    // (each part < 2^31)
-    uint64_t packed = 0;
-    for (int j = threadIdx.x; j <= sym && j < V; j += kCdfThreads) {
-      const uint64_t g = gfloor(exp2_fixed(__ldg(z + j), st.m, H, L), st);
-      packed += j < sym ? (g << 32) : g;
+    uint32_t k = 0u;
+    if (vec) {
+      const float4* z4 = reinterpret_cast<const float4*>(z);
+      for (int j = lane; j < (V >> 2); j += 32) {
+        const float4 v = __ldg(z4 + j);
+        k = max(max(k, max(float_key(__float_as_uint(v.x)), float_key(__float_as_uint(v.y)))),
+                max(float_key(__float_as_uint(v.z)), float_key(__float_as_uint(v.w))));
+      }
+    } else {
+      for (int j = lane; j < V; j += 32) k = max(k, float_key(__float_as_uint(__ldg(z + j))));
     }
-    if (need_resid) gall = block_sum_u64(gall, redu);
-    packed = block_sum_u64(packed, redu);
-    const uint64_t gbelow = packed >> 32, gsym = packed & 0xFFFFFFFFull;
-    if (threadIdx.x == 0) {
-      uint64_t resid = st.Mq - gall;
-      start[out_idx] = (uint32_t)(sym + gbelow + (st.amax < sym ? resid : 0ull));
-      freq[out_idx] = (uint32_t)(1ull + gsym + (st.amax == sym ? resid : 0ull));
-    }
+    k = __reduce_max_sync(0xffffffffu, k);
+    if (lane == 0) row_max[r] = k;
   }
 }
 
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
-                      int64_t n_tok, int W, int64_t first_win, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0, const uint32_t* row_max) {
+                      int64_t n_tok, int W, int64_t first_win, uint32_t* start, uint32_t* freq, int mode,
+                      cudaStream_t s, int64_t pair_win0, uint32_t* row_max, bool have_max) {
   if (rows <= 0) return;
-  if (!row_max) {
-    // a kernel-side max pass reads each row twice: the block-per-row form keeps the second read in
-    // L2 (measured: 2.28 against 2.52 ms for 65,536 rows of 32,000 logits)
-    const unsigned blocks = (unsigned)std::min<int64_t>(rows, 152 * 4 * 8);
-    note_launch();
-    k_cdf_pairs_block<<<blocks, kCdfThreads, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
-                                                     start, freq, mode, pair_win0, nullptr);
-    return;
-  }
-  // one wave of resident blocks, each warp walking rows
   static int resident = 0;
   if (!resident) {
     int dev = 0, sms = 0, per_sm = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_cdf_pairs, 32 * kPairWarps, 0);
+    cudaFuncSetAttribute(k_cdf_pairs, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_cdf_pairs, 32 * kPairWarps, kPairSmem);
     resident = std::max(1, sms * per_sm);
   }
+  if (!have_max) {
+    note_launch();
+    k_row_max_key<<<(unsigned)std::min<int64_t>((rows + 7) / 8, 152 * 8), 256, 0, s>>>(logits, rows, V, row_max);
+  }
+  // one wave of resident blocks, each warp walking rows
   const int64_t blocks = std::min<int64_t>((rows + kPairWarps - 1) / kPairWarps, resident);
   note_launch();
-  k_cdf_pairs<<<(unsigned)blocks, 32 * kPairWarps, 0, s>>>(logits, rows, V, P, tab, tok, n_tok, W, first_win,
-                                                          start, freq, mode, pair_win0, row_max);
+  k_cdf_pairs<<<(unsigned)blocks, 32 * kPairWarps, kPairSmem, s>>>(logits, rows, V, P, tab, tok, n_tok, W,
+                                                                   first_win, start, freq, mode, pair_win0, row_max);
 }
 
 // Block inclusive scan of one u64 per thread; returns the inclusive prefix; *total the tile sum.

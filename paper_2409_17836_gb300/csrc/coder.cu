@@ -22,9 +22,10 @@
 // leave for the stream's slot in 16-byte chunks, at most two per 8 tokens: scattered 4-byte
 // stores from 32 lanes to 32 slots would cost one memory transaction each.
 //
-// Layout: one stream per thread, 32 windows per warp. Pairs are read from window tiles (the
-// encode path; a warp reads one contiguous kilobyte per array per 8 tokens) or at
-// start[w*stride_win + i*stride_pos] (lmgc_range_encode's general layout, 8 tokens ahead).
+// Layout: one stream per thread, 32 windows per warp. Pairs come from window tiles (the encode
+// path; a warp's 8 tokens are one contiguous kilobyte per array, staged through shared memory by
+// bulk copies) or from start[w*stride_win + i*stride_pos] (lmgc_range_encode's general layout,
+// loaded 8 tokens ahead).
 // Slot words are stored in native byte order; the pack step writes the bytes most significant
 // first.
 #include <algorithm>
@@ -55,9 +56,19 @@ struct Stream {
   uint32_t chk;        // OR of s | (f - 1) | (s + f - 1) over the tokens: >= T iff a pair was invalid
   uint32_t max_words;
   uint32_t* slot;
-  uint32_t* ring;
+  uint32_t ring;        // shared-memory address of this thread's ring (kRingWords words)
   bool overflow;
 
+  // ring words through shared-state-space instructions (a generic pointer would make every
+  // read of the ring wait like a global load)
+  __device__ __forceinline__ uint32_t ring_ld(int32_t i) const {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(ring + 4u * (uint32_t)(i & (kRingWords - 1))) : "memory");
+    return v;
+  }
+  __device__ __forceinline__ void ring_st(int32_t i, uint32_t v) const {
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(ring + 4u * (uint32_t)(i & (kRingWords - 1))), "r"(v) : "memory");
+  }
   __device__ __forceinline__ void init(int P, uint32_t* sl, uint32_t mw, uint32_t* rg) {
     const uint64_t r0 = 1ull << (62 - P);  // R = 2^62
     rlo = (uint32_t)r0;
@@ -69,7 +80,7 @@ struct Stream {
     chk = 0u;
     max_words = mw;
     slot = sl;
-    ring = rg;
+    ring = (uint32_t)__cvta_generic_to_shared(rg);
     overflow = false;
   }
   // +1 into the completed words before a0 (ring or slot); a carry past word 0 cannot happen for
@@ -78,8 +89,8 @@ struct Stream {
     for (int32_t i = w - 1; i >= 0; --i) {
       uint32_t v;
       if (i >= fw) {
-        v = ring[i & (kRingWords - 1)] + 1u;
-        ring[i & (kRingWords - 1)] = v;
+        v = ring_ld(i) + 1u;
+        ring_st(i, v);
       } else {
         if ((uint32_t)i >= max_words) break;
         v = slot[i] + 1u;
@@ -130,7 +141,7 @@ struct Stream {
     asm("shr.u32 %0, %1, %2;" : "=r"(rhi) : "r"(phi), "r"(s2));
     sh -= k;
     const bool full = sh < 0;
-    if (full) ring[w & (kRingWords - 1)] = a0;
+    if (full) ring_st(w, a0);
     a0 = full ? a1 : a0;
     a1 = full ? a2 : a1;
     a2 = full ? 0u : a2;
@@ -144,7 +155,11 @@ struct Stream {
 #pragma unroll
     for (int q = 0; q < CHUNKS; q++) {
       if (w - fw >= 4) {
-        const uint4 v = *reinterpret_cast<const uint4*>(ring + (fw & (kRingWords - 1)));
+        uint4 v;
+        asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "r"(ring + 4u * (uint32_t)(fw & (kRingWords - 1)))
+                     : "memory");
         if ((uint32_t)(fw + 3) < max_words) *reinterpret_cast<uint4*>(slot + fw) = v;
         fw += 4;
       }
@@ -169,18 +184,56 @@ struct Stream {
       nbits = (uint64_t)w * 32u + (uint64_t)nrem;
     }
     for (int32_t i = fw; i < w; i++)
-      if ((uint32_t)i < max_words) slot[i] = ring[i & (kRingWords - 1)];
+      if ((uint32_t)i < max_words) slot[i] = ring_ld(i);
     if ((uint32_t)w < max_words) slot[w] = nrem >= 32 ? a0 : a0 & ~(0xFFFFFFFFu >> nrem);
     if (nrem > 32 && (uint32_t)(w + 1) < max_words) slot[w + 1] = a1 & ~(0xFFFFFFFFu >> (nrem - 32));
     return nbits;
   }
 };
 
-// One stream per thread. TILED: pairs in window tiles (vector loads, 8 tokens a group);
-// otherwise at start[w*stride_win + i*stride_pos], loaded 8 tokens ahead. PT: P at compile
-// time (0: P_rt). CHECK: validate the pairs (a window stops after the group holding an invalid
-// pair, and the error word reports it).
-template <int PT, bool CHECK, bool TILED>
+// mbarrier and bulk-copy helpers for the staged tiles (shared::cta addresses)
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ bool bar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded wait for a phase: false (and kErrLimit) after about 2 s
+__device__ __forceinline__ bool bar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
+  if (bar_try(a, parity)) return true;
+  uint64_t t0, t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  for (uint32_t i = 1; i < (1u << 26); ++i) {
+    if (bar_try(a, parity)) return true;
+    if ((i & 63) == 0) {
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+      if (t - t0 > 2000000000ull) break;
+    }
+  }
+  atomicOr(err, kErrLimit);
+  return false;
+}
+// one group's start and freq tiles (1 KiB each) into a stage, completing on its barrier
+__device__ __forceinline__ void stage_tiles(uint32_t bar, uint32_t dst_s, uint32_t dst_f, const uint32_t* src_s,
+                                            const uint32_t* src_f) {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], 2048;" ::"r"(bar) : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 1024, [%2];" ::"r"(dst_s),
+               "l"(src_s), "r"(bar)
+               : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 1024, [%2];" ::"r"(dst_f),
+               "l"(src_f), "r"(bar)
+               : "memory");
+}
+
+// One stream per thread, pairs at start[w*stride_win + i*stride_pos] (lmgc_range_encode's general
+// layout), loaded 8 tokens ahead. PT: P at compile time (0: P_rt). CHECK: validate the pairs (a
+// window stops after the group holding an invalid pair, and the error word reports it).
+template <int PT, bool CHECK>
 __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
     const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
     int64_t win_tokens, const uint32_t* __restrict__ win_len, int64_t stride_win, int64_t stride_pos,
@@ -196,24 +249,104 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
   Stream c;
   c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz), (uint32_t)(slot_sz / 4),
          rings + threadIdx.x * kRingStride);
-  if (TILED) {
-    const int64_t groups = pair_tile_groups(win_tokens);
-    const int64_t g_end = (n + 7) >> 3;
-    const int64_t e0 = pair_tile_index(w, 0, groups);
-    const uint4* qs = reinterpret_cast<const uint4*>(start + e0);
-    const uint4* qf = reinterpret_cast<const uint4*>(freq + e0);
-    uint4 s0 = make_uint4(0, 0, 0, 0), s1 = s0, f0 = s0, f1 = s0;
-    if (g_end > 0) {
-      s0 = __ldcs(qs); s1 = __ldcs(qs + 1); f0 = __ldcs(qf); f1 = __ldcs(qf + 1);
-    }
-    for (int64_t g = 0; g < g_end; g++) {
-      const uint32_t cs[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-      const uint32_t cf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
-      if (g + 1 < g_end) {  // the next tile of this window block: 256 elements on
-        qs += 64;
-        qf += 64;
-        s0 = __ldcs(qs); s1 = __ldcs(qs + 1); f0 = __ldcs(qf); f1 = __ldcs(qf + 1);
+  constexpr int kPre = 8;
+  const uint32_t* qs = start + w * stride_win;
+  const uint32_t* qf = freq + w * stride_win;
+  uint32_t bs[kPre], bf[kPre];
+#pragma unroll
+  for (int j = 0; j < kPre; j++) {
+    bs[j] = j < n ? __ldcs(qs) : 0u;
+    bf[j] = j < n ? __ldcs(qf) : 1u;
+    qs += stride_pos;
+    qf += stride_pos;
+  }
+  for (int64_t i0 = 0; i0 < n; i0 += kPre) {
+    uint32_t cs[kPre], cf[kPre];
+    const bool full_next = i0 + 2 * kPre <= n;
+#pragma unroll
+    for (int j = 0; j < kPre; j++) {
+      cs[j] = bs[j];
+      cf[j] = bf[j];
+      if (full_next || i0 + kPre + j < n) {
+        bs[j] = __ldcs(qs);
+        bf[j] = __ldcs(qf);
       }
+      qs += stride_pos;
+      qf += stride_pos;
+    }
+    if (i0 + kPre <= n) {
+#pragma unroll
+      for (int j = 0; j < kPre; j++) c.template token<CHECK>(cs[j], cf[j], P);
+    } else {
+      const int jn = (int)(n - i0);
+#pragma unroll
+      for (int j = 0; j < kPre; j++)
+        if (j < jn) c.template token<CHECK>(cs[j], cf[j], P);
+    }
+    c.template flush<2>();
+    if (CHECK && c.chk >= T) break;
+  }
+  bitlen[w] = (uint32_t)c.finish();
+  if (bad || c.overflow || (CHECK && c.chk >= T)) atomicOr(err, kErrCorrupt);
+}
+
+// Pairs in window tiles (the encode path): a warp codes the 32 windows of one tile column, whose
+// 8-position groups are contiguous 1 KiB tiles of starts and of freqs. The warp stages them
+// through a two-stage ring in shared memory: lane 0 fills a stage with bulk copies that complete
+// on the stage's mbarrier, every lane waits for it (bounded), reads its window's 8 pairs (two
+// 16-byte loads per array), codes them, and then the stage is refilled with the tiles two
+// groups on, which thus have a whole group of coding to land. No register holds pairs ahead.
+template <int PT, bool CHECK>
+__global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
+    const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
+    int64_t win_tokens, const uint32_t* __restrict__ win_len, uint8_t* __restrict__ slots, size_t slot_sz,
+    uint32_t* __restrict__ bitlen, uint32_t* err) {
+  constexpr int kWarps = kCoderThreads / 32;
+  __shared__ __align__(16) uint32_t rings[kCoderThreads * kRingStride];
+  __shared__ __align__(128) uint32_t tiles[kWarps][2][2][256];  // [warp][stage][start, freq][32 x 8]
+  __shared__ __align__(8) uint64_t full[kWarps][2];
+  const int P = PT ? PT : P_rt;
+  const uint32_t T = 1u << P;
+  const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
+  const int64_t w = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t w0 = w - lane;  // the tile column's first window
+  if (w0 >= n_win) return;      // warp-uniform
+  const bool live = w < n_win;
+  int64_t n = live ? (win_len ? (int64_t)win_len[w] : win_tokens) : 0;
+  const bool bad = n > win_tokens;
+  if (bad) n = 0;  // a window longer than its slot is not coded
+  const int64_t groups = pair_tile_groups(win_tokens);
+  int64_t g_all = (n + 7) >> 3;  // groups any window of the warp codes (warp-uniform after the max)
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) g_all = max(g_all, (int64_t)__shfl_xor_sync(0xffffffffu, (long long)g_all, o));
+  Stream c;
+  c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)(live ? w : w0) * slot_sz), (uint32_t)(slot_sz / 4),
+         rings + threadIdx.x * kRingStride);
+  const int64_t col = pair_tile_index(w0, 0, groups);  // element of the column's first tile
+  const uint32_t* ts = start + col;
+  const uint32_t* tf = freq + col;
+  const uint32_t bar0 = smem_addr(&full[wp][0]), bar1 = smem_addr(&full[wp][1]);
+  if (lane == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar0) : "memory");
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar1) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    for (int st = 0; st < 2 && st < g_all; st++)
+      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((int64_t)st << 8),
+                  tf + ((int64_t)st << 8));
+  }
+  __syncwarp();
+  bool ok = true, stopped = false;
+  int64_t g = 0;
+  for (; g < g_all; g++) {
+    const int st = (int)(g & 1);
+    ok = __all_sync(0xffffffffu, bar_wait(st ? bar1 : bar0, (uint32_t)(g >> 1) & 1u, err));
+    if (!ok) break;
+    const uint4* qs = reinterpret_cast<const uint4*>(tiles[wp][st][0] + 8 * lane);
+    const uint4* qf = reinterpret_cast<const uint4*>(tiles[wp][st][1] + 8 * lane);
+    const uint4 s0 = qs[0], s1 = qs[1], f0 = qf[0], f1 = qf[1];
+    const uint32_t cs[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+    const uint32_t cf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+    if (!stopped && 8 * g < n) {
       if (8 * g + 8 <= n) {
 #pragma unroll
         for (int j = 0; j < 8; j++) c.template token<CHECK>(cs[j], cf[j], P);
@@ -224,65 +357,56 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
           if (j < jn) c.template token<CHECK>(cs[j], cf[j], P);
       }
       c.template flush<2>();
-      if (CHECK && c.chk >= T) break;
+      if (CHECK && c.chk >= T) stopped = true;
     }
-  } else {
-    constexpr int kPre = 8;
-    const uint32_t* qs = start + w * stride_win;
-    const uint32_t* qf = freq + w * stride_win;
-    uint32_t bs[kPre], bf[kPre];
-#pragma unroll
-    for (int j = 0; j < kPre; j++) {
-      bs[j] = j < n ? __ldcs(qs) : 0u;
-      bf[j] = j < n ? __ldcs(qf) : 1u;
-      qs += stride_pos;
-      qf += stride_pos;
-    }
-    for (int64_t i0 = 0; i0 < n; i0 += kPre) {
-      uint32_t cs[kPre], cf[kPre];
-      const bool full_next = i0 + 2 * kPre <= n;
-#pragma unroll
-      for (int j = 0; j < kPre; j++) {
-        cs[j] = bs[j];
-        cf[j] = bf[j];
-        if (full_next || i0 + kPre + j < n) {
-          bs[j] = __ldcs(qs);
-          bf[j] = __ldcs(qf);
-        }
-        qs += stride_pos;
-        qf += stride_pos;
-      }
-      if (i0 + kPre <= n) {
-#pragma unroll
-        for (int j = 0; j < kPre; j++) c.template token<CHECK>(cs[j], cf[j], P);
-      } else {
-        const int jn = (int)(n - i0);
-#pragma unroll
-        for (int j = 0; j < kPre; j++)
-          if (j < jn) c.template token<CHECK>(cs[j], cf[j], P);
-      }
-      c.template flush<2>();
-      if (CHECK && c.chk >= T) break;
-    }
+    __syncwarp();  // every lane has read the stage
+    if (lane == 0 && g + 2 < g_all)
+      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((g + 2) << 8),
+                  tf + ((g + 2) << 8));
   }
+  if (!ok) {
+    // a wait gave up: let this warp's copies still in flight land before the block's shared
+    // memory is released (bounded again), and report the window as failed
+    if (lane == 0) {
+      for (int64_t h = g; h < g + 2 && h < g_all; h++) bar_wait((h & 1) ? bar1 : bar0, (uint32_t)(h >> 1) & 1u, err);
+    }
+    __syncwarp();
+  }
+  if (!live) return;
   bitlen[w] = (uint32_t)c.finish();
-  if (bad || c.overflow || (CHECK && c.chk >= T)) atomicOr(err, kErrCorrupt);
+  if (bad || !ok || c.overflow || (CHECK && c.chk >= T)) atomicOr(err, kErrCorrupt);
 }
 
-template <bool CHECK, bool TILED>
+template <bool CHECK>
 static void launch_coder(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
                          const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
                          size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s) {
   const unsigned g = (unsigned)((n_win + kCoderThreads - 1) / kCoderThreads);
   if (P == 24)
-    k_range_encode<24, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
-                                                                 stride_pos, slots, slot_sz, bitlen, err);
+    k_range_encode<24, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                          stride_pos, slots, slot_sz, bitlen, err);
   else if (P == 16)
-    k_range_encode<16, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
-                                                                 stride_pos, slots, slot_sz, bitlen, err);
+    k_range_encode<16, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                          stride_pos, slots, slot_sz, bitlen, err);
   else
-    k_range_encode<0, CHECK, TILED><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
-                                                                stride_pos, slots, slot_sz, bitlen, err);
+    k_range_encode<0, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, stride_win,
+                                                         stride_pos, slots, slot_sz, bitlen, err);
+}
+
+template <bool CHECK>
+static void launch_coder_tiles(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
+                               const uint32_t* win_len, uint8_t* slots, size_t slot_sz, uint32_t* bitlen,
+                               uint32_t* err, cudaStream_t s) {
+  const unsigned g = (unsigned)((n_win + kCoderThreads - 1) / kCoderThreads);
+  if (P == 24)
+    k_range_encode_tiles<24, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, slots,
+                                                                slot_sz, bitlen, err);
+  else if (P == 16)
+    k_range_encode_tiles<16, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, slots,
+                                                                slot_sz, bitlen, err);
+  else
+    k_range_encode_tiles<0, CHECK><<<g, kCoderThreads, 0, s>>>(start, freq, P, n_win, win_tokens, win_len, slots,
+                                                               slot_sz, bitlen, err);
 }
 
 void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int64_t n_win, int64_t win_tokens,
@@ -291,11 +415,11 @@ void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int
   if (n_win <= 0) return;
   note_launch();
   if (tiled) {
-    if (check) launch_coder<true, true>(start, freq, P, n_win, win_tokens, win_len, 0, 0, slots, slot_sz, bitlen, err, s);
-    else launch_coder<false, true>(start, freq, P, n_win, win_tokens, win_len, 0, 0, slots, slot_sz, bitlen, err, s);
+    if (check) launch_coder_tiles<true>(start, freq, P, n_win, win_tokens, win_len, slots, slot_sz, bitlen, err, s);
+    else launch_coder_tiles<false>(start, freq, P, n_win, win_tokens, win_len, slots, slot_sz, bitlen, err, s);
   } else {
-    launch_coder<true, false>(start, freq, P, n_win, win_tokens, win_len, stride_win, stride_pos, slots, slot_sz,
-                              bitlen, err, s);
+    launch_coder<true>(start, freq, P, n_win, win_tokens, win_len, stride_win, stride_pos, slots, slot_sz, bitlen,
+                       err, s);
   }
 }
 

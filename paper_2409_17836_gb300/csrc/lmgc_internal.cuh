@@ -206,12 +206,13 @@ void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t ds
 
 // cdf.cu
 void upload_exp2_tables(uint32_t* d_tab, cudaStream_t s);  // builds H and L on the host
-// mode 1: pair index i * pair_stride_pos + (window - pair_win0)
-// row_max (optional): float_key of each row's maximum, which replaces the kernel's max pass
+// mode 0: row r codes tok[r], pair r; mode 1: row r is position r % W of window first_win + r / W,
+// its pair goes to element pair_tile_index(window - pair_win0, position) of the window tiles.
+// row_max: [rows] float_key of each row's maximum; have_max false: computed into it first
 void launch_cdf_pairs(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, const uint16_t* tok,
                       int64_t n_tok, int W, int64_t first_win, uint32_t* start,
-                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0 = 0,
-                      const uint32_t* row_max = nullptr);
+                      uint32_t* freq, int mode, cudaStream_t s, int64_t pair_win0, uint32_t* row_max,
+                      bool have_max);
 void launch_quantize_cdf(const float* logits, int64_t rows, int V, int P, const uint32_t* tab, uint32_t* cdf,
                          cudaStream_t s);
 // launch_cdf_pairs over the restricted alphabet (no row_max input); a token outside it sets
