@@ -39,20 +39,25 @@
 namespace lmgc {
 namespace attn {
 
-constexpr int BQ = 128, BKV = 64;
+constexpr int BQ = 128;
 constexpr int kThreads = 256;  // K TMA warp, S-MMA warp, 4 softmax warps, V TMA warp, PV-MMA warp
 constexpr float kMaxBlockSum = 4096.f;  // the reference moves when a block's P sum would exceed 2^12
 
 template <int HD>
 struct Shape {
+  // keys per block: 64 at hd 64 (two CTAs per SM fit in tensor memory), 128 at hd 128, where
+  // S = Q K^T then runs as MMAs of N = 128 (half as many MMA issues per key) and the softmax's
+  // per-block costs (barrier waits, tensor-memory round trips, the arrive) cover twice the keys
+  static constexpr int BKV = HD == 128 ? 128 : 64;
+  static constexpr int NS = 3;                          // S buffers: S(kb) is issued NS - 1 blocks ahead
   static constexpr int KCH = HD / 64;                   // 64-column (128-byte) chunks of a row
   static constexpr uint32_t Q_BYTES = BQ * HD * 2;
-  static constexpr uint32_t KV_CHUNK = BKV * 128;       // one 64x64 bf16 chunk (8 KiB)
+  static constexpr uint32_t KV_CHUNK = BKV * 128;       // one BKV x 64 fp16 chunk
   static constexpr uint32_t K_BYTES = BKV * HD * 2;
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
-  static constexpr int KSK = 3, KSV = 2;                // stages of the K ring and of the V ring
-  static constexpr uint32_t TMEM_S = 0;                 // S ring: columns 0..191 (P in the first 32 of each)
-  static constexpr uint32_t TMEM_O = HD == 64 ? 192 : 256;  // O: HD columns
+  static constexpr int KSK = NS, KSV = 2;               // stages of the K ring (one per S buffer) and of the V ring
+  static constexpr uint32_t TMEM_S = 0;                 // S ring: NS x BKV columns (P in the first BKV / 2 of each)
+  static constexpr uint32_t TMEM_O = NS * BKV;          // O: HD columns (192 at hd 64, 384 at hd 128)
   static constexpr uint32_t TMEM_COLS = HD == 64 ? 256 : 512;
   static constexpr size_t SMEM = Q_BYTES + KSK * K_BYTES + KSV * V_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
@@ -220,14 +225,18 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const uint32_t sv = sk + S::KSK * S::K_BYTES;        // V ring
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (sv + S::KSV * S::V_BYTES - sq));
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
-  // barriers: 0 Q loaded | 1-3 S ready | 4-6 P written (128 arrivals) | 7-8 P V done (by the
-  //           parity of the block) | 9-11 K stage loaded | 15-16 V stage loaded
+  // barriers, per S buffer i = kb % NS: 0 Q loaded | 1-3 S(kb) ready | 4-6 P(kb) written (128
+  //   arrivals) | 7-9 P V(kb) done | 10-12 K stage loaded | 15-16 V stage (kb % 2) loaded.
+  // Waits go by the parity of a block's phase, (kb / NS) & 1 (V: (kb / 2) & 1). Such a wait is
+  // sound when the previous phase of the barrier has completed and the next cannot complete
+  // before the waiter moves on; the comments at each wait say why both hold.
   const uint32_t b_q = smem_u32(bars + 0);
   auto b_s = [&](int i) { return smem_u32(bars + 1 + i); };
   auto b_p = [&](int i) { return smem_u32(bars + 4 + i); };
   auto b_pv = [&](int i) { return smem_u32(bars + 7 + i); };
-  auto b_kfull = [&](int i) { return smem_u32(bars + 9 + i); };
+  auto b_kfull = [&](int i) { return smem_u32(bars + 10 + i); };
   auto b_vfull = [&](int i) { return smem_u32(bars + 15 + i); };
+  constexpr int BKV = S::BKV, NS = S::NS;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y;  // query head; with packing, the KV head
@@ -239,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   const int64_t rem = p.pos_first + p.n_pos - pos0;
   const int nrows = PACKED ? p.packed : (rem < BQ ? (int)rem : BQ);  // valid rows
   const int64_t last_pos = PACKED ? pos0 : pos0 + nrows - 1;
-  const int nkb = (int)(last_pos / BKV) + 1;
+  const int nkb = (int)(last_pos / S::BKV) + 1;
   const int q_row0 = (int)(w * p.q_win_stride + (pos0 - p.pos_first));
   const int kv_row0 = (int)(w * p.W);
 
@@ -251,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);  // 12-14, 17-18 unused
+    for (int i = 0; i < 19; i++) mbar_init(smem_u32(bars + i), (i >= 4 && i <= 6) ? 128 : 1);  // 13-14, 17-18 unused
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -284,10 +293,11 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     }
     __syncwarp();
     for (int kb = 0; kb < nkb; kb++) {
-      const int ks = kb % S::KSK;  // == kb % 3, the S buffer index of block kb
-      // stage free once S(kb - 3), which read it, is done
+      const int ks = kb % S::KSK;  // == kb % NS, the S buffer index of block kb
+      // stage free once S(kb - NS), which read it, is done (this warp saw S(kb - 2 NS) done, and
+      // S(kb) needs the stage it is about to load)
       if (kb >= S::KSK &&
-          !__all_sync(0xffffffffu, mbar_wait(b_s(ks), (uint32_t)((kb - S::KSK) / 3) & 1u, p.err)))
+          !__all_sync(0xffffffffu, mbar_wait(b_s(ks), (uint32_t)((kb - S::KSK) / NS) & 1u, p.err)))
         break;
       if (lane == 0) {
         mbar_expect_tx(b_kfull(ks), S::K_BYTES);
@@ -301,10 +311,12 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
   } else if (warp == 6) {
     // ---------------- TMA producer: V blocks ----------------
     for (int kb = 0; kb < nkb; kb++) {
-      const int vs = kb % S::KSV;  // == kb & 1, the P V-done barrier index of block kb
-      // stage free once P V(kb - 2), which read it, is done
-      if (kb >= S::KSV &&
-          !__all_sync(0xffffffffu, mbar_wait(b_pv(vs), (uint32_t)((kb - S::KSV) >> 1) & 1u, p.err)))
+      const int vs = kb % S::KSV;
+      // stage free once P V(kb - 2), which read it, is done (P V completes in order and this warp
+      // saw P V(kb - 3) done; the next phase of that barrier, P V(kb - 2 + NS), needs V stages
+      // this warp has not loaded yet)
+      if (kb >= S::KSV && !__all_sync(0xffffffffu, mbar_wait(b_pv((kb - S::KSV) % NS),
+                                                             (uint32_t)((kb - S::KSV) / NS) & 1u, p.err)))
         break;
       if (lane == 0) {
         mbar_expect_tx(b_vfull(vs), S::V_BYTES);
@@ -319,10 +331,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     // ---------------- S issuer: S(kb) = Q K(kb)^T two blocks ahead of the softmax ----------------
     bool ok = __all_sync(0xffffffffu, mbar_wait(b_q, 0, p.err));
     for (int kb = 0; kb < nkb && ok; kb++) {
-      const int ks = kb % S::KSK, sb = kb % 3;
-      // S(kb) overwrites the buffer from which P V(kb-3) read P(kb-3)
-      if (kb >= 3 && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv((kb - 3) & 1), (uint32_t)((kb - 3) >> 1) & 1u,
-                                                              p.err))))
+      const int ks = kb % S::KSK, sb = kb % NS;
+      // S(kb) overwrites the buffer from which P V(kb - NS) read P(kb - NS) (this warp saw
+      // P V(kb - 2 NS) done; the barrier's next phase, P V(kb), needs S(kb))
+      if (kb >= NS && !(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(sb), (uint32_t)((kb - NS) / NS) & 1u, p.err))))
         break;
       if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_kfull(ks), (uint32_t)(kb / S::KSK) & 1u, p.err)))) break;
       tc_fence_after();
@@ -332,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
 #pragma unroll
         for (int k = 0; k < HD / 16; k++) {
           const int c = k >> 2, o = (k & 3) * 32;
-          tc_mma(tmem + S::TMEM_S + sb * 64, desc_kmajor(sq + c * (BQ * 128) + o),
+          tc_mma(tmem + S::TMEM_S + sb * BKV, desc_kmajor(sq + c * (BQ * 128) + o),
                  desc_kmajor(kbase + c * S::KV_CHUNK + o), S::IDESC_S, k > 0 ? 1u : 0u);
         }
         tc_commit(b_s(sb));
@@ -343,20 +355,20 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     // ---------------- P V issuer ----------------
     bool ok = true;
     for (int kb = 0; kb < nkb && ok; kb++) {
-      const int sb = kb % 3, vs = kb % S::KSV;
+      const int sb = kb % NS, vs = kb % S::KSV;
       ok = __all_sync(0xffffffffu, mbar_wait(b_vfull(vs), (uint32_t)(kb / S::KSV) & 1u, p.err));
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(sb), (uint32_t)(kb / 3) & 1u, p.err));
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(b_p(sb), (uint32_t)(kb / NS) & 1u, p.err));
       if (!ok) break;
       tc_fence_after();
       if (lane == 0) {
         const uint32_t vbase = sv + vs * S::V_BYTES;
-        // O += P V over the 64 keys in steps of 16: P (in TMEM) advances 8 columns, V advances
-        // 16 rows (2 KiB)
+        // O += P V over the block's keys in steps of 16: P (in TMEM) advances 8 columns, V
+        // advances 16 rows (2 KiB)
 #pragma unroll
         for (int k = 0; k < BKV / 16; k++)
-          tc_mma_ts(tmem + S::TMEM_O, tmem + S::TMEM_S + sb * 64 + 8 * k, desc_mnmajor(vbase + k * 2048, S::KV_CHUNK),
+          tc_mma_ts(tmem + S::TMEM_O, tmem + S::TMEM_S + sb * BKV + 8 * k, desc_mnmajor(vbase + k * 2048, S::KV_CHUNK),
                     S::IDESC_PV, (kb > 0 || k > 0) ? 1u : 0u);
-        tc_commit(b_pv(kb & 1));
+        tc_commit(b_pv(sb));
       }
       __syncwarp();
     }
@@ -374,29 +386,29 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int kb = 0; kb < nkb; kb++) {
-      const int sb = kb % 3;
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / 3) & 1u, p.err)))) break;
+      const int sb = kb % NS;
+      if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_s(sb), (uint32_t)(kb / NS) & 1u, p.err)))) break;
       if (!live) {
         mbar_arrive(b_p(sb));
         continue;
       }
       tc_fence_after();
-      float s[64];
+      float s[BKV];
       // S row of this block into s[], causally masked (only on blocks that reach past the tile's
       // first position)
       auto load_s = [&]() {
-        uint32_t a[32], b[32];
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64, a);
-        tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * 64 + 32, b);
+        // every 32-column load of the row in flight, then one wait
+        uint32_t a[BKV / 32][32];
+#pragma unroll
+        for (int q = 0; q < BKV / 32; q++) tmem_ld32_nowait(tmem + tl + S::TMEM_S + sb * BKV + 32 * q, a[q]);
         tmem_wait();
 #pragma unroll
-        for (int j = 0; j < 32; j++) {
-          s[j] = __uint_as_float(a[j]);
-          s[32 + j] = __uint_as_float(b[j]);
-        }
+        for (int q = 0; q < BKV / 32; q++)
+#pragma unroll
+          for (int j = 0; j < 32; j++) s[32 * q + j] = __uint_as_float(a[q][j]);
         if ((int)(kb * BKV + BKV - 1) > pos0_i) {
 #pragma unroll
-          for (int j = 0; j < 64; j++)
+          for (int j = 0; j < BKV; j++)
             if (kb * BKV + j > qpos_i) s[j] = -INFINITY;
         }
       };
@@ -406,7 +418,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         const uint64_t c2 = f2pack(c, c), nb2 = f2pack(nb, nb);
         uint64_t acc0 = 0ull, acc1 = 0ull;  // (+0, +0) packed
 #pragma unroll
-        for (int j = 0; j < 64; j += 2) {
+        for (int j = 0; j < BKV; j += 2) {
           float t0, t1;
           f2unpack(ffma2(f2pack(s[j], s[j + 1]), c2, nb2), t0, t1);
           s[j] = ex2_approx(t0);
@@ -435,7 +447,7 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
 #pragma unroll
           for (int i = 0; i < 4; i++) mx4[i] = s[i];
 #pragma unroll
-          for (int j = 4; j < 64; j += 2) mx4[(j >> 1) & 3] = fmax3(mx4[(j >> 1) & 3], s[j], s[j + 1]);
+          for (int j = 4; j < BKV; j += 2) mx4[(j >> 1) & 3] = fmax3(mx4[(j >> 1) & 3], s[j], s[j + 1]);
           const float mx = fmaxf(fmax3(mx4[0], mx4[1], mx4[2]), mx4[3]);  // finite: key 0 is unmasked
           corr = kb == 0 ? 0.f : ex2_approx((m - mx) * c);
           l *= corr;
@@ -443,10 +455,10 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         }
         if (kb > 0) {
           // scale this warp's rows of O (factor 1 for rows that did not move) once the previous
-          // block's P V has landed in TMEM (its barrier is read by parity: P V(kb-3) has
-          // completed, as S(kb) has)
-          const int pst = (kb - 1) & 1;
-          if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv(pst), (uint32_t)((kb - 1) >> 1) & 1u, p.err)))) break;
+          // block's P V has landed in TMEM (P V(kb - 1 - NS) has completed, as S(kb) has; the
+          // barrier's next phase, P V(kb - 1 + NS), needs P from these warps)
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(b_pv((kb - 1) % NS), (uint32_t)((kb - 1) / NS) & 1u, p.err))))
+            break;
           tc_fence_after();
 #pragma unroll 1
           for (int cc = 0; cc < HD / 32; cc++) {
@@ -462,25 +474,25 @@ __global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
         bsum = exp_block();
       }
       l += bsum;
-      // P as fp16 pairs over the first 32 columns of this block's S buffer (already read)
-      {
+      // P as fp16 pairs over the first BKV / 2 columns of this block's S buffer (already read)
+#pragma unroll
+      for (int h2 = 0; h2 < BKV / 2; h2 += 32) {
         uint32_t pw[32];
 #pragma unroll
         for (int j = 0; j < 32; j++) {
-          __half2 hb = __floats2half2_rn(s[2 * j], s[2 * j + 1]);
+          __half2 hb = __floats2half2_rn(s[2 * (h2 + j)], s[2 * (h2 + j) + 1]);
           pw[j] = *reinterpret_cast<uint32_t*>(&hb);
         }
-        tmem_st32(tmem + tl + S::TMEM_S + sb * 64, pw);
-        tmem_st_wait();
+        tmem_st32(tmem + tl + S::TMEM_S + sb * BKV + h2, pw);
       }
+      tmem_st_wait();
       tc_fence_before();
       mbar_arrive(b_p(sb));
     }
-    // O / l once the last P V has completed
-    // (P V(j)'s barrier is read by parity, which is only meaningful once P V(j-2) has completed:
-    // S(last) implies P V(last-3), so P V(last-1) is awaited before P V(last))
+    // O / l once the last P V has completed (S(last) implies P V(last - NS), the previous phase of
+    // P V(last)'s barrier and, as P V completes in order, of P V(last - 1)'s)
     for (int j = nkb >= 2 ? nkb - 2 : 0; j < nkb && ok; j++)
-      ok = __all_sync(0xffffffffu, mbar_wait(b_pv(j & 1), (uint32_t)(j >> 1) & 1u, p.err));
+      ok = __all_sync(0xffffffffu, mbar_wait(b_pv(j % NS), (uint32_t)(j / NS) & 1u, p.err));
     if (ok && live) {
       tc_fence_after();
       const float inv = 1.f / l;
@@ -558,7 +570,7 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
   std::call_once(g_once, init_once);
   CUtensorMap tq, tkv;
   if (!make_map(&tq, q, (uint64_t)qkv_dim, (uint64_t)q_rows, BQ) ||
-      !make_map(&tkv, kv, (uint64_t)qkv_dim, (uint64_t)kv_rows, BKV)) {
+      !make_map(&tkv, kv, (uint64_t)qkv_dim, (uint64_t)kv_rows, hd == 128 ? Shape<128>::BKV : Shape<64>::BKV)) {
     set_thread_error("cuTensorMapEncodeTiled failed (attention)");
     return;
   }
