@@ -346,21 +346,32 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> 
         start[b0:b0 + nb] = st.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
         freq[b0:b0 + nb] = fr.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
         del row, sym, st, fr
-    payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None)
-    torch.cuda.synchronize()
-    L.lmgc_profile(None, True)
-    for _ in range(reps):
-        payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None, out=payload)
-    st = L.lmgc_kernel_stats(None)["range_encode"]
-    L.lmgc_profile(None, False)
-    kms = st["ms"] / max(1, st["launches"])
-    rd = 8.0 * W * n_win
-    wr = float(payload.numel())
-    out["range_encode"] = {"windows": n_win, "tokens": W * n_win, "ms": kms, "read_bytes": rd, "write_bytes": wr,
-                           "bits_per_token": 8.0 * wr / (W * n_win), "achieved": (rd + wr) / kms / 1e6,
-                           "unit": "GB/s", "frac": (rd + wr) / kms / 1e6 / pk["hbm"],
-                           "tokens_per_s": W * n_win / (kms / 1e3)}
-    del start, freq, payload
+    # "range_encode": the coder as the encode path runs it (its pairs, valid by construction, are
+    # not checked again); "range_encode_validated": the same with every pair checked, as for a
+    # caller's pairs. The codes must be identical.
+    for key, validate in (("range_encode", False), ("range_encode_validated", True)):
+        payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None, validate=validate)
+        torch.cuda.synchronize()
+        L.lmgc_profile(None, True)
+        for _ in range(reps):
+            payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None, out=payload, validate=validate)
+        st = L.lmgc_kernel_stats(None)["range_encode"]
+        L.lmgc_profile(None, False)
+        kms = st["ms"] / max(1, st["launches"])
+        rd = 8.0 * W * n_win
+        wr = float(payload.numel())
+        out[key] = {"windows": n_win, "tokens": W * n_win, "ms": kms, "read_bytes": rd, "write_bytes": wr,
+                    "bits_per_token": 8.0 * wr / (W * n_win), "achieved": (rd + wr) / kms / 1e6,
+                    "unit": "GB/s", "frac": (rd + wr) / kms / 1e6 / pk["hbm"],
+                    "tokens_per_s": W * n_win / (kms / 1e3)}
+        if validate:
+            same = torch.equal(payload, ref_payload)
+            out[key]["codes_equal_unchecked"] = bool(same)
+            if not same:
+                raise RuntimeError("coder microbenchmark: checked and unchecked codes differ")
+        else:
+            ref_payload = payload.clone()
+    del start, freq, payload, ref_payload
     torch.cuda.empty_cache()
     return out
 

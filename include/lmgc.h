@@ -197,10 +197,15 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * d_freq), arrays of lmgc_pair_tile_elems(n_win, win_tokens) elements, 16-byte aligned (INVALID
  * otherwise; elements past a window's length or past n_win are read but not used). Each thread
  * codes one window; a warp stages its 32 windows' tiles through shared memory with bulk copies.
- * Same arithmetic, output, scratch and errors as lmgc_range_encode. Syncs. */
+ * validate != 0: every pair is checked as in lmgc_range_encode. validate == 0: the caller vouches
+ * that every pair satisfies 0 < freq < 2^cdf_bits and start + freq <= 2^cdf_bits (as the encode
+ * path's own pairs from its CDF kernels do) and the check is skipped, as the encode path skips
+ * it; pairs that break this give unspecified codes and bit lengths (each at most its slot's
+ * size) but no access outside the call's buffers. Same arithmetic, output, scratch and errors as
+ * lmgc_range_encode. Syncs. */
 lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
-                                    size_t win_tokens, const uint32_t* d_win_len, uint8_t* d_out, size_t cap,
-                                    size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream);
+                                    size_t win_tokens, const uint32_t* d_win_len, int validate, uint8_t* d_out,
+                                    size_t cap, size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream);
 
 /* Elements of one window-tiled pair array for n_win windows of win_tokens positions
  * (ceil(n_win / 32) * ceil(win_tokens / 8) * 256). */

@@ -608,12 +608,12 @@ lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, co
 
 }  // extern "C"
 
-// lmgc_range_encode and lmgc_range_encode_tiled: the coder over a caller's pairs (validated),
-// with stream-ordered scratch
+// lmgc_range_encode and lmgc_range_encode_tiled: the coder over a caller's pairs (validated
+// unless the caller vouches for them), with stream-ordered scratch
 static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
                                     size_t win_tokens, const uint32_t* d_win_len, size_t stride_win,
-                                    size_t stride_pos, bool tiled, uint8_t* d_out, size_t cap, size_t* out_bytes,
-                                    uint32_t* d_bitlen, lmgc_stream stream) {
+                                    size_t stride_pos, bool tiled, bool validate, uint8_t* d_out, size_t cap,
+                                    size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream) {
   if (!out_bytes || (n_win && (!d_start || !d_freq || !d_bitlen)))
     return fail(nullptr, LMGC_ERR_INVALID, "null argument");
   if (cdf_bits < 1 || cdf_bits > 30) return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must be in 1..30");
@@ -638,7 +638,8 @@ static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_f
     {
       ProfScope ps(nullptr, kCoder, 8.0 * (double)n_win * (double)win_tokens, s);
       launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
-                          (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s, tiled, true);
+                          (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s, tiled,
+                          validate);
     }
     launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
     uint64_t total = 0;
@@ -673,14 +674,14 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
                               uint8_t* d_out, size_t cap, size_t* out_bytes, uint32_t* d_bitlen,
                               lmgc_stream stream) {
   return range_encode_any(d_start, d_freq, cdf_bits, n_win, win_tokens, d_win_len, stride_win, stride_pos, false,
-                          d_out, cap, out_bytes, d_bitlen, stream);
+                          true, d_out, cap, out_bytes, d_bitlen, stream);
 }
 
 lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
-                                    size_t win_tokens, const uint32_t* d_win_len, uint8_t* d_out, size_t cap,
-                                    size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream) {
-  return range_encode_any(d_start, d_freq, cdf_bits, n_win, win_tokens, d_win_len, 0, 0, true, d_out, cap,
-                          out_bytes, d_bitlen, stream);
+                                    size_t win_tokens, const uint32_t* d_win_len, int validate, uint8_t* d_out,
+                                    size_t cap, size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream) {
+  return range_encode_any(d_start, d_freq, cdf_bits, n_win, win_tokens, d_win_len, 0, 0, true, validate != 0, d_out,
+                          cap, out_bytes, d_bitlen, stream);
 }
 
 lmgc_status lmgc_pair_tile_elems(size_t n_win, size_t win_tokens, size_t* elems) {

@@ -43,7 +43,7 @@ size_t slot_bytes(size_t win_tokens, int P) {
   return ((words * 4 + 15) / 16) * 16;
 }
 
-constexpr int kRingWords = 16;   // completed words not yet written (at most 3 + 8 between flushes)
+constexpr int kRingWords = 16;   // completed words not yet written (at most 4 + 8 between flushes)
 constexpr int kRingStride = 20;  // words per thread in shared memory: 16-byte aligned, few bank conflicts
 constexpr int kCoderThreads = 128;
 
@@ -131,11 +131,16 @@ struct Stream {
         : "=r"(plo), "=r"(phi)
         : "r"(rlo), "r"(f), "r"(rhi));
     // k = 62 - bitlen(r f): clz of the high word less 2, plus 1 for r f = 2^62 (f = T). For any
-    // input k lies in [0, 30], so sh and w stay bounded whatever the pairs hold.
+    // input k lies in [0, 30], so sh and w stay bounded whatever the pairs hold. Unchecked pairs
+    // (the encode path's, from the CDF kernels) have f < T, so r f < 2^62 and the correction is
+    // never needed there; garbage pairs then give k in [-2, 30], with sh and w still bounded.
     int32_t k;
-    asm("{\n\t.reg .u32 z, t;\n\tclz.b32 z, %1;\n\tshr.u32 t, %1, 30;\n\tadd.u32 z, z, t;\n\tsub.s32 %0, z, 2;\n\t}"
-        : "=r"(k)
-        : "r"(phi));
+    if (CHECK)
+      asm("{\n\t.reg .u32 z, t;\n\tclz.b32 z, %1;\n\tshr.u32 t, %1, 30;\n\tadd.u32 z, z, t;\n\tsub.s32 %0, z, 2;\n\t}"
+          : "=r"(k)
+          : "r"(phi));
+    else
+      asm("{\n\t.reg .u32 z;\n\tclz.b32 z, %1;\n\tsub.s32 %0, z, 2;\n\t}" : "=r"(k) : "r"(phi));
     const int32_t s2 = P - k;  // in [0, P] for valid pairs
     asm("shf.r.wrap.b32 %0, %1, %2, %3;" : "=r"(rlo) : "r"(plo), "r"(phi), "r"(s2));
     asm("shr.u32 %0, %1, %2;" : "=r"(rhi) : "r"(phi), "r"(s2));
@@ -148,13 +153,16 @@ struct Stream {
     sh += full ? 32 : 0;
     w += full ? 1 : 0;
   }
-  // the completed 16-byte chunks of the ring to the slot: k <= 30 per token, so at most 8 words
-  // complete per 8 tokens and two chunks leave at most 3 + 8 - 8 words behind
+  // the completed 16-byte chunks of the ring to the slot, keeping at least the last completed
+  // word in the ring: a carry out of a0 (not rare while the window's offset is small) then
+  // lands in shared memory instead of a global read-modify-write of the slot. k <= 30 per token,
+  // so at most 8 words complete per 8 tokens; two chunks leave at most 4 words behind, and at
+  // most 12 of the ring's 16 are ever pending.
   template <int CHUNKS>
   __device__ __forceinline__ void flush() {
 #pragma unroll
     for (int q = 0; q < CHUNKS; q++) {
-      if (w - fw >= 4) {
+      if (w - fw >= 5) {
         uint4 v;
         asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
                      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
@@ -187,7 +195,10 @@ struct Stream {
       if ((uint32_t)i < max_words) slot[i] = ring_ld(i);
     if ((uint32_t)w < max_words) slot[w] = nrem >= 32 ? a0 : a0 & ~(0xFFFFFFFFu >> nrem);
     if (nrem > 32 && (uint32_t)(w + 1) < max_words) slot[w + 1] = a1 & ~(0xFFFFFFFFu >> (nrem - 32));
-    return nbits;
+    // a valid code fits its slot; pairs that were not checked may yield any length, which must
+    // not send the packing step past the slot
+    const uint64_t cap_bits = (uint64_t)max_words * 32u;
+    return nbits < cap_bits ? nbits : cap_bits;
   }
 };
 
@@ -202,9 +213,19 @@ __device__ __forceinline__ bool bar_try(uint32_t a, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// non-blocking probe of a phase (cheaper than try_wait when the phase has completed)
+__device__ __forceinline__ bool bar_test(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 // bounded wait for a phase: false (and kErrLimit) after about 2 s
 __device__ __forceinline__ bool bar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
-  if (bar_try(a, parity)) return true;
+  if (bar_test(a, parity) || bar_try(a, parity)) return true;
   uint64_t t0, t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
   for (uint32_t i = 1; i < (1u << 26); ++i) {
@@ -293,9 +314,10 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
 // Pairs in window tiles (the encode path): a warp codes the 32 windows of one tile column, whose
 // 8-position groups are contiguous 1 KiB tiles of starts and of freqs. The warp stages them
 // through a two-stage ring in shared memory: lane 0 fills a stage with bulk copies that complete
-// on the stage's mbarrier, every lane waits for it (bounded), reads its window's 8 pairs (two
-// 16-byte loads per array), codes them, and then the stage is refilled with the tiles two
-// groups on, which thus have a whole group of coding to land. No register holds pairs ahead.
+// on the stage's mbarrier, every lane waits for it (bounded) and reads its window's 8 pairs (two
+// 16-byte loads per array), and once every lane has read it the stage is refilled with the
+// tiles two groups on, which thus have two groups of coding to land. No register holds pairs
+// ahead beyond the group being coded.
 template <int PT, bool CHECK>
 __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
     const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
@@ -346,6 +368,10 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
     const uint4 s0 = qs[0], s1 = qs[1], f0 = qf[0], f1 = qf[1];
     const uint32_t cs[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
     const uint32_t cf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+    __syncwarp();  // every lane has read the stage
+    if (lane == 0 && g + 2 < g_all)
+      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((g + 2) << 8),
+                  tf + ((g + 2) << 8));
     if (!stopped && 8 * g < n) {
       if (8 * g + 8 <= n) {
 #pragma unroll
@@ -359,10 +385,6 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
       c.template flush<2>();
       if (CHECK && c.chk >= T) stopped = true;
     }
-    __syncwarp();  // every lane has read the stage
-    if (lane == 0 && g + 2 < g_all)
-      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((g + 2) << 8),
-                  tf + ((g + 2) << 8));
   }
   if (!ok) {
     // a wait gave up: let this warp's copies still in flight land before the block's shared

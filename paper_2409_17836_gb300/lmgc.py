@@ -85,7 +85,8 @@ SYMBOLS = {
     "lmgc_range_encode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p, C.c_size_t,
                                     C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p, C.c_void_p]),
     "lmgc_range_encode_tiled": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p,
-                                          C.c_void_p, C.c_size_t, C.POINTER(C.c_size_t), C.c_void_p, C.c_void_p]),
+                                          C.c_int, C.c_void_p, C.c_size_t, C.POINTER(C.c_size_t), C.c_void_p,
+                                          C.c_void_p]),
     "lmgc_pair_tile_elems": (C.c_int, [C.c_size_t, C.c_size_t, C.POINTER(C.c_size_t)]),
     "lmgc_range_encode_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int, C.c_size_t, C.c_size_t, C.c_void_p,
                                             C.c_size_t, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p,
@@ -268,18 +269,21 @@ def lmgc_pair_tile_elems(n_win: int, win_tokens: int) -> int:
 
 
 def lmgc_range_encode_tiled(start: torch.Tensor, freq: torch.Tensor, cdf_bits: int, n_win: int, win_tokens: int,
-                            win_len: torch.Tensor | None, out: torch.Tensor | None = None, stream=None):
+                            win_len: torch.Tensor | None, out: torch.Tensor | None = None, stream=None,
+                            validate: bool = True):
     """The coder over pairs in window tiles (lmgc_pair_tile_elems elements per array); returns
-    (payload bytes, bitlen)."""
+    (payload bytes, bitlen). validate=False skips the per-pair check, as the encode path does for
+    its own pairs (the caller vouches for 0 < freq < 2^cdf_bits and start + freq <= 2^cdf_bits)."""
     bitlen = torch.empty(max(n_win, 1), dtype=torch.int32, device=start.device)
     nbytes = C.c_size_t()
+    v = 1 if validate else 0
     if out is None:
-        st = load().lmgc_range_encode_tiled(_ptr(start), _ptr(freq), cdf_bits, n_win, win_tokens, _ptr(win_len), None,
-                                            0, C.byref(nbytes), _ptr(bitlen), _stream(stream))
+        st = load().lmgc_range_encode_tiled(_ptr(start), _ptr(freq), cdf_bits, n_win, win_tokens, _ptr(win_len), v,
+                                            None, 0, C.byref(nbytes), _ptr(bitlen), _stream(stream))
         if st not in (OK, ERR_NO_SPACE):
             _check(None, st)
         out = torch.empty(max(nbytes.value, 1), dtype=torch.uint8, device=start.device)
-    st = load().lmgc_range_encode_tiled(_ptr(start), _ptr(freq), cdf_bits, n_win, win_tokens, _ptr(win_len),
+    st = load().lmgc_range_encode_tiled(_ptr(start), _ptr(freq), cdf_bits, n_win, win_tokens, _ptr(win_len), v,
                                         _ptr(out), out.numel(), C.byref(nbytes), _ptr(bitlen), _stream(stream))
     _check(None, st)
     return out[: nbytes.value], bitlen[:n_win]

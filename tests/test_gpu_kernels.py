@@ -154,13 +154,15 @@ def test_cdf_bit_exact(V, P, rows):
 
 def coder(start, freq, P, n_win, W, lens, layout):
     """The GPU coder on [n_win][W] pairs passed in the given layout: row-major and position-major
-    through lmgc_range_encode's strides, window tiles through lmgc_range_encode_tiled."""
+    through lmgc_range_encode's strides, window tiles through lmgc_range_encode_tiled, checked
+    ("tile") or vouched for as the encode path does ("tile-trusted")."""
     wl = torch.from_numpy(lens.view(np.int32)).cuda() if lens is not None else None
-    if layout == "tile":
+    if layout in ("tile", "tile-trusted"):
         st, fr = to_pair_tiles(start), to_pair_tiles(freq)
         assert st.size == L.lmgc_pair_tile_elems(n_win, W)
         return L.lmgc_range_encode_tiled(torch.from_numpy(st.view(np.int32)).cuda(),
-                                         torch.from_numpy(fr.view(np.int32)).cuda(), P, n_win, W, wl)
+                                         torch.from_numpy(fr.view(np.int32)).cuda(), P, n_win, W, wl,
+                                         validate=layout == "tile")
     if layout == "row":
         s_dev, f_dev, sw, sp = start, freq, W, 1
     else:
@@ -182,10 +184,12 @@ def check_codes(out, bitlen, start, freq, P, lens):
 
 
 @pytest.mark.parametrize("P,layout", [(16, "row"), (24, "pos"), (24, "row"), (30, "pos"), (16, "tile"), (24, "tile"),
-                                      (30, "tile"), (7, "tile")])
+                                      (30, "tile"), (7, "tile"), (16, "tile-trusted"), (24, "tile-trusted"),
+                                      (30, "tile-trusted"), (7, "tile-trusted")])
 def test_range_encode_bit_exact(P, layout):
     """Ragged windows (lengths 1..300, one of 17) over random integer CDFs, 70 windows (two full
-    32-window blocks and a partial one), W = 300 (not a multiple of the 8-position tile group)."""
+    32-window blocks and a partial one), W = 300 (not a multiple of the 8-position tile group).
+    Every freq is below 2^P (at least V symbols share the range), so the unchecked form applies."""
     rng = np.random.default_rng(P)
     n_win, W = 70, 300
     V = 32 if P <= 16 else 1000
