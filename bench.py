@@ -188,9 +188,10 @@ def run_full(args, cfg, ctx, vals):
 
 
 def run_decode(args, cfg, ctx, vals):
-    """lmgc_decode of every window of an encoded stream (--decode-windows full windows, default one
-    batch), timed with CUDA events around the call; the restored tokens are compared with the
-    serialised input. The library decodes as many windows per step as its KV cache budget holds."""
+    """lmgc_decode of every window of an encoded stream (--decode-windows full windows; default as
+    many as one decode batch takes, that is as many as the library's KV cache budget holds, at
+    most the whole stream), timed with CUDA events around the call; the restored tokens are
+    compared with the serialised input."""
     import numpy as np
     import torch
 
@@ -198,7 +199,10 @@ def run_decode(args, cfg, ctx, vals):
     from paper_2409_17836_gb300 import lmgc as L
 
     W = cfg.window
-    n_dec = args.decode_windows or cfg.batch_windows
+    n_all = -(-L.lmgc_serial_tokens(ctx, vals.size) // W)
+    # (the encode below takes a little device memory of its own: keep 5% of the batch as slack so
+    # that the decode still runs as one batch)
+    n_dec = args.decode_windows or max(1, min(n_all, (L.lmgc_decode_batch_windows(ctx) * 19) // 20))
     n = values_for_tokens(lambda m: L.lmgc_serial_tokens(ctx, m), vals.size, n_dec * W)
     v = vals[:n]
     d = torch.from_numpy(v.view(np.int32) if v.dtype == np.float32 else v).cuda()

@@ -275,14 +275,21 @@ lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t*
  * container d_in (device, in_bytes) into d_tok (device, [n_ids][W] uint16; a partial last window
  * fills only its length). Each decode step runs the same kernels as lmgc_encode on one row per
  * window, so its logits -- and hence its CDFs -- are bit-identical to the encoder's. Windows
- * are decoded in batches of as many as a KV cache of half the free device memory (at most
- * 64 GiB) holds; the context keeps that cache for later calls (lmgc_destroy frees it).
+ * are decoded in batches of as many as a KV cache of half the free device memory holds (the
+ * cache keeps each position's keys and values, 2 n_kv_heads hd values per layer); the context
+ * keeps that cache for later calls (lmgc_destroy frees it).
  * Errors: CORRUPT (bad header, a model or serialisation word -- separators, byte grouping and
  * order, alphabet -- other than the context's, a code that leaves its interval, or a restored
  * window whose token checksum differs from the container's), INVALID
  * (window id out of range), NO_SPACE (cap_tok < n_ids * W), CUDA. Syncs. */
 lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, const uint32_t* h_win_ids,
                         size_t n_ids, uint16_t* d_tok, size_t cap_tok, lmgc_stream stream);
+
+/* The number of windows lmgc_decode would take per batch if called now: as many as a KV cache of
+ * half the free device memory (or the cache the context already holds, if larger) takes, at most
+ * batch_windows * W (one workspace row per window). A build choice with no counterpart in the
+ * paper, for callers sizing their decode requests. Errors: INVALID (null argument), CUDA. */
+lmgc_status lmgc_decode_batch_windows(lmgc_ctx* ctx, size_t* n);
 
 /* Per-stage device time of the last lmgc_encode call, in milliseconds (CUDA events):
  * ms[0] serialise, ms[1] model forward (all layers and the vocabulary projection),

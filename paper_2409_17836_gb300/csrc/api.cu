@@ -136,21 +136,25 @@ static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M
                      s);  // kSwiGLU never reaches here
 }
 
+// kv: the qkv rows themselves (prefill), or the decoder's cache (from_cache), whose rows hold a
+// position's keys and values only: [K heads | V heads], 2 n_kv_heads hd wide
 static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, int64_t n_win, int64_t pos_first,
-                      int n_pos, int64_t q_win_stride, cudaStream_t s) {
+                      int n_pos, int64_t q_win_stride, cudaStream_t s, bool from_cache = false) {
   const lmgc_config& c = ctx->cfg;
   // algorithmic flops: QK^T and PV over the causal triangle, 4*hd per (query, key) pair per head
   double pairs = 0;
   for (int64_t p = pos_first; p < pos_first + n_pos; p++) pairs += (double)(p + 1);
   ProfScope ps(ctx, kAttn, 4.0 * ctx->hd * c.n_heads * pairs * (double)n_win, s);
   const int qd = c.n_heads * ctx->hd, kd = c.n_kv_heads * ctx->hd;
+  const int64_t kv_dim = from_cache ? 2 * kd : ctx->qkv_dim;
+  const int k_off = from_cache ? 0 : qd, v_off = k_off + kd;
   if (c.dtype == LMGC_BF16) {  // lmgc_create admitted only head layouts the tcgen05 kernel takes
     const int64_t q_rows = q_win_stride == 1 ? n_win : n_win * c.window;
-    launch_attention_tc(q, q_rows, kv, n_win * c.window, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads,
+    launch_attention_tc(q, q_rows, ctx->qkv_dim, kv, n_win * c.window, kv_dim, k_off, v_off, out, qd, c.n_heads,
                         c.n_kv_heads, ctx->hd, c.window, n_win, pos_first, n_pos, q_win_stride, ctx->d_err, s);
   } else {
-    launch_attention(q, ctx->qkv_dim, kv, ctx->qkv_dim, qd, qd + kd, out, qd, c.n_heads, c.n_kv_heads, ctx->hd,
-                     c.window, n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
+    launch_attention(q, ctx->qkv_dim, kv, kv_dim, k_off, v_off, out, qd, c.n_heads, c.n_kv_heads, ctx->hd, c.window,
+                     n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
   }
 }
 
@@ -183,9 +187,11 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
       if (!decode) {
         attention(ctx, ws.qkv, ws.qkv, ws.att, n_win, 0, c.window, W, s);
       } else {
-        char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->qkv_dim * ctx->elt;
-        launch_copy_rows(ws.qkv, ctx->qkv_dim, cache_l, W, pos, n_win, ctx->qkv_dim, c.dtype, s);
-        attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s);
+        // the cache keeps each position's keys and values (columns [qd, qd + 2 kd) of its qkv row)
+        char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->kv_dim * ctx->elt;
+        launch_copy_rows((const char*)ws.qkv + (size_t)qd * ctx->elt, ctx->qkv_dim, cache_l, W, pos, n_win,
+                         ctx->kv_dim, c.dtype, s);
+        attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s, true);
       }
       // the O projection (K = qd, a short main loop) takes the 8-warp residual epilogue, whose
       // sums of squares come in 128-column parts; the choice depends on the shape only, so a
@@ -225,9 +231,10 @@ static void forward_layers(lmgc_ctx* ctx, int64_t rows, int64_t n_win, bool deco
     if (!decode) {
       attention(ctx, ws.qkv, ws.qkv, ws.att, n_win, 0, c.window, W, s);
     } else {
-      char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->qkv_dim * ctx->elt;
-      launch_copy_rows(ws.qkv, ctx->qkv_dim, cache_l, W, pos, n_win, ctx->qkv_dim, c.dtype, s);
-      attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s);
+      char* cache_l = (char*)ctx->kv_cache + (size_t)l * (size_t)n_win * W * ctx->kv_dim * ctx->elt;
+      launch_copy_rows((const char*)ws.qkv + (size_t)qd * ctx->elt, ctx->qkv_dim, cache_l, W, pos, n_win,
+                       ctx->kv_dim, c.dtype, s);
+      attention(ctx, ws.qkv, cache_l, ws.att, n_win, pos, 1, 1, s, true);
     }
     gemm(ctx, ws.att, L.wo, ws.x, rows, d, qd, kAddResidual, s);
     {
@@ -398,12 +405,13 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   cudaGetDevice(&ctx->device);
   ctx->hd = hd;
   ctx->qkv_dim = (c.n_heads + 2 * c.n_kv_heads) * hd;
+  ctx->kv_dim = 2 * c.n_kv_heads * hd;
   ctx->tpv = tpv;
   ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
   if (c.dtype == LMGC_BF16) {
     // a bf16 model has one backend, the tcgen05 kernels: without the tensor-map encoder (or on a
     // device they do not run on) the context is refused instead of computing on CUDA cores
-    const bool tc = tc_attention_supported(hd, ctx->qkv_dim) &&
+    const bool tc = tc_attention_supported(hd, ctx->qkv_dim) && tc_attention_supported(hd, ctx->kv_dim) &&
                     tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kStore) &&
                     tc_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd, kAddResidual) &&
                     tc_gemm_supported(1, 2 * (int64_t)c.d_ffn, c.d_model, kStore) &&
@@ -908,6 +916,22 @@ lmgc_status lmgc_encode_host(lmgc_ctx* ctx, const void* h_in, size_t n, uint8_t*
   return LMGC_OK;
 }
 
+// bytes of KV cache one decoded window needs: every layer's keys and values at W positions
+static size_t decode_kv_per_window(const lmgc_ctx* ctx) {
+  return (size_t)std::max(1, ctx->cfg.n_layers) * (size_t)ctx->cfg.window * (size_t)ctx->kv_dim * ctx->elt;
+}
+
+// windows per decode batch: a KV cache of half the free device memory (or the context's cache if
+// larger), at most one workspace row per window (batch_windows * W rows)
+static cudaError_t decode_batch(const lmgc_ctx* ctx, size_t* n) {
+  size_t free_b = 0, total_b = 0;
+  const cudaError_t e = cudaMemGetInfo(&free_b, &total_b);
+  if (e != cudaSuccess) return e;
+  const size_t budget = std::max<size_t>(ctx->kv_cap, free_b / 2);
+  *n = std::min<size_t>(budget / decode_kv_per_window(ctx), (size_t)ctx->cfg.batch_windows * ctx->cfg.window);
+  return cudaSuccess;
+}
+
 lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, const uint32_t* h_win_ids,
                         size_t n_ids, uint16_t* d_tok, size_t cap_tok, lmgc_stream stream) {
   if (!ctx || !d_in || (n_ids && (!h_win_ids || !d_tok))) return fail(ctx, LMGC_ERR_INVALID, "null argument");
@@ -951,16 +975,12 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   if (off[n_win] > in_bytes) return fail(ctx, LMGC_ERR_CORRUPT, "container payload truncated");
   for (size_t i = 0; i < n_ids; i++)
     if (h_win_ids[i] >= n_win) return fail(ctx, LMGC_ERR_INVALID, "window id out of range");
-  const size_t kv_per_win = (size_t)std::max(1, c.n_layers) * W * ctx->qkv_dim * ctx->elt;
+  const size_t kv_per_win = decode_kv_per_window(ctx);
   // decode batch: as many of the requested windows as a KV cache of half the free device memory
-  // (at most 64 GiB) holds -- a step's GEMMs cost about the same for 64 rows as for 256
-  size_t free_b = 0, total_b = 0;
-  LMGC_CUDA(ctx, cudaMemGetInfo(&free_b, &total_b));
-  const size_t kv_budget = std::max<size_t>(ctx->kv_cap, std::min<size_t>(free_b / 2, 64ull << 30));
-  // (one workspace row per window: at most batch_windows * W of them)
-  const int64_t nd_max = std::max<int64_t>(
-      1, std::min<int64_t>(std::min<int64_t>((int64_t)std::max<size_t>(n_ids, 1), (int64_t)(kv_budget / kv_per_win)),
-                           (int64_t)c.batch_windows * W));
+  // holds -- a step's GEMMs cost about the same for 64 rows as for 256
+  size_t batch = 0;
+  LMGC_CUDA(ctx, decode_batch(ctx, &batch));
+  const int64_t nd_max = std::max<int64_t>(1, std::min<int64_t>((int64_t)std::max<size_t>(n_ids, 1), (int64_t)batch));
   const size_t kv_need = kv_per_win * (size_t)nd_max;
   if (ctx->kv_cap < kv_need || !ctx->kv_cache) {
     LMGC_CUDA(ctx, ensure(&ctx->kv_cache, &ctx->kv_cap, kv_need));
@@ -1022,6 +1042,12 @@ lmgc_status lmgc_decode(lmgc_ctx* ctx, const uint8_t* d_in, size_t in_bytes, con
   cudaStreamSynchronize(s);
   if (ctx->prof.enabled) prof_collect(ctx);
   return st;
+}
+
+lmgc_status lmgc_decode_batch_windows(lmgc_ctx* ctx, size_t* n) {
+  if (!ctx || !n) return fail(ctx, LMGC_ERR_INVALID, "null argument");
+  LMGC_CUDA(ctx, decode_batch(ctx, n));
+  return LMGC_OK;
 }
 
 lmgc_status lmgc_launch_count(uint64_t* n) {

@@ -563,14 +563,15 @@ bool tc_attention_supported(int hd, int64_t qkv_dim) {
   return attn::g_encode != nullptr && (hd == 64 || hd == 128) && qkv_dim % 64 == 0;
 }
 
-void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t kv_rows, int64_t qkv_dim, int k_off,
-                         int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
-                         int64_t pos_first, int n_pos, int64_t q_win_stride, uint32_t* err, cudaStream_t s) {
+void launch_attention_tc(const void* q, int64_t q_rows, int64_t q_dim, const void* kv, int64_t kv_rows,
+                         int64_t kv_dim, int k_off, int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd,
+                         int W, int64_t n_win, int64_t pos_first, int n_pos, int64_t q_win_stride, uint32_t* err,
+                         cudaStream_t s) {
   using namespace attn;
   std::call_once(g_once, init_once);
   CUtensorMap tq, tkv;
-  if (!make_map(&tq, q, (uint64_t)qkv_dim, (uint64_t)q_rows, BQ) ||
-      !make_map(&tkv, kv, (uint64_t)qkv_dim, (uint64_t)kv_rows, hd == 128 ? Shape<128>::BKV : Shape<64>::BKV)) {
+  if (!make_map(&tq, q, (uint64_t)q_dim, (uint64_t)q_rows, BQ) ||
+      !make_map(&tkv, kv, (uint64_t)kv_dim, (uint64_t)kv_rows, hd == 128 ? Shape<128>::BKV : Shape<64>::BKV)) {
     set_thread_error("cuTensorMapEncodeTiled failed (attention)");
     return;
   }
@@ -591,7 +592,7 @@ void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t 
   // a decode step (one query row per window) packs the query heads of each KV head into one tile
   const int group = nq / nkv;
   p.packed = (n_pos == 1 && q_win_stride == 1 && group > 1 && group <= 32) ? group : 0;
-  if (p.packed && !make_map(&tq, q, (uint64_t)qkv_dim, (uint64_t)q_rows, 1)) {
+  if (p.packed && !make_map(&tq, q, (uint64_t)q_dim, (uint64_t)q_rows, 1)) {
     set_thread_error("cuTensorMapEncodeTiled failed (attention)");
     return;
   }

@@ -73,6 +73,7 @@ struct lmgc_ctx {
   lmgc_config cfg;
   int device = 0;
   int hd = 0, qkv_dim = 0, tpv = 0;
+  int kv_dim = 0;  // 2 n_kv_heads hd: a KV-cache row (keys, then values)
   size_t elt = 4;  // bytes per weight / activation element
   void* w_embed = nullptr;
   void* w_head = nullptr;
@@ -257,10 +258,12 @@ size_t dec_state_bytes();
 void launch_dec_init(const uint8_t* codes, const uint64_t* code_off, const uint32_t* bitlen, int64_t n,
                      void* state, cudaStream_t s);
 
-// attn_tc.cu (tcgen05)
+// attn_tc.cu (tcgen05). q: [q_rows][q_dim] (query head h at column h * hd); kv: [kv_rows][kv_dim]
+// (key head j at column k_off + j * hd, value head j at v_off + j * hd)
 bool tc_attention_supported(int hd, int64_t qkv_dim);
-void launch_attention_tc(const void* q, int64_t q_rows, const void* kv, int64_t kv_rows, int64_t qkv_dim, int k_off,
-                         int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
+void launch_attention_tc(const void* q, int64_t q_rows, int64_t q_dim, const void* kv, int64_t kv_rows,
+                         int64_t kv_dim, int k_off, int v_off, void* out, int64_t out_stride, int nq, int nkv, int hd,
+                         int W, int64_t n_win,
                          int64_t pos_first, int n_pos, int64_t q_win_stride, uint32_t* err, cudaStream_t s);
 
 // gemm_tc.cu (tcgen05)

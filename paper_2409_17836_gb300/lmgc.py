@@ -100,6 +100,7 @@ SYMBOLS = {
                                    C.c_void_p]),
     "lmgc_decode": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, C.c_size_t,
                               C.c_void_p]),
+    "lmgc_decode_batch_windows": (C.c_int, [C.c_void_p, C.POINTER(C.c_size_t)]),
     "lmgc_stage_times": (C.c_int, [C.c_void_p, C.c_void_p, C.c_size_t]),
     "lmgc_launch_count": (C.c_int, [C.c_void_p]),
     "lmgc_profile": (C.c_int, [C.c_void_p, C.c_int]),
@@ -346,6 +347,13 @@ def lmgc_encode_host(ctx: Context, values: torch.Tensor, out: torch.Tensor, stre
     _check(ctx, load().lmgc_encode_host(ctx.handle, _ptr(values), values.numel(), _ptr(out), out.numel(),
                                         C.byref(nb), _stream(stream)))
     return nb.value
+
+
+def lmgc_decode_batch_windows(ctx: Context) -> int:
+    """Windows lmgc_decode would take per batch with the device memory free now."""
+    n = C.c_size_t()
+    _check(ctx, load().lmgc_decode_batch_windows(ctx.handle, C.byref(n)))
+    return n.value
 
 
 def lmgc_decode(ctx: Context, container: torch.Tensor, win_ids, out: torch.Tensor | None = None,

@@ -47,6 +47,21 @@ def test_tiny_full_encode_decode_and_oracle_size():
     ctx.close()
 
 
+def test_decode_batch_windows():
+    """The decode batch query: at least one window, at most one workspace row per window, and a
+    batch that covers the KV cache the context already holds after a decode."""
+    cfg = configs.TINY
+    ctx = L.Context(cfg)
+    n = L.lmgc_decode_batch_windows(ctx)
+    assert 1 <= n <= cfg.batch_windows * cfg.window
+    vals = I.tiny_gradient(0)[:200]  # 1800 tokens: 8 windows of 256 (the last partial)
+    buf = encode(ctx, vals)
+    toks = decode_all(ctx, buf, list(range(8)))
+    assert np.array_equal(toks.reshape(-1)[:1800], O.serialize(vals, 0))
+    assert L.lmgc_decode_batch_windows(ctx) >= min(8, n)
+    ctx.close()
+
+
 def test_tiny_pairs_and_codes_given_gpu_logits():
     """CDF pairs bit-exact given the GPU's logits; codes bit-exact given those pairs."""
     cfg = configs.TINY
