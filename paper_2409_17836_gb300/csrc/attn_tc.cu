@@ -48,8 +48,8 @@ struct Shape {
   // keys per block: 64 at hd 64 (two CTAs per SM fit in tensor memory), 128 at hd 128, where
   // S = Q K^T then runs as MMAs of N = 128 (half as many MMA issues per key) and the softmax's
   // per-block costs (barrier waits, tensor-memory round trips, the arrive) cover twice the keys
-  static constexpr int BKV = HD == 128 ? 128 : 64;
-  static constexpr int NS = 3;                          // S buffers: S(kb) is issued NS - 1 blocks ahead
+  static constexpr int BKV = 64;
+  static constexpr int NS = HD == 128 ? 2 : 3;          // S buffers: S(kb) is issued NS - 1 blocks ahead
   static constexpr int KCH = HD / 64;                   // 64-column (128-byte) chunks of a row
   static constexpr uint32_t Q_BYTES = BQ * HD * 2;
   static constexpr uint32_t KV_CHUNK = BKV * 128;       // one BKV x 64 fp16 chunk
@@ -57,8 +57,8 @@ struct Shape {
   static constexpr uint32_t V_BYTES = BKV * HD * 2;
   static constexpr int KSK = NS, KSV = 2;               // stages of the K ring (one per S buffer) and of the V ring
   static constexpr uint32_t TMEM_S = 0;                 // S ring: NS x BKV columns (P in the first BKV / 2 of each)
-  static constexpr uint32_t TMEM_O = NS * BKV;          // O: HD columns (192 at hd 64, 384 at hd 128)
-  static constexpr uint32_t TMEM_COLS = HD == 64 ? 256 : 512;
+  static constexpr uint32_t TMEM_O = NS * BKV;          // O: HD columns (192 at hd 64, 128 at hd 128)
+  static constexpr uint32_t TMEM_COLS = 256;            // two CTAs per SM
   static constexpr size_t SMEM = Q_BYTES + KSK * K_BYTES + KSV * V_BYTES + 1024 + 256 + 3 * 1024;
   // S: M 128, N 64; PV: M 128, N HD, B (V) MN-major (bit 16)
   static constexpr uint32_t IDESC_S = (1u << 4) | ((uint32_t)(BKV >> 3) << 17) |
@@ -215,7 +215,7 @@ struct Params {
 };
 
 template <int HD, bool PACKED>
-__global__ void __launch_bounds__(kThreads, HD == 64 ? 2 : 1)
+__global__ void __launch_bounds__(kThreads, 2)
     k_attn_tc(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tkv, Params p) {
   using S = Shape<HD>;
   extern __shared__ uint8_t smem_raw[];
