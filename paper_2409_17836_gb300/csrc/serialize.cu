@@ -117,20 +117,68 @@ static void ser_dispatch(bool vec, const void* in, int64_t n, uint16_t* tok, uin
   else k_serialize<ND, NS, false><<<(unsigned)blocks, kSerThreads, 0, s>>>(in, n, tok, s0, s1);
 }
 
-// Byte-grouped layout: a block takes kGrpTile consecutive groups of g bytes; each thread writes
-// its groups' 2g digits and separator tokens into shared memory, and the block stores the tile's
-// tokens as 16-byte vectors (a tile starts at token k0 (2g + ns), k0 a multiple of kGrpTile, so
-// on a 16-byte boundary). Byte b of the stream is byte b mod 4 of fp32 value b / 4 (most
-// significant first, or least with le) or uint8 code b.
+// Byte-grouped layout. Byte b of the stream is byte b mod 4 of fp32 value b / 4 (most
+// significant first, or least with le) or uint8 code b. Tokens of group k start at k (2g + ns).
+//
+// k_serialize_units (whole tiles of a word-aligned stream): a thread takes one unit of lcm(g, 4)
+// bytes -- whole words, lcm(g, 4) / g whole groups -- loads its words, writes the unit's digit and
+// separator tokens into shared memory, and the block stores the tile's tokens as 16-byte vectors.
+// k_serialize_grouped (the rest, from group k_base): a block takes kGrpTile consecutive groups,
+// a thread a group at a time, bytes loaded one by one (it also takes the stream's short last
+// group). Both tiles start on 16-byte boundaries of the token array (their first group is a
+// multiple of 256 groups), and the shared tile is sized for the launch's g and ns.
 constexpr int kGrpThreads = 256, kGrpTile = 4 * kGrpThreads;
 
+template <int G>
+struct GroupUnit {
+  static constexpr int kBytes = G % 4 == 0 ? G : (G % 2 == 0 ? 2 * G : 4 * G);  // lcm(G, 4)
+  static constexpr int kWords = kBytes / 4;
+  static constexpr int kGroups = kBytes / G;
+};
+
+template <int G>
+__global__ void __launch_bounds__(kGrpThreads, 8) k_serialize_units(const uint32_t* __restrict__ in, int ns,
+                                                                 int swap, uint16_t* __restrict__ tok,
+                                                                 uint16_t sep0, uint16_t sep1) {
+  using U = GroupUnit<G>;
+  extern __shared__ __align__(16) uint16_t ubuf[];  // kGrpThreads * U::kGroups * (2 G + ns) tokens
+  const int tpg = 2 * G + ns, ut = U::kGroups * tpg;
+  const int t = threadIdx.x;
+  const uint32_t* src = in + ((int64_t)blockIdx.x * kGrpThreads + t) * U::kWords;
+  uint32_t w[U::kWords];
+#pragma unroll
+  for (int i = 0; i < U::kWords; i++) {
+    w[i] = __ldcs(src + i);
+    if (swap) w[i] = __byte_perm(w[i], 0u, 0x0123);  // most significant byte first: byte j at bits 8j
+  }
+  uint16_t* o = ubuf + t * ut;
+#pragma unroll
+  for (int k = 0; k < U::kGroups; k++) {
+#pragma unroll
+    for (int i = 0; i < G; i++) {
+      const int b = k * G + i;  // the unit's byte b: byte b & 3 of word b >> 2
+      const uint32_t byte = (w[b >> 2] >> (8 * (b & 3))) & 0xFFu;
+      o[2 * i] = (uint16_t)(byte >> 4);
+      o[2 * i + 1] = (uint16_t)(byte & 0xFu);
+    }
+    if (ns >= 1) o[2 * G] = sep0;
+    if (ns >= 2) o[2 * G + 1] = sep1;
+    o += tpg;
+  }
+  __syncthreads();
+  const int nt = kGrpThreads * ut;  // a multiple of 8
+  const uint4* s4 = reinterpret_cast<const uint4*>(ubuf);
+  uint4* d4 = reinterpret_cast<uint4*>(tok + (int64_t)blockIdx.x * nt);
+  for (int q = t; q < nt / 8; q += kGrpThreads) __stcs(d4 + q, s4[q]);
+}
+
 __global__ void __launch_bounds__(kGrpThreads) k_serialize_grouped(const void* __restrict__ in, int64_t n, int bv,
-                                                                   int g, int ns, int le,
+                                                                   int g, int ns, int le, int64_t k_base,
                                                                    uint16_t* __restrict__ tok, uint16_t sep0,
                                                                    uint16_t sep1, bool vec) {
-  __shared__ __align__(16) uint16_t buf[kGrpTile * (2 * 8 + 2)];
+  extern __shared__ __align__(16) uint16_t buf[];  // kGrpTile * (2 g + ns) tokens
   const int64_t nb = n * bv, n_groups = (nb + g - 1) / g;
-  const int64_t k0 = (int64_t)blockIdx.x * kGrpTile;
+  const int64_t k0 = k_base + (int64_t)blockIdx.x * kGrpTile;
   const int tpg = 2 * g + ns;
   const int ng = n_groups - k0 < kGrpTile ? (int)(n_groups - k0) : kGrpTile;
   for (int i = threadIdx.x; i < ng; i += kGrpThreads) {
@@ -176,8 +224,41 @@ void launch_serialize(int input_kind, int sep_mode, int byte_group, int byte_ord
     const int bv = (int)bytes_per_value(input_kind), g = byte_group ? byte_group : bv;
     const int64_t groups = (n * bv + g - 1) / g;
     const bool vec = ((uintptr_t)tok) % 16 == 0;  // tiles start on 16-byte boundaries then
-    k_serialize_grouped<<<(unsigned)((groups + kGrpTile - 1) / kGrpTile), kGrpThreads, 0, s>>>(
-        in, n, bv, g, sep_count(sep_mode), byte_order, tok, s0, s1, vec);
+    const int ns = sep_count(sep_mode);
+    const int64_t nb = n * bv;
+    // whole tiles of units (word loads need a word-aligned stream; the tile stores 16-byte ones)
+    int64_t k_base = 0;
+    if (vec && (bv == 4 || ((uintptr_t)in) % 4 == 0)) {
+      const int swap = bv == 4 && !byte_order;  // fp32 bytes most significant first
+      const uint32_t* w = reinterpret_cast<const uint32_t*>(in);
+#define LMGC_UNITS(GV)                                                                                          \
+  do {                                                                                                           \
+    using U = GroupUnit<GV>;                                                                                     \
+    const int64_t tiles = nb / ((int64_t)kGrpThreads * U::kBytes);                                               \
+    if (tiles > 0) {                                                                                             \
+      const size_t sm = (size_t)kGrpThreads * U::kGroups * (size_t)(2 * GV + ns) * sizeof(uint16_t);            \
+      k_serialize_units<GV><<<(unsigned)tiles, kGrpThreads, sm, s>>>(w, ns, swap, tok, s0, s1);                 \
+      k_base = tiles * kGrpThreads * U::kGroups;                                                                  \
+    }                                                                                                            \
+  } while (0)
+      switch (g) {
+        case 1: LMGC_UNITS(1); break;
+        case 2: LMGC_UNITS(2); break;
+        case 3: LMGC_UNITS(3); break;
+        case 4: LMGC_UNITS(4); break;
+        case 5: LMGC_UNITS(5); break;
+        case 6: LMGC_UNITS(6); break;
+        case 7: LMGC_UNITS(7); break;
+        default: LMGC_UNITS(8); break;
+      }
+#undef LMGC_UNITS
+    }
+    if (k_base < groups) {
+      if (k_base > 0) note_launch();
+      const size_t smem = (size_t)kGrpTile * (size_t)(2 * g + ns) * sizeof(uint16_t);  // <= 36 KB (g <= 8)
+      k_serialize_grouped<<<(unsigned)((groups - k_base + kGrpTile - 1) / kGrpTile), kGrpThreads, smem, s>>>(
+          in, n, bv, g, ns, byte_order, k_base, tok, s0, s1, vec);
+    }
     return;
   }
   int ns = sep_mode == LMGC_SEP_NONE ? 0 : (sep_mode == LMGC_SEP_COMMA_SPACE ? 2 : 1);

@@ -63,12 +63,14 @@ def test_serialize_unaligned_input_and_u8():
     ctx.close()
 
 
-@pytest.mark.parametrize("group,order", [(1, 0), (2, 1), (3, 0), (3, 1), (4, 1), (8, 0), (8, 1)])
+@pytest.mark.parametrize("group,order", [(1, 0), (2, 1), (3, 0), (3, 1), (4, 1), (5, 1), (6, 0), (7, 1), (8, 0),
+                                         (8, 1)])
 @pytest.mark.parametrize("sep_mode", [0, 2, 4])
 def test_serialize_byte_groups_bit_exact(group, order, sep_mode):
     """Byte grouping (Sec. 5.3): tokens bit-exact with the oracle for fp32 values (either byte
     order) and uint8 codes, ragged counts whose last group is partial; round trip; the token
-    count through lmgc_serial_tokens."""
+    count through lmgc_serial_tokens. The counts span whole tiles of word-aligned units (the
+    unit kernel, one instantiation per group width) and the rest (the per-group kernel)."""
     ctx = ctx_for(sep_mode=sep_mode, byte_group=group, byte_order=order)
     rng = np.random.default_rng(10 * group + order + sep_mode)
     for n in (1, 2, 3, 1001, 65537):
@@ -83,7 +85,7 @@ def test_serialize_byte_groups_bit_exact(group, order, sep_mode):
         assert L.lmgc_deserialize(ctx, tok, back) == n
         assert np.array_equal(back.cpu().numpy().view(np.uint32), bits), n
     # a per-value token count exists unless groups cross values and carry separators
-    assert (ctx.tpv is None) == (group in (3, 8) and sep_mode != 4)
+    assert (ctx.tpv is None) == (group in (3, 5, 6, 7, 8) and sep_mode != 4)
     ctx.close()
     ctx = ctx_for(sep_mode=sep_mode, byte_group=group, input_kind=L.IN_U8)
     codes = rng.integers(0, 256, 4099).astype(np.uint8)
