@@ -166,10 +166,12 @@ lmgc_status lmgc_quantize_cdf(lmgc_ctx* ctx, const float* d_logits, size_t rows,
 
 /* The coder's per-token input without materialising CDFs: for row r with symbol d_sym[r],
  * d_start[r] = cdf_r[sym] and d_freq[r] = cdf_r[sym + 1] - cdf_r[sym] under the quantiser of
- * lmgc_quantize_cdf. All arrays are indexed by row. With alphabet 1 the quantiser runs over the
- * restricted alphabet's logits of each row (V' ids), sym is the index of d_sym[r] among them,
- * and the call syncs to report a d_sym[r] outside the alphabet (CORRUPT; its pair is (0, 1)).
- * Errors: INVALID, CORRUPT, CUDA. */
+ * lmgc_quantize_cdf. All arrays are indexed by row. It runs the encode path's kernel, after a
+ * pass that takes each row's maximum into stream-ordered scratch of 4 bytes per row (allocated
+ * and freed on the stream). With alphabet 1 the quantiser runs over the restricted alphabet's
+ * logits of each row (V' ids), sym is the index of d_sym[r] among them, and the call syncs to
+ * report a d_sym[r] outside the alphabet (CORRUPT; its pair is (0, 1)).
+ * Errors: INVALID, CORRUPT, CUDA (including a failed scratch allocation). */
 lmgc_status lmgc_cdf_pairs(lmgc_ctx* ctx, const float* d_logits, size_t rows, const uint16_t* d_sym,
                            uint32_t* d_start, uint32_t* d_freq, lmgc_stream stream);
 
