@@ -261,6 +261,21 @@ def test_range_encode_rejects_bad_pairs():
         assert e.value.status == L.ERR_INVALID, bad
 
 
+def test_range_encode_tiled_rejects_misaligned_pairs():
+    """The tiles are staged by bulk copies, whose sources must be 16-byte aligned: a pair array
+    that starts 4 bytes into an allocation is refused on the host (INVALID), before any launch."""
+    st = np.zeros((32, 8), np.uint32)
+    fr = np.full((32, 8), 2, np.uint32)
+    s = torch.from_numpy(np.concatenate([[0], to_pair_tiles(st)]).astype(np.uint32).view(np.int32)).cuda()
+    f = torch.from_numpy(np.concatenate([[0], to_pair_tiles(fr)]).astype(np.uint32).view(np.int32)).cuda()
+    for validate in (True, False):
+        with pytest.raises(L.LmgcError) as e:
+            L.lmgc_range_encode_tiled(s[1:], f[1:], 16, 32, 8, None, validate=validate)
+        assert e.value.status == L.ERR_INVALID
+    out, bitlen = L.lmgc_range_encode_tiled(s[1:].clone(), f[1:].clone(), 16, 32, 8, None)
+    check_codes(out, bitlen, st, fr, 16, np.full(32, 8, np.uint32))
+
+
 @pytest.mark.parametrize("sep_mode,V,P", [(0, 32, 16), (2, 1000, 20), (4, 32000, 24)])
 def test_cdf_pairs_alphabet_bit_exact(sep_mode, V, P):
     """Restricted-alphabet pairs: the quantiser over each row's alphabet logits (ascending ids)
