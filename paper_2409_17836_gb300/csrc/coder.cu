@@ -13,10 +13,12 @@
 // before it, so L is the sum of the addends at their positions. A thread keeps stream bits
 // [32 w, 32 w + 96) in three registers a0:a1:a2 and adds each addend at offset off = B - 32 w,
 // which stays in [3, 34] between tokens (sh = 34 - off is a funnel-shift count below 32). Word a0
-// is complete when off reaches 35: it leaves, the window moves one word on. A carry out of a0
-// increments the completed words before it (never beyond word 0: L + R stays below 2^(B+62)).
+// is complete when off reaches 35: it moves to a fourth register am1, the window moves one word
+// on, and the word am1 held leaves. A carry out of a0 goes into am1 within the same add; one out
+// of am1 (only when am1 is all ones) increments the completed words before it (never beyond
+// word 0: L + R stays below 2^(B+62)).
 //
-// Per token: two 32x32->64 multiply-adds per product, three funnel shifts, a three-word add with
+// Per token: two 32x32->64 multiply-adds per product, three funnel shifts, a four-word add with
 // carry, a count of leading zeros and a handful of selects (the step is inline PTX so that each
 // operation is one instruction). Completed words go to a per-thread ring in shared memory and
 // leave for the stream's slot in 16-byte chunks, at most two per 8 tokens: scattered 4-byte
@@ -50,9 +52,11 @@ constexpr int kCoderThreads = 128;
 struct Stream {
   uint32_t rlo, rhi;   // r = R >> P
   uint32_t a0, a1, a2; // stream bits [32 w, 32 w + 96)
+  uint32_t am1;        // word w - 1, the last completed one (a carry out of a0 lands here)
+  uint32_t nz;         // OR of the words below word 0 as they completed (checked form; zero for valid input)
   int32_t sh;          // 34 - (B - 32 w), in [0, 31] between tokens
   int32_t w;           // word index of a0 (-1 before the first word completes)
-  int32_t fw;          // words [0, fw) are in the slot, [fw, w) only in the ring
+  int32_t fw;          // words [0, fw) are in the slot, [fw, w - 1) only in the ring
   uint32_t chk;        // OR of s | (f - 1) | (s + f - 1) over the tokens: >= T iff a pair was invalid
   uint32_t max_words;
   uint32_t* slot;
@@ -73,7 +77,7 @@ struct Stream {
     const uint64_t r0 = 1ull << (62 - P);  // R = 2^62
     rlo = (uint32_t)r0;
     rhi = (uint32_t)(r0 >> 32);
-    a0 = a1 = a2 = 0u;
+    a0 = a1 = a2 = am1 = nz = 0u;
     sh = 2;  // B = 0 at w = -1: off = 32
     w = -1;
     fw = 0;
@@ -83,10 +87,10 @@ struct Stream {
     ring = (uint32_t)__cvta_generic_to_shared(rg);
     overflow = false;
   }
-  // +1 into the completed words before a0 (ring or slot); a carry past word 0 cannot happen for
+  // +1 into the completed words before am1 (ring or slot); a carry past word 0 cannot happen for
   // valid input and is reported
   __device__ __forceinline__ void carry() {
-    for (int32_t i = w - 1; i >= 0; --i) {
+    for (int32_t i = w - 2; i >= 0; --i) {
       uint32_t v;
       if (i >= fw) {
         v = ring_ld(i) + 1u;
@@ -100,18 +104,20 @@ struct Stream {
     }
     overflow = true;
   }
-  // a0:a1:a2 += chi:clo placed with its bit 61 at stream position B; returns the carry out of a0
+  // am1:a0:a1:a2 += chi:clo placed with its bit 61 at stream position B; returns the carry out of
+  // am1 (which needs am1 = 2^32 - 1, so almost never happens)
   __device__ __forceinline__ uint32_t add(uint32_t clo, uint32_t chi) {
     uint32_t cy;
     asm("{\n\t.reg .u32 x0, x1, x2;\n\t"
-        "shf.l.wrap.b32 x2, 0, %4, %6;\n\t"
-        "shf.l.wrap.b32 x1, %4, %5, %6;\n\t"
-        "shf.l.wrap.b32 x0, %5, 0, %6;\n\t"
+        "shf.l.wrap.b32 x2, 0, %5, %7;\n\t"
+        "shf.l.wrap.b32 x1, %5, %6, %7;\n\t"
+        "shf.l.wrap.b32 x0, %6, 0, %7;\n\t"
         "add.cc.u32 %2, %2, x2;\n\t"
         "addc.cc.u32 %1, %1, x1;\n\t"
         "addc.cc.u32 %0, %0, x0;\n\t"
+        "addc.cc.u32 %4, %4, 0;\n\t"
         "addc.u32 %3, 0, 0;\n\t}"
-        : "+r"(a0), "+r"(a1), "+r"(a2), "=r"(cy)
+        : "+r"(a0), "+r"(a1), "+r"(a2), "=r"(cy), "+r"(am1)
         : "r"(clo), "r"(chi), "r"(sh));
     return cy;
   }
@@ -134,19 +140,24 @@ struct Stream {
     // input k lies in [0, 30], so sh and w stay bounded whatever the pairs hold. Unchecked pairs
     // (the encode path's, from the CDF kernels) have f < T, so r f < 2^62 and the correction is
     // never needed there; garbage pairs then give k in [-2, 30], with sh and w still bounded.
-    int32_t k;
-    if (CHECK)
-      asm("{\n\t.reg .u32 z, t;\n\tclz.b32 z, %1;\n\tshr.u32 t, %1, 30;\n\tadd.u32 z, z, t;\n\tsub.s32 %0, z, 2;\n\t}"
-          : "=r"(k)
-          : "r"(phi));
-    else
-      asm("{\n\t.reg .u32 z;\n\tclz.b32 z, %1;\n\tsub.s32 %0, z, 2;\n\t}" : "=r"(k) : "r"(phi));
-    const int32_t s2 = P - k;  // in [0, P] for valid pairs
+    // (k + 2 is kept, so that P - k and sh - k are each one add of a constant)
+    int32_t z;
+    asm("clz.b32 %0, %1;" : "=r"(z) : "r"(phi));
+    if (CHECK) z += (int32_t)(phi >> 30);
+    const int32_t s2 = (P + 2) - z;  // P - k, in [0, P] for valid pairs
     asm("shf.r.wrap.b32 %0, %1, %2, %3;" : "=r"(rlo) : "r"(plo), "r"(phi), "r"(s2));
     asm("shr.u32 %0, %1, %2;" : "=r"(rhi) : "r"(phi), "r"(s2));
-    sh -= k;
+    sh = (sh + 2) - z;
     const bool full = sh < 0;
-    if (full) ring_st(w, a0);
+    // the completed word before a0 leaves for the ring (words -2 and -1, which the first two
+    // completions retire, land in ring slots that are rewritten before any read; they are
+    // nonzero only after a carry past word 0, impossible for valid pairs, so only the checked
+    // form looks at them)
+    if (full) {
+      ring_st(w - 1, am1);
+      if (CHECK) nz |= w <= 0 ? am1 : 0u;
+    }
+    am1 = full ? a0 : am1;
     a0 = full ? a1 : a0;
     a1 = full ? a2 : a1;
     a2 = full ? 0u : a2;
@@ -177,6 +188,11 @@ struct Stream {
   // returns B + 2 and writes every remaining word
   __device__ __forceinline__ uint64_t finish() {
     if (add(0xFFFFFFFFu, 0x0FFFFFFFu)) carry();
+    // am1 back into the ring (word w - 1), or, below word 0, checked to be zero like the words
+    // below word 0 that completed earlier
+    if (w >= 1) ring_st(w - 1, am1);
+    else nz |= am1;
+    overflow |= nz != 0u;
     const int32_t off = 34 - sh;
     int32_t nrem;  // bits of the code in a0 (and a1)
     uint64_t nbits;

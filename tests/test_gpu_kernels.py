@@ -204,7 +204,7 @@ def test_range_encode_bit_exact(P, layout):
     check_codes(out, bitlen, start, freq, P, lens)
 
 
-@pytest.mark.parametrize("layout", ["tile", "pos"])
+@pytest.mark.parametrize("layout", ["tile", "tile-trusted", "pos"])
 @pytest.mark.parametrize("P", [16, 24])
 def test_range_encode_carry_heavy(P, layout):
     """Streams built to carry: mostly tokens at the top of the range (start = T - freq) with small
