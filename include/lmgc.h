@@ -198,7 +198,8 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * i of window w is element ((w / 32) * G + i / 8) * 256 + (w % 32) * 8 + i % 8 of d_start (and of
  * d_freq), arrays of lmgc_pair_tile_elems(n_win, win_tokens) elements, 16-byte aligned (INVALID
  * otherwise; elements past a window's length or past n_win are read but not used). Each thread
- * codes one window; a warp stages its 32 windows' tiles through shared memory with bulk copies.
+ * codes one window; a warp stages its 32 windows' tiles through shared memory with asynchronous
+ * 16-byte copies.
  * validate != 0: every pair is checked as in lmgc_range_encode. validate == 0: the caller vouches
  * that every pair satisfies 0 < freq < 2^cdf_bits and start + freq <= 2^cdf_bits (as the encode
  * path's own pairs from its CDF kernels do) and the check is skipped, as the encode path skips

@@ -26,7 +26,7 @@
 //
 // Layout: one stream per thread, 32 windows per warp. Pairs come from window tiles (the encode
 // path; a warp's 8 tokens are one contiguous kilobyte per array, staged through shared memory by
-// bulk copies) or from start[w*stride_win + i*stride_pos] (lmgc_range_encode's general layout,
+// asynchronous copies) or from start[w*stride_win + i*stride_pos] (lmgc_range_encode's general layout,
 // loaded 8 tokens ahead).
 // Slot words are stored in native byte order; the pack step writes the bytes most significant
 // first.
@@ -218,54 +218,7 @@ struct Stream {
   }
 };
 
-// mbarrier and bulk-copy helpers for the staged tiles (shared::cta addresses)
 __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-__device__ __forceinline__ bool bar_try(uint32_t a, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(a), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// non-blocking probe of a phase (cheaper than try_wait when the phase has completed)
-__device__ __forceinline__ bool bar_test(uint32_t a, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(a), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// bounded wait for a phase: false (and kErrLimit) after about 2 s
-__device__ __forceinline__ bool bar_wait(uint32_t a, uint32_t parity, uint32_t* err) {
-  if (bar_test(a, parity) || bar_try(a, parity)) return true;
-  uint64_t t0, t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
-  for (uint32_t i = 1; i < (1u << 26); ++i) {
-    if (bar_try(a, parity)) return true;
-    if ((i & 63) == 0) {
-      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-      if (t - t0 > 2000000000ull) break;
-    }
-  }
-  atomicOr(err, kErrLimit);
-  return false;
-}
-// one group's start and freq tiles (1 KiB each) into a stage, completing on its barrier
-__device__ __forceinline__ void stage_tiles(uint32_t bar, uint32_t dst_s, uint32_t dst_f, const uint32_t* src_s,
-                                            const uint32_t* src_f) {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], 2048;" ::"r"(bar) : "memory");
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 1024, [%2];" ::"r"(dst_s),
-               "l"(src_s), "r"(bar)
-               : "memory");
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], 1024, [%2];" ::"r"(dst_f),
-               "l"(src_f), "r"(bar)
-               : "memory");
-}
 
 // One stream per thread, pairs at start[w*stride_win + i*stride_pos] (lmgc_range_encode's general
 // layout), loaded 8 tokens ahead. PT: P at compile time (0: P_rt). CHECK: validate the pairs (a
@@ -329,11 +282,11 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
 
 // Pairs in window tiles (the encode path): a warp codes the 32 windows of one tile column, whose
 // 8-position groups are contiguous 1 KiB tiles of starts and of freqs. The warp stages them
-// through a two-stage ring in shared memory: lane 0 fills a stage with bulk copies that complete
-// on the stage's mbarrier, every lane waits for it (bounded) and reads its window's 8 pairs (two
-// 16-byte loads per array), and once every lane has read it the stage is refilled with the
-// tiles two groups on, which thus have two groups of coding to land. No register holds pairs
-// ahead beyond the group being coded.
+// through a two-stage ring in shared memory with asynchronous 16-byte copies (every lane copies
+// its share of each tile, so that a copy instruction of the warp covers 512 contiguous bytes):
+// the copies of group g + 2 are issued once every lane has read group g's stage, and so have two
+// groups of coding to land. (Kilobyte bulk copies completing on an mbarrier, one lane issuing,
+// were 1-2% slower.) No register holds pairs ahead beyond the group being coded.
 template <int PT, bool CHECK>
 __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
     const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
@@ -342,7 +295,6 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
   constexpr int kWarps = kCoderThreads / 32;
   __shared__ __align__(16) uint32_t rings[kCoderThreads * kRingStride];
   __shared__ __align__(128) uint32_t tiles[kWarps][2][2][256];  // [warp][stage][start, freq][32 x 8]
-  __shared__ __align__(8) uint64_t full[kWarps][2];
   const int P = PT ? PT : P_rt;
   const uint32_t T = 1u << P;
   const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
@@ -363,31 +315,37 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
   const int64_t col = pair_tile_index(w0, 0, groups);  // element of the column's first tile
   const uint32_t* ts = start + col;
   const uint32_t* tf = freq + col;
-  const uint32_t bar0 = smem_addr(&full[wp][0]), bar1 = smem_addr(&full[wp][1]);
-  if (lane == 0) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar0) : "memory");
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar1) : "memory");
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    for (int st = 0; st < 2 && st < g_all; st++)
-      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((int64_t)st << 8),
-                  tf + ((int64_t)st << 8));
-  }
-  __syncwarp();
-  bool ok = true, stopped = false;
-  int64_t g = 0;
-  for (; g < g_all; g++) {
+  // Each lane copies 16 bytes of each half kilobyte of a group's two tiles (every copy
+  // instruction of the warp covers 512 contiguous bytes); a lane's own 32 bytes of an array thus
+  // come from two other lanes, and __syncwarp after the wait makes them visible.
+  const uint32_t stage0 = smem_addr(tiles[wp][0][0]);  // stage t, array a at + (2 t + a) KiB
+  auto issue = [&](int64_t gg) {
+    if (gg < g_all) {
+      const uint32_t d = stage0 + (uint32_t)(gg & 1) * 2048u + 16u * (uint32_t)lane;
+      const uint32_t* src_s = ts + (gg << 8) + 4 * lane;
+      const uint32_t* src_f = tf + (gg << 8) + 4 * lane;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src_s) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d + 512u), "l"(src_s + 128) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d + 1024u), "l"(src_f) : "memory");
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d + 1536u), "l"(src_f + 128) : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  issue(0);
+  issue(1);
+  const bool ok = true;
+  bool stopped = false;
+  for (int64_t g = 0; g < g_all; g++) {
     const int st = (int)(g & 1);
-    ok = __all_sync(0xffffffffu, bar_wait(st ? bar1 : bar0, (uint32_t)(g >> 1) & 1u, err));
-    if (!ok) break;
+    asm volatile("cp.async.wait_group 1;" ::: "memory");  // this lane's copies of group g
+    __syncwarp();                                          // and every other lane's
     const uint4* qs = reinterpret_cast<const uint4*>(tiles[wp][st][0] + 8 * lane);
     const uint4* qf = reinterpret_cast<const uint4*>(tiles[wp][st][1] + 8 * lane);
     const uint4 s0 = qs[0], s1 = qs[1], f0 = qf[0], f1 = qf[1];
     const uint32_t cs[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
     const uint32_t cf[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
     __syncwarp();  // every lane has read the stage
-    if (lane == 0 && g + 2 < g_all)
-      stage_tiles(st ? bar1 : bar0, smem_addr(tiles[wp][st][0]), smem_addr(tiles[wp][st][1]), ts + ((g + 2) << 8),
-                  tf + ((g + 2) << 8));
+    issue(g + 2);
     if (!stopped && 8 * g < n) {
       if (8 * g + 8 <= n) {
 #pragma unroll
@@ -402,14 +360,7 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
       if (CHECK && c.chk >= T) stopped = true;
     }
   }
-  if (!ok) {
-    // a wait gave up: let this warp's copies still in flight land before the block's shared
-    // memory is released (bounded again), and report the window as failed
-    if (lane == 0) {
-      for (int64_t h = g; h < g + 2 && h < g_all; h++) bar_wait((h & 1) ? bar1 : bar0, (uint32_t)(h >> 1) & 1u, err);
-    }
-    __syncwarp();
-  }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   if (!live) return;
   bitlen[w] = (uint32_t)c.finish();
   if (bad || !ok || c.overflow || (CHECK && c.chk >= T)) atomicOr(err, kErrCorrupt);
