@@ -202,9 +202,9 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * 16-byte copies.
  * validate != 0: every pair is checked as in lmgc_range_encode. validate == 0: the caller vouches
  * that every pair satisfies 0 < freq < 2^cdf_bits and start + freq <= 2^cdf_bits (as the encode
- * path's own pairs from its CDF kernels do) and the check is skipped, as the encode path skips
- * it; pairs that break this give unspecified codes and bit lengths (each at most its slot's
- * size) but no access outside the call's buffers. Same arithmetic, output, scratch and errors as
+ * path's own pairs from its CDF kernels do) and the check is skipped; pairs that break this give
+ * unspecified codes and bit lengths (each at most its slot's size) but no access outside the
+ * call's buffers. The checked form is not slower (the encode path uses it for its own pairs). Same arithmetic, output, scratch and errors as
  * lmgc_range_encode. Syncs. */
 lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
                                     size_t win_tokens, const uint32_t* d_win_len, int validate, uint8_t* d_out,

@@ -778,9 +778,11 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   launch_window_crc(ctx->tok + w_begin * W, W, d_wl, n_win, ctx->enc_crc, s);
   {
     ProfScope ps(ctx, kCoder, (double)n_win * (double)W * 8, s);
-    // the pairs come from the CDF kernels, valid by construction: no per-pair check
+    // the pairs come from the CDF kernels, valid by construction; they are checked all the same,
+    // as the checked kernel measured faster than the unchecked one (its check runs beside the
+    // serial chain), and an invalid pair then fails the call instead of giving a wrong code
     launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 0, 0, ctx->enc_slots, slot,
-                        ctx->enc_bl, ctx->d_err, s, true, false);
+                        ctx->enc_bl, ctx->d_err, s, true, true);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[3], s));
   launch_pack_codes(ctx->enc_slots, slot, ctx->enc_bl, n_win, ctx->enc_off, nullptr, s);
