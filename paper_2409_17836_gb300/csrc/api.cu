@@ -125,15 +125,15 @@ static void prof_collect(lmgc_ctx* ctx) {
 }
 
 // ---- GEMM dispatch by the model's dtype: a bf16-weight model runs every contraction on the
-// tcgen05 kernel (lmgc_create rejects shapes it does not take), an fp32 model on CUDA cores ----
+// fp16 tcgen05 kernel, an fp32 model on the three-pass TF32 tcgen05 kernel (lmgc_create rejects
+// shapes and devices they do not take) ----
 static void gemm(lmgc_ctx* ctx, const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int epi,
                  cudaStream_t s, const RopeArgs* rope = nullptr, const NormArgs* norm = nullptr) {
   ProfScope ps(ctx, kGemm, 2.0 * (double)M * (double)N * (double)K, s);
   if (ctx->cfg.dtype == LMGC_BF16)
     launch_gemm_tc(A, B, C, M, N, K, epi, ctx->d_err, s, rope, norm);
-  else
-    launch_gemm_simt(A, B, C, M, N, K, ctx->cfg.dtype, epi == kAddResidualWide ? (int)kAddResidual : epi,
-                     s);  // kSwiGLU never reaches here
+  else  // kSwiGLU and kQKVRope never reach here
+    launch_gemm_tf32((const float*)A, (const float*)B, (float*)C, M, N, K, epi, ctx->d_err, s);
 }
 
 // kv: the qkv rows themselves (prefill), or the decoder's cache (from_cache), whose rows hold a
@@ -410,7 +410,7 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
   ctx->elt = c.dtype == LMGC_BF16 ? 2 : 4;
   if (c.dtype == LMGC_BF16) {
     // a bf16 model has one backend, the tcgen05 kernels: without the tensor-map encoder (or on a
-    // device they do not run on) the context is refused instead of computing on CUDA cores
+    // device they do not run on) the context is refused instead of computing another way
     const bool tc = tc_attention_supported(hd, ctx->qkv_dim) && tc_attention_supported(hd, ctx->kv_dim) &&
                     tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kStore) &&
                     tc_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd, kAddResidual) &&
@@ -421,6 +421,18 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
       delete ctx;
       return fail(nullptr, LMGC_ERR_INVALID,
                   "bf16 models need the tcgen05 kernels: a Blackwell device and the driver's tensor-map encoder");
+    }
+  } else {
+    // an fp32 model's contractions run on the tcgen05 TF32 kernel, likewise with no other backend
+    const bool tc = tf32_gemm_supported(1, ctx->qkv_dim, c.d_model) &&
+                    tf32_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd) &&
+                    tf32_gemm_supported(1, 2 * (int64_t)c.d_ffn, c.d_model) &&
+                    tf32_gemm_supported(1, c.d_model, c.d_ffn) && tf32_gemm_supported(1, c.vocab, c.d_model);
+    if (!tc) {
+      delete ctx;
+      return fail(nullptr, LMGC_ERR_INVALID,
+                  "fp32 models need the tcgen05 TF32 kernel: a Blackwell device, the driver's tensor-map encoder "
+                  "and inner dimensions that are multiples of 4");
     }
   }
   ctx->fused_rope = c.dtype == LMGC_BF16 && tc_gemm_supported(1, ctx->qkv_dim, c.d_model, kQKVRope);
@@ -1067,6 +1079,11 @@ lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epi 3 needs the bf16 tensor-core path and N % 256 == 0");
   if (ctx->cfg.dtype == LMGC_BF16 && M && N && !tc_gemm_supported(M, N, K, epi))
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: shape outside the tcgen05 kernel");
+  if (ctx->cfg.dtype != LMGC_BF16 && (epi == kSwiGLU || epi == kQKVRope))
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epilogue 3 is for bf16 models");
+  // the operands are read by TMA, whose global addresses must be 16-byte aligned
+  if (((uintptr_t)d_a | (uintptr_t)d_b) & 15)
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: A and B must be 16-byte aligned");
   cudaStream_t s = (cudaStream_t)stream;
   gemm(ctx, d_a, d_b, d_c, (int64_t)M, (int64_t)N, (int64_t)K, epi, s);
   LMGC_CUDA(ctx, cudaGetLastError());

@@ -1,5 +1,6 @@
 // lm.cu -- the LM prior of Eq. 2 (a Llama-family decoder, Sec. 5.1): weight generation,
-// embedding, RMSNorm, RoPE, causal GQA attention, SwiGLU, and a CUDA-core GEMM.
+// embedding, RMSNorm, RoPE, causal GQA attention on CUDA cores (fp32 models), SwiGLU. The dense
+// contractions are on the tensor cores (gemm_tc.cu, gemm_tf32.cu).
 //
 // Every kernel here is row-invariant: a row's result depends only on that row's inputs (and, for
 // attention, on the keys/values of its window), never on M, the batch or the row's place in a
@@ -189,113 +190,6 @@ void launch_rmsnorm(const float* x, int64_t rows, int d, float eps, void* out, i
   unsigned blocks = (unsigned)((rows + 7) / 8);
   if (dtype == LMGC_BF16) k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (__half*)out);
   else k_rmsnorm<<<blocks, 256, 0, s>>>(x, rows, d, eps, (float*)out);
-}
-
-// ------------------------------------------------------------------------------------------
-// CUDA-core GEMM: C[M][N] (op)= A[M][K] . B[N][K]^T, fp32 accumulation in k order.
-// 128x128 tile, 256 threads, 8x8 outputs per thread. Used for the fp32 model and as the bf16
-// path where the tensor-core GEMM does not apply.
-// Epilogues: kStore (C has A's type), kAddResidual (C fp32 += acc), kStoreF32 (C fp32 = acc).
-// ------------------------------------------------------------------------------------------
-constexpr int GBM = 128, GBN = 128, GBK = 16;
-
-template <typename T>
-__device__ __forceinline__ void load8(const T* p, float* v, bool ok);
-template <>
-__device__ __forceinline__ void load8<float>(const float* p, float* v, bool ok) {
-  if (ok) {
-    float4 a = *reinterpret_cast<const float4*>(p);
-    float4 b = *reinterpret_cast<const float4*>(p + 4);
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; i++) v[i] = 0.f;
-  }
-}
-template <>
-__device__ __forceinline__ void load8<__half>(const __half* p, float* v, bool ok) {
-  if (ok) {
-    uint4 q = *reinterpret_cast<const uint4*>(p);
-    const __half2* h = reinterpret_cast<const __half2*>(&q);
-#pragma unroll
-    for (int i = 0; i < 4; i++) {
-      float2 f = __half22float2(h[i]);
-      v[2 * i] = f.x;
-      v[2 * i + 1] = f.y;
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; i++) v[i] = 0.f;
-  }
-}
-
-template <typename T>
-__global__ void __launch_bounds__(256) k_gemm_simt(const T* __restrict__ A, const T* __restrict__ B, void* C,
-                                                   int64_t M, int64_t N, int64_t K, int epi) {
-  __shared__ __align__(16) float As[GBK][GBM + 4];
-  __shared__ __align__(16) float Bs[GBK][GBN + 4];
-  const int t = threadIdx.x;
-  const int tx = t & 15, ty = t >> 4;
-  const int64_t m0 = (int64_t)blockIdx.y * GBM, n0 = (int64_t)blockIdx.x * GBN;
-  // loader: each thread loads 8 consecutive k of one row of A and of B per k-tile
-  const int lr = t >> 1, lk = (t & 1) * 8;
-  float acc[8][8];
-#pragma unroll
-  for (int i = 0; i < 8; i++)
-#pragma unroll
-    for (int j = 0; j < 8; j++) acc[i][j] = 0.f;
-  for (int64_t k0 = 0; k0 < K; k0 += GBK) {
-    float va[8], vb[8];
-    int64_t ar = m0 + lr, br = n0 + lr;
-    bool kok = k0 + lk < K;  // K % 8 == 0
-    load8<T>(A + ar * K + k0 + lk, va, ar < M && kok);
-    load8<T>(B + br * K + k0 + lk, vb, br < N && kok);
-    __syncthreads();
-#pragma unroll
-    for (int i = 0; i < 8; i++) {
-      As[lk + i][lr] = va[i];
-      Bs[lk + i][lr] = vb[i];
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < GBK; kk++) {
-      float a[8], b[8];
-      float4 a0 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-      float4 a1 = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
-      float4 b0 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
-      float4 b1 = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
-      a[0] = a0.x; a[1] = a0.y; a[2] = a0.z; a[3] = a0.w; a[4] = a1.x; a[5] = a1.y; a[6] = a1.z; a[7] = a1.w;
-      b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w; b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
-#pragma unroll
-      for (int i = 0; i < 8; i++)
-#pragma unroll
-        for (int j = 0; j < 8; j++) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < 8; i++) {
-    int64_t m = m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + i - 4);
-    if (m >= M) continue;
-#pragma unroll
-    for (int j = 0; j < 8; j++) {
-      int64_t n = n0 + (j < 4 ? tx * 4 + j : 64 + tx * 4 + j - 4);
-      if (n >= N) continue;
-      if (epi == kStore) reinterpret_cast<T*>(C)[m * N + n] = from_f<T>(acc[i][j]);
-      else if (epi == kAddResidual) reinterpret_cast<float*>(C)[m * N + n] += acc[i][j];
-      else reinterpret_cast<float*>(C)[m * N + n] = acc[i][j];
-    }
-  }
-}
-
-void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
-                      cudaStream_t s) {
-  if (M <= 0 || N <= 0) return;
-  note_launch();
-  dim3 grid((unsigned)((N + GBN - 1) / GBN), (unsigned)((M + GBM - 1) / GBM));
-  if (dtype == LMGC_BF16)
-    k_gemm_simt<<<grid, 256, 0, s>>>((const __half*)A, (const __half*)B, C, M, N, K, epi);
-  else
-    k_gemm_simt<<<grid, 256, 0, s>>>((const float*)A, (const float*)B, C, M, N, K, epi);
 }
 
 // ------------------------------------------------------------------------------------------

@@ -194,8 +194,11 @@ struct RopeArgs {
   int pos_mod;       // row m sits at position pos0 + m % pos_mod
   int64_t pos0;
 };
-void launch_gemm_simt(const void* A, const void* B, void* C, int64_t M, int64_t N, int64_t K, int dtype, int epi,
-                      cudaStream_t s);
+// fp32 models: C (op)= A . B^T on the tensor cores in three-pass TF32 form (gemm_tf32.cu);
+// epi kStore / kStoreF32 (C = acc) or kAddResidual (C += acc), C fp32 [M][N]
+bool tf32_gemm_supported(int64_t M, int64_t N, int64_t K);
+void launch_gemm_tf32(const float* A, const float* B, float* C, int64_t M, int64_t N, int64_t K, int epi,
+                      uint32_t* err, cudaStream_t s);
 void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
                  int64_t pos_first, int64_t q_win_stride, int n_pos, int dtype, cudaStream_t s);
 void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,

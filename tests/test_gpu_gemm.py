@@ -1,12 +1,12 @@
 """The model's dense contraction (lmgc_gemm): C = A . B^T for the linear layers and the
-vocabulary projection of the Eq. 2 model. A bf16-weight model computes with fp16 operands on the
-tcgen05 kernel (its bf16 weight values are exact in fp16), an fp32 model on CUDA cores; compared
-with the fp64 definition. Bound per element: accumulation error
-<= 2^-19 * sum_k |a_k b_k| on the tensor cores (their fp32 accumulation aligns products
-with truncation, measured at up to 1.4 x 2^-22 * sum |a b|), and the standard bound of sequential fp32 summation,
-K * 2^-24 * sum |a b|, on CUDA cores; plus one fp16 rounding of the output for epilogues 0 and 3:
-2^-11 relative (2^-10 allowed), and below 2^-14 the fixed 2^-24 spacing of fp16 subnormals
-(2^-25 absolute)."""
+vocabulary projection of the Eq. 2 model, compared with the fp64 definition. A bf16-weight model
+computes with fp16 operands on the tcgen05 kernel (its bf16 weight values are exact in fp16); an
+fp32 model with fp32 operands on the tcgen05 kernel in three-pass TF32 form. Bound per element:
+accumulation error <= 2^-19 * sum_k |a_k b_k| on the tensor cores (their fp32 accumulation aligns
+products with truncation, measured at up to 1.4 x 2^-22 * sum |a b|); for the TF32 form also the
+split's terms (see test_gemm_fp32_tf32x3); plus one fp16 rounding of the output for epilogues 0
+and 3: 2^-11 relative (2^-10 allowed), and below 2^-14 the fixed 2^-24 spacing of fp16
+subnormals (2^-25 absolute)."""
 import numpy as np
 import pytest
 import torch
@@ -84,17 +84,64 @@ def test_gemm_tc_row_invariance(ctx_f16):
     assert torch.equal(part, full[517:520])
 
 
-def test_gemm_fp32_simt():
-    ctx = L.Context(configs.with_(configs.TINY, batch_windows=1))
-    g = torch.Generator().manual_seed(1)
-    a = torch.randn(300, 136, generator=g)
-    b = torch.randn(520, 136, generator=g)
-    c = torch.empty(300, 520, device="cuda")
-    L.lmgc_gemm(ctx, a.cuda(), b.cuda(), c, 2)
-    ref = O.gemm_nt(a.numpy(), b.numpy())
-    bound = 136 * 2.0 ** -24 * O.gemm_nt(np.abs(a.numpy()), np.abs(b.numpy()))
-    assert np.all(np.abs(c.cpu().numpy() - ref) <= bound)
-    ctx.close()
+@pytest.fixture(scope="module")
+def ctx_f32():
+    c = L.Context(configs.with_(configs.TINY, batch_windows=1))
+    yield c
+    c.close()
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 520, 136), (128, 128, 32), (1, 384, 128), (36864 // 9, 1024, 128),
+                                   (257, 32, 512), (5, 17, 8), (1000, 130, 520)])
+@pytest.mark.parametrize("epi", [0, 1, 2])
+def test_gemm_fp32_tf32x3(ctx_f32, M, N, K, epi):
+    """An fp32 model's contraction on the tcgen05 TF32 kernel in three passes (lo_A hi_B + hi_A lo_B
+    + hi_A hi_B, hi = x with its low 13 bits cleared). Bound per element: the dropped lo_A lo_B
+    term (< 2^-20 |a b|), the truncation of each lo to TF32 in the two cross terms (< 2^-20 |a b|
+    each) and the tensor cores' fp32 accumulation (2^-19 sum |a b|, as for the fp16 kernel):
+    2^-19 + 3 2^-20 < 2^-17 of sum_k |a_k b_k|, plus one fp32 rounding of C += for epilogue 1.
+    Shapes with ragged M and N tiles, N <= 32 (the narrow tile), K not a multiple of the 32-wide K
+    step, and M = 1 (a decode step)."""
+    g = torch.Generator().manual_seed(M + N + K + epi)
+    a = torch.randn(M, K, generator=g)
+    b = torch.randn(N, K, generator=g)
+    c0 = torch.randn(M, N, generator=g)
+    c = c0.clone().cuda() if epi == 1 else torch.full((M, N), float("nan"), device="cuda")
+    L.lmgc_gemm(ctx_f32, a.cuda(), b.cuda(), c, epi)
+    an, bn = a.numpy().astype(np.float64), b.numpy().astype(np.float64)
+    ref = O.gemm_nt(an, bn)
+    bound = 2.0 ** -17 * O.gemm_nt(np.abs(an), np.abs(bn)) + 1e-30
+    if epi == 1:
+        ref = ref + c0.numpy().astype(np.float64)
+        bound += 2.0 ** -23 * np.abs(ref)
+    got = c.cpu().numpy().astype(np.float64)
+    err = np.abs(got - ref)
+    assert np.all(err <= bound), float((err / bound).max())
+
+
+def test_gemm_fp32_rows_independent_of_m(ctx_f32):
+    """Each row of C is the same whatever M and the row's place in a tile (the decoder's one-row
+    steps reproduce the encoder's logits bit for bit)."""
+    g = torch.Generator().manual_seed(7)
+    a = torch.randn(700, 128, generator=g).cuda()
+    b = torch.randn(384, 128, generator=g).cuda()
+    full = torch.empty(700, 384, device="cuda")
+    L.lmgc_gemm(ctx_f32, a, b, full, 2)
+    for r in (0, 127, 128, 333, 699):
+        one = torch.empty(1, 384, device="cuda")
+        L.lmgc_gemm(ctx_f32, a[r:r + 1].contiguous(), b, one, 2)
+        assert torch.equal(one[0], full[r])
+    part = torch.empty(3, 384, device="cuda")
+    L.lmgc_gemm(ctx_f32, a[517:520].contiguous(), b, part, 2)
+    assert torch.equal(part, full[517:520])
+
+
+def test_gemm_rejects_misaligned_operands(ctx_f32):
+    a = torch.randn(9, 64, device="cuda")
+    b = torch.randn(32, 64, device="cuda")
+    with pytest.raises(L.LmgcError) as e:
+        L.lmgc_gemm(ctx_f32, a.view(-1)[1:1 + 8 * 64].view(8, 64), b, torch.zeros(8, 32, device="cuda"), 2)
+    assert e.value.status == L.ERR_INVALID
 
 
 def test_gemm_rejects_bad_k(ctx_f16):
