@@ -148,14 +148,15 @@ static void attention(lmgc_ctx* ctx, const void* q, const void* kv, void* out, i
   const int qd = c.n_heads * ctx->hd, kd = c.n_kv_heads * ctx->hd;
   const int64_t kv_dim = from_cache ? 2 * kd : ctx->qkv_dim;
   const int k_off = from_cache ? 0 : qd, v_off = k_off + kd;
-  if (c.dtype == LMGC_BF16) {  // lmgc_create admitted only head layouts the tcgen05 kernel takes
-    const int64_t q_rows = q_win_stride == 1 ? n_win : n_win * c.window;
+  // lmgc_create admitted only head layouts the tcgen05 kernels take
+  const int64_t q_rows = q_win_stride == 1 ? n_win : n_win * c.window;
+  if (c.dtype == LMGC_BF16)
     launch_attention_tc(q, q_rows, ctx->qkv_dim, kv, n_win * c.window, kv_dim, k_off, v_off, out, qd, c.n_heads,
                         c.n_kv_heads, ctx->hd, c.window, n_win, pos_first, n_pos, q_win_stride, ctx->d_err, s);
-  } else {
-    launch_attention(q, ctx->qkv_dim, kv, kv_dim, k_off, v_off, out, qd, c.n_heads, c.n_kv_heads, ctx->hd, c.window,
-                     n_win, pos_first, n_pos, q_win_stride, c.dtype, s);
-  }
+  else
+    launch_attention_tf32((const float*)q, q_rows, ctx->qkv_dim, (const float*)kv, n_win * c.window, kv_dim, k_off,
+                          v_off, (float*)out, qd, c.n_heads, c.n_kv_heads, ctx->hd, c.window, n_win, pos_first,
+                          n_pos, q_win_stride, ctx->d_err, s);
 }
 
 // One forward of the model over `rows` input rows already embedded into ws.x.
@@ -379,9 +380,10 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
       c.d_model % c.n_heads || c.n_heads % c.n_kv_heads || c.vocab < 20 || c.window < 1 || c.batch_windows < 1)
     return fail(nullptr, LMGC_ERR_INVALID, "bad model shape");
   const int hd = c.d_model / c.n_heads;
-  if (hd != 32 && hd != 64 && hd != 128) return fail(nullptr, LMGC_ERR_INVALID, "head dim must be 32, 64 or 128");
-  if (c.dtype == LMGC_BF16 && hd == 32)
+  if (c.dtype == LMGC_BF16 && hd != 64 && hd != 128)
     return fail(nullptr, LMGC_ERR_INVALID, "head dim of a bf16 model must be 64 or 128 (tcgen05 attention)");
+  if (c.dtype != LMGC_BF16 && hd != 32 && hd != 64)
+    return fail(nullptr, LMGC_ERR_INVALID, "head dim of an fp32 model must be 32 or 64 (tcgen05 TF32 attention)");
   if (c.d_model % 8 || c.d_ffn % 8) return fail(nullptr, LMGC_ERR_INVALID, "d_model and d_ffn must be multiples of 8");
   if (c.cdf_bits < 1 || c.cdf_bits > 30 || (int64_t)c.vocab >= (1ll << c.cdf_bits))
     return fail(nullptr, LMGC_ERR_INVALID, "cdf_bits must satisfy vocab < 2^cdf_bits <= 2^30");
@@ -424,14 +426,16 @@ lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out) {
     }
   } else {
     // an fp32 model's contractions run on the tcgen05 TF32 kernel, likewise with no other backend
-    const bool tc = tf32_gemm_supported(1, ctx->qkv_dim, c.d_model) &&
+    const bool tc = tf32_attention_supported(hd, ctx->qkv_dim, ctx->qkv_dim) &&
+                    tf32_attention_supported(hd, ctx->qkv_dim, ctx->kv_dim) &&
+                    tf32_gemm_supported(1, ctx->qkv_dim, c.d_model) &&
                     tf32_gemm_supported(1, c.d_model, (int64_t)c.n_heads * hd) &&
                     tf32_gemm_supported(1, 2 * (int64_t)c.d_ffn, c.d_model) &&
                     tf32_gemm_supported(1, c.d_model, c.d_ffn) && tf32_gemm_supported(1, c.vocab, c.d_model);
     if (!tc) {
       delete ctx;
       return fail(nullptr, LMGC_ERR_INVALID,
-                  "fp32 models need the tcgen05 TF32 kernel: a Blackwell device, the driver's tensor-map encoder "
+                  "fp32 models need the tcgen05 TF32 kernels: a Blackwell device, the driver's tensor-map encoder "
                   "and inner dimensions that are multiples of 4");
     }
   }

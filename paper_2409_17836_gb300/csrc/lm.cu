@@ -1,6 +1,7 @@
 // lm.cu -- the LM prior of Eq. 2 (a Llama-family decoder, Sec. 5.1): weight generation,
-// embedding, RMSNorm, RoPE, causal GQA attention on CUDA cores (fp32 models), SwiGLU. The dense
-// contractions are on the tensor cores (gemm_tc.cu, gemm_tf32.cu).
+// embedding, RMSNorm, RoPE, SwiGLU (the kernels bf16 models do not fold into their GEMM
+// epilogues, and fp32 models use). The dense contractions and attention are on the tensor cores
+// (gemm_tc.cu, attn_tc.cu; gemm_tf32.cu, attn_tf32.cu for fp32 models).
 //
 // Every kernel here is row-invariant: a row's result depends only on that row's inputs (and, for
 // attention, on the keys/values of its window), never on M, the batch or the row's place in a
@@ -227,174 +228,6 @@ void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, 
   if (dtype == LMGC_BF16)
     k_rope<<<blocks, 256, 0, s>>>((__half*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
   else k_rope<<<blocks, 256, 0, s>>>((float*)qkv, rows, qkv_dim, n_rot_heads, hd, cs, pos_first, q_win_stride);
-}
-
-// ------------------------------------------------------------------------------------------
-// Causal softmax attention with grouped-query heads, CUDA cores, fp32 online softmax.
-// Block (qb, h, w): query positions pos_first + qb*64 + [0, 64) of window w (at most n_pos of
-// them); query row for position p: w*q_win_stride + (p - pos_first). Keys/values of window w at
-// position j: kv row w*W + j (k at column k_off + kvh*hd, v at v_off + kvh*hd). Key blocks are
-// 64-aligned and visited in order 0, 1, ..., so a row's arithmetic is the same whether it is
-// computed in a full prefill block or alone in a decode step.
-// ------------------------------------------------------------------------------------------
-constexpr int ABQ = 64, ABK = 64;
-
-template <typename T, int HD>
-__global__ void __launch_bounds__(256) k_attention(const T* __restrict__ q, int64_t q_stride,
-                                                   const T* __restrict__ kv, int64_t kv_stride, int k_off, int v_off,
-                                                   T* __restrict__ out, int64_t out_stride, int nq, int nkv, int W,
-                                                   int64_t pos_first, int n_pos, int64_t q_win_stride, float scale) {
-  extern __shared__ __align__(16) float sm[];
-  float* Qs = sm;                       // [ABQ][HD]
-  float* Kt = Qs + ABQ * HD;            // [HD][ABK] (transposed)
-  float* Vs = Kt + HD * ABK;            // [ABK][HD]
-  float* Ps = Vs + ABK * HD;            // [ABQ][ABK + 1]
-  const int t = threadIdx.x, tx = t & 15, ty = t >> 4;
-  const int qb = blockIdx.x, h = blockIdx.y;
-  const int64_t w = blockIdx.z;
-  const int kvh = h / (nq / nkv);
-  const int64_t p_lo = pos_first + (int64_t)qb * ABQ;
-  const int64_t rem_pos = pos_first + n_pos - p_lo;
-  const int nrows = rem_pos < ABQ ? (int)rem_pos : ABQ;
-  if (nrows <= 0) return;
-  const int64_t p_hi = p_lo + nrows - 1;
-  for (int e = t; e < ABQ * HD; e += 256) {
-    int r = e / HD, c = e - r * HD;
-    float v = 0.f;
-    if (r < nrows) v = to_f<T>(q[(w * q_win_stride + (p_lo + r - pos_first)) * q_stride + (int64_t)h * HD + c]);
-    Qs[e] = v;
-  }
-  constexpr int OC = HD / 16;
-  float m[4], l[4], o[4][OC];
-#pragma unroll
-  for (int r = 0; r < 4; r++) {
-    m[r] = -INFINITY;
-    l[r] = 0.f;
-#pragma unroll
-    for (int c = 0; c < OC; c++) o[r][c] = 0.f;
-  }
-  const int nkb = (int)(p_hi / ABK) + 1;
-  for (int kb = 0; kb < nkb; kb++) {
-    __syncthreads();
-    for (int e = t; e < ABK * HD; e += 256) {
-      int j = e / HD, c = e - j * HD;
-      int64_t pj = (int64_t)kb * ABK + j;
-      float kvv = 0.f, vvv = 0.f;
-      if (pj <= p_hi) {
-        const T* row = kv + (w * W + pj) * kv_stride;
-        kvv = to_f<T>(row[k_off + kvh * HD + c]);
-        vvv = to_f<T>(row[v_off + kvh * HD + c]);
-      }
-      Kt[c * ABK + j] = kvv;
-      Vs[j * HD + c] = vvv;
-    }
-    __syncthreads();
-    float s[4][4];
-#pragma unroll
-    for (int r = 0; r < 4; r++)
-#pragma unroll
-      for (int c = 0; c < 4; c++) s[r][c] = 0.f;
-#pragma unroll 4
-    for (int d = 0; d < HD; d++) {
-      float4 kk = *reinterpret_cast<const float4*>(&Kt[d * ABK + tx * 4]);
-#pragma unroll
-      for (int r = 0; r < 4; r++) {
-        float qv = Qs[(ty * 4 + r) * HD + d];
-        s[r][0] = fmaf(qv, kk.x, s[r][0]);
-        s[r][1] = fmaf(qv, kk.y, s[r][1]);
-        s[r][2] = fmaf(qv, kk.z, s[r][2]);
-        s[r][3] = fmaf(qv, kk.w, s[r][3]);
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 4; r++) {
-      const int64_t p = p_lo + ty * 4 + r;
-      float mx = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < 4; c++) {
-        int64_t j = (int64_t)kb * ABK + tx * 4 + c;
-        s[r][c] = (j <= p) ? s[r][c] * scale : -INFINITY;
-        mx = fmaxf(mx, s[r][c]);
-      }
-#pragma unroll
-      for (int off = 8; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      const float mn = fmaxf(m[r], mx);
-      const float corr = (mn == -INFINITY) ? 1.f : expf(m[r] - mn);
-      float rs = 0.f;
-#pragma unroll
-      for (int c = 0; c < 4; c++) {
-        float pv = (s[r][c] == -INFINITY) ? 0.f : expf(s[r][c] - mn);
-        s[r][c] = pv;
-        rs += pv;
-      }
-#pragma unroll
-      for (int off = 8; off > 0; off >>= 1) rs += __shfl_xor_sync(0xffffffffu, rs, off);
-      l[r] = l[r] * corr + rs;
-      m[r] = mn;
-#pragma unroll
-      for (int c = 0; c < OC; c++) o[r][c] *= corr;
-#pragma unroll
-      for (int c = 0; c < 4; c++) Ps[(ty * 4 + r) * (ABK + 1) + tx * 4 + c] = s[r][c];
-    }
-    __syncthreads();
-#pragma unroll 4
-    for (int j = 0; j < ABK; j++) {
-      float vv[OC];
-#pragma unroll
-      for (int c = 0; c < OC; c++) vv[c] = Vs[j * HD + tx + 16 * c];
-#pragma unroll
-      for (int r = 0; r < 4; r++) {
-        float pv = Ps[(ty * 4 + r) * (ABK + 1) + j];
-#pragma unroll
-        for (int c = 0; c < OC; c++) o[r][c] = fmaf(pv, vv[c], o[r][c]);
-      }
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < 4; r++) {
-    int rr = ty * 4 + r;
-    if (rr >= nrows) continue;
-    float inv = 1.f / l[r];
-    T* orow = out + (w * q_win_stride + (p_lo + rr - pos_first)) * out_stride + (int64_t)h * HD;
-#pragma unroll
-    for (int c = 0; c < OC; c++) orow[tx + 16 * c] = from_f<T>(o[r][c] * inv);
-  }
-}
-
-template <typename T, int HD>
-static void attn_launch(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
-                        void* out, int64_t out_stride, int nq, int nkv, int W, int64_t n_win, int64_t pos_first,
-                        int n_pos, int64_t q_win_stride, cudaStream_t s) {
-  size_t smem = sizeof(float) * (ABQ * HD + HD * ABK + ABK * HD + ABQ * (ABK + 1));
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaFuncSetAttribute(k_attention<T, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    attr_done = true;
-  }
-  dim3 grid((unsigned)((n_pos + ABQ - 1) / ABQ), (unsigned)nq, (unsigned)n_win);
-  float scale = 1.0f / sqrtf((float)HD);
-  note_launch();
-  k_attention<T, HD><<<grid, 256, smem, s>>>((const T*)q, q_stride, (const T*)kv, kv_stride, k_off, v_off, (T*)out,
-                                             out_stride, nq, nkv, W, pos_first, n_pos, q_win_stride, scale);
-}
-
-void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
-                      void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
-                      int64_t pos_first, int n_pos, int64_t q_win_stride, int dtype, cudaStream_t s) {
-  if (n_win <= 0 || n_pos <= 0) return;
-#define LMGC_ATT(T, HDV)                                                                                        \
-  attn_launch<T, HDV>(q, q_stride, kv, kv_stride, k_off, v_off, out, out_stride, nq, nkv, W, n_win, pos_first, \
-                      n_pos, q_win_stride, s)
-  if (dtype == LMGC_BF16) {
-    if (hd == 32) LMGC_ATT(__half, 32);
-    else if (hd == 64) LMGC_ATT(__half, 64);
-    else LMGC_ATT(__half, 128);
-  } else {
-    if (hd == 32) LMGC_ATT(float, 32);
-    else if (hd == 64) LMGC_ATT(float, 64);
-    else LMGC_ATT(float, 128);
-  }
-#undef LMGC_ATT
 }
 
 // act[r][j] = silu(g) * u, g = gu[r][j], u = gu[r][ffn + j]

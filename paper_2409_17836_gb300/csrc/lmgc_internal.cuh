@@ -201,9 +201,13 @@ void launch_gemm_tf32(const float* A, const float* B, float* C, int64_t M, int64
                       uint32_t* err, cudaStream_t s);
 void launch_rope(void* qkv, int64_t rows, int qkv_dim, int n_rot_heads, int hd, const float2* cs, int W,
                  int64_t pos_first, int64_t q_win_stride, int n_pos, int dtype, cudaStream_t s);
-void launch_attention(const void* q, int64_t q_stride, const void* kv, int64_t kv_stride, int k_off, int v_off,
-                      void* out, int64_t out_stride, int nq, int nkv, int hd, int W, int64_t n_win,
-                      int64_t pos_first, int n_pos, int64_t q_win_stride, int dtype, cudaStream_t s);
+// fp32 models: causal attention on the tensor cores in three-pass TF32 form (attn_tf32.cu), head
+// dim 32 or 64; arguments as launch_attention_tc's
+bool tf32_attention_supported(int hd, int64_t q_dim, int64_t kv_dim);
+void launch_attention_tf32(const float* q, int64_t q_rows, int64_t q_dim, const float* kv, int64_t kv_rows,
+                           int64_t kv_dim, int k_off, int v_off, float* out, int64_t out_stride, int nq, int nkv,
+                           int hd, int W, int64_t n_win, int64_t pos_first, int n_pos, int64_t q_win_stride,
+                           uint32_t* err, cudaStream_t s);
 void launch_swiglu(const void* gu, int64_t rows, int ffn, void* act, int dtype, cudaStream_t s);
 void launch_copy_rows(const void* src, int64_t src_stride, void* dst, int64_t dst_win_stride, int64_t dst_pos,
                       int64_t n_rows, int64_t row_elems, int dtype, cudaStream_t s);

@@ -53,6 +53,19 @@ def test_tiny_fp32_all_positions():
     compare(configs.TINY, tok, [0, 3, 5], 256)
 
 
+@pytest.mark.parametrize("hd,nkv", [(32, 2), (64, 2), (64, 1)])
+def test_small_fp32_ragged(hd, nkv):
+    """fp32 on the tcgen05 TF32 kernels: GQA, head dims 32 and 64, a window of 200 positions
+    (three full 64-key blocks and a ragged fourth, two 128-row query tiles), a partial last
+    window, and weights large enough (init_std 0.2) for the softmax maximum to move between
+    key blocks."""
+    cfg = L.ModelConfig(n_layers=2, d_model=128, n_heads=128 // hd, n_kv_heads=nkv, d_ffn=256, vocab=40,
+                        dtype=L.F32, window=200, cdf_bits=16, init_std=0.2)
+    rng = np.random.default_rng(100 + hd + nkv)
+    tok = tokens(rng, 200 * 3 + 57)
+    compare(cfg, tok, [0, 2, 3], 200, batch=2)
+
+
 @pytest.mark.parametrize("hd,nkv", [(64, 2), (128, 2), (64, 1)])
 def test_small_bf16_ragged(hd, nkv):
     """bf16, several GEMM tiles, GQA, a ragged window (130 = 2*64 + 2) and a partial last window."""

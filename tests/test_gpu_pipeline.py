@@ -47,6 +47,23 @@ def test_tiny_full_encode_decode_and_oracle_size():
     ctx.close()
 
 
+def test_fp32_gqa_hd64_round_trip():
+    """An fp32 model with head dim 64 and grouped-query heads (the other shape of the TF32
+    attention): encode then decode of every window is lossless, the decoder's one-row steps
+    (keys and values from the cache) reproducing the encoder's logits; 14 windows of 200 tokens
+    (the last partial) in batches of 4."""
+    cfg = L.ModelConfig(n_layers=2, d_model=128, n_heads=2, n_kv_heads=1, d_ffn=256, vocab=32, dtype=L.F32,
+                        window=200, cdf_bits=16, batch_windows=4, init_std=0.1)
+    ctx = L.Context(cfg)
+    vals = I.tiny_gradient(0)[:300]  # 2700 tokens
+    buf = encode(ctx, vals)
+    h = parse(buf)
+    assert h["n_win"] == 14
+    toks = decode_all(ctx, buf, list(range(14)))
+    assert np.array_equal(toks.reshape(-1)[:2700], O.serialize(vals, 0))
+    ctx.close()
+
+
 def test_decode_batch_windows():
     """The decode batch query: at least one window, at most one workspace row per window, and a
     batch that covers the KV cache the context already holds after a decode."""
