@@ -91,11 +91,12 @@ typedef struct {
 
 /* Create a context on the current CUDA device: validates the configuration, allocates the
  * weights and the workspace for `batch_windows` windows and generates the weights on the device.
- * *out receives the context. A bf16 model computes every contraction on the tcgen05 kernels and
- * has no other backend. Errors: INVALID (bad shape: d_model % n_heads, n_heads % n_kv_heads,
- * head dim not 32, 64 or 128 -- 64 or 128 for LMGC_BF16 --, vocab < 20, cdf_bits out of range;
- * LMGC_BF16 on a device or driver without the tcgen05 kernels and the tensor-map encoder),
- * NOMEM, CUDA. */
+ * *out receives the context. Every contraction (the linear layers, attention, the vocabulary
+ * projection) runs on the tcgen05 kernels, fp16 operands for LMGC_BF16 and three-pass TF32 for
+ * LMGC_F32, with no other backend. Errors: INVALID (bad shape: d_model % n_heads,
+ * n_heads % n_kv_heads, head dim not 64 or 128 for LMGC_BF16 or not 32 or 64 for LMGC_F32,
+ * vocab < 20, cdf_bits out of range; a device or driver without the tcgen05 kernels and the
+ * tensor-map encoder), NOMEM, CUDA. */
 lmgc_status lmgc_create(const lmgc_config* cfg, lmgc_ctx** out);
 
 /* Free everything the context owns. NULL is accepted. */
