@@ -143,7 +143,7 @@ lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, si
 
 /* The model's dense contraction (every linear layer of the Eq. 2 model and its vocabulary
  * projection), exposed for parity tests of the GEMM kernels: C[M][N] (op)= A[M][K] . B[N][K]^T,
- * A and B row-major and 16-byte aligned (bf16-weight contexts: fp16 on the tcgen05 kernel; fp32
+ * A, B and C row-major and 16-byte aligned (bf16-weight contexts: fp16 on the tcgen05 kernel; fp32
  * contexts: fp32 on the tcgen05 kernel in three-pass TF32 form, each operand split into a TF32
  * high part and the remainder), fp32 accumulation in k order (for LMGC_BF16 contexts A and B are
  * fp16, see lmgc_config.dtype).
@@ -152,7 +152,7 @@ lmgc_status lmgc_lm_probs(lmgc_ctx* ctx, const uint16_t* d_tok, size_t n_tok, si
  * rows interleaved in 128-row blocks (rows 256t..256t+127 gate, 256t+128..256t+255 up) and
  * C[M][N/2] (fp16) = silu(gate) * up, i.e. C[m][128t+j] = silu(R[m][256t+j]) * R[m][256t+128+j];
  * 5: as 1, through the tensor-core kernel's 8-warp epilogue (the O projection's form).
- * Errors: INVALID (K % 8 != 0, A or B not 16-byte aligned, epi outside 0..3 and 5, epi 3
+ * Errors: INVALID (K % 8 != 0, A, B or C not 16-byte aligned, epi outside 0..3 and 5, epi 3
  * unsupported), LIMIT, CUDA. Syncs. */
 lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c, size_t M, size_t N, size_t K,
                       int epi, lmgc_stream stream);

@@ -1085,9 +1085,10 @@ lmgc_status lmgc_gemm(lmgc_ctx* ctx, const void* d_a, const void* d_b, void* d_c
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: shape outside the tcgen05 kernel");
   if (ctx->cfg.dtype != LMGC_BF16 && (epi == kSwiGLU || epi == kQKVRope))
     return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: epilogue 3 is for bf16 models");
-  // the operands are read by TMA, whose global addresses must be 16-byte aligned
-  if (((uintptr_t)d_a | (uintptr_t)d_b) & 15)
-    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: A and B must be 16-byte aligned");
+  // the operands are read by TMA, whose global addresses must be 16-byte aligned, and the
+  // epilogues write C with 16-byte vector stores
+  if (((uintptr_t)d_a | (uintptr_t)d_b | (uintptr_t)d_c) & 15)
+    return fail(ctx, LMGC_ERR_INVALID, "lmgc_gemm: A, B and C must be 16-byte aligned");
   cudaStream_t s = (cudaStream_t)stream;
   gemm(ctx, d_a, d_b, d_c, (int64_t)M, (int64_t)N, (int64_t)K, epi, s);
   LMGC_CUDA(ctx, cudaGetLastError());

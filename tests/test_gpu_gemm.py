@@ -137,11 +137,17 @@ def test_gemm_fp32_rows_independent_of_m(ctx_f32):
 
 
 def test_gemm_rejects_misaligned_operands(ctx_f32):
+    """TMA reads A and B and the epilogues store C with 16-byte vectors: an operand 4 bytes off a
+    16-byte boundary is refused (INVALID) before any launch."""
     a = torch.randn(9, 64, device="cuda")
     b = torch.randn(32, 64, device="cuda")
-    with pytest.raises(L.LmgcError) as e:
-        L.lmgc_gemm(ctx_f32, a.view(-1)[1:1 + 8 * 64].view(8, 64), b, torch.zeros(8, 32, device="cuda"), 2)
-    assert e.value.status == L.ERR_INVALID
+    c = torch.zeros(8 * 32 + 1, device="cuda")
+    for args in ((a.view(-1)[1:1 + 8 * 64].view(8, 64), b[:32], c[:256].view(8, 32)),
+                 (a[:8], b.view(-1)[1:1 + 31 * 64].view(31, 64), c[:248].view(8, 31)),
+                 (a[:8], b, c[1:].view(8, 32))):
+        with pytest.raises(L.LmgcError) as e:
+            L.lmgc_gemm(ctx_f32, *args, 2)
+        assert e.value.status == L.ERR_INVALID
 
 
 def test_gemm_rejects_bad_k(ctx_f16):
