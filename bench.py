@@ -350,10 +350,10 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> 
         start[b0:b0 + nb] = st.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
         freq[b0:b0 + nb] = fr.int().view(G, 8, nb, 32).permute(2, 0, 3, 1)
         del row, sym, st, fr
-    # "range_encode": the coder as the encode path runs it, every pair checked (the checked kernel
-    # is the faster of the two: its check runs beside the serial chain); "range_encode_unchecked":
-    # the form a caller that vouches for its pairs may ask for. The codes must be identical.
-    for key, validate in (("range_encode", True), ("range_encode_unchecked", False)):
+    # "range_encode": the coder as the encode path runs it (its pairs, valid by construction, are
+    # not checked again); "range_encode_validated": the same with every pair checked, as for a
+    # caller's pairs. The codes must be identical.
+    for key, validate in (("range_encode", False), ("range_encode_validated", True)):
         payload, _ = L.lmgc_range_encode_tiled(start, freq, P, n_win, W, None, validate=validate)
         torch.cuda.synchronize()
         L.lmgc_profile(None, True)
@@ -368,9 +368,9 @@ def microbenchmarks(L, ctx, pk, reps: int = 3, coder_windows: int = 1 << 20) -> 
                     "bits_per_token": 8.0 * wr / (W * n_win), "achieved": (rd + wr) / kms / 1e6,
                     "unit": "GB/s", "frac": (rd + wr) / kms / 1e6 / pk["hbm"],
                     "tokens_per_s": W * n_win / (kms / 1e3)}
-        if not validate:
+        if validate:
             same = torch.equal(payload, ref_payload)
-            out[key]["codes_equal_checked"] = bool(same)
+            out[key]["codes_equal_unchecked"] = bool(same)
             if not same:
                 raise RuntimeError("coder microbenchmark: checked and unchecked codes differ")
         else:

@@ -208,8 +208,9 @@ lmgc_status lmgc_range_encode(const uint32_t* d_start, const uint32_t* d_freq, i
  * that every pair satisfies 0 < freq < 2^cdf_bits and start + freq <= 2^cdf_bits (as the encode
  * path's own pairs from its CDF kernels do) and the check is skipped; pairs that break this give
  * unspecified codes and bit lengths (each at most its slot's size) but no access outside the
- * call's buffers. The checked form is not slower (the encode path uses it for its own pairs). Same arithmetic, output, scratch and errors as
- * lmgc_range_encode. Syncs. */
+ * call's buffers; the encode path runs this form on its own pairs. Same arithmetic, output and
+ * errors as lmgc_range_encode; its scratch holds one code slot per window for whole blocks of 32
+ * windows (the codes of a block are interleaved in 16-byte chunks). Syncs. */
 lmgc_status lmgc_range_encode_tiled(const uint32_t* d_start, const uint32_t* d_freq, int cdf_bits, size_t n_win,
                                     size_t win_tokens, const uint32_t* d_win_len, int validate, uint8_t* d_out,
                                     size_t cap, size_t* out_bytes, uint32_t* d_bitlen, lmgc_stream stream);

@@ -651,7 +651,8 @@ static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_f
   uint8_t* slots = nullptr;
   uint64_t* offs = nullptr;
   uint32_t* derr = nullptr;
-  cudaError_t e = cudaMallocAsync((void**)&slots, slot * n_win, s);
+  // the tiled coder keeps each 32-window block's slots as one interleaved table: whole blocks
+  cudaError_t e = cudaMallocAsync((void**)&slots, slot * (tiled ? (n_win + 31) / 32 * 32 : n_win), s);
   if (e == cudaSuccess) e = cudaMallocAsync((void**)&offs, (n_win + 1) * 8 + 16, s);
   if (e == cudaSuccess) e = cudaMallocAsync((void**)&derr, 16, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(derr, 0, 4, s);
@@ -665,7 +666,7 @@ static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_f
                           (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s, tiled,
                           validate);
     }
-    launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
+    launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s, tiled);
     uint64_t total = 0;
     uint32_t herr = 0;
     e = cudaMemcpyAsync(&total, offs + n_win, 8, cudaMemcpyDeviceToHost, s);
@@ -677,7 +678,7 @@ static lmgc_status range_encode_any(const uint32_t* d_start, const uint32_t* d_f
       *out_bytes = total;
       if (cap < total) st = fail(nullptr, LMGC_ERR_NO_SPACE, "range_encode: output too small");
       else {
-        launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s);
+        launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s, tiled);
         e = cudaGetLastError();
         if (e != cudaSuccess) st = cuda_fail(nullptr, e, "range_encode pack");
       }
@@ -746,7 +747,8 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   const size_t tbl = ((size_t)n_win * 4 + 255) / 256 * 256;
   const size_t wl_off = 0, bl_off = tbl, cr_off = 2 * tbl, of_off = 3 * tbl,
                sl_off = of_off + (((size_t)n_win + 1) * 8 + 255) / 256 * 256;
-  LMGC_CUDA(ctx, ensure(&ctx->win_len, &ctx->win_cap, sl_off + slot * (size_t)n_win));
+  // the tiled coder keeps each 32-window block's slots as one interleaved table: whole blocks
+  LMGC_CUDA(ctx, ensure(&ctx->win_len, &ctx->win_cap, sl_off + slot * (((size_t)n_win + 31) / 32 * 32)));
   uint32_t* d_wl = (uint32_t*)((char*)ctx->win_len + wl_off);
   ctx->enc_bl = (uint32_t*)((char*)ctx->win_len + bl_off);
   ctx->enc_crc = (uint32_t*)((char*)ctx->win_len + cr_off);
@@ -794,14 +796,12 @@ static lmgc_status encode_codes(lmgc_ctx* ctx, const void* d_in, size_t n, int64
   launch_window_crc(ctx->tok + w_begin * W, W, d_wl, n_win, ctx->enc_crc, s);
   {
     ProfScope ps(ctx, kCoder, (double)n_win * (double)W * 8, s);
-    // the pairs come from the CDF kernels, valid by construction; they are checked all the same,
-    // as the checked kernel measured faster than the unchecked one (its check runs beside the
-    // serial chain), and an invalid pair then fails the call instead of giving a wrong code
+    // the pairs come from the CDF kernels, valid by construction: no per-pair check
     launch_range_encode(ctx->pair_start, ctx->pair_freq, (int)P, n_win, W, d_wl, 0, 0, ctx->enc_slots, slot,
-                        ctx->enc_bl, ctx->d_err, s, true, true);
+                        ctx->enc_bl, ctx->d_err, s, true, false);
   }
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[3], s));
-  launch_pack_codes(ctx->enc_slots, slot, ctx->enc_bl, n_win, ctx->enc_off, nullptr, s);
+  launch_pack_codes(ctx->enc_slots, slot, ctx->enc_bl, n_win, ctx->enc_off, nullptr, s, true);
   LMGC_CUDA(ctx, cudaMemcpyAsync(payload, ctx->enc_off + n_win, 8, cudaMemcpyDeviceToHost, s));
   lmgc_status st = check_err_word(ctx, s, "encode");
   ctx->enc_batches = n_batches;
@@ -815,7 +815,7 @@ static lmgc_status encode_pack(lmgc_ctx* ctx, uint8_t* d_payload, uint32_t* d_bi
   const int64_t n_win = ctx->enc_nwin;
   LMGC_CUDA(ctx, cudaMemcpyAsync(d_bitlen, ctx->enc_bl, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
   LMGC_CUDA(ctx, cudaMemcpyAsync(d_crc, ctx->enc_crc, 4 * (size_t)n_win, cudaMemcpyDeviceToDevice, s));
-  launch_pack_codes(ctx->enc_slots, ctx->enc_slot, ctx->enc_bl, n_win, ctx->enc_off, d_payload, s);
+  launch_pack_codes(ctx->enc_slots, ctx->enc_slot, ctx->enc_bl, n_win, ctx->enc_off, d_payload, s, true);
   LMGC_CUDA(ctx, cudaEventRecord(ctx->ev[5], s));
   LMGC_CUDA(ctx, cudaStreamSynchronize(s));
   LMGC_CUDA(ctx, cudaGetLastError());

@@ -22,7 +22,10 @@
 // carry, a count of leading zeros and a handful of selects (the step is inline PTX so that each
 // operation is one instruction). Completed words go to a per-thread ring in shared memory and
 // leave for the stream's slot in 16-byte chunks, at most two per 8 tokens: scattered 4-byte
-// stores from 32 lanes to 32 slots would cost one memory transaction each.
+// stores from 32 lanes to 32 slots would cost one memory transaction each. The tiled coder
+// interleaves the slots of a warp's 32 windows chunk by chunk (chunk c of window w at
+// (c * 32 + w % 32) * 16 bytes into the block's table), so that the chunks the 32 streams flush
+// at about the same point of their codes share memory lines.
 //
 // Layout: one stream per thread, 32 windows per warp. Pairs come from window tiles (the encode
 // path; a warp's 8 tokens are one contiguous kilobyte per array, staged through shared memory by
@@ -49,6 +52,7 @@ constexpr int kRingWords = 16;   // completed words not yet written (at most 4 +
 constexpr int kRingStride = 20;  // words per thread in shared memory: 16-byte aligned, few bank conflicts
 constexpr int kCoderThreads = 128;
 
+template <bool ILV>
 struct Stream {
   uint32_t rlo, rhi;   // r = R >> P
   uint32_t a0, a1, a2; // stream bits [32 w, 32 w + 96)
@@ -59,7 +63,8 @@ struct Stream {
   int32_t fw;          // words [0, fw) are in the slot, [fw, w - 1) only in the ring
   uint32_t chk;        // OR of s | (f - 1) | (s + f - 1) over the tokens: >= T iff a pair was invalid
   uint32_t max_words;
-  uint32_t* slot;
+  uint32_t* slot;       // the window's slot, or (ILV) the warp's table of 32 interleaved slots
+  uint32_t lane;        // ILV: this window's column of the table
   uint32_t ring;        // shared-memory address of this thread's ring (kRingWords words)
   bool overflow;
 
@@ -73,7 +78,14 @@ struct Stream {
   __device__ __forceinline__ void ring_st(int32_t i, uint32_t v) const {
     asm volatile("st.shared.u32 [%0], %1;" ::"r"(ring + 4u * (uint32_t)(i & (kRingWords - 1))), "r"(v) : "memory");
   }
-  __device__ __forceinline__ void init(int P, uint32_t* sl, uint32_t mw, uint32_t* rg) {
+  // word i of the code: slot[i], or (ILV) 16-byte chunk i / 4 of the window's column, so that
+  // the chunks the 32 windows of a warp write at about the same point of their codes lie side by
+  // side (a warp's chunk stores then touch few memory lines instead of 32)
+  __device__ __forceinline__ uint32_t* word(int32_t i) const {
+    return ILV ? slot + ((size_t)(uint32_t)(i >> 2) * 32u + lane) * 4u + (uint32_t)(i & 3) : slot + i;
+  }
+  __device__ __forceinline__ void init(int P, uint32_t* sl, uint32_t mw, uint32_t* rg, uint32_t ln = 0) {
+    lane = ln;
     const uint64_t r0 = 1ull << (62 - P);  // R = 2^62
     rlo = (uint32_t)r0;
     rhi = (uint32_t)(r0 >> 32);
@@ -97,8 +109,8 @@ struct Stream {
         ring_st(i, v);
       } else {
         if ((uint32_t)i >= max_words) break;
-        v = slot[i] + 1u;
-        slot[i] = v;
+        v = *word(i) + 1u;
+        *word(i) = v;
       }
       if (v != 0u) return;
     }
@@ -179,7 +191,7 @@ struct Stream {
                      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                      : "r"(ring + 4u * (uint32_t)(fw & (kRingWords - 1)))
                      : "memory");
-        if ((uint32_t)(fw + 3) < max_words) *reinterpret_cast<uint4*>(slot + fw) = v;
+        if ((uint32_t)(fw + 3) < max_words) *reinterpret_cast<uint4*>(word(fw)) = v;
         fw += 4;
       }
     }
@@ -208,9 +220,9 @@ struct Stream {
       nbits = (uint64_t)w * 32u + (uint64_t)nrem;
     }
     for (int32_t i = fw; i < w; i++)
-      if ((uint32_t)i < max_words) slot[i] = ring_ld(i);
-    if ((uint32_t)w < max_words) slot[w] = nrem >= 32 ? a0 : a0 & ~(0xFFFFFFFFu >> nrem);
-    if (nrem > 32 && (uint32_t)(w + 1) < max_words) slot[w + 1] = a1 & ~(0xFFFFFFFFu >> (nrem - 32));
+      if ((uint32_t)i < max_words) *word(i) = ring_ld(i);
+    if ((uint32_t)w < max_words) *word(w) = nrem >= 32 ? a0 : a0 & ~(0xFFFFFFFFu >> nrem);
+    if (nrem > 32 && (uint32_t)(w + 1) < max_words) *word(w + 1) = a1 & ~(0xFFFFFFFFu >> (nrem - 32));
     // a valid code fits its slot; pairs that were not checked may yield any length, which must
     // not send the packing step past the slot
     const uint64_t cap_bits = (uint64_t)max_words * 32u;
@@ -236,7 +248,7 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
   int64_t n = win_len ? (int64_t)win_len[w] : win_tokens;
   bool bad = n > win_tokens;
   if (bad) n = 0;  // a window longer than its slot is not coded
-  Stream c;
+  Stream<false> c;
   c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)w * slot_sz), (uint32_t)(slot_sz / 4),
          rings + threadIdx.x * kRingStride);
   constexpr int kPre = 8;
@@ -286,7 +298,8 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode(
 // its share of each tile, so that a copy instruction of the warp covers 512 contiguous bytes):
 // the copies of group g + 2 are issued once every lane has read group g's stage, and so have two
 // groups of coding to land. (Kilobyte bulk copies completing on an mbarrier, one lane issuing,
-// were 1-2% slower.) No register holds pairs ahead beyond the group being coded.
+// were 1-2% slower.) No register holds pairs ahead beyond the group being coded. The codes go to
+// the block's interleaved slot table (the slots array holds whole 32-window tables).
 template <int PT, bool CHECK>
 __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
     const uint32_t* __restrict__ start, const uint32_t* __restrict__ freq, int P_rt, int64_t n_win,
@@ -309,9 +322,9 @@ __global__ void __launch_bounds__(kCoderThreads) k_range_encode_tiles(
   int64_t g_all = (n + 7) >> 3;  // groups any window of the warp codes (warp-uniform after the max)
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) g_all = max(g_all, (int64_t)__shfl_xor_sync(0xffffffffu, (long long)g_all, o));
-  Stream c;
-  c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)(live ? w : w0) * slot_sz), (uint32_t)(slot_sz / 4),
-         rings + threadIdx.x * kRingStride);
+  Stream<true> c;
+  c.init(P, reinterpret_cast<uint32_t*>(slots + (size_t)w0 * slot_sz), (uint32_t)(slot_sz / 4),
+         rings + threadIdx.x * kRingStride, (uint32_t)lane);
   const int64_t col = pair_tile_index(w0, 0, groups);  // element of the column's first tile
   const uint32_t* ts = start + col;
   const uint32_t* tf = freq + col;
@@ -454,25 +467,33 @@ __global__ void __launch_bounds__(1024) k_scan_lengths(const uint32_t* __restric
 }
 
 __global__ void k_copy_codes(const uint8_t* __restrict__ slots, size_t slot_sz, const uint32_t* __restrict__ bitlen,
-                             const uint64_t* __restrict__ off, int64_t n, uint8_t* __restrict__ out) {
+                             const uint64_t* __restrict__ off, int64_t n, uint8_t* __restrict__ out, bool ilv) {
   for (int64_t w = blockIdx.x; w < n; w += gridDim.x) {
     const uint32_t nb = (bitlen[w] + 7u) / 8u;
-    const uint8_t* src = slots + (size_t)w * slot_sz;
     uint8_t* dst = out + off[w];
     // slot words are in native (little-endian) byte order; the code's bytes go most significant first
-    for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x) dst[b] = src[b ^ 3u];
+    if (!ilv) {
+      const uint8_t* src = slots + (size_t)w * slot_sz;
+      for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x) dst[b] = src[b ^ 3u];
+    } else {
+      // the warp's table: 16-byte chunk c of window w at ((c * 32 + w % 32) * 16) from its base
+      const uint8_t* base = slots + (size_t)(w & ~(int64_t)31) * slot_sz;
+      const uint32_t col = (uint32_t)(w & 31);
+      for (uint32_t b = threadIdx.x; b < nb; b += blockDim.x)
+        dst[b] = base[((size_t)(b >> 4) * 32u + col) * 16u + ((b & 15u) ^ 3u)];
+    }
   }
 }
 
 void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win, uint64_t* offsets,
-                       uint8_t* out, cudaStream_t s) {
+                       uint8_t* out, cudaStream_t s, bool interleaved) {
   if (n_win <= 0) return;
   note_launch();
   k_scan_lengths<<<1, 1024, 0, s>>>(bitlen, n_win, offsets);
   if (out) {
     unsigned blocks = (unsigned)std::min<int64_t>(n_win, 152 * 16);
     note_launch();
-    k_copy_codes<<<blocks, 128, 0, s>>>(slots, slot_sz, bitlen, offsets, n_win, out);
+    k_copy_codes<<<blocks, 128, 0, s>>>(slots, slot_sz, bitlen, offsets, n_win, out, interleaved);
   }
 }
 
@@ -603,7 +624,7 @@ extern "C" lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const 
   if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: clear");
   launch_range_encode(d_start, d_freq, cdf_bits, (int64_t)n_win, (int64_t)win_tokens, d_win_len,
                       (int64_t)stride_win, (int64_t)stride_pos, slots, slot, d_bitlen, derr, s);
-  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s);
+  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, nullptr, s, false);
   // a failed launch must not let the previous call's total (still in the array) be read back
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: launch");
@@ -616,7 +637,7 @@ extern "C" lmgc_status lmgc_range_encode_noalloc(const uint32_t* d_start, const 
   if (herr) return fail(nullptr, LMGC_ERR_INVALID, "lmgc_range_encode_noalloc: invalid (start, freq) or window length");
   *out_bytes = total;
   if (cap < total) return fail(nullptr, LMGC_ERR_NO_SPACE, "lmgc_range_encode_noalloc: output too small");
-  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s);
+  launch_pack_codes(slots, slot, d_bitlen, (int64_t)n_win, offs, d_out, s, false);
   e = cudaStreamSynchronize(s);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(nullptr, e, "lmgc_range_encode_noalloc: pack");

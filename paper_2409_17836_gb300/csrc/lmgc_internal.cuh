@@ -256,8 +256,10 @@ void launch_range_encode(const uint32_t* start, const uint32_t* freq, int P, int
                          const uint32_t* win_len, int64_t stride_win, int64_t stride_pos, uint8_t* slots,
                          size_t slot_sz, uint32_t* bitlen, uint32_t* err, cudaStream_t s, bool tiled = false,
                          bool check = true);
+// interleaved: the slots as the tiled coder leaves them, each 32-window block one table whose
+// 16-byte chunk c of window w lies at ((c * 32 + w % 32) * 16) from the block's first slot
 void launch_pack_codes(const uint8_t* slots, size_t slot_sz, const uint32_t* bitlen, int64_t n_win,
-                       uint64_t* offsets /* [n_win+1] scratch */, uint8_t* out, cudaStream_t s);
+                       uint64_t* offsets /* [n_win+1] scratch */, uint8_t* out, cudaStream_t s, bool interleaved);
 // crc32 of the little-endian bytes of tok[w * stride .. w * stride + len[w]) for each w < n_win
 void launch_window_crc(const uint16_t* tok, int64_t stride, const uint32_t* len, int64_t n_win, uint32_t* out,
                        cudaStream_t s);
